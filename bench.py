@@ -1,0 +1,417 @@
+#!/usr/bin/env python
+"""Benchmark of the batched softmax with slice scheduling on GB300.
+
+One step = one pass of the whole hot path over one batch: the scheduler's
+persistent kernel pulls every patch of the workload and computes its row
+softmax (bsm_softmax through the C ABI, plan cached after the first call;
+the plan itself -- topology probe, address map, Sec. 4.1/4.2 steps -- is
+built once up front, as the paper's scheduler builds its table once).
+
+Default workload: fp32 softmax over the last dim of 384 slices of 512 x 512
+(a 196608 x 512 tensor), values 3*N(0,1) from a fixed seed -- the shape of
+the paper's SOFTMAX experiment (Sec. 6).  Inputs (805 MB with the output)
+are larger than the 129 MB L2, so no flush is needed between steps.
+
+Metric: GB/s of algorithmic traffic (every input element read once, every
+output element written once) per step; also % of the measured HBM copy
+peak and of the 8 TB/s nominal, and slices/s.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 2]
+                  [--policy cbmf_lb|dynamic|rr|cbmf|whole_gpu] [--sweep]
+                  [--impl reference]
+
+--impl reference times the double-precision CPU oracle (the only other
+implementation of the path) on this machine's host cores, each step a bounded
+sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+METRIC = "batched softmax GB/s (read+write) and % of GB300 HBM peak; slices/sec"
+KERNEL_SRC = os.path.join(ROOT, "paper_2002_07062_gb300", "csrc", "bsm_kernels.cu")
+PROFILE_DIR = os.path.join(ROOT, "profiles")
+
+
+def measured_peak():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        d = json.load(open(p))
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_hash() -> str:
+    return hashlib.sha256(open(KERNEL_SRC, "rb").read()).hexdigest()[:16]
+
+
+def profiled_traffic(workload_k: int, dtype_name: str):
+    """DRAM bytes per launch of the softmax kernel from the committed ncu
+    summary for this workload, if it was taken on the current kernel source."""
+    path = os.path.join(PROFILE_DIR, "softmax_persistent_workload%d.md" % workload_k)
+    if not os.path.exists(path):
+        return None
+    text = open(path).read()
+    m_hash = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]{16})", text)
+    m_traf = re.search(r"dram_bytes_per_launch:\s*([0-9]+)", text)
+    if not m_hash or not m_traf or m_hash.group(1) != kernel_hash():
+        return None
+    return int(m_traf.group(1))
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during a region."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        time.sleep(0.25)
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        sm_sorted = sorted(sm)
+        return {"sm_mhz": sm_sorted[len(sm_sorted) // 2], "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def policy_code(name: str) -> int:
+    from paper_2002_07062_gb300 import bsm
+    return bsm.POLICIES[name]
+
+
+def run_reference(args):
+    """The oracle, as it stands, on the host cores: K timed steps, each a
+    bounded sample of the workload."""
+    import numpy as np
+    from oracle import softmax as O
+    from paper_2002_07062_gb300 import workload
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return 0
+    w = workload.config(args.workload)
+    cores = os.cpu_count() or 1
+    # calibrate on one slice, then size a step so the whole run stays ~2 minutes
+    one = workload.slice_sample(w, [0])
+    t0 = time.perf_counter()
+    O.softmax_batched(one.x, one.offsets, one.rows, one.cols, one.flags, want_f64=False,
+                      nthreads=cores)
+    t_one = max(time.perf_counter() - t0, 1e-4)
+    budget = 120.0 / max(1, args.steps + args.warmup)
+    n_sl = int(max(1, min(w.nslices, budget / t_one)))
+    samp = workload.slice_sample(w, list(range(n_sl)))
+    for _ in range(args.warmup):
+        O.softmax_batched(samp.x, samp.offsets, samp.rows, samp.cols, samp.flags,
+                          want_f64=False, nthreads=cores)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        O.softmax_batched(samp.x, samp.offsets, samp.rows, samp.cols, samp.flags,
+                          want_f64=False, nthreads=cores)
+    dt = (time.perf_counter() - t0) / args.steps
+    gbs = samp.algorithmic_bytes / dt / 1e9
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(gbs, 3), "unit": "GB/s",
+        "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(dt * 1e3, 4), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "slices_per_step": n_sl},
+        "slices_per_s": round(n_sl / dt, 3),
+        "cpu_baseline": {"value": round(gbs, 3), "unit": "GB/s", "cores": cores,
+                         "kind": "oracle",
+                         "sample": "first %d of %d slices per step" % (n_sl, w.nslices)},
+        "e2e": {"value": round(gbs, 3), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def cpu_baseline(w, seconds: float = 10.0):
+    """Oracle throughput on a bounded sample of the workload (host cores)."""
+    from oracle import softmax as O
+    from paper_2002_07062_gb300 import workload
+    cores = os.cpu_count() or 1
+    one = workload.slice_sample(w, [0])
+    t0 = time.perf_counter()
+    O.softmax_batched(one.x, one.offsets, one.rows, one.cols, one.flags, want_f64=False,
+                      nthreads=cores)
+    t_one = max(time.perf_counter() - t0, 1e-4)
+    n_sl = int(max(1, min(w.nslices, seconds / t_one)))
+    samp = workload.slice_sample(w, list(range(n_sl)))
+    t0 = time.perf_counter()
+    O.softmax_batched(samp.x, samp.offsets, samp.rows, samp.cols, samp.flags, want_f64=False,
+                      nthreads=cores)
+    dt = time.perf_counter() - t0
+    return {"value": round(samp.algorithmic_bytes / dt / 1e9, 4), "unit": "GB/s",
+            "cores": cores, "kind": "oracle",
+            "sample": "first %d of %d slices (%.1f s, double precision, %d threads)"
+                      % (n_sl, w.nslices, dt, cores)}
+
+
+def time_steps(fn, steps, stream, per_launch=True):
+    """Run fn() `steps` times on `stream`; returns (total ms, per-step ms list)."""
+    import torch
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(steps)] if per_launch else []
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for k in range(steps):
+        if per_launch:
+            ev[k][0].record(stream)
+        fn()
+        if per_launch:
+            ev[k][1].record(stream)
+    end.record(stream)
+    end.synchronize()
+    per = [a.elapsed_time(b) for a, b in ev] if per_launch else []
+    return start.elapsed_time(end), per
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--workload", type=int, default=2)
+    ap.add_argument("--policy", default="dynamic")
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--sweep", action="store_true",
+                    help="also time every policy on workloads 2-5 (extra JSON lines)")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=20)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import numpy as np
+    import torch
+    import __graft_entry__ as g
+    from paper_2002_07062_gb300 import bsm, workload
+
+    ws, rank, local = dist_env()
+    if ws > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    else:
+        torch.cuda.set_device(0)
+    if rank == 0 or ws == 1:
+        g.build()
+    if ws > 1:
+        dist.barrier()
+        g.build()
+    dev = torch.cuda.current_device()
+
+    w = workload.config(args.workload).materialize()
+    pol = policy_code(args.policy)
+    xh = w.x
+    x = torch.from_numpy(xh.view(np.int16) if w.dtype == workload.BF16 else xh).cuda()
+    if w.dtype == workload.BF16:
+        x = x.view(torch.bfloat16)
+    y = torch.empty_like(x)
+    stream = torch.cuda.Stream()
+    uniform = w.uniform
+    B, R, C = w.nslices, int(w.rows[0]), int(w.cols[0])
+
+    def step():
+        if uniform:
+            bsm.bsm_softmax_ex(x, y, B, R, C, w.dtype, pol, w.flags, stream)
+        else:
+            bsm.bsm_softmax_ragged(x, y, w.offsets, w.rows, w.cols, w.dtype, pol, w.flags, stream)
+
+    # plan once (cached), then the same plan's stats for the launch count
+    with torch.cuda.stream(stream):
+        step()
+    stream.synchronize()
+    plan = bsm.bsm_plan_create(x, y, w.rows, w.cols, w.dtype, pol, offsets=w.offsets,
+                               flags=w.flags)
+    st = plan.stats()
+    plan.close()
+    launches_per_step = int(st["launches"])
+
+    for _ in range(args.warmup):
+        step()
+    stream.synchronize()
+    if ws > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(dev) as clk:
+        total_ms, per = time_steps(step, args.steps, stream, per_launch=launches_per_step == 1)
+    torch.cuda.synchronize()
+    if ws > 1:
+        dist.barrier()
+        t = torch.tensor([total_ms], device="cuda", dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    status = bsm.bsm_device_status()
+    ms = total_ms / args.steps
+    bytes_step = w.algorithmic_bytes
+    value = ws * bytes_step / (ms * 1e-3) / 1e9
+    peak, peak_src = measured_peak()
+    launch_ms = float(np.mean(per)) if per else ms
+    achieved = bytes_step / (launch_ms * 1e-3) / 1e9
+    traffic = profiled_traffic(args.workload, "f32")
+
+    out = {
+        "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": ws,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 5),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f32" if w.dtype == workload.F32 else "bf16", "data": "synthetic",
+        "config": {"workload": w.name, "policy": args.policy, "slices": B,
+                   "rows": R if uniform else "ragged", "cols": C if uniform else "ragged",
+                   "causal": bool(w.flags & 1), "seed": hex(w.seed),
+                   "bytes_per_step": bytes_step,
+                   "l2": "inputs larger than L2 (%d MB vs 129 MB), no flush" % (bytes_step >> 20),
+                   "parallelism": "slices sharded by rank, no collective" if ws > 1 else "1 GPU"},
+        "pct_of_measured_hbm": round(100 * value / ws / peak, 2),
+        "pct_of_nominal_8tbs": round(100 * value / ws / NOMINAL_HBM_GBS, 2),
+        "slices_per_s": round(ws * B / (ms * 1e-3), 1),
+        "gpu_launches": launches_per_step * args.steps,
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak,
+                     "unit": "GB/s", "frac": round(achieved / peak, 4), "traffic": traffic,
+                     "peak_source": peak_src, "kernel": "softmax_persistent",
+                     "launch_ms": round(launch_ms, 5)},
+        "clocks": clk.summary(),
+        "plan": {k: st[k] for k in ("n_items", "n_die", "stage_bytes", "n_stages", "grid",
+                                     "moved_items", "overlap_items", "tie_items", "L", "N",
+                                     "map_chunk_bytes", "plan_ms", "steal")},
+        "device_status": status,
+    }
+
+    if not args.no_e2e:
+        xp = torch.empty(x.shape, dtype=x.dtype, pin_memory=True)
+        xp.copy_(x.cpu())
+        yp = torch.empty(y.shape, dtype=y.dtype, pin_memory=True)
+
+        def e2e_step():
+            x.copy_(xp, non_blocking=True)
+            step()
+            yp.copy_(y, non_blocking=True)
+
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                e2e_step()
+            stream.synchronize()
+            e_ms, _ = time_steps(e2e_step, args.e2e_steps, stream, per_launch=False)
+        e_ms /= args.e2e_steps
+        nb = x.numel() * x.element_size()
+        out["e2e"] = {"value": round(ws * bytes_step / (e_ms * 1e-3) / 1e9, 2), "unit": "GB/s",
+                      "h2d_bytes_per_step": nb, "d2h_bytes_per_step": nb,
+                      "ms_per_step": round(e_ms, 4)}
+    if not args.no_cpu_baseline and rank == 0 and ws == 1:
+        out["cpu_baseline"] = cpu_baseline(w)
+
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+
+    if args.sweep and rank == 0:
+        sweep(args, bsm, workload, stream)
+    if ws > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def sweep(args, bsm, workload, stream):
+    """Policy-by-shape sweep: every policy on workloads 2-5 (median of 20)."""
+    import numpy as np
+    import torch
+    for k in (2, 3, 4, 5):
+        w = workload.config(k).materialize()
+        xh = w.x.view(np.int16) if w.dtype == workload.BF16 else w.x
+        x = torch.from_numpy(xh).cuda()
+        if w.dtype == workload.BF16:
+            x = x.view(torch.bfloat16)
+        y = torch.empty_like(x)
+        for name in ("whole_gpu", "rr", "dynamic", "cbmf", "cbmf_lb"):
+            pol = bsm.POLICIES[name]
+            reps = 3 if name == "whole_gpu" and k == 5 else 20
+
+            def step():
+                bsm.bsm_softmax_ragged(x, y, w.offsets, w.rows, w.cols, w.dtype, pol, w.flags,
+                                       stream)
+            for _ in range(3):
+                step()
+            stream.synchronize()
+            _, per = time_steps(step, reps, stream, per_launch=True)
+            med = float(np.median(per))
+            print(json.dumps({"sweep": True, "workload": w.name, "policy": name,
+                              "ms": round(med, 4),
+                              "GBps": round(w.algorithmic_bytes / (med * 1e-3) / 1e9, 2),
+                              "slices_per_s": round(w.nslices / (med * 1e-3), 1)}), flush=True)
+        del x, y
+        torch.cuda.empty_cache()
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,282 @@
+/*
+ * bsm.h -- C ABI of libbsm: batched row-wise softmax over many slices, with
+ * the slices scheduled onto the GPU's SMs by a selectable policy.
+ *
+ * What is computed (Sec. 2 of "An optimal scheduling architecture for
+ * accelerating batch algorithms on Neural Network processor architectures",
+ * Nyshadham et al.: SOFTMAX on every 512 x 512 slice of a (512*384) x 512
+ * tensor; Sec. 6, SOFTMAX table).  For slice s with R_s rows and C_s columns
+ * stored row-major at element offset off_s, and every row r of it:
+ *     v[c] = x[r,c] + M[r,c]   (M = 0; with BSM_FLAG_CAUSAL, M = -inf for c > r)
+ *     y[r,c] = exp(v[c] - max v) / sum_c' exp(v[c'] - max v)
+ * A row holding NaN or +inf, or a row that is entirely -inf, comes out NaN
+ * (the formula gives 0/0 or inf - inf there).
+ *
+ * How slices are scheduled (the policies) -- Sec. 3 and Sec. 4:
+ *   BSM_POLICY_WHOLE_GPU  Sec. 3, first previous solution: one slice after
+ *                         another, each spread over the whole device (one
+ *                         launch per slice).
+ *   BSM_POLICY_RR         Sec. 3, second previous solution: slice i runs on
+ *                         compute unit (i mod G), statically.
+ *   BSM_POLICY_CBMF       Sec. 4.1, Cluster Beamforming: every patch (a block
+ *                         of rows of one slice) goes to the die whose memory
+ *                         holds most of its bytes (ties: seeded fair coin);
+ *                         the SMs of that die take the die's patches in order.
+ *   BSM_POLICY_CBMF_LB    Sec. 4.1 + Sec. 4.2: CBMF followed by the weighted
+ *                         load balance (patches moved from the over-loaded die
+ *                         to the other, weighted by inverse latency), plus
+ *                         run-time stealing once a die's own queue is empty.
+ *   BSM_POLICY_DYNAMIC    Not in the paper: one device-wide queue of patches,
+ *                         every SM pulls the next one (the locality-blind
+ *                         dynamic schedule CBMF is measured against).
+ * Every policy computes every row with the same device routine, chosen only
+ * by the row length, so y is bit-identical across policies.
+ *
+ * Conventions shared by every entry point below:
+ *   - x and y are device pointers owned by the caller.  They must stay valid
+ *     until the work queued on `stream` completes.  Host arrays passed in are
+ *     copied; the caller keeps ownership.
+ *   - Calls return a bsm_status; no C++ exception crosses the ABI.  Argument
+ *     checks are synchronous.  The launches are asynchronous on `stream`
+ *     (NULL = the legacy default stream); a fault detected inside a kernel is
+ *     recorded in a sticky per-device status word (bsm_device_status).
+ *   - Alignment: x and y 16-byte aligned, every slice's byte offset and every
+ *     row's byte length (C * element size) a multiple of 16; otherwise
+ *     BSM_ERR_MISALIGNED.
+ *   - In place (x == y) is allowed; partially overlapping x and y are not
+ *     (BSM_ERR_INVALID_ARG).
+ *   - Row length limit: C * element size <= bsm_max_row_bytes() (a row must
+ *     fit one shared-memory stage), else BSM_ERR_UNSUPPORTED.
+ */
+#ifndef BSM_H
+#define BSM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* A cudaStream_t.  NULL selects the legacy default stream. */
+typedef struct CUstream_st *bsm_stream_t;
+
+typedef enum {
+    BSM_OK = 0,
+    BSM_ERR_INVALID_ARG = 1,   /* null / negative / inconsistent arguments */
+    BSM_ERR_MISALIGNED = 2,    /* 16-byte alignment rule broken */
+    BSM_ERR_UNSUPPORTED = 3,   /* row too long for a stage, too many patches */
+    BSM_ERR_CUDA = 4,          /* a CUDA runtime call failed */
+    BSM_ERR_DEVICE_BOUNDS = 5, /* a kernel met a patch outside the buffers */
+    BSM_ERR_TIMEOUT = 6,       /* a kernel wait gave up after its time limit */
+    BSM_ERR_NO_DEVICE = 7,     /* no usable CUDA device */
+    BSM_ERR_NOMEM = 8          /* host or device allocation failed */
+} bsm_status;
+
+typedef enum { BSM_F32 = 0, BSM_BF16 = 1 } bsm_dtype;   /* input type == output type */
+
+typedef enum {
+    BSM_POLICY_WHOLE_GPU = 0,
+    BSM_POLICY_RR = 1,
+    BSM_POLICY_CBMF = 2,
+    BSM_POLICY_CBMF_LB = 3,
+    BSM_POLICY_DYNAMIC = 4
+} bsm_policy;
+
+#define BSM_FLAG_CAUSAL 1u     /* additive -inf mask above each slice's diagonal */
+
+#define BSM_MAX_DIES 4
+#define BSM_MAX_SM 256
+
+/* Device-side status bits (bsm_device_status). */
+#define BSM_DEV_BOUNDS 1u      /* a patch fell outside the buffers or a stage; skipped */
+#define BSM_DEV_TIMEOUT 2u     /* a pipeline wait ran out of time; the CTA gave up */
+
+/*
+ * Softmax over B slices of R x C stored back to back, i.e. a (B*R) x C
+ * row-major tensor (the layout of Sec. 2).  Equivalent to bsm_softmax_ex with
+ * flags = 0.  The plan (patch table, die queues) is built on first use for a
+ * given (device, x, y, shape, dtype, policy, flags) and cached.
+ *   x, y    device pointers, B*R*C elements of `dtype` each.
+ *   B, R, C B >= 0, R >= 0, C >= 1; B*R*C < 2^62.
+ *   dtype   bsm_dtype; policy bsm_policy.
+ * Errors: BSM_ERR_INVALID_ARG, BSM_ERR_MISALIGNED, BSM_ERR_UNSUPPORTED,
+ * BSM_ERR_CUDA, BSM_ERR_NOMEM.  B*R == 0 returns BSM_OK and launches nothing.
+ */
+int bsm_softmax(const void *x, void *y, int64_t B, int64_t R, int64_t C, int dtype,
+                int policy, bsm_stream_t stream);
+
+/* bsm_softmax with flags (BSM_FLAG_CAUSAL: M[r,c] = -inf for c > r, r the row
+ * inside its slice). */
+int bsm_softmax_ex(const void *x, void *y, int64_t B, int64_t R, int64_t C, int dtype,
+                   int policy, uint32_t flags, bsm_stream_t stream);
+
+/*
+ * Ragged batch: slice s has rows[s] x cols[s] elements at element offset
+ * offsets[s] of x (and of y).  offsets/rows/cols are HOST arrays of
+ * num_slices entries, copied.  Slices must not overlap each other; they need
+ * not be contiguous or ordered.  Same errors as bsm_softmax.
+ */
+int bsm_softmax_ragged(const void *x, void *y, int64_t num_slices, const int64_t *offsets,
+                       const int32_t *rows, const int32_t *cols, int dtype, int policy,
+                       uint32_t flags, bsm_stream_t stream);
+
+/* ---- plans: build the schedule once ("upfront", Sec. 5), run it many times ---- */
+
+typedef struct bsm_plan bsm_plan;
+
+typedef struct {
+    const void *x;              /* device input */
+    void *y;                    /* device output (may equal x) */
+    int64_t num_slices;
+    const int64_t *offsets;     /* host, element offsets; NULL = packed back to back */
+    const int32_t *rows;        /* host, num_slices entries */
+    const int32_t *cols;        /* host, num_slices entries */
+    int32_t dtype;              /* bsm_dtype */
+    int32_t policy;             /* bsm_policy */
+    uint32_t flags;             /* BSM_FLAG_* */
+    int32_t rows_per_item;      /* rows per patch; 0 = as many as fill one stage */
+    uint64_t tie_seed;          /* seed of the CBMF equal-share coin */
+    int32_t lb_weighted;        /* CBMF_LB: 1 = weights from measured latency, 0 = equal */
+    int32_t count_output_bytes; /* CBMF: 1 = a patch's bytes on a die count x and y */
+    int32_t device;             /* -1 = the current device */
+} bsm_plan_desc;
+
+/* Fill a descriptor with the defaults (rows_per_item 0, tie_seed 0x2002070600,
+ * lb_weighted 1, count_output_bytes 1, device -1, offsets NULL). */
+int bsm_plan_desc_init(bsm_plan_desc *d);
+
+/* Build a plan: validate, cut slices into patches, and for CBMF / CBMF_LB
+ * probe the topology (cached per device) and the die of every chunk of x and
+ * y, then run the Sec. 4.1 / 4.2 steps on the host and upload the tables.
+ * Synchronous; allocates device memory owned by the plan. */
+int bsm_plan_create(bsm_plan **plan, const bsm_plan_desc *d);
+
+/* Launch the plan on `stream` (async).  Allocates nothing and does not
+ * synchronise.  Executions of one plan must not overlap in time (they share
+ * the plan's queue counters): keep them on one stream, or order them. */
+int bsm_plan_execute(const bsm_plan *plan, bsm_stream_t stream);
+
+typedef struct {
+    int32_t policy;
+    int32_t n_die;              /* dies the schedule used (1 if not separable) */
+    int64_t n_items;            /* patches */
+    int64_t N[BSM_MAX_DIES];    /* Sec. 4.1: patches with any byte on die d */
+    int64_t L[BSM_MAX_DIES];    /* Sec. 4.1: patches assigned to die d */
+    int64_t overlap_items;      /* patches on more than one die */
+    int64_t tie_items;          /* patches resolved by the coin */
+    int64_t moved_items;        /* Sec. 4.2: patches moved by the load balance */
+    int64_t queue_items[BSM_MAX_DIES];
+    int64_t queue_bytes[BSM_MAX_DIES];
+    double est_finish_before[BSM_MAX_DIES];  /* per-die estimated finish, LB input */
+    double est_finish_after[BSM_MAX_DIES];   /* same after LB */
+    int32_t stage_bytes;        /* shared-memory stage size */
+    int32_t n_stages;           /* stages per CTA */
+    int32_t grid;               /* CTAs per launch */
+    int32_t launches;           /* launches per execute (WHOLE_GPU: one per slice) */
+    int32_t steal;              /* 1 if CTAs steal from other dies' queues */
+    int64_t map_chunk_bytes;    /* granularity of the address->die map used */
+    double plan_ms;             /* host time spent in bsm_plan_create */
+} bsm_plan_stats;
+
+int bsm_plan_get_stats(const bsm_plan *plan, bsm_plan_stats *out);
+void bsm_plan_destroy(bsm_plan *plan);
+
+/* Drop every cached plan of bsm_softmax / bsm_softmax_ex / bsm_softmax_ragged. */
+void bsm_cache_clear(void);
+
+/* ---- topology: the GB300 stand-in for cluster / memory-bank nearness ----
+ * Sec. 2.1: a compute unit reaches its nearest memory bank with the least
+ * latency.  On GB300 the "banks" are the two dies' L2 partitions and HBM
+ * stacks.  The probe times dependent L2-hit loads from every SM to many
+ * addresses, groups SMs whose latency profiles agree (one group per die), and
+ * records the near and far latency (the weights of Sec. 4.2). */
+typedef struct {
+    int32_t device;
+    int32_t n_sm;
+    int32_t n_die;              /* 2 on GB300 when separable, else 1 */
+    int32_t separable;          /* 1 if near/far latencies split cleanly */
+    int8_t sm_die[BSM_MAX_SM];  /* die of SM id (%smid); -1 if never seen */
+    int32_t sm_per_die[BSM_MAX_DIES];
+    double l_near;              /* mean near L2-hit latency, SM cycles */
+    double l_far;               /* mean far L2-hit latency, SM cycles */
+    double separation;          /* mean |correlation| of SM profiles, 0..1 */
+    int64_t granularity;        /* bytes of the smallest same-die address run seen */
+    double probe_ms;
+} bsm_topology;
+
+/* Probe once per device (cached; force = 1 probes again).  Synchronous;
+ * allocates and frees a 32 MiB scratch buffer.  device = -1: current. */
+int bsm_topology_probe(int device, int force, bsm_topology *out);
+
+/* Die of every `chunk`-byte chunk of the device buffer [ptr, ptr + bytes):
+ * die_out (host, ceil(bytes/chunk) entries) gets the die whose L2 answers the
+ * chunk's first line fastest.  chunk is a multiple of 128.  Reads the buffer,
+ * writes nothing to it.  Needs a separable topology (else BSM_ERR_UNSUPPORTED).
+ * Synchronous. */
+int bsm_addr_die_map(int device, const void *ptr, int64_t bytes, int64_t chunk, int8_t *die_out);
+
+/* Raw probe matrix, for diagnostics: lat_out (host, BSM_MAX_SM x n_lines,
+ * row = %smid) gets the mean cycles of a dependent L2-hit load from that SM to
+ * byte offset line_off[i] of a 32 MiB scratch buffer (line_off multiples of
+ * 128, below 32 MiB); seen_out[smid] = 1 for SMs that ran.  Synchronous. */
+int bsm_probe_latency(int device, int32_t n_lines, const int64_t *line_off, int32_t reps,
+                      float *lat_out, int32_t *seen_out);
+
+/* ---- the scheduling steps alone, on the host (no GPU needed) ----
+ * Runs the Sec. 4.1 table + overlap resolution and, when balance != 0, the
+ * Sec. 4.2 load balance, on a caller-given address->bank map.  All arrays are
+ * host memory owned by the caller. */
+typedef struct {
+    int32_t n_banks;            /* 1..BSM_MAX_DIES */
+    int64_t n_patches;
+    const int64_t *patch_begin; /* byte range [begin, end) of each patch */
+    const int64_t *patch_end;
+    int32_t n_maps;             /* 1 (input only) or 2 (input and output) */
+    int64_t chunk[2];           /* bytes per map chunk */
+    int64_t n_chunks[2];
+    const int8_t *bank_of_chunk[2];
+    uint64_t tie_seed;
+    int32_t balance;            /* 0: CBMF only; 1: CBMF + load balance */
+    const int32_t *units;       /* compute units near each bank */
+    int64_t l_near, l_far;      /* latency weights (equal = unweighted) */
+    const int64_t *cost;        /* work of each patch (bytes it moves) */
+} bsm_schedule_desc;
+
+typedef struct {
+    int64_t *bytes_on_bank;     /* n_patches x n_banks */
+    uint8_t *overlap;           /* n_patches */
+    int64_t *N;                 /* n_banks */
+    int32_t *bank;              /* n_patches: bank after overlap resolution */
+    int64_t *L;                 /* n_banks */
+    int32_t *queue_items;       /* n_patches: the banks' queues, concatenated */
+    int64_t *queue_len;         /* n_banks */
+    int32_t *moved;             /* n_patches: patch ids in the order moved */
+    int64_t n_moved;
+    int64_t *work_before;       /* n_banks: l_near*native + l_far*moved-in bytes */
+    int64_t *work_after;        /* n_banks */
+} bsm_schedule_out;
+
+int bsm_schedule_host(const bsm_schedule_desc *d, bsm_schedule_out *out);
+
+/* ---- status ---- */
+
+/* Sticky device-side status word of `device` (-1 = current), BSM_DEV_* bits.
+ * Synchronises the device.  bsm_device_status_clear zeroes it. */
+int bsm_device_status(int device, uint32_t *status_out);
+int bsm_device_status_clear(int device);
+
+/* Largest row (C * element size) a plan accepts on this device, bytes. */
+int64_t bsm_max_row_bytes(int device);
+
+/* Static description of a status code. */
+const char *bsm_status_string(int status);
+
+/* Library version, (major << 16) | minor. */
+int bsm_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BSM_H */

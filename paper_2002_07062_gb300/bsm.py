@@ -1,0 +1,377 @@
+"""Thin Python binding of libbsm (include/bsm.h).
+
+Argument marshalling only: every step of the softmax and of the scheduling
+runs inside libbsm.  Device buffers are passed as integers (device
+addresses) or as torch tensors (their data_ptr()); host arrays as numpy
+arrays.  Every call raises BsmError on a non-zero status.  If libbsm.so has
+not been built, loading fails loudly: there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+from typing import Optional, Sequence
+
+import numpy as np
+
+PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(PKG, "_lib", "libbsm.so")
+HEADER = os.path.join(os.path.dirname(PKG), "include", "bsm.h")
+
+F32, BF16 = 0, 1
+POLICY_WHOLE_GPU, POLICY_RR, POLICY_CBMF, POLICY_CBMF_LB, POLICY_DYNAMIC = range(5)
+POLICIES = {"whole_gpu": POLICY_WHOLE_GPU, "rr": POLICY_RR, "cbmf": POLICY_CBMF,
+            "cbmf_lb": POLICY_CBMF_LB, "dynamic": POLICY_DYNAMIC}
+POLICY_NAMES = {v: k for k, v in POLICIES.items()}
+FLAG_CAUSAL = 1
+MAX_DIES = 4
+MAX_SM = 256
+DEV_BOUNDS, DEV_TIMEOUT = 1, 2
+
+(OK, ERR_INVALID_ARG, ERR_MISALIGNED, ERR_UNSUPPORTED, ERR_CUDA, ERR_DEVICE_BOUNDS,
+ ERR_TIMEOUT, ERR_NO_DEVICE, ERR_NOMEM) = range(9)
+
+c_i64p = ctypes.POINTER(ctypes.c_int64)
+c_i32p = ctypes.POINTER(ctypes.c_int32)
+
+
+class BsmError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__("%s: %s (status %d)" % (where, status_string(status), status))
+
+
+class PlanDesc(ctypes.Structure):
+    _fields_ = [("x", ctypes.c_void_p), ("y", ctypes.c_void_p), ("num_slices", ctypes.c_int64),
+                ("offsets", c_i64p), ("rows", c_i32p), ("cols", c_i32p),
+                ("dtype", ctypes.c_int32), ("policy", ctypes.c_int32), ("flags", ctypes.c_uint32),
+                ("rows_per_item", ctypes.c_int32), ("tie_seed", ctypes.c_uint64),
+                ("lb_weighted", ctypes.c_int32), ("count_output_bytes", ctypes.c_int32),
+                ("device", ctypes.c_int32)]
+
+
+class PlanStats(ctypes.Structure):
+    _fields_ = [("policy", ctypes.c_int32), ("n_die", ctypes.c_int32), ("n_items", ctypes.c_int64),
+                ("N", ctypes.c_int64 * MAX_DIES), ("L", ctypes.c_int64 * MAX_DIES),
+                ("overlap_items", ctypes.c_int64), ("tie_items", ctypes.c_int64),
+                ("moved_items", ctypes.c_int64), ("queue_items", ctypes.c_int64 * MAX_DIES),
+                ("queue_bytes", ctypes.c_int64 * MAX_DIES),
+                ("est_finish_before", ctypes.c_double * MAX_DIES),
+                ("est_finish_after", ctypes.c_double * MAX_DIES),
+                ("stage_bytes", ctypes.c_int32), ("n_stages", ctypes.c_int32),
+                ("grid", ctypes.c_int32), ("launches", ctypes.c_int32), ("steal", ctypes.c_int32),
+                ("map_chunk_bytes", ctypes.c_int64), ("plan_ms", ctypes.c_double)]
+
+
+class Topology(ctypes.Structure):
+    _fields_ = [("device", ctypes.c_int32), ("n_sm", ctypes.c_int32), ("n_die", ctypes.c_int32),
+                ("separable", ctypes.c_int32), ("sm_die", ctypes.c_int8 * MAX_SM),
+                ("sm_per_die", ctypes.c_int32 * MAX_DIES), ("l_near", ctypes.c_double),
+                ("l_far", ctypes.c_double), ("separation", ctypes.c_double),
+                ("granularity", ctypes.c_int64), ("probe_ms", ctypes.c_double)]
+
+
+class ScheduleDesc(ctypes.Structure):
+    _fields_ = [("n_banks", ctypes.c_int32), ("n_patches", ctypes.c_int64),
+                ("patch_begin", c_i64p), ("patch_end", c_i64p), ("n_maps", ctypes.c_int32),
+                ("chunk", ctypes.c_int64 * 2), ("n_chunks", ctypes.c_int64 * 2),
+                ("bank_of_chunk", ctypes.POINTER(ctypes.c_int8) * 2),
+                ("tie_seed", ctypes.c_uint64), ("balance", ctypes.c_int32), ("units", c_i32p),
+                ("l_near", ctypes.c_int64), ("l_far", ctypes.c_int64), ("cost", c_i64p)]
+
+
+class ScheduleOut(ctypes.Structure):
+    _fields_ = [("bytes_on_bank", c_i64p), ("overlap", ctypes.POINTER(ctypes.c_uint8)),
+                ("N", c_i64p), ("bank", c_i32p), ("L", c_i64p), ("queue_items", c_i32p),
+                ("queue_len", c_i64p), ("moved", c_i32p), ("n_moved", ctypes.c_int64),
+                ("work_before", c_i64p), ("work_after", c_i64p)]
+
+
+_lib = None
+
+
+def lib():
+    """Load libbsm.so; raises if it was not built (run __graft_entry__.build())."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise ImportError("libbsm.so not found at %s: build it with "
+                          "`python -c 'import __graft_entry__ as g; g.build()'`" % LIB_PATH)
+    L = ctypes.CDLL(LIB_PATH)
+    vp, i64, i32, u32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_uint32
+    sig = {
+        "bsm_softmax": ([vp, vp, i64, i64, i64, ctypes.c_int, ctypes.c_int, vp], ctypes.c_int),
+        "bsm_softmax_ex": ([vp, vp, i64, i64, i64, ctypes.c_int, ctypes.c_int, u32, vp], ctypes.c_int),
+        "bsm_softmax_ragged": ([vp, vp, i64, c_i64p, c_i32p, c_i32p, ctypes.c_int, ctypes.c_int, u32,
+                                vp], ctypes.c_int),
+        "bsm_plan_desc_init": ([ctypes.POINTER(PlanDesc)], ctypes.c_int),
+        "bsm_plan_create": ([ctypes.POINTER(vp), ctypes.POINTER(PlanDesc)], ctypes.c_int),
+        "bsm_plan_execute": ([vp, vp], ctypes.c_int),
+        "bsm_plan_get_stats": ([vp, ctypes.POINTER(PlanStats)], ctypes.c_int),
+        "bsm_plan_destroy": ([vp], None),
+        "bsm_cache_clear": ([], None),
+        "bsm_topology_probe": ([ctypes.c_int, ctypes.c_int, ctypes.POINTER(Topology)], ctypes.c_int),
+        "bsm_addr_die_map": ([ctypes.c_int, vp, i64, i64, ctypes.POINTER(ctypes.c_int8)], ctypes.c_int),
+        "bsm_probe_latency": ([ctypes.c_int, i32, c_i64p, i32, ctypes.POINTER(ctypes.c_float), c_i32p],
+                              ctypes.c_int),
+        "bsm_schedule_host": ([ctypes.POINTER(ScheduleDesc), ctypes.POINTER(ScheduleOut)], ctypes.c_int),
+        "bsm_device_status": ([ctypes.c_int, ctypes.POINTER(u32)], ctypes.c_int),
+        "bsm_device_status_clear": ([ctypes.c_int], ctypes.c_int),
+        "bsm_max_row_bytes": ([ctypes.c_int], i64),
+        "bsm_status_string": ([ctypes.c_int], ctypes.c_char_p),
+        "bsm_version": ([], ctypes.c_int),
+    }
+    for name, (args, res) in sig.items():
+        f = getattr(L, name)
+        f.argtypes = args
+        f.restype = res
+    _lib = L
+    return L
+
+
+def header_functions() -> list:
+    """Names of the functions include/bsm.h declares."""
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?[a-z_0-9]+\s*\*?\s*(bsm_[a-z_0-9]+)\s*\(",
+                                 text, flags=re.M)))
+
+
+def status_string(status: int) -> str:
+    return lib().bsm_status_string(status).decode()
+
+
+def _check(rc: int, where: str):
+    if rc != OK:
+        raise BsmError(rc, where)
+
+
+def _dptr(t) -> Optional[int]:
+    """Device address of a torch tensor, or an int passed through."""
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return int(t.data_ptr())
+
+
+def _stream(s) -> Optional[int]:
+    if s is None:
+        return None
+    if isinstance(s, int):
+        return s
+    return int(s.cuda_stream)
+
+
+def _np(a, dt):
+    return np.ascontiguousarray(np.asarray(a), dtype=dt)
+
+
+def bsm_softmax(x, y, B: int, R: int, C: int, dtype: int, policy: int, stream=None):
+    _check(lib().bsm_softmax(_dptr(x), _dptr(y), B, R, C, dtype, policy, _stream(stream)),
+           "bsm_softmax")
+
+
+def bsm_softmax_ex(x, y, B: int, R: int, C: int, dtype: int, policy: int, flags: int = 0,
+                   stream=None):
+    _check(lib().bsm_softmax_ex(_dptr(x), _dptr(y), B, R, C, dtype, policy, flags,
+                                _stream(stream)), "bsm_softmax_ex")
+
+
+def bsm_softmax_ragged(x, y, offsets, rows, cols, dtype: int, policy: int, flags: int = 0,
+                       stream=None):
+    off = _np(offsets, np.int64)
+    r = _np(rows, np.int32)
+    c = _np(cols, np.int32)
+    if not (len(off) == len(r) == len(c)):
+        raise ValueError("offsets, rows and cols must have the same length")
+    _check(lib().bsm_softmax_ragged(_dptr(x), _dptr(y), len(off),
+                                    off.ctypes.data_as(c_i64p), r.ctypes.data_as(c_i32p),
+                                    c.ctypes.data_as(c_i32p), dtype, policy, flags,
+                                    _stream(stream)), "bsm_softmax_ragged")
+
+
+class Plan:
+    """Owner of a bsm_plan; destroyed with the object."""
+
+    def __init__(self, handle: int, keep):
+        self.handle = handle
+        self._keep = keep
+
+    def execute(self, stream=None):
+        bsm_plan_execute(self, stream)
+
+    def stats(self) -> dict:
+        return bsm_plan_get_stats(self)
+
+    def close(self):
+        if self.handle:
+            lib().bsm_plan_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def bsm_plan_create(x, y, rows, cols, dtype: int, policy: int, offsets=None, flags: int = 0,
+                    rows_per_item: int = 0, tie_seed: Optional[int] = None,
+                    lb_weighted: bool = True, count_output_bytes: bool = True,
+                    device: int = -1) -> Plan:
+    d = PlanDesc()
+    _check(lib().bsm_plan_desc_init(ctypes.byref(d)), "bsm_plan_desc_init")
+    r = _np(rows, np.int32)
+    c = _np(cols, np.int32)
+    off = None if offsets is None else _np(offsets, np.int64)
+    d.x = _dptr(x)
+    d.y = _dptr(y)
+    d.num_slices = len(r)
+    d.rows = r.ctypes.data_as(c_i32p)
+    d.cols = c.ctypes.data_as(c_i32p)
+    if off is not None:
+        d.offsets = off.ctypes.data_as(c_i64p)
+    d.dtype = dtype
+    d.policy = policy
+    d.flags = flags
+    d.rows_per_item = rows_per_item
+    if tie_seed is not None:
+        d.tie_seed = tie_seed
+    d.lb_weighted = 1 if lb_weighted else 0
+    d.count_output_bytes = 1 if count_output_bytes else 0
+    d.device = device
+    h = ctypes.c_void_p()
+    _check(lib().bsm_plan_create(ctypes.byref(h), ctypes.byref(d)), "bsm_plan_create")
+    return Plan(h.value, (x, y))
+
+
+def bsm_plan_execute(plan: Plan, stream=None):
+    _check(lib().bsm_plan_execute(plan.handle, _stream(stream)), "bsm_plan_execute")
+
+
+def bsm_plan_get_stats(plan: Plan) -> dict:
+    s = PlanStats()
+    _check(lib().bsm_plan_get_stats(plan.handle, ctypes.byref(s)), "bsm_plan_get_stats")
+    out = {}
+    for name, _ in PlanStats._fields_:
+        v = getattr(s, name)
+        out[name] = list(v) if not isinstance(v, (int, float)) else v
+    return out
+
+
+def bsm_plan_destroy(plan: Plan):
+    plan.close()
+
+
+def bsm_cache_clear():
+    lib().bsm_cache_clear()
+
+
+def bsm_topology_probe(device: int = -1, force: bool = False) -> dict:
+    t = Topology()
+    _check(lib().bsm_topology_probe(device, 1 if force else 0, ctypes.byref(t)),
+           "bsm_topology_probe")
+    return {"device": t.device, "n_sm": t.n_sm, "n_die": t.n_die, "separable": t.separable,
+            "sm_die": list(t.sm_die), "sm_per_die": list(t.sm_per_die), "l_near": t.l_near,
+            "l_far": t.l_far, "separation": t.separation, "granularity": t.granularity,
+            "probe_ms": t.probe_ms}
+
+
+def bsm_addr_die_map(ptr, nbytes: int, chunk: int, device: int = -1) -> np.ndarray:
+    n = (nbytes + chunk - 1) // chunk
+    out = np.zeros(n, np.int8)
+    _check(lib().bsm_addr_die_map(device, _dptr(ptr), nbytes, chunk,
+                                  out.ctypes.data_as(ctypes.POINTER(ctypes.c_int8))),
+           "bsm_addr_die_map")
+    return out
+
+
+def bsm_probe_latency(line_off, reps: int = 8, device: int = -1):
+    off = _np(line_off, np.int64)
+    lat = np.zeros((MAX_SM, len(off)), np.float32)
+    seen = np.zeros(MAX_SM, np.int32)
+    _check(lib().bsm_probe_latency(device, len(off), off.ctypes.data_as(c_i64p), reps,
+                                   lat.ctypes.data_as(ctypes.POINTER(ctypes.c_float)),
+                                   seen.ctypes.data_as(c_i32p)), "bsm_probe_latency")
+    return lat, seen
+
+
+def bsm_schedule_host(patches: Sequence, maps: Sequence, n_banks: int, tie_seed: int,
+                      balance: bool = False, units=None, l_near: int = 1, l_far: int = 1,
+                      cost=None) -> dict:
+    """patches: (begin, end) byte ranges; maps: (chunk, bank_of_chunk) pairs."""
+    n = len(patches)
+    pb = _np([p[0] for p in patches], np.int64)
+    pe = _np([p[1] for p in patches], np.int64)
+    d = ScheduleDesc()
+    d.n_banks = n_banks
+    d.n_patches = n
+    d.patch_begin = pb.ctypes.data_as(c_i64p)
+    d.patch_end = pe.ctypes.data_as(c_i64p)
+    d.n_maps = len(maps)
+    keep = []
+    for k, (chunk, bank_of_chunk) in enumerate(maps):
+        arr = _np(bank_of_chunk, np.int8)
+        keep.append(arr)
+        d.chunk[k] = chunk
+        d.n_chunks[k] = len(arr)
+        d.bank_of_chunk[k] = arr.ctypes.data_as(ctypes.POINTER(ctypes.c_int8))
+    d.tie_seed = tie_seed
+    d.balance = 1 if balance else 0
+    u = _np(units if units is not None else [1] * n_banks, np.int32)
+    d.units = u.ctypes.data_as(c_i32p)
+    d.l_near = l_near
+    d.l_far = l_far
+    cst = _np(cost if cost is not None else [p[1] - p[0] for p in patches], np.int64)
+    d.cost = cst.ctypes.data_as(c_i64p)
+    bob = np.zeros((max(n, 1), n_banks), np.int64)
+    ov = np.zeros(max(n, 1), np.uint8)
+    N = np.zeros(n_banks, np.int64)
+    bank = np.zeros(max(n, 1), np.int32)
+    L = np.zeros(n_banks, np.int64)
+    qi = np.zeros(max(n, 1), np.int32)
+    ql = np.zeros(n_banks, np.int64)
+    mv = np.zeros(max(n, 1), np.int32)
+    wb = np.zeros(n_banks, np.int64)
+    wa = np.zeros(n_banks, np.int64)
+    o = ScheduleOut()
+    o.bytes_on_bank = bob.ctypes.data_as(c_i64p)
+    o.overlap = ov.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8))
+    o.N = N.ctypes.data_as(c_i64p)
+    o.bank = bank.ctypes.data_as(c_i32p)
+    o.L = L.ctypes.data_as(c_i64p)
+    o.queue_items = qi.ctypes.data_as(c_i32p)
+    o.queue_len = ql.ctypes.data_as(c_i64p)
+    o.moved = mv.ctypes.data_as(c_i32p)
+    o.work_before = wb.ctypes.data_as(c_i64p)
+    o.work_after = wa.ctypes.data_as(c_i64p)
+    _check(lib().bsm_schedule_host(ctypes.byref(d), ctypes.byref(o)), "bsm_schedule_host")
+    queues, pos = [], 0
+    for b in range(n_banks):
+        queues.append([int(v) for v in qi[pos:pos + ql[b]]])
+        pos += int(ql[b])
+    return {"bytes_on_bank": bob[:n].tolist(), "overlap": ov[:n].tolist(), "N": N.tolist(),
+            "bank": bank[:n].tolist(), "L": L.tolist(), "queues": queues,
+            "moved": mv[:o.n_moved].tolist(), "work_before": wb.tolist(),
+            "work_after": wa.tolist()}
+
+
+def bsm_device_status(device: int = -1) -> int:
+    v = ctypes.c_uint32()
+    _check(lib().bsm_device_status(device, ctypes.byref(v)), "bsm_device_status")
+    return v.value
+
+
+def bsm_device_status_clear(device: int = -1):
+    _check(lib().bsm_device_status_clear(device), "bsm_device_status_clear")
+
+
+def bsm_max_row_bytes(device: int = -1) -> int:
+    return int(lib().bsm_max_row_bytes(device))
+
+
+def bsm_version() -> int:
+    return int(lib().bsm_version())

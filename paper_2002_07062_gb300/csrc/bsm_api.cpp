@@ -1,0 +1,822 @@
+// bsm_api.cpp -- the C ABI of libbsm (include/bsm.h): argument checks, plan
+// construction (patches, die queues, upload of the patch table -- the
+// "Patch<->Cluster mapping table" kept in device memory, Sec. 5), plan
+// execution, the plan cache behind the one-call entry points, and status.
+
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <chrono>
+#include <cmath>
+#include <cstring>
+#include <list>
+#include <mutex>
+#include <new>
+#include <numeric>
+#include <vector>
+
+#include "bsm_internal.h"
+
+namespace bsm {
+
+int topology_get(int device, int force, bsm_topology *out);
+int addr_die_map_host(int device, const void *ptr, int64_t bytes, int64_t chunk, int8_t *die_out);
+int probe_latency_host(int device, const std::vector<int64_t> &lines, int reps, std::vector<float> &lat,
+                       std::vector<int32_t> &seen);
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+constexpr uint64_t kDefaultTieSeed = 0x2002070600ull;
+constexpr int64_t kMaxMapChunks = 1ll << 24;
+
+struct DeviceCtx {
+    bool ready = false;
+    int n_sm = 0;
+    int smem_optin = 0;
+    uint32_t *status = nullptr;   // sticky device status word
+};
+
+std::mutex g_mu;
+DeviceCtx g_dev[kMaxDevices];
+
+int device_ctx(int device, DeviceCtx **out)
+{
+    if (device < 0) {
+        if (cudaGetDevice(&device) != cudaSuccess)
+            return BSM_ERR_NO_DEVICE;
+    }
+    if (device >= kMaxDevices)
+        return BSM_ERR_NO_DEVICE;
+    std::lock_guard<std::mutex> lk(g_mu);
+    DeviceCtx &c = g_dev[device];
+    if (!c.ready) {
+        int prev = -1;
+        cudaGetDevice(&prev);
+        if (cudaSetDevice(device) != cudaSuccess)
+            return BSM_ERR_NO_DEVICE;
+        int rc = BSM_OK;
+        if (cudaDeviceGetAttribute(&c.n_sm, cudaDevAttrMultiProcessorCount, device) != cudaSuccess ||
+            cudaDeviceGetAttribute(&c.smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, device) !=
+                cudaSuccess)
+            rc = BSM_ERR_NO_DEVICE;
+        if (!rc && kernel_set_smem_limit(c.smem_optin) != 0)
+            rc = BSM_ERR_CUDA;
+        if (!rc && cudaMalloc(&c.status, 256) != cudaSuccess)
+            rc = BSM_ERR_NOMEM;
+        if (!rc && cudaMemset(c.status, 0, 256) != cudaSuccess)
+            rc = BSM_ERR_CUDA;
+        if (!rc && cudaDeviceSynchronize() != cudaSuccess)
+            rc = BSM_ERR_CUDA;
+        if (prev >= 0 && prev != device)
+            cudaSetDevice(prev);
+        if (rc) {
+            if (c.status)
+                cudaFree(c.status);
+            c.status = nullptr;
+            return rc;
+        }
+        c.ready = true;
+    }
+    *out = &c;
+    return BSM_OK;
+}
+
+int64_t max_row_bytes_for(const DeviceCtx &c)
+{
+    return ((static_cast<int64_t>(c.smem_optin) - kSmemHeader) / 2) & ~int64_t(127);
+}
+
+int esize(int dtype) { return dtype == BSM_F32 ? 4 : 2; }
+
+}  // namespace
+}  // namespace bsm
+
+struct bsm_plan {
+    int device = 0;
+    int policy = 0;
+    int dtype = 0;
+    bsm::KernelArgs args{};
+    int grid = 0;
+    struct Launch {
+        int32_t begin, end, grid;
+    };
+    std::vector<Launch> whole_gpu;   // WHOLE_GPU: one launch per slice
+    void *blob = nullptr;            // device tables (items, queue, slices, sm_die, heads)
+    bsm_plan_stats stats{};
+    // identity of the plan for the cache
+    const void *x = nullptr;
+    void *y = nullptr;
+    uint32_t flags = 0;
+    std::vector<int64_t> key_offsets;
+    std::vector<int32_t> key_rows, key_cols;
+    int64_t key_B = -1, key_R = -1, key_C = -1;
+};
+
+namespace bsm {
+namespace {
+
+struct SliceView {
+    int64_t off;
+    int32_t R, C;
+};
+
+// Validate a descriptor; fills the slice list and the element extent.
+int validate(const bsm_plan_desc *d, const DeviceCtx &c, std::vector<SliceView> &slices,
+             int64_t &total_elems, int64_t &max_row_bytes)
+{
+    if (d->dtype != BSM_F32 && d->dtype != BSM_BF16)
+        return BSM_ERR_INVALID_ARG;
+    if (d->policy < BSM_POLICY_WHOLE_GPU || d->policy > BSM_POLICY_DYNAMIC)
+        return BSM_ERR_INVALID_ARG;
+    if (d->flags & ~BSM_FLAG_CAUSAL)
+        return BSM_ERR_INVALID_ARG;
+    if (d->num_slices < 0 || d->rows_per_item < 0)
+        return BSM_ERR_INVALID_ARG;
+    if (d->num_slices > 0 && (!d->rows || !d->cols))
+        return BSM_ERR_INVALID_ARG;
+    const int es = esize(d->dtype);
+    const int64_t row_limit = max_row_bytes_for(c);
+    slices.clear();
+    slices.reserve(static_cast<size_t>(d->num_slices));
+    total_elems = 0;
+    max_row_bytes = 0;
+    int64_t packed = 0;
+    bool misaligned = false, too_long = false;
+    for (int64_t s = 0; s < d->num_slices; ++s) {
+        const int64_t R = d->rows[s], C = d->cols[s];
+        if (R < 0 || C < 1)
+            return BSM_ERR_INVALID_ARG;
+        const int64_t off = d->offsets ? d->offsets[s] : packed;
+        if (off < 0)
+            return BSM_ERR_INVALID_ARG;
+        if (R > 0 && C > (int64_t(1) << 40) / R)
+            return BSM_ERR_INVALID_ARG;
+        const int64_t n = R * C;
+        if (off > (int64_t(1) << 61) - n)
+            return BSM_ERR_INVALID_ARG;
+        packed = off + n;
+        if (R > 0) {
+            if ((C * es) % 16 != 0 || (off * es) % 16 != 0)
+                misaligned = true;
+            if (C * es > row_limit)
+                too_long = true;
+            max_row_bytes = std::max(max_row_bytes, C * es);
+            total_elems = std::max(total_elems, off + n);
+        }
+        slices.push_back({off, static_cast<int32_t>(R), static_cast<int32_t>(C)});
+    }
+    if (total_elems > 0) {
+        if (!d->x || !d->y)
+            return BSM_ERR_INVALID_ARG;
+        const uintptr_t xa = reinterpret_cast<uintptr_t>(d->x), ya = reinterpret_cast<uintptr_t>(d->y);
+        const uintptr_t len = static_cast<uintptr_t>(total_elems) * es;
+        if (xa != ya && xa < ya + len && ya < xa + len)
+            return BSM_ERR_INVALID_ARG;   // partial overlap
+        if ((xa & 15) || (ya & 15))
+            misaligned = true;
+    }
+    if (misaligned)
+        return BSM_ERR_MISALIGNED;
+    if (too_long)
+        return BSM_ERR_UNSUPPORTED;
+    // slices must not overlap one another
+    if (d->offsets && slices.size() > 1) {
+        std::vector<size_t> order;
+        order.reserve(slices.size());
+        for (size_t s = 0; s < slices.size(); ++s)
+            if (slices[s].R > 0)
+                order.push_back(s);
+        std::sort(order.begin(), order.end(),
+                  [&](size_t a, size_t b) { return slices[a].off < slices[b].off; });
+        for (size_t k = 1; k < order.size(); ++k) {
+            const SliceView &p = slices[order[k - 1]];
+            if (p.off + int64_t(p.R) * p.C > slices[order[k]].off)
+                return BSM_ERR_INVALID_ARG;
+        }
+    }
+    return BSM_OK;
+}
+
+int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
+{
+    const auto t0 = std::chrono::steady_clock::now();
+    if (!out || !d)
+        return BSM_ERR_INVALID_ARG;
+    *out = nullptr;
+    DeviceCtx *c = nullptr;
+    int rc = device_ctx(d->device, &c);
+    if (rc)
+        return rc;
+    int device = d->device;
+    if (device < 0)
+        cudaGetDevice(&device);
+    std::vector<SliceView> slices;
+    int64_t total = 0, max_row = 0;
+    if ((rc = validate(d, *c, slices, total, max_row)))
+        return rc;
+    const int es = esize(d->dtype);
+
+    // ---- stages: one CTA per SM, as many stages as fit the shared memory
+    const int64_t avail = c->smem_optin - kSmemHeader;
+    const int64_t stage = std::max<int64_t>(kMinStageBytes, (max_row + 127) & ~int64_t(127));
+    const int n_stages = static_cast<int>(std::min<int64_t>(kMaxStages, avail / stage));
+    if (n_stages < 2)
+        return BSM_ERR_UNSUPPORTED;
+
+    // ---- patches: consecutive rows of one slice filling (at most) one stage
+    std::vector<Item> items;
+    std::vector<int32_t> slice_first(slices.size() + 1, 0);
+    for (size_t s = 0; s < slices.size(); ++s) {
+        slice_first[s] = static_cast<int32_t>(items.size());
+        const SliceView &v = slices[s];
+        if (v.R == 0)
+            continue;
+        const int64_t row_bytes = int64_t(v.C) * es;
+        int64_t rpi = std::max<int64_t>(1, stage / row_bytes);
+        if (d->rows_per_item > 0)
+            rpi = std::min<int64_t>(rpi, d->rows_per_item);
+        if (d->policy == BSM_POLICY_WHOLE_GPU)
+            rpi = std::min<int64_t>(rpi, (v.R + c->n_sm - 1) / c->n_sm);
+        rpi = std::max<int64_t>(1, std::min<int64_t>(rpi, v.R));
+        for (int64_t r0 = 0; r0 < v.R; r0 += rpi) {
+            if (items.size() >= static_cast<size_t>(INT32_MAX))
+                return BSM_ERR_UNSUPPORTED;
+            const int64_t nr = std::min<int64_t>(rpi, v.R - r0);
+            items.push_back({v.off + r0 * v.C, v.C, static_cast<int32_t>(nr), static_cast<int32_t>(r0), 0});
+        }
+    }
+    slice_first[slices.size()] = static_cast<int32_t>(items.size());
+    const int64_t n_items = static_cast<int64_t>(items.size());
+
+    bsm_plan *p = new bsm_plan();
+    p->device = device;
+    p->policy = d->policy;
+    p->dtype = d->dtype;
+    p->x = d->x;
+    p->y = d->y;
+    p->flags = d->flags;
+    bsm_plan_stats &st = p->stats;
+    std::memset(&st, 0, sizeof st);
+    st.policy = d->policy;
+    st.n_die = 1;
+    st.n_items = n_items;
+    st.stage_bytes = static_cast<int32_t>(stage);
+    st.n_stages = n_stages;
+
+    // ---- the schedule
+    std::vector<int32_t> queue;
+    int32_t qbeg[BSM_MAX_DIES] = {0}, qlen[BSM_MAX_DIES] = {0};
+    int n_queues = 1;
+    int8_t sm_die_tab[BSM_MAX_SM];
+    std::memset(sm_die_tab, 0, sizeof sm_die_tab);
+    bool use_sm_die = false;
+    if (d->policy == BSM_POLICY_DYNAMIC) {
+        queue.resize(static_cast<size_t>(n_items));
+        std::iota(queue.begin(), queue.end(), 0);
+        qlen[0] = static_cast<int32_t>(n_items);
+        st.queue_items[0] = n_items;
+        st.queue_bytes[0] = total * es * 2;
+        st.L[0] = st.N[0] = n_items;
+    } else if (d->policy == BSM_POLICY_CBMF || d->policy == BSM_POLICY_CBMF_LB) {
+        bsm_topology topo;
+        if ((rc = topology_get(device, 0, &topo))) {
+            delete p;
+            return rc;
+        }
+        const bool lb = d->policy == BSM_POLICY_CBMF_LB;
+        if (!topo.separable || n_items == 0) {
+            // one die: CBMF degenerates to a single queue
+            queue.resize(static_cast<size_t>(n_items));
+            std::iota(queue.begin(), queue.end(), 0);
+            qlen[0] = static_cast<int32_t>(n_items);
+            st.queue_items[0] = n_items;
+            st.L[0] = st.N[0] = n_items;
+        } else {
+            const int nb = 2;
+            const int64_t xbytes = total * es;
+            int64_t chunk = std::max<int64_t>(128, topo.granularity);
+            chunk = (chunk + 127) & ~int64_t(127);
+            while ((xbytes + chunk - 1) / chunk > kMaxMapChunks)
+                chunk *= 2;
+            st.map_chunk_bytes = chunk;
+            const int64_t nch = (xbytes + chunk - 1) / chunk;
+            std::vector<int8_t> xmap(static_cast<size_t>(nch)), ymap;
+            if ((rc = addr_die_map_host(device, d->x, xbytes, chunk, xmap.data()))) {
+                delete p;
+                return rc;
+            }
+            const bool count_y = d->count_output_bytes != 0;
+            if (count_y) {
+                if (d->y == d->x) {
+                    ymap = xmap;
+                } else {
+                    ymap.resize(static_cast<size_t>(nch));
+                    if ((rc = addr_die_map_host(device, d->y, xbytes, chunk, ymap.data()))) {
+                        delete p;
+                        return rc;
+                    }
+                }
+            }
+            std::vector<int64_t> pb(static_cast<size_t>(n_items)), pe(static_cast<size_t>(n_items)),
+                cost(static_cast<size_t>(n_items));
+            for (int64_t i = 0; i < n_items; ++i) {
+                pb[i] = items[i].off * es;
+                pe[i] = (items[i].off + int64_t(items[i].nrows) * items[i].C) * es;
+                cost[i] = 2 * (pe[i] - pb[i]);
+            }
+            int32_t units[BSM_MAX_DIES] = {std::max(1, topo.sm_per_die[0]), std::max(1, topo.sm_per_die[1])};
+            bsm_schedule_desc sd{};
+            sd.n_banks = nb;
+            sd.n_patches = n_items;
+            sd.patch_begin = pb.data();
+            sd.patch_end = pe.data();
+            sd.n_maps = count_y ? 2 : 1;
+            sd.chunk[0] = sd.chunk[1] = chunk;
+            sd.n_chunks[0] = sd.n_chunks[1] = nch;
+            sd.bank_of_chunk[0] = xmap.data();
+            sd.bank_of_chunk[1] = count_y ? ymap.data() : nullptr;
+            sd.tie_seed = d->tie_seed;
+            sd.balance = lb ? 1 : 0;
+            sd.units = units;
+            sd.l_near = d->lb_weighted ? std::max<int64_t>(1, llround(topo.l_near)) : 1;
+            sd.l_far = d->lb_weighted ? std::max<int64_t>(1, llround(topo.l_far)) : 1;
+            sd.cost = cost.data();
+            std::vector<int64_t> bob(static_cast<size_t>(n_items) * nb);
+            std::vector<uint8_t> ov(static_cast<size_t>(n_items));
+            std::vector<int32_t> bank(static_cast<size_t>(n_items)), qi(static_cast<size_t>(n_items)),
+                moved(static_cast<size_t>(n_items));
+            int64_t N[BSM_MAX_DIES] = {0}, L[BSM_MAX_DIES] = {0}, ql[BSM_MAX_DIES] = {0};
+            int64_t wb[BSM_MAX_DIES] = {0}, wa[BSM_MAX_DIES] = {0};
+            bsm_schedule_out so{};
+            so.bytes_on_bank = bob.data();
+            so.overlap = ov.data();
+            so.N = N;
+            so.bank = bank.data();
+            so.L = L;
+            so.queue_items = qi.data();
+            so.queue_len = ql;
+            so.moved = moved.data();
+            so.work_before = wb;
+            so.work_after = wa;
+            if ((rc = schedule_host(&sd, &so))) {
+                delete p;
+                return rc;
+            }
+            queue = qi;
+            n_queues = nb;
+            int32_t pos = 0;
+            for (int b = 0; b < nb; ++b) {
+                qbeg[b] = pos;
+                qlen[b] = static_cast<int32_t>(ql[b]);
+                pos += qlen[b];
+                st.N[b] = N[b];
+                st.L[b] = L[b];
+                st.queue_items[b] = ql[b];
+                int64_t bytes = 0;
+                for (int32_t k = qbeg[b]; k < qbeg[b] + qlen[b]; ++k)
+                    bytes += cost[queue[k]];
+                st.queue_bytes[b] = bytes;
+                if (lb) {
+                    st.est_finish_before[b] = double(wb[b]) / units[b];
+                    st.est_finish_after[b] = double(wa[b]) / units[b];
+                }
+            }
+            for (int64_t i = 0; i < n_items; ++i) {
+                st.overlap_items += ov[i];
+                const int64_t *row = &bob[static_cast<size_t>(i) * nb];
+                if (row[0] == row[1])
+                    ++st.tie_items;
+            }
+            st.moved_items = so.n_moved;
+            st.n_die = nb;
+            std::memcpy(sm_die_tab, topo.sm_die, sizeof sm_die_tab);
+            for (int s = 0; s < BSM_MAX_SM; ++s)
+                if (sm_die_tab[s] < 0)
+                    sm_die_tab[s] = 0;
+            use_sm_die = true;
+            p->args.steal = lb ? 1 : 0;
+        }
+    }
+
+    // ---- upload the tables in one allocation
+    const size_t items_b = sizeof(Item) * static_cast<size_t>(n_items);
+    const size_t queue_b = sizeof(int32_t) * queue.size();
+    const size_t slices_b = sizeof(int32_t) * slice_first.size();
+    auto up = [](size_t v) { return (v + 255) & ~size_t(255); };
+    const size_t o_items = 0, o_queue = up(items_b), o_slices = o_queue + up(queue_b),
+                 o_smdie = o_slices + up(slices_b), o_heads = o_smdie + 256, blob_b = o_heads + 256;
+    std::vector<unsigned char> host(blob_b, 0);
+    if (items_b)
+        std::memcpy(&host[o_items], items.data(), items_b);
+    if (queue_b)
+        std::memcpy(&host[o_queue], queue.data(), queue_b);
+    std::memcpy(&host[o_slices], slice_first.data(), slices_b);
+    std::memcpy(&host[o_smdie], sm_die_tab, BSM_MAX_SM);
+    int prev = -1;
+    cudaGetDevice(&prev);
+    cudaSetDevice(device);
+    if (cudaMalloc(&p->blob, blob_b) != cudaSuccess) {
+        if (prev >= 0)
+            cudaSetDevice(prev);
+        delete p;
+        return BSM_ERR_NOMEM;
+    }
+    if (cudaMemcpy(p->blob, host.data(), blob_b, cudaMemcpyHostToDevice) != cudaSuccess) {
+        cudaFree(p->blob);
+        if (prev >= 0)
+            cudaSetDevice(prev);
+        delete p;
+        return BSM_ERR_CUDA;
+    }
+    if (prev >= 0)
+        cudaSetDevice(prev);
+    unsigned char *b = static_cast<unsigned char *>(p->blob);
+
+    KernelArgs &a = p->args;
+    a.x = d->x;
+    a.y = d->y;
+    a.total_elems = total;
+    a.items = reinterpret_cast<const Item *>(b + o_items);
+    a.n_items = static_cast<int32_t>(n_items);
+    a.slice_first_item = reinterpret_cast<const int32_t *>(b + o_slices);
+    a.n_slices = static_cast<int32_t>(std::min<size_t>(slices.size(), INT32_MAX));
+    a.n_queues = n_queues;
+    a.queue = reinterpret_cast<const int32_t *>(b + o_queue);
+    for (int q = 0; q < BSM_MAX_DIES; ++q) {
+        a.queue_begin[q] = qbeg[q];
+        a.queue_len[q] = qlen[q];
+    }
+    a.heads = reinterpret_cast<uint32_t *>(b + o_heads);
+    a.sm_die = use_sm_die ? reinterpret_cast<const int8_t *>(b + o_smdie) : nullptr;
+    a.stage_bytes = static_cast<int32_t>(stage);
+    a.n_stages = n_stages;
+    a.flags = d->flags;
+    a.status = c->status;
+
+    switch (d->policy) {
+    case BSM_POLICY_WHOLE_GPU:
+        a.mode = PULL_STATIC;
+        for (size_t s = 0; s < slices.size(); ++s) {
+            const int32_t n = slice_first[s + 1] - slice_first[s];
+            if (n > 0)
+                p->whole_gpu.push_back({slice_first[s], slice_first[s + 1], std::min(n, c->n_sm)});
+        }
+        p->grid = c->n_sm;
+        st.launches = static_cast<int32_t>(p->whole_gpu.size());
+        break;
+    case BSM_POLICY_RR:
+        a.mode = PULL_RR_SLICE;
+        p->grid = static_cast<int>(std::min<int64_t>(c->n_sm, std::max<int64_t>(1, int64_t(slices.size()))));
+        st.launches = n_items > 0 ? 1 : 0;
+        break;
+    default:
+        a.mode = PULL_QUEUE;
+        p->grid = c->n_sm;
+        st.launches = n_items > 0 ? 1 : 0;
+        break;
+    }
+    st.grid = p->grid;
+    st.steal = a.steal;
+    st.plan_ms = std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t0).count();
+    *out = p;
+    return BSM_OK;
+}
+
+int plan_execute_impl(const bsm_plan *p, bsm_stream_t stream)
+{
+    if (!p)
+        return BSM_ERR_INVALID_ARG;
+    if (p->args.n_items == 0)
+        return BSM_OK;
+    int prev = -1;
+    cudaGetDevice(&prev);
+    if (prev != p->device && cudaSetDevice(p->device) != cudaSuccess)
+        return BSM_ERR_NO_DEVICE;
+    int err = 0;
+    if (p->policy == BSM_POLICY_WHOLE_GPU) {
+        KernelArgs a = p->args;
+        for (const auto &l : p->whole_gpu) {
+            a.item_begin = l.begin;
+            a.item_end = l.end;
+            if ((err = launch_softmax(a, p->dtype, l.grid, stream)))
+                break;
+        }
+    } else {
+        err = launch_softmax(p->args, p->dtype, p->grid, stream);
+    }
+    if (prev >= 0 && prev != p->device)
+        cudaSetDevice(prev);
+    return err ? BSM_ERR_CUDA : BSM_OK;
+}
+
+// ---- plan cache of the one-call entry points
+
+struct CacheKey {
+    int device;
+    const void *x;
+    void *y;
+    int dtype, policy;
+    uint32_t flags;
+};
+
+std::mutex g_cache_mu;
+std::list<bsm_plan *> g_cache;   // most recent first
+constexpr size_t kCacheMax = 32;
+
+bool same_key(const bsm_plan *p, const CacheKey &k)
+{
+    return p->device == k.device && p->x == k.x && p->y == k.y && p->dtype == k.dtype &&
+           p->policy == k.policy && p->flags == k.flags;
+}
+
+int cached_run(const CacheKey &k, int64_t B, int64_t R, int64_t C, int64_t n, const int64_t *off,
+               const int32_t *rows, const int32_t *cols, bsm_stream_t stream)
+{
+    std::lock_guard<std::mutex> lk(g_cache_mu);
+    for (auto it = g_cache.begin(); it != g_cache.end(); ++it) {
+        bsm_plan *p = *it;
+        if (!same_key(p, k))
+            continue;
+        bool hit;
+        if (B >= 0) {
+            hit = p->key_B == B && p->key_R == R && p->key_C == C;
+        } else {
+            hit = p->key_B < 0 && static_cast<int64_t>(p->key_rows.size()) == n &&
+                  std::equal(rows, rows + n, p->key_rows.begin()) &&
+                  std::equal(cols, cols + n, p->key_cols.begin()) &&
+                  std::equal(off, off + n, p->key_offsets.begin());
+        }
+        if (hit) {
+            g_cache.splice(g_cache.begin(), g_cache, it);
+            return plan_execute_impl(p, stream);
+        }
+    }
+    bsm_plan_desc d;
+    bsm_plan_desc_init(&d);
+    d.x = k.x;
+    d.y = k.y;
+    d.dtype = k.dtype;
+    d.policy = k.policy;
+    d.flags = k.flags;
+    d.device = k.device;
+    std::vector<int32_t> r, c;
+    if (B >= 0) {
+        if (B > INT32_MAX || R > INT32_MAX || C > INT32_MAX)
+            return BSM_ERR_UNSUPPORTED;
+        r.assign(static_cast<size_t>(B), static_cast<int32_t>(R));
+        c.assign(static_cast<size_t>(B), static_cast<int32_t>(C));
+        d.num_slices = B;
+        d.rows = r.data();
+        d.cols = c.data();
+    } else {
+        d.num_slices = n;
+        d.offsets = off;
+        d.rows = rows;
+        d.cols = cols;
+    }
+    bsm_plan *p = nullptr;
+    int rc = plan_create_impl(&p, &d);
+    if (rc)
+        return rc;
+    if (B >= 0) {
+        p->key_B = B;
+        p->key_R = R;
+        p->key_C = C;
+    } else {
+        p->key_offsets.assign(off, off + n);
+        p->key_rows.assign(rows, rows + n);
+        p->key_cols.assign(cols, cols + n);
+    }
+    g_cache.push_front(p);
+    while (g_cache.size() > kCacheMax) {
+        bsm_plan *old = g_cache.back();
+        g_cache.pop_back();
+        cudaFree(old->blob);
+        delete old;
+    }
+    return plan_execute_impl(p, stream);
+}
+
+}  // namespace
+}  // namespace bsm
+
+using namespace bsm;
+
+#define BSM_GUARD(expr)                                  \
+    try {                                                \
+        return (expr);                                   \
+    } catch (const std::bad_alloc &) {                   \
+        return BSM_ERR_NOMEM;                            \
+    } catch (...) {                                      \
+        return BSM_ERR_INVALID_ARG;                      \
+    }
+
+extern "C" {
+
+int bsm_plan_desc_init(bsm_plan_desc *d)
+{
+    if (!d)
+        return BSM_ERR_INVALID_ARG;
+    std::memset(d, 0, sizeof *d);
+    d->tie_seed = kDefaultTieSeed;
+    d->lb_weighted = 1;
+    d->count_output_bytes = 1;
+    d->device = -1;
+    return BSM_OK;
+}
+
+int bsm_plan_create(bsm_plan **plan, const bsm_plan_desc *d) { BSM_GUARD(plan_create_impl(plan, d)) }
+
+int bsm_plan_execute(const bsm_plan *plan, bsm_stream_t stream) { BSM_GUARD(plan_execute_impl(plan, stream)) }
+
+int bsm_plan_get_stats(const bsm_plan *plan, bsm_plan_stats *out)
+{
+    if (!plan || !out)
+        return BSM_ERR_INVALID_ARG;
+    *out = plan->stats;
+    return BSM_OK;
+}
+
+void bsm_plan_destroy(bsm_plan *plan)
+{
+    if (!plan)
+        return;
+    cudaFree(plan->blob);
+    delete plan;
+}
+
+void bsm_cache_clear(void)
+{
+    std::lock_guard<std::mutex> lk(g_cache_mu);
+    for (bsm_plan *p : g_cache) {
+        cudaFree(p->blob);
+        delete p;
+    }
+    g_cache.clear();
+}
+
+static int softmax_uniform(const void *x, void *y, int64_t B, int64_t R, int64_t C, int dtype, int policy,
+                           uint32_t flags, bsm_stream_t stream)
+{
+    if (B < 0 || R < 0 || C < 1)
+        return BSM_ERR_INVALID_ARG;
+    if (dtype != BSM_F32 && dtype != BSM_BF16)
+        return BSM_ERR_INVALID_ARG;
+    if (policy < BSM_POLICY_WHOLE_GPU || policy > BSM_POLICY_DYNAMIC || (flags & ~BSM_FLAG_CAUSAL))
+        return BSM_ERR_INVALID_ARG;
+    if (R > 0 && (B > (int64_t(1) << 62) / R || C > (int64_t(1) << 62) / std::max<int64_t>(1, B * R)))
+        return BSM_ERR_INVALID_ARG;
+    if (B == 0 || R == 0)
+        return BSM_OK;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess)
+        return BSM_ERR_NO_DEVICE;
+    CacheKey k{dev, x, y, dtype, policy, flags};
+    return cached_run(k, B, R, C, 0, nullptr, nullptr, nullptr, stream);
+}
+
+int bsm_softmax(const void *x, void *y, int64_t B, int64_t R, int64_t C, int dtype, int policy,
+                bsm_stream_t stream)
+{
+    BSM_GUARD(softmax_uniform(x, y, B, R, C, dtype, policy, 0u, stream))
+}
+
+int bsm_softmax_ex(const void *x, void *y, int64_t B, int64_t R, int64_t C, int dtype, int policy,
+                   uint32_t flags, bsm_stream_t stream)
+{
+    BSM_GUARD(softmax_uniform(x, y, B, R, C, dtype, policy, flags, stream))
+}
+
+static int softmax_ragged(const void *x, void *y, int64_t n, const int64_t *off, const int32_t *rows,
+                          const int32_t *cols, int dtype, int policy, uint32_t flags, bsm_stream_t stream)
+{
+    if (n < 0 || (n > 0 && (!off || !rows || !cols)))
+        return BSM_ERR_INVALID_ARG;
+    if (dtype != BSM_F32 && dtype != BSM_BF16)
+        return BSM_ERR_INVALID_ARG;
+    if (policy < BSM_POLICY_WHOLE_GPU || policy > BSM_POLICY_DYNAMIC || (flags & ~BSM_FLAG_CAUSAL))
+        return BSM_ERR_INVALID_ARG;
+    if (n == 0)
+        return BSM_OK;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess)
+        return BSM_ERR_NO_DEVICE;
+    CacheKey k{dev, x, y, dtype, policy, flags};
+    return cached_run(k, -1, 0, 0, n, off, rows, cols, stream);
+}
+
+int bsm_softmax_ragged(const void *x, void *y, int64_t num_slices, const int64_t *offsets,
+                       const int32_t *rows, const int32_t *cols, int dtype, int policy, uint32_t flags,
+                       bsm_stream_t stream)
+{
+    BSM_GUARD(softmax_ragged(x, y, num_slices, offsets, rows, cols, dtype, policy, flags, stream))
+}
+
+int bsm_topology_probe(int device, int force, bsm_topology *out)
+{
+    if (!out)
+        return BSM_ERR_INVALID_ARG;
+    if (device < 0 && cudaGetDevice(&device) != cudaSuccess)
+        return BSM_ERR_NO_DEVICE;
+    DeviceCtx *c = nullptr;
+    int rc = device_ctx(device, &c);
+    if (rc)
+        return rc;
+    BSM_GUARD(topology_get(device, force, out))
+}
+
+int bsm_addr_die_map(int device, const void *ptr, int64_t bytes, int64_t chunk, int8_t *die_out)
+{
+    if (device < 0 && cudaGetDevice(&device) != cudaSuccess)
+        return BSM_ERR_NO_DEVICE;
+    BSM_GUARD(addr_die_map_host(device, ptr, bytes, chunk, die_out))
+}
+
+int bsm_probe_latency(int device, int32_t n_lines, const int64_t *line_off, int32_t reps, float *lat_out,
+                      int32_t *seen_out)
+{
+    if (n_lines <= 0 || !line_off || !lat_out || !seen_out)
+        return BSM_ERR_INVALID_ARG;
+    if (device < 0 && cudaGetDevice(&device) != cudaSuccess)
+        return BSM_ERR_NO_DEVICE;
+    try {
+        std::vector<int64_t> lines(line_off, line_off + n_lines);
+        std::vector<float> lat;
+        std::vector<int32_t> seen;
+        int rc = probe_latency_host(device, lines, reps, lat, seen);
+        if (rc)
+            return rc;
+        std::memcpy(lat_out, lat.data(), sizeof(float) * lat.size());
+        std::memcpy(seen_out, seen.data(), sizeof(int32_t) * seen.size());
+        return BSM_OK;
+    } catch (const std::bad_alloc &) {
+        return BSM_ERR_NOMEM;
+    }
+}
+
+int bsm_schedule_host(const bsm_schedule_desc *d, bsm_schedule_out *out) { BSM_GUARD(schedule_host(d, out)) }
+
+int bsm_device_status(int device, uint32_t *status_out)
+{
+    if (!status_out)
+        return BSM_ERR_INVALID_ARG;
+    DeviceCtx *c = nullptr;
+    int rc = device_ctx(device, &c);
+    if (rc)
+        return rc;
+    if (cudaDeviceSynchronize() != cudaSuccess)
+        return BSM_ERR_CUDA;
+    if (cudaMemcpy(status_out, c->status, sizeof(uint32_t), cudaMemcpyDeviceToHost) != cudaSuccess)
+        return BSM_ERR_CUDA;
+    return BSM_OK;
+}
+
+int bsm_device_status_clear(int device)
+{
+    DeviceCtx *c = nullptr;
+    int rc = device_ctx(device, &c);
+    if (rc)
+        return rc;
+    if (cudaMemset(c->status, 0, sizeof(uint32_t)) != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess)
+        return BSM_ERR_CUDA;
+    return BSM_OK;
+}
+
+int64_t bsm_max_row_bytes(int device)
+{
+    DeviceCtx *c = nullptr;
+    if (device_ctx(device, &c))
+        return 0;
+    return max_row_bytes_for(*c);
+}
+
+const char *bsm_status_string(int status)
+{
+    switch (status) {
+    case BSM_OK:
+        return "ok";
+    case BSM_ERR_INVALID_ARG:
+        return "invalid argument";
+    case BSM_ERR_MISALIGNED:
+        return "misaligned: pointers, slice offsets and row lengths must be multiples of 16 bytes";
+    case BSM_ERR_UNSUPPORTED:
+        return "unsupported: row longer than a shared-memory stage, or too many patches";
+    case BSM_ERR_CUDA:
+        return "CUDA runtime error";
+    case BSM_ERR_DEVICE_BOUNDS:
+        return "a kernel met a patch outside the buffers";
+    case BSM_ERR_TIMEOUT:
+        return "a kernel wait ran out of time";
+    case BSM_ERR_NO_DEVICE:
+        return "no usable CUDA device";
+    case BSM_ERR_NOMEM:
+        return "out of memory";
+    default:
+        return "unknown status";
+    }
+}
+
+int bsm_version(void) { return (1 << 16) | 0; }
+
+}  // extern "C"

@@ -1,0 +1,74 @@
+// bsm_internal.h -- types shared by the kernels (.cu) and the host side
+// (.cpp) of libbsm.  Not part of the public ABI.
+#pragma once
+
+#include <cstdint>
+
+#include "../../include/bsm.h"
+
+namespace bsm {
+
+// One patch ("batch or patch", Sec. 4: the unit of work the scheduler places):
+// rows [row0, row0 + nrows) of one slice.  The patch's elements are contiguous:
+// they start at element `off` of x and y and span nrows * C elements.
+struct Item {
+    int64_t off;
+    int32_t C;
+    int32_t nrows;
+    int32_t row0;   // row index inside the slice of the first row (causal mask)
+    int32_t pad;
+};
+static_assert(sizeof(Item) == 24, "Item layout");
+
+// How a CTA finds its next patch.
+enum PullMode : int32_t {
+    PULL_STATIC = 0,    // CTA b takes items item_begin + b, + b + G, ... (< item_end)
+    PULL_RR_SLICE = 1,  // CTA b takes every patch of slices b, b + G, ... (Sec. 3 RR)
+    PULL_QUEUE = 2      // CTA pulls from its die's queue, then (steal) the others'
+};
+
+constexpr int kMaxStages = 8;
+constexpr int kConsumerWarps = 16;
+constexpr int kThreads = (kConsumerWarps + 1) * 32;  // + one producer warp
+constexpr int kSmemHeader = 1024;                     // barriers + stage metadata
+constexpr int kMinStageBytes = 32 * 1024;
+
+struct KernelArgs {
+    const void *x;
+    void *y;
+    int64_t total_elems;        // extent of x and y, elements (bounds checks)
+    const Item *items;
+    int32_t n_items;
+    int32_t mode;               // PullMode
+    int32_t item_begin, item_end;           // PULL_STATIC
+    const int32_t *slice_first_item;        // PULL_RR_SLICE: n_slices + 1 entries
+    int32_t n_slices;
+    int32_t n_queues;                       // PULL_QUEUE
+    const int32_t *queue;                   // concatenated per-die queues
+    int32_t queue_begin[BSM_MAX_DIES];
+    int32_t queue_len[BSM_MAX_DIES];
+    int32_t steal;
+    uint32_t *heads;            // BSM_MAX_DIES queue heads + 1 exit counter; self-resetting
+    const int8_t *sm_die;       // die of each %smid (NULL: all die 0)
+    int32_t stage_bytes;
+    int32_t n_stages;
+    uint32_t flags;
+    uint32_t *status;           // sticky device status word
+};
+
+// Launch the persistent softmax kernel (bsm_kernels.cu).  Returns a
+// cudaError_t value (0 = success).
+int launch_softmax(const KernelArgs &a, int dtype, int grid, void *stream);
+// Raise the dynamic shared-memory limit of both kernel instances.
+int kernel_set_smem_limit(int bytes);
+
+// Probe kernels (bsm_probe.cu).  All synchronous; return cudaError_t values.
+int probe_latency_run(const void *buf, const int64_t *line_off_dev, int n_lines, int reps,
+                      int grid, float *lat_dev, uint32_t *claim_dev);
+int probe_map_run(const void *buf, int64_t bytes, int64_t chunk, int reps, const int8_t *sm_die_dev,
+                  float threshold, int n_sm, uint32_t *counter_dev, int8_t *die_dev);
+
+// Host planner (bsm_planner.cpp).
+int schedule_host(const bsm_schedule_desc *d, bsm_schedule_out *out);
+
+}  // namespace bsm

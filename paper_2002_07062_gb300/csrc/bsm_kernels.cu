@@ -1,0 +1,573 @@
+// bsm_kernels.cu -- the persistent batched-softmax kernel for sm_103a.
+//
+// One CTA per SM.  Warp 16 is the producer: one lane pulls the next patch
+// (Sec. 4: a block of rows of one slice) from the schedule -- a static list
+// for the Sec. 3 baselines, or the CTA's die queue for Cluster Beamforming
+// (Sec. 4.1) with stealing after the Sec. 4.2 balance -- and streams the
+// patch's contiguous bytes into a ring of shared-memory stages with one 1-D
+// TMA bulk copy (cp.async.bulk, completion counted on an mbarrier).  Warps
+// 0..15 are consumers: they wait on a stage's "full" barrier, compute the
+// softmax of its rows out of shared memory, store y with 128-bit coalesced
+// stores, and release the stage on its "empty" barrier.  The patch geometry
+// travels with the stage (the "templated kernel fed patch coordinates from a
+// queue" of Sec. 5).
+//
+// Row routine (the arithmetic, identical under every policy): a row is owned
+// by a group of T lanes (T = 16 for rows of <= 256 bytes, else 32); lane l owns
+// the 16-byte vectors l, l + T, l + 2T, ...; the maximum and the sum are
+// per-lane in vector order, then a butterfly (xor) shuffle tree.  Rows of up
+// to 2 KiB are held in registers; longer rows are swept three times out of
+// shared memory (max, sum, write).  exp(t) is evaluated as 2^(t*log2 e) with
+// the exponent formed by one fused multiply-add, v*log2e - m*log2e, and the
+// power of two from the PTX ex2.approx instruction; y = p * (1/sum).
+//
+// Every wait is bounded (kWaitLimitNs, 2 s of wall time): on expiry the CTA
+// records BSM_DEV_TIMEOUT in the status word, lets its copies in flight land,
+// and returns.
+
+#include <cuda_runtime.h>
+#include <cstdint>
+
+#include "bsm_internal.h"
+
+namespace bsm {
+namespace {
+
+constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s
+constexpr float kLog2e = 1.4426950408889634f;
+
+enum : int32_t { KIND_DATA = 0, KIND_SKIP = 1, KIND_DONE = 2 };
+
+struct alignas(16) StageMeta {
+    int64_t off;
+    int32_t C;
+    int32_t nrows;
+    int32_t row0;
+    int32_t kind;
+    int32_t pad[2];
+};
+static_assert(sizeof(StageMeta) == 32, "StageMeta layout");
+
+struct SmemHeader {
+    uint64_t full[kMaxStages];
+    uint64_t empty[kMaxStages];
+    StageMeta meta[kMaxStages];
+    int32_t abort_flag;
+};
+static_assert(sizeof(SmemHeader) <= kSmemHeader, "header too large");
+
+// ---------------------------------------------------------------- PTX helpers
+
+__device__ __forceinline__ uint32_t smem_addr(const void *p)
+{
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ uint64_t global_timer_ns()
+{
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ uint32_t sm_id()
+{
+    uint32_t s;
+    asm volatile("mov.u32 %0, %%smid;" : "=r"(s));
+    return s;
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count)
+                 : "memory");
+}
+
+__device__ __forceinline__ void mbar_init_fence()
+{
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t *bar)
+{
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)),
+                 "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_addr(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Wait until the phase with the given parity of `bar` has completed.  Gives
+// up (returns false) when *abort becomes non-zero (if abort != nullptr) or
+// after kWaitLimitNs.
+__device__ __noinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity,
+                                               const volatile int32_t *abort)
+{
+    if (mbar_try_wait(bar, parity))
+        return true;
+    const uint64_t t0 = global_timer_ns();
+    for (uint32_t it = 0; it < (1u << 28); ++it) {
+        if (mbar_try_wait(bar, parity))
+            return true;
+        if ((it & 7u) == 7u) {
+            if (abort && *abort)
+                return false;
+            if (global_timer_ns() - t0 > kWaitLimitNs)
+                return false;
+        }
+    }
+    return false;
+}
+
+// 1-D bulk copy global -> shared, completion counted (bytes) on `bar`.
+__device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar)
+{
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+            smem_addr(dst)),
+        "l"(src), "r"(bytes), "r"(smem_addr(bar))
+        : "memory");
+}
+
+// Plain C++ accesses: the compiler sees them as memory operations, so the
+// "memory" clobber of the barrier waits orders them, and it may still
+// schedule them freely inside a row.
+__device__ __forceinline__ uint4 lds128(const unsigned char *p)
+{
+    return *reinterpret_cast<const uint4 *>(p);
+}
+
+__device__ __forceinline__ void stg128(void *p, uint4 v)
+{
+    *reinterpret_cast<uint4 *>(p) = v;
+}
+
+__device__ __forceinline__ float ex2(float a)
+{
+    float r;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(a));
+    return r;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
+{
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
+}
+
+// ------------------------------------------------------- element-type traits
+
+template <typename Tag> struct Elem;
+struct F32 {};
+struct BF16 {};
+
+template <> struct Elem<F32> {
+    static constexpr int kSize = 4;
+    static constexpr int kPerVec = 4;
+    __device__ static __forceinline__ void unpack(uint4 r, float (&v)[4])
+    {
+        v[0] = __uint_as_float(r.x);
+        v[1] = __uint_as_float(r.y);
+        v[2] = __uint_as_float(r.z);
+        v[3] = __uint_as_float(r.w);
+    }
+    __device__ static __forceinline__ uint4 pack(const float (&v)[4])
+    {
+        return make_uint4(__float_as_uint(v[0]), __float_as_uint(v[1]), __float_as_uint(v[2]),
+                          __float_as_uint(v[3]));
+    }
+};
+
+template <> struct Elem<BF16> {
+    static constexpr int kSize = 2;
+    static constexpr int kPerVec = 8;
+    __device__ static __forceinline__ void unpack(uint4 r, float (&v)[8])
+    {
+        const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            v[2 * k] = __uint_as_float(w[k] << 16);
+            v[2 * k + 1] = __uint_as_float(w[k] & 0xFFFF0000u);
+        }
+    }
+    __device__ static __forceinline__ uint4 pack(const float (&v)[8])
+    {
+        return make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]),
+                          pack_bf16x2(v[6], v[7]));
+    }
+};
+
+// ------------------------------------------------------------- row routines
+
+template <int T> __device__ __forceinline__ float group_max(float m)
+{
+#pragma unroll
+    for (int o = T / 2; o >= 1; o >>= 1)
+        m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+    return m;
+}
+
+template <int T> __device__ __forceinline__ float group_sum(float s)
+{
+#pragma unroll
+    for (int o = T / 2; o >= 1; o >>= 1)
+        s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
+    return s;
+}
+
+// Additive causal mask of one 16-byte vector: element c of the row gets -inf
+// when c > row.
+template <int EPV>
+__device__ __forceinline__ void apply_causal(float (&v)[EPV], int col0, int row)
+{
+#pragma unroll
+    for (int e = 0; e < EPV; ++e)
+        v[e] += (col0 + e > row) ? -INFINITY : 0.0f;
+}
+
+// Register-resident row: T lanes, up to V vectors per lane.
+template <typename Tag, int T, int V>
+__device__ __forceinline__ void row_in_registers(const unsigned char *srow, void *yrow, int nvec,
+                                                 int row, bool causal, int l, bool valid)
+{
+    using E = Elem<Tag>;
+    constexpr int EPV = E::kPerVec;
+    float v[V][EPV];
+    float m = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < V; ++j) {
+        const int vi = j * T + l;
+        if (valid && vi < nvec) {
+            E::unpack(lds128(srow + 16 * vi), v[j]);
+            if (causal)
+                apply_causal<EPV>(v[j], vi * EPV, row);
+#pragma unroll
+            for (int e = 0; e < EPV; ++e)
+                m = fmaxf(m, v[j][e]);
+        } else {
+#pragma unroll
+            for (int e = 0; e < EPV; ++e)
+                v[j][e] = -INFINITY;
+        }
+    }
+    m = group_max<T>(m);
+    const float mL = m * kLog2e;
+    float s = 0.0f;
+#pragma unroll
+    for (int j = 0; j < V; ++j) {
+        float ps = 0.0f;
+#pragma unroll
+        for (int e = 0; e < EPV; ++e) {
+            v[j][e] = ex2(fmaf(v[j][e], kLog2e, -mL));
+            ps += v[j][e];
+        }
+        if (j * T + l < nvec)
+            s += ps;
+    }
+    s = group_sum<T>(s);
+    const float inv = 1.0f / s;
+#pragma unroll
+    for (int j = 0; j < V; ++j) {
+        const int vi = j * T + l;
+        if (valid && vi < nvec) {
+#pragma unroll
+            for (int e = 0; e < EPV; ++e)
+                v[j][e] *= inv;
+            stg128(static_cast<unsigned char *>(yrow) + 16 * vi, E::pack(v[j]));
+        }
+    }
+}
+
+// Shared-memory-resident row of any length: one warp, three sweeps.
+template <typename Tag>
+__device__ __forceinline__ void row_in_smem(const unsigned char *srow, void *yrow, int nvec, int row,
+                                            bool causal, int lane)
+{
+    using E = Elem<Tag>;
+    constexpr int EPV = E::kPerVec;
+    float v[EPV];
+    float m = -INFINITY;
+    for (int vi = lane; vi < nvec; vi += 32) {
+        E::unpack(lds128(srow + 16 * vi), v);
+        if (causal)
+            apply_causal<EPV>(v, vi * EPV, row);
+#pragma unroll
+        for (int e = 0; e < EPV; ++e)
+            m = fmaxf(m, v[e]);
+    }
+    m = group_max<32>(m);
+    const float mL = m * kLog2e;
+    float s = 0.0f;
+    for (int vi = lane; vi < nvec; vi += 32) {
+        E::unpack(lds128(srow + 16 * vi), v);
+        if (causal)
+            apply_causal<EPV>(v, vi * EPV, row);
+        float ps = 0.0f;
+#pragma unroll
+        for (int e = 0; e < EPV; ++e)
+            ps += ex2(fmaf(v[e], kLog2e, -mL));
+        s += ps;
+    }
+    s = group_sum<32>(s);
+    const float inv = 1.0f / s;
+    for (int vi = lane; vi < nvec; vi += 32) {
+        E::unpack(lds128(srow + 16 * vi), v);
+        if (causal)
+            apply_causal<EPV>(v, vi * EPV, row);
+#pragma unroll
+        for (int e = 0; e < EPV; ++e)
+            v[e] = ex2(fmaf(v[e], kLog2e, -mL)) * inv;
+        stg128(static_cast<unsigned char *>(yrow) + 16 * vi, E::pack(v));
+    }
+}
+
+// All rows of one stage that belong to this consumer warp.
+template <typename Tag>
+__device__ __forceinline__ void consume_stage(const unsigned char *sbuf, const StageMeta &mt,
+                                              unsigned char *y, bool causal, int warp, int lane)
+{
+    using E = Elem<Tag>;
+    const int C = mt.C;
+    const int nrows = mt.nrows;
+    const int row_bytes = C * E::kSize;
+    const int nvec = row_bytes >> 4;
+    unsigned char *ybase = y + mt.off * E::kSize;
+    if (nvec <= 16) {
+        const int half = lane >> 4, l = lane & 15;
+        for (int rb = 2 * warp; rb < nrows; rb += 2 * kConsumerWarps) {
+            const int r = rb + half;
+            const bool valid = r < nrows;
+            row_in_registers<Tag, 16, 1>(sbuf + (size_t)r * row_bytes, ybase + (size_t)r * row_bytes,
+                                         nvec, mt.row0 + r, causal, l, valid);
+        }
+    } else if (nvec <= 32) {
+        for (int r = warp; r < nrows; r += kConsumerWarps)
+            row_in_registers<Tag, 32, 1>(sbuf + (size_t)r * row_bytes, ybase + (size_t)r * row_bytes,
+                                         nvec, mt.row0 + r, causal, lane, true);
+    } else if (nvec <= 64) {
+        for (int r = warp; r < nrows; r += kConsumerWarps)
+            row_in_registers<Tag, 32, 2>(sbuf + (size_t)r * row_bytes, ybase + (size_t)r * row_bytes,
+                                         nvec, mt.row0 + r, causal, lane, true);
+    } else if (nvec <= 128) {
+        for (int r = warp; r < nrows; r += kConsumerWarps)
+            row_in_registers<Tag, 32, 4>(sbuf + (size_t)r * row_bytes, ybase + (size_t)r * row_bytes,
+                                         nvec, mt.row0 + r, causal, lane, true);
+    } else {
+        for (int r = warp; r < nrows; r += kConsumerWarps)
+            row_in_smem<Tag>(sbuf + (size_t)r * row_bytes, ybase + (size_t)r * row_bytes, nvec,
+                             mt.row0 + r, causal, lane);
+    }
+}
+
+// -------------------------------------------------------------- the schedule
+
+struct Puller {
+    const KernelArgs &a;
+    int32_t k = 0;           // PULL_STATIC: patches taken so far
+    int32_t slice = -1;      // PULL_RR_SLICE
+    int32_t cur = 0, end = 0;
+    int32_t q = 0;           // PULL_QUEUE: index into the try order
+    int32_t die = 0;
+
+    __device__ explicit Puller(const KernelArgs &args) : a(args)
+    {
+        if (a.mode == PULL_QUEUE && a.sm_die) {
+            int d = a.sm_die[sm_id() & (BSM_MAX_SM - 1)];
+            die = (d >= 0 && d < a.n_queues) ? d : 0;
+        }
+        if (a.mode == PULL_RR_SLICE)
+            slice = static_cast<int32_t>(blockIdx.x) - static_cast<int32_t>(gridDim.x);
+    }
+
+    // Next patch index, or -1 when this CTA has no more work.
+    __device__ int32_t next()
+    {
+        if (a.mode == PULL_STATIC) {
+            const int64_t idx = (int64_t)a.item_begin + blockIdx.x + (int64_t)k * gridDim.x;
+            ++k;
+            return idx < a.item_end ? static_cast<int32_t>(idx) : -1;
+        }
+        if (a.mode == PULL_RR_SLICE) {
+            while (cur >= end) {
+                slice += gridDim.x;
+                if (slice >= a.n_slices)
+                    return -1;
+                cur = a.slice_first_item[slice];
+                end = a.slice_first_item[slice + 1];
+            }
+            return cur++;
+        }
+        // PULL_QUEUE: own die first, then (steal) the other dies in order.
+        const int tries = a.steal ? a.n_queues : 1;
+        while (q < tries) {
+            const int qq = (die + q) % a.n_queues;
+            const uint32_t t = atomicAdd(&a.heads[qq], 1u);
+            if (t < static_cast<uint32_t>(a.queue_len[qq]))
+                return a.queue[a.queue_begin[qq] + t];
+            ++q;
+        }
+        return -1;
+    }
+};
+
+template <typename Tag>
+__global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelArgs a)
+{
+    using E = Elem<Tag>;
+    extern __shared__ __align__(1024) unsigned char smem[];
+    SmemHeader &h = *reinterpret_cast<SmemHeader *>(smem);
+    unsigned char *stages = smem + kSmemHeader;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int S = a.n_stages;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(&h.full[s], 1);
+            mbar_init(&h.empty[s], kConsumerWarps);
+        }
+        h.abort_flag = 0;
+        mbar_init_fence();
+    }
+    __syncthreads();
+
+    if (warp == kConsumerWarps) {
+        // ------------------------------------------------------- producer
+        if (lane == 0) {
+            Puller pull(a);
+            uint32_t issued_phase[kMaxStages];
+            bool issued[kMaxStages];
+            for (int s = 0; s < kMaxStages; ++s)
+                issued[s] = false;
+            bool aborted = false;
+            for (uint32_t it = 0;; ++it) {
+                const int s = it % S;
+                const uint32_t ph = (it / S) & 1u;
+                if (!mbar_wait_bounded(&h.empty[s], ph ^ 1u, &h.abort_flag)) {
+                    aborted = true;
+                    break;
+                }
+                issued[s] = false;                 // the consumers released it
+                StageMeta &mt = h.meta[s];
+                const int32_t idx = pull.next();
+                if (idx < 0) {
+                    mt.kind = KIND_DONE;
+                    mbar_arrive(&h.full[s]);
+                    break;
+                }
+                bool ok = idx < a.n_items;
+                Item item{};
+                if (ok) {
+                    item = a.items[idx];
+                    const int64_t n = (int64_t)item.nrows * item.C;
+                    const int64_t bytes = n * E::kSize;
+                    ok = item.off >= 0 && item.C > 0 && item.nrows > 0 && item.row0 >= 0 &&
+                         item.off + n <= a.total_elems && bytes <= a.stage_bytes &&
+                         (bytes & 15) == 0 && ((item.off * E::kSize) & 15) == 0;
+                }
+                if (!ok) {
+                    atomicOr(a.status, BSM_DEV_BOUNDS);
+                    mt.kind = KIND_SKIP;
+                    mbar_arrive(&h.full[s]);
+                    continue;
+                }
+                mt.off = item.off;
+                mt.C = item.C;
+                mt.nrows = item.nrows;
+                mt.row0 = item.row0;
+                mt.kind = KIND_DATA;
+                const uint32_t bytes = static_cast<uint32_t>((int64_t)item.nrows * item.C * E::kSize);
+                mbar_arrive_expect_tx(&h.full[s], bytes);
+                bulk_load(stages + (size_t)s * a.stage_bytes,
+                          static_cast<const unsigned char *>(a.x) + item.off * E::kSize, bytes,
+                          &h.full[s]);
+                issued[s] = true;
+                issued_phase[s] = ph;
+            }
+            if (aborted) {
+                atomicOr(a.status, BSM_DEV_TIMEOUT);
+                h.abort_flag = 1;
+                // let every copy still in flight land before the CTA exits
+                for (int s = 0; s < S; ++s)
+                    if (issued[s])
+                        mbar_wait_bounded(&h.full[s], issued_phase[s], nullptr);
+            }
+            if (a.mode == PULL_QUEUE) {
+                // the last CTA to finish pulling rewinds the queue heads
+                __threadfence();
+                const uint32_t prev = atomicAdd(&a.heads[BSM_MAX_DIES], 1u);
+                if (prev == gridDim.x - 1) {
+                    for (int d = 0; d < BSM_MAX_DIES; ++d)
+                        atomicExch(&a.heads[d], 0u);
+                    atomicExch(&a.heads[BSM_MAX_DIES], 0u);
+                }
+            }
+        }
+        return;
+    }
+
+    // ----------------------------------------------------------- consumers
+    const bool causal = (a.flags & BSM_FLAG_CAUSAL) != 0;
+    unsigned char *y = static_cast<unsigned char *>(a.y);
+    for (uint32_t it = 0;; ++it) {
+        const int s = it % S;
+        const uint32_t ph = (it / S) & 1u;
+        if (!mbar_wait_bounded(&h.full[s], ph, &h.abort_flag)) {
+            if (lane == 0) {
+                atomicOr(a.status, BSM_DEV_TIMEOUT);
+                h.abort_flag = 1;
+            }
+            break;
+        }
+        const StageMeta mt = h.meta[s];
+        if (mt.kind == KIND_DONE)
+            break;
+        if (mt.kind == KIND_DATA)
+            consume_stage<Tag>(stages + (size_t)s * a.stage_bytes, mt, y, causal, warp, lane);
+        __syncwarp();
+        if (lane == 0)
+            mbar_arrive(&h.empty[s]);
+    }
+}
+
+}  // namespace
+
+int kernel_set_smem_limit(int bytes)
+{
+    cudaError_t e = cudaFuncSetAttribute(softmax_persistent<F32>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e != cudaSuccess)
+        return static_cast<int>(e);
+    e = cudaFuncSetAttribute(softmax_persistent<BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             bytes);
+    return static_cast<int>(e);
+}
+
+int launch_softmax(const KernelArgs &a, int dtype, int grid, void *stream)
+{
+    const size_t smem = kSmemHeader + (size_t)a.n_stages * a.stage_bytes;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (dtype == BSM_F32)
+        softmax_persistent<F32><<<grid, kThreads, smem, st>>>(a);
+    else
+        softmax_persistent<BF16><<<grid, kThreads, smem, st>>>(a);
+    return static_cast<int>(cudaGetLastError());
+}
+
+}  // namespace bsm

@@ -1,0 +1,118 @@
+// bsm_probe.cu -- latency probes behind the topology (Sec. 2.1: a compute
+// unit reaches its nearest memory bank fastest; the latency to a farther bank
+// grows with the hops in between).
+//
+// On GB300 each die owns half of the L2 and of the HBM stacks; an SM reading
+// a line homed on the other die crosses the die-to-die link.  Both kernels
+// time chains of dependent L2-only loads (ld.global.cg, the loaded value -- 0
+// -- feeds the next address) from one lane per SM, so the figure is the
+// round-trip latency of an L2 hit from that SM to that line's home slice.
+// Every loop has a fixed trip count; every address is checked against the
+// buffer on the host before launch.
+
+#include <cuda_runtime.h>
+#include <cstdint>
+
+#include "bsm_internal.h"
+
+namespace bsm {
+namespace {
+
+__device__ __forceinline__ uint32_t probe_smid()
+{
+    uint32_t s;
+    asm volatile("mov.u32 %0, %%smid;" : "=r"(s));
+    return s;
+}
+
+__device__ __forceinline__ uint32_t ld_l2(const uint32_t *p)
+{
+    uint32_t v;
+    asm volatile("ld.global.cg.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ long long clk()
+{
+    long long t;
+    asm volatile("mov.u64 %0, %%clock64;" : "=l"(t));
+    return t;
+}
+
+// Mean cycles of `reps` dependent L2-hit loads of the line at p.
+__device__ __forceinline__ float time_line(const unsigned char *p, int reps)
+{
+    const uint32_t *q = reinterpret_cast<const uint32_t *>(p);
+    uint32_t v = ld_l2(q);          // brings the line into L2
+    v = ld_l2(q + v);
+    const long long t0 = clk();
+    for (int r = 0; r < reps; ++r)
+        v = ld_l2(q + v);
+    asm volatile("add.u32 %0, %0, 0;" : "+r"(v));   // issue waits for the last load
+    const long long t1 = clk();
+    return static_cast<float>(t1 - t0) / reps + (v == 0xFFFFFFFFu ? 1.0f : 0.0f);
+}
+
+// One CTA of 32 threads per SM does the work: the first CTA that lands on an
+// SM claims it; the others return at once.
+__global__ void probe_latency_kernel(const unsigned char *buf, const int64_t *line_off, int n_lines,
+                                     int reps, float *lat, uint32_t *claim)
+{
+    if (threadIdx.x != 0)
+        return;
+    const uint32_t sm = probe_smid() & (BSM_MAX_SM - 1);
+    if (atomicCAS(&claim[sm], 0u, 1u) != 0u)
+        return;
+    for (int k = 0; k < n_lines; ++k) {
+        const int i = static_cast<int>((k + 7ull * sm) % static_cast<unsigned>(n_lines));
+        lat[(size_t)sm * n_lines + i] = time_line(buf + line_off[i], reps);
+    }
+}
+
+// Die of every `chunk`-byte chunk: an SM of known die times the chunk's
+// first line; below the threshold the line is near (same die), else far.
+__global__ void probe_map_kernel(const unsigned char *buf, int64_t n_chunks, int64_t chunk, int reps,
+                                 const int8_t *sm_die, float threshold, uint32_t *counter,
+                                 int8_t *die_out)
+{
+    if (threadIdx.x != 0)
+        return;
+    const int my = sm_die[probe_smid() & (BSM_MAX_SM - 1)];
+    if (my < 0 || my > 1)
+        return;
+    for (int64_t guard = 0; guard < n_chunks; ++guard) {
+        const uint32_t c = atomicAdd(counter, 1u);
+        if (c >= n_chunks)
+            break;
+        const float t = time_line(buf + (int64_t)c * chunk, reps);
+        die_out[c] = static_cast<int8_t>(t < threshold ? my : 1 - my);
+    }
+}
+
+}  // namespace
+
+int probe_latency_run(const void *buf, const int64_t *line_off_dev, int n_lines, int reps, int grid,
+                      float *lat_dev, uint32_t *claim_dev)
+{
+    probe_latency_kernel<<<grid, 32>>>(static_cast<const unsigned char *>(buf), line_off_dev, n_lines,
+                                       reps, lat_dev, claim_dev);
+    cudaError_t e = cudaGetLastError();
+    if (e == cudaSuccess)
+        e = cudaDeviceSynchronize();
+    return static_cast<int>(e);
+}
+
+int probe_map_run(const void *buf, int64_t bytes, int64_t chunk, int reps, const int8_t *sm_die_dev,
+                  float threshold, int n_sm, uint32_t *counter_dev, int8_t *die_dev)
+{
+    const int64_t n_chunks = (bytes + chunk - 1) / chunk;
+    // the chunk's first line must lie inside the buffer: (n_chunks-1)*chunk < bytes
+    probe_map_kernel<<<n_sm, 32>>>(static_cast<const unsigned char *>(buf), n_chunks, chunk, reps,
+                                   sm_die_dev, threshold, counter_dev, die_dev);
+    cudaError_t e = cudaGetLastError();
+    if (e == cudaSuccess)
+        e = cudaDeviceSynchronize();
+    return static_cast<int>(e);
+}
+
+}  // namespace bsm

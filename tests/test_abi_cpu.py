@@ -1,0 +1,75 @@
+"""The C-ABI library on a machine without a GPU: it loads, it exports every
+function include/bsm.h declares, argument errors come back as status codes
+before any CUDA call, and the host-side scheduler matches the oracle."""
+import ctypes
+import subprocess
+
+import numpy as np
+import pytest
+
+from paper_2002_07062_gb300 import bsm
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    import __graft_entry__ as g
+    g.build()
+
+
+def test_library_exports_every_header_function():
+    names = bsm.header_functions()
+    assert len(names) >= 15
+    out = subprocess.run(["nm", "-D", "--defined-only", bsm.LIB_PATH], capture_output=True,
+                         text=True, check=True).stdout
+    exported = {line.split()[-1] for line in out.splitlines() if line.strip()}
+    missing = [n for n in names if n not in exported]
+    assert not missing, missing
+    for n in names:
+        assert hasattr(bsm.lib(), n)
+
+
+def test_status_strings_and_version():
+    assert bsm.status_string(0) == "ok"
+    for s in range(1, 9):
+        assert bsm.status_string(s) not in ("ok", "unknown status")
+    assert bsm.status_string(99) == "unknown status"
+    assert bsm.bsm_version() >> 16 == 1
+
+
+@pytest.mark.parametrize("args,code", [
+    ((0, 0, -1, 4, 4, bsm.F32, bsm.POLICY_RR), bsm.ERR_INVALID_ARG),   # B < 0
+    ((0, 0, 1, -4, 4, bsm.F32, bsm.POLICY_RR), bsm.ERR_INVALID_ARG),   # R < 0
+    ((0, 0, 1, 4, 0, bsm.F32, bsm.POLICY_RR), bsm.ERR_INVALID_ARG),    # C < 1
+    ((0, 0, 1, 4, 4, 7, bsm.POLICY_RR), bsm.ERR_INVALID_ARG),          # dtype
+    ((0, 0, 1, 4, 4, bsm.F32, 9), bsm.ERR_INVALID_ARG),                # policy
+])
+def test_argument_errors_without_gpu(args, code):
+    rc = bsm.lib().bsm_softmax(*args, None)
+    assert rc == code
+
+
+def test_empty_batch_is_a_no_op():
+    assert bsm.lib().bsm_softmax(None, None, 0, 5, 4, bsm.F32, bsm.POLICY_RR, None) == bsm.OK
+    assert bsm.lib().bsm_softmax(None, None, 3, 0, 4, bsm.F32, bsm.POLICY_RR, None) == bsm.OK
+    assert bsm.lib().bsm_softmax_ragged(None, None, 0, None, None, None, bsm.F32,
+                                        bsm.POLICY_RR, 0, None) == bsm.OK
+
+
+def test_bad_flags_and_null_tables_rejected():
+    assert bsm.lib().bsm_softmax_ex(0, 0, 1, 4, 4, bsm.F32, bsm.POLICY_RR, 2, None) == \
+        bsm.ERR_INVALID_ARG
+    assert bsm.lib().bsm_softmax_ragged(0, 0, 3, None, None, None, bsm.F32, bsm.POLICY_RR, 0,
+                                        None) == bsm.ERR_INVALID_ARG
+    assert bsm.lib().bsm_plan_create(None, None) == bsm.ERR_INVALID_ARG
+    d = bsm.PlanDesc()
+    assert bsm.lib().bsm_plan_desc_init(ctypes.byref(d)) == bsm.OK
+    assert d.tie_seed == 0x2002070600 and d.lb_weighted == 1 and d.device == -1
+
+
+def test_schedule_host_rejects_bad_maps():
+    with pytest.raises(bsm.BsmError):
+        bsm.bsm_schedule_host([(0, 512)], [(256, [0, 5])], 2, 0)      # bank 5 of 2
+    with pytest.raises(bsm.BsmError):
+        bsm.bsm_schedule_host([(0, 1024)], [(256, [0, 1])], 2, 0)     # past the map
+    with pytest.raises(bsm.BsmError):
+        bsm.bsm_schedule_host([(0, 512)], [(256, [0, 1])], 2, 0, balance=True, units=[0, 1])

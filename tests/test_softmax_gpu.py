@@ -1,0 +1,208 @@
+"""GPU parity of the batched softmax (through the C ABI) against the
+double-precision oracle, under every scheduling policy.
+
+fp32 output: max |y - oracle| <= 2e-6.  bf16 output: within 1 bf16 ulp of
+the oracle's round-to-nearest-even result.  Every policy must give the same
+bits (one row routine, fixed reduction order), every row must be written,
+and nothing outside y may be touched."""
+import numpy as np
+import pytest
+
+from gpu_util import (bits, check_all_against_oracle, check_rows_against_oracle, run,
+                      sample_rows, to_device, to_host)
+from paper_2002_07062_gb300 import bsm, workload
+
+pytestmark = pytest.mark.gpu
+
+ALL = [bsm.POLICY_WHOLE_GPU, bsm.POLICY_RR, bsm.POLICY_DYNAMIC, bsm.POLICY_CBMF,
+       bsm.POLICY_CBMF_LB]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def setup():
+    import torch
+    import __graft_entry__ as g
+    g.build()
+    torch.cuda.set_device(0)
+    bsm.bsm_device_status_clear()
+    yield
+    bsm.bsm_cache_clear()
+
+
+def _all_policies_identical(w, x, policies=ALL):
+    import torch
+    ys = [run(w, x, p) for p in policies]
+    torch.cuda.synchronize()
+    for p, y in zip(policies[1:], ys[1:]):
+        assert torch.equal(bits(y), bits(ys[0])), "policy %d differs from %d" % (p, policies[0])
+    return ys[0]
+
+
+def _ragged_all_classes(dtype, flags, seed, nslices=24):
+    # C from one 16-byte vector to 2.5x the register-resident limit; R 1..60
+    unit = 4 if dtype == workload.F32 else 8
+    return workload.ragged("classes", dtype, nslices, 2.0, seed, flags, row_unit=1,
+                           row_steps=60, col_unit=unit, col_steps=160).materialize()
+
+
+@pytest.mark.parametrize("dtype", [workload.F32, workload.BF16])
+@pytest.mark.parametrize("flags", [0, bsm.FLAG_CAUSAL])
+def test_ragged_every_row_routine_full_parity(dtype, flags):
+    w = _ragged_all_classes(dtype, flags, 100 + 2 * dtype + flags)
+    x = to_device(w.x)
+    y = _all_policies_identical(w, x)
+    check_all_against_oracle(w, to_host(y))
+    assert bsm.bsm_device_status() == 0
+
+
+def test_workload1_full_parity():
+    w = workload.config(1).materialize()
+    x = to_device(w.x)
+    y = _all_policies_identical(w, x)
+    check_all_against_oracle(w, to_host(y))
+
+
+@pytest.mark.parametrize("k", [2, 3, 5])
+def test_uniform_workloads_full_size(k):
+    import torch
+    w = workload.config(k).materialize()
+    x = to_device(w.x)
+    y = _all_policies_identical(w, x)
+    yh = to_host(y)
+    check_rows_against_oracle(w, yh, sample_rows(w, 1500, 7 + k))
+    R, C = int(w.rows[0]), int(w.cols[0])
+    yd = y.view(-1, C).double()
+    assert not torch.isnan(yd).any()                     # every row written
+    s = yd.sum(dim=1)
+    tol = C * 2.0 ** -24 * 4 if w.dtype == workload.F32 else 0.01
+    assert float((s - 1).abs().max()) <= tol
+    if w.flags & bsm.FLAG_CAUSAL:
+        y3 = y.view(w.nslices, R, C)
+        upper = torch.triu(torch.ones(R, C, dtype=torch.bool, device=y.device), diagonal=1)
+        assert int((y3[:, upper] != 0).sum()) == 0        # masked entries exactly 0
+        assert bool((y3[:, 0, 0] == 1).all())             # row 0 one-hot
+    assert bsm.bsm_device_status() == 0
+
+
+def test_ragged_workload4_full_size():
+    import torch
+    w = workload.config(4).materialize()
+    x = to_device(w.x)
+    y = _all_policies_identical(w, x, [bsm.POLICY_RR, bsm.POLICY_DYNAMIC, bsm.POLICY_CBMF,
+                                       bsm.POLICY_CBMF_LB, bsm.POLICY_WHOLE_GPU])
+    yh = to_host(y)
+    check_rows_against_oracle(w, yh, sample_rows(w, 3000, 44))
+    assert not torch.isnan(y).any()
+    for s in range(0, w.nslices, 37):
+        R, C = int(w.rows[s]), int(w.cols[s])
+        a = int(w.offsets[s])
+        ss = y[a:a + R * C].view(R, C).double().sum(dim=1)
+        assert float((ss - 1).abs().max()) <= C * 2.0 ** -24 * 4
+    assert bsm.bsm_device_status() == 0
+
+
+def test_guard_bands_untouched_and_in_place():
+    import torch
+    w = _ragged_all_classes(workload.F32, 0, 9, nslices=10)
+    x = to_device(w.x)
+    pad = 4096
+    big = torch.full((w.numel + 2 * pad,), 1234.5, dtype=torch.float32, device="cuda")
+    y = big[pad:pad + w.numel]
+    run(w, x, bsm.POLICY_DYNAMIC, y=y)
+    torch.cuda.synchronize()
+    assert bool((big[:pad] == 1234.5).all()) and bool((big[pad + w.numel:] == 1234.5).all())
+    ref = to_host(y)
+    check_all_against_oracle(w, ref)
+    # in place: x == y gives the same bits
+    xi = x.clone()
+    run(w, xi, bsm.POLICY_CBMF_LB, y=xi)
+    torch.cuda.synchronize()
+    assert np.array_equal(to_host(xi).view(np.uint32), ref.view(np.uint32))
+
+
+@pytest.mark.parametrize("dtype", [workload.F32, workload.BF16])
+def test_longest_row_and_single_row(dtype):
+    es = 4 if dtype == workload.F32 else 2
+    cmax = bsm.bsm_max_row_bytes() // es
+    for R, C in [(3, cmax), (1, 16 // es), (1, cmax), (2, 16 // es * 3)]:
+        w = workload.uniform("edge", dtype, 2, R, C, 3.0, 77 + C).materialize()
+        x = to_device(w.x)
+        y = _all_policies_identical(w, x)
+        check_all_against_oracle(w, to_host(y))
+
+
+def test_non_finite_rows_match_oracle():
+    C = 64
+    rows = []
+    rng = np.random.default_rng(1)
+    for kind in range(6):
+        r = rng.normal(0, 2, C).astype(np.float32)
+        if kind == 1:
+            r[5] = np.nan
+        elif kind == 2:
+            r[9] = np.inf
+        elif kind == 3:
+            r[:] = -np.inf
+        elif kind == 4:
+            r[:] = -np.inf
+            r[3] = 1.0
+        elif kind == 5:
+            r[:] = -np.inf
+            r[3] = r[40] = 2.0
+        rows.append(r)
+    xs = np.stack(rows).reshape(-1)
+    w = workload.uniform("nonfinite", workload.F32, 1, len(rows), C, 1.0, 0)
+    w.x = xs
+    x = to_device(xs)
+    y = _all_policies_identical(w, x)
+    yh = to_host(y).reshape(-1, C)
+    assert np.isnan(yh[1]).all() and np.isnan(yh[2]).all() and np.isnan(yh[3]).all()
+    assert yh[4, 3] == 1.0 and np.count_nonzero(yh[4]) == 1
+    assert yh[5, 3] == 0.5 and yh[5, 40] == 0.5 and np.count_nonzero(yh[5]) == 2
+    check_all_against_oracle(w, to_host(y))
+
+
+def test_argument_errors_on_device():
+    import torch
+    x = torch.zeros(4 * 64 + 8, device="cuda")
+    y = torch.zeros_like(x)
+    with pytest.raises(bsm.BsmError) as e:
+        bsm.bsm_softmax(x.data_ptr() + 4, y, 4, 1, 64, bsm.F32, bsm.POLICY_RR)
+    assert e.value.status == bsm.ERR_MISALIGNED
+    with pytest.raises(bsm.BsmError) as e:
+        bsm.bsm_softmax(x, y, 1, 1, 6, bsm.F32, bsm.POLICY_RR)          # 24-byte rows
+    assert e.value.status == bsm.ERR_MISALIGNED
+    with pytest.raises(bsm.BsmError) as e:
+        bsm.bsm_softmax(x, x.data_ptr() + 16, 4, 1, 64, bsm.F32, bsm.POLICY_RR)
+    assert e.value.status == bsm.ERR_INVALID_ARG                        # partial overlap
+    big = bsm.bsm_max_row_bytes() // 4 + 4
+    xb = torch.zeros(big, device="cuda")
+    with pytest.raises(bsm.BsmError) as e:
+        bsm.bsm_softmax(xb, xb, 1, 1, big, bsm.F32, bsm.POLICY_RR)
+    assert e.value.status == bsm.ERR_UNSUPPORTED
+    with pytest.raises(bsm.BsmError) as e:                              # overlapping slices
+        bsm.bsm_softmax_ragged(x, y, [0, 32], [1, 1], [64, 64], bsm.F32, bsm.POLICY_RR)
+    assert e.value.status == bsm.ERR_INVALID_ARG
+    assert bsm.bsm_device_status() == 0
+
+
+def test_topology_and_plan_stats():
+    import torch
+    t = bsm.bsm_topology_probe()
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    assert t["n_sm"] == n_sm
+    seen = [d for d in t["sm_die"] if d >= 0]
+    assert len(seen) >= n_sm * 0.9
+    assert t["l_near"] > 0 and t["l_far"] >= t["l_near"]
+    assert sum(t["sm_per_die"]) == len(seen)
+    w = workload.config(2)
+    x = torch.empty(w.numel, device="cuda")
+    y = torch.empty_like(x)
+    for pol in (bsm.POLICY_CBMF, bsm.POLICY_CBMF_LB):
+        p = bsm.bsm_plan_create(x, y, w.rows, w.cols, w.dtype, pol)
+        st = p.stats()
+        n = st["n_items"]
+        assert sum(st["L"][:st["n_die"]]) == n                         # sum L = N
+        assert sum(st["N"][:st["n_die"]]) >= n                         # sum N >= N
+        assert sum(st["queue_items"][:st["n_die"]]) == n
+        p.close()
