@@ -91,6 +91,7 @@ typedef enum {
 /* Device-side status bits (bsm_device_status). */
 #define BSM_DEV_BOUNDS 1u      /* a patch fell outside the buffers or a stage; skipped */
 #define BSM_DEV_TIMEOUT 2u     /* a pipeline wait ran out of time; the CTA gave up */
+#define BSM_DEV_CHECK 4u       /* the checking kernel caught an out-of-range access; skipped */
 
 /*
  * Softmax over B slices of R x C stored back to back, i.e. a (B*R) x C
@@ -265,6 +266,24 @@ int bsm_schedule_host(const bsm_schedule_desc *d, bsm_schedule_out *out);
  * Synchronises the device.  bsm_device_status_clear zeroes it. */
 int bsm_device_status(int device, uint32_t *status_out);
 int bsm_device_status_clear(int device);
+
+/* The 8-word device status block of `device` (-1 = current): word 0 is the
+ * sticky BSM_DEV_* bits; when BSM_DEV_CHECK is set, words 1..7 describe the
+ * first caught access (1 = kind: 1 shared read, 2 global store, 3 bulk copy,
+ * 4 stage geometry; 2 = block; 3 = thread; 4..5 = offset, 6..7 = extent).
+ * Synchronises the device. */
+int bsm_device_debug(int device, uint32_t out[8]);
+
+/* Select the self-checking kernel instantiation (on != 0) for launches made
+ * after this call, in every thread: every shared-memory read, global store
+ * and bulk copy is checked against its stage or buffer and skipped (and
+ * recorded, see bsm_device_debug) when out of range.  Slower; for diagnosis. */
+void bsm_set_device_checks(int on);
+
+/* Name and description of the last CUDA runtime error a bsm call saw in this
+ * thread ("" if none).  The string stays valid until the next bsm call in
+ * the same thread. */
+const char *bsm_last_cuda_error(void);
 
 /* Largest row (C * element size) a plan accepts on this device, bytes. */
 int64_t bsm_max_row_bytes(int device);

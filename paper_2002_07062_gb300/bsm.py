@@ -27,7 +27,7 @@ POLICY_NAMES = {v: k for k, v in POLICIES.items()}
 FLAG_CAUSAL = 1
 MAX_DIES = 4
 MAX_SM = 256
-DEV_BOUNDS, DEV_TIMEOUT = 1, 2
+DEV_BOUNDS, DEV_TIMEOUT, DEV_CHECK = 1, 2, 4
 
 (OK, ERR_INVALID_ARG, ERR_MISALIGNED, ERR_UNSUPPORTED, ERR_CUDA, ERR_DEVICE_BOUNDS,
  ERR_TIMEOUT, ERR_NO_DEVICE, ERR_NOMEM) = range(9)
@@ -39,7 +39,10 @@ c_i32p = ctypes.POINTER(ctypes.c_int32)
 class BsmError(RuntimeError):
     def __init__(self, status: int, where: str):
         self.status = status
-        super().__init__("%s: %s (status %d)" % (where, status_string(status), status))
+        msg = "%s: %s (status %d)" % (where, status_string(status), status)
+        if status == ERR_CUDA:
+            msg += " [%s]" % bsm_last_cuda_error()
+        super().__init__(msg)
 
 
 class PlanDesc(ctypes.Structure):
@@ -122,6 +125,9 @@ def lib():
         "bsm_max_row_bytes": ([ctypes.c_int], i64),
         "bsm_status_string": ([ctypes.c_int], ctypes.c_char_p),
         "bsm_version": ([], ctypes.c_int),
+        "bsm_device_debug": ([ctypes.c_int, ctypes.POINTER(ctypes.c_uint32)], ctypes.c_int),
+        "bsm_set_device_checks": ([ctypes.c_int], None),
+        "bsm_last_cuda_error": ([], ctypes.c_char_p),
     }
     for name, (args, res) in sig.items():
         f = getattr(L, name)
@@ -367,6 +373,20 @@ def bsm_device_status(device: int = -1) -> int:
 
 def bsm_device_status_clear(device: int = -1):
     _check(lib().bsm_device_status_clear(device), "bsm_device_status_clear")
+
+
+def bsm_device_debug(device: int = -1) -> list:
+    out = (ctypes.c_uint32 * 8)()
+    _check(lib().bsm_device_debug(device, out), "bsm_device_debug")
+    return list(out)
+
+
+def bsm_set_device_checks(on: bool):
+    lib().bsm_set_device_checks(1 if on else 0)
+
+
+def bsm_last_cuda_error() -> str:
+    return lib().bsm_last_cuda_error().decode()
 
 
 def bsm_max_row_bytes(device: int = -1) -> int:

@@ -6,6 +6,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <chrono>
 #include <cmath>
 #include <cstring>
@@ -13,11 +14,23 @@
 #include <mutex>
 #include <new>
 #include <numeric>
+#include <string>
 #include <vector>
 
 #include "bsm_internal.h"
 
 namespace bsm {
+
+namespace {
+thread_local std::string t_last_error;
+}
+
+int record_cuda_error(int cuda_error, const char *where)
+{
+    const cudaError_t e = static_cast<cudaError_t>(cuda_error);
+    t_last_error = std::string(where) + ": " + cudaGetErrorName(e) + " (" + cudaGetErrorString(e) + ")";
+    return BSM_ERR_CUDA;
+}
 
 int topology_get(int device, int force, bsm_topology *out);
 int addr_die_map_host(int device, const void *ptr, int64_t bytes, int64_t chunk, int8_t *die_out);
@@ -39,6 +52,9 @@ struct DeviceCtx {
 
 std::mutex g_mu;
 DeviceCtx g_dev[kMaxDevices];
+std::atomic<int> g_checked{0};
+
+int cuda_error(cudaError_t e, const char *where) { return record_cuda_error(static_cast<int>(e), where); }
 
 int device_ctx(int device, DeviceCtx **out)
 {
@@ -60,14 +76,15 @@ int device_ctx(int device, DeviceCtx **out)
             cudaDeviceGetAttribute(&c.smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, device) !=
                 cudaSuccess)
             rc = BSM_ERR_NO_DEVICE;
-        if (!rc && kernel_set_smem_limit(c.smem_optin) != 0)
-            rc = BSM_ERR_CUDA;
-        if (!rc && cudaMalloc(&c.status, 256) != cudaSuccess)
-            rc = BSM_ERR_NOMEM;
-        if (!rc && cudaMemset(c.status, 0, 256) != cudaSuccess)
-            rc = BSM_ERR_CUDA;
-        if (!rc && cudaDeviceSynchronize() != cudaSuccess)
-            rc = BSM_ERR_CUDA;
+        cudaError_t e = cudaSuccess;
+        if (!rc && (e = static_cast<cudaError_t>(kernel_set_smem_limit(c.smem_optin))) != cudaSuccess)
+            rc = cuda_error(e, "cudaFuncSetAttribute");
+        if (!rc && (e = cudaMalloc(&c.status, 256)) != cudaSuccess)
+            rc = cuda_error(e, "cudaMalloc(status)");
+        if (!rc && (e = cudaMemset(c.status, 0, 256)) != cudaSuccess)
+            rc = cuda_error(e, "cudaMemset(status)");
+        if (!rc && (e = cudaDeviceSynchronize()) != cudaSuccess)
+            rc = cuda_error(e, "cudaDeviceSynchronize");
         if (prev >= 0 && prev != device)
             cudaSetDevice(prev);
         if (rc) {
@@ -422,12 +439,12 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
         delete p;
         return BSM_ERR_NOMEM;
     }
-    if (cudaMemcpy(p->blob, host.data(), blob_b, cudaMemcpyHostToDevice) != cudaSuccess) {
+    if (cudaError_t e = cudaMemcpy(p->blob, host.data(), blob_b, cudaMemcpyHostToDevice)) {
         cudaFree(p->blob);
         if (prev >= 0)
             cudaSetDevice(prev);
         delete p;
-        return BSM_ERR_CUDA;
+        return cuda_error(e, "cudaMemcpy(plan tables)");
     }
     if (prev >= 0)
         cudaSetDevice(prev);
@@ -494,20 +511,21 @@ int plan_execute_impl(const bsm_plan *p, bsm_stream_t stream)
     if (prev != p->device && cudaSetDevice(p->device) != cudaSuccess)
         return BSM_ERR_NO_DEVICE;
     int err = 0;
+    const bool checked = g_checked.load(std::memory_order_relaxed) != 0;
     if (p->policy == BSM_POLICY_WHOLE_GPU) {
         KernelArgs a = p->args;
         for (const auto &l : p->whole_gpu) {
             a.item_begin = l.begin;
             a.item_end = l.end;
-            if ((err = launch_softmax(a, p->dtype, l.grid, stream)))
+            if ((err = launch_softmax(a, p->dtype, l.grid, stream, checked)))
                 break;
         }
     } else {
-        err = launch_softmax(p->args, p->dtype, p->grid, stream);
+        err = launch_softmax(p->args, p->dtype, p->grid, stream, checked);
     }
     if (prev >= 0 && prev != p->device)
         cudaSetDevice(prev);
-    return err ? BSM_ERR_CUDA : BSM_OK;
+    return err ? cuda_error(static_cast<cudaError_t>(err), "kernel launch") : BSM_OK;
 }
 
 // ---- plan cache of the one-call entry points
@@ -765,10 +783,10 @@ int bsm_device_status(int device, uint32_t *status_out)
     int rc = device_ctx(device, &c);
     if (rc)
         return rc;
-    if (cudaDeviceSynchronize() != cudaSuccess)
-        return BSM_ERR_CUDA;
-    if (cudaMemcpy(status_out, c->status, sizeof(uint32_t), cudaMemcpyDeviceToHost) != cudaSuccess)
-        return BSM_ERR_CUDA;
+    if (cudaError_t e = cudaDeviceSynchronize())
+        return cuda_error(e, "cudaDeviceSynchronize");
+    if (cudaError_t e = cudaMemcpy(status_out, c->status, sizeof(uint32_t), cudaMemcpyDeviceToHost))
+        return cuda_error(e, "cudaMemcpy(status)");
     return BSM_OK;
 }
 
@@ -778,10 +796,31 @@ int bsm_device_status_clear(int device)
     int rc = device_ctx(device, &c);
     if (rc)
         return rc;
-    if (cudaMemset(c->status, 0, sizeof(uint32_t)) != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess)
-        return BSM_ERR_CUDA;
+    if (cudaError_t e = cudaMemset(c->status, 0, 8 * sizeof(uint32_t)))
+        return cuda_error(e, "cudaMemset(status)");
+    if (cudaError_t e = cudaDeviceSynchronize())
+        return cuda_error(e, "cudaDeviceSynchronize");
     return BSM_OK;
 }
+
+int bsm_device_debug(int device, uint32_t out[8])
+{
+    if (!out)
+        return BSM_ERR_INVALID_ARG;
+    DeviceCtx *c = nullptr;
+    int rc = device_ctx(device, &c);
+    if (rc)
+        return rc;
+    if (cudaError_t e = cudaDeviceSynchronize())
+        return cuda_error(e, "cudaDeviceSynchronize");
+    if (cudaError_t e = cudaMemcpy(out, c->status, 8 * sizeof(uint32_t), cudaMemcpyDeviceToHost))
+        return cuda_error(e, "cudaMemcpy(status)");
+    return BSM_OK;
+}
+
+void bsm_set_device_checks(int on) { g_checked.store(on ? 1 : 0); }
+
+const char *bsm_last_cuda_error(void) { return t_last_error.c_str(); }
 
 int64_t bsm_max_row_bytes(int device)
 {

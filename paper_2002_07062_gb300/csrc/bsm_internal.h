@@ -58,7 +58,7 @@ struct KernelArgs {
 
 // Launch the persistent softmax kernel (bsm_kernels.cu).  Returns a
 // cudaError_t value (0 = success).
-int launch_softmax(const KernelArgs &a, int dtype, int grid, void *stream);
+int launch_softmax(const KernelArgs &a, int dtype, int grid, void *stream, bool checked);
 // Raise the dynamic shared-memory limit of both kernel instances.
 int kernel_set_smem_limit(int bytes);
 
@@ -67,6 +67,10 @@ int probe_latency_run(const void *buf, const int64_t *line_off_dev, int n_lines,
                       int grid, float *lat_dev, uint32_t *claim_dev);
 int probe_map_run(const void *buf, int64_t bytes, int64_t chunk, int reps, const int8_t *sm_die_dev,
                   float threshold, int n_sm, uint32_t *counter_dev, int8_t *die_dev);
+
+// Remember a failing CUDA call for bsm_last_cuda_error (bsm_api.cpp);
+// returns BSM_ERR_CUDA.
+int record_cuda_error(int cuda_error, const char *where);
 
 // Host planner (bsm_planner.cpp).
 int schedule_host(const bsm_schedule_desc *d, bsm_schedule_out *out);

@@ -158,6 +158,52 @@ __device__ __forceinline__ void stg128(void *p, uint4 v)
     *reinterpret_cast<uint4 *>(p) = v;
 }
 
+// ---------------------------------------------------------- self-checks
+// The checking instantiation (Checked = true) verifies every shared-memory
+// read, global store and bulk copy against the stage and buffer extents; a
+// violation is recorded (BSM_DEV_CHECK, plus the first one's details in words
+// 1..7 of the status block) and the access is skipped.
+
+struct Bounds {
+    const unsigned char *s_lo, *s_hi;   // bytes of the current stage that hold the patch
+    const unsigned char *y_lo, *y_hi;   // the output buffer
+    uint32_t *status;
+};
+
+__device__ __noinline__ void check_fail(uint32_t *status, uint32_t kind, uint64_t a, uint64_t b)
+{
+    atomicOr(status, BSM_DEV_CHECK);
+    if (atomicCAS(&status[1], 0u, kind) == 0u) {
+        status[2] = blockIdx.x;
+        status[3] = threadIdx.x;
+        status[4] = static_cast<uint32_t>(a);
+        status[5] = static_cast<uint32_t>(a >> 32);
+        status[6] = static_cast<uint32_t>(b);
+        status[7] = static_cast<uint32_t>(b >> 32);
+    }
+}
+
+template <bool Checked>
+__device__ __forceinline__ bool load_vec(const unsigned char *p, const Bounds &b, uint4 &out)
+{
+    if (Checked && (p < b.s_lo || p + 16 > b.s_hi || (reinterpret_cast<uintptr_t>(p) & 15))) {
+        check_fail(b.status, 1, static_cast<uint64_t>(p - b.s_lo), static_cast<uint64_t>(b.s_hi - b.s_lo));
+        return false;
+    }
+    out = lds128(p);
+    return true;
+}
+
+template <bool Checked>
+__device__ __forceinline__ void store_vec(unsigned char *p, const Bounds &b, uint4 v)
+{
+    if (Checked && (p < b.y_lo || p + 16 > b.y_hi || (reinterpret_cast<uintptr_t>(p) & 15))) {
+        check_fail(b.status, 2, static_cast<uint64_t>(p - b.y_lo), static_cast<uint64_t>(b.y_hi - b.y_lo));
+        return;
+    }
+    stg128(p, v);
+}
+
 __device__ __forceinline__ float ex2(float a)
 {
     float r;
@@ -243,9 +289,10 @@ __device__ __forceinline__ void apply_causal(float (&v)[EPV], int col0, int row)
 }
 
 // Register-resident row: T lanes, up to V vectors per lane.
-template <typename Tag, int T, int V>
-__device__ __forceinline__ void row_in_registers(const unsigned char *srow, void *yrow, int nvec,
-                                                 int row, bool causal, int l, bool valid)
+template <typename Tag, bool Checked, int T, int V>
+__device__ __forceinline__ void row_in_registers(const unsigned char *srow, unsigned char *yrow,
+                                                 int nvec, int row, bool causal, int l, bool valid,
+                                                 const Bounds &bd)
 {
     using E = Elem<Tag>;
     constexpr int EPV = E::kPerVec;
@@ -254,8 +301,9 @@ __device__ __forceinline__ void row_in_registers(const unsigned char *srow, void
 #pragma unroll
     for (int j = 0; j < V; ++j) {
         const int vi = j * T + l;
-        if (valid && vi < nvec) {
-            E::unpack(lds128(srow + 16 * vi), v[j]);
+        uint4 raw;
+        if (valid && vi < nvec && load_vec<Checked>(srow + 16 * vi, bd, raw)) {
+            E::unpack(raw, v[j]);
             if (causal)
                 apply_causal<EPV>(v[j], vi * EPV, row);
 #pragma unroll
@@ -290,22 +338,25 @@ __device__ __forceinline__ void row_in_registers(const unsigned char *srow, void
 #pragma unroll
             for (int e = 0; e < EPV; ++e)
                 v[j][e] *= inv;
-            stg128(static_cast<unsigned char *>(yrow) + 16 * vi, E::pack(v[j]));
+            store_vec<Checked>(yrow + 16 * vi, bd, E::pack(v[j]));
         }
     }
 }
 
 // Shared-memory-resident row of any length: one warp, three sweeps.
-template <typename Tag>
-__device__ __forceinline__ void row_in_smem(const unsigned char *srow, void *yrow, int nvec, int row,
-                                            bool causal, int lane)
+template <typename Tag, bool Checked>
+__device__ __forceinline__ void row_in_smem(const unsigned char *srow, unsigned char *yrow, int nvec,
+                                            int row, bool causal, int lane, const Bounds &bd)
 {
     using E = Elem<Tag>;
     constexpr int EPV = E::kPerVec;
     float v[EPV];
+    uint4 raw;
     float m = -INFINITY;
     for (int vi = lane; vi < nvec; vi += 32) {
-        E::unpack(lds128(srow + 16 * vi), v);
+        if (!load_vec<Checked>(srow + 16 * vi, bd, raw))
+            continue;
+        E::unpack(raw, v);
         if (causal)
             apply_causal<EPV>(v, vi * EPV, row);
 #pragma unroll
@@ -316,7 +367,9 @@ __device__ __forceinline__ void row_in_smem(const unsigned char *srow, void *yro
     const float mL = m * kLog2e;
     float s = 0.0f;
     for (int vi = lane; vi < nvec; vi += 32) {
-        E::unpack(lds128(srow + 16 * vi), v);
+        if (!load_vec<Checked>(srow + 16 * vi, bd, raw))
+            continue;
+        E::unpack(raw, v);
         if (causal)
             apply_causal<EPV>(v, vi * EPV, row);
         float ps = 0.0f;
@@ -328,20 +381,23 @@ __device__ __forceinline__ void row_in_smem(const unsigned char *srow, void *yro
     s = group_sum<32>(s);
     const float inv = 1.0f / s;
     for (int vi = lane; vi < nvec; vi += 32) {
-        E::unpack(lds128(srow + 16 * vi), v);
+        if (!load_vec<Checked>(srow + 16 * vi, bd, raw))
+            continue;
+        E::unpack(raw, v);
         if (causal)
             apply_causal<EPV>(v, vi * EPV, row);
 #pragma unroll
         for (int e = 0; e < EPV; ++e)
             v[e] = ex2(fmaf(v[e], kLog2e, -mL)) * inv;
-        stg128(static_cast<unsigned char *>(yrow) + 16 * vi, E::pack(v));
+        store_vec<Checked>(yrow + 16 * vi, bd, E::pack(v));
     }
 }
 
 // All rows of one stage that belong to this consumer warp.
-template <typename Tag>
+template <typename Tag, bool Checked>
 __device__ __forceinline__ void consume_stage(const unsigned char *sbuf, const StageMeta &mt,
-                                              unsigned char *y, bool causal, int warp, int lane)
+                                              unsigned char *y, bool causal, int warp, int lane,
+                                              Bounds bd)
 {
     using E = Elem<Tag>;
     const int C = mt.C;
@@ -349,30 +405,36 @@ __device__ __forceinline__ void consume_stage(const unsigned char *sbuf, const S
     const int row_bytes = C * E::kSize;
     const int nvec = row_bytes >> 4;
     unsigned char *ybase = y + mt.off * E::kSize;
+    bd.s_lo = sbuf;
+    bd.s_hi = sbuf + (size_t)nrows * row_bytes;
     if (nvec <= 16) {
         const int half = lane >> 4, l = lane & 15;
         for (int rb = 2 * warp; rb < nrows; rb += 2 * kConsumerWarps) {
             const int r = rb + half;
             const bool valid = r < nrows;
-            row_in_registers<Tag, 16, 1>(sbuf + (size_t)r * row_bytes, ybase + (size_t)r * row_bytes,
-                                         nvec, mt.row0 + r, causal, l, valid);
+            row_in_registers<Tag, Checked, 16, 1>(sbuf + (size_t)r * row_bytes,
+                                                  ybase + (size_t)r * row_bytes, nvec, mt.row0 + r,
+                                                  causal, l, valid, bd);
         }
     } else if (nvec <= 32) {
         for (int r = warp; r < nrows; r += kConsumerWarps)
-            row_in_registers<Tag, 32, 1>(sbuf + (size_t)r * row_bytes, ybase + (size_t)r * row_bytes,
-                                         nvec, mt.row0 + r, causal, lane, true);
+            row_in_registers<Tag, Checked, 32, 1>(sbuf + (size_t)r * row_bytes,
+                                                  ybase + (size_t)r * row_bytes, nvec, mt.row0 + r,
+                                                  causal, lane, true, bd);
     } else if (nvec <= 64) {
         for (int r = warp; r < nrows; r += kConsumerWarps)
-            row_in_registers<Tag, 32, 2>(sbuf + (size_t)r * row_bytes, ybase + (size_t)r * row_bytes,
-                                         nvec, mt.row0 + r, causal, lane, true);
+            row_in_registers<Tag, Checked, 32, 2>(sbuf + (size_t)r * row_bytes,
+                                                  ybase + (size_t)r * row_bytes, nvec, mt.row0 + r,
+                                                  causal, lane, true, bd);
     } else if (nvec <= 128) {
         for (int r = warp; r < nrows; r += kConsumerWarps)
-            row_in_registers<Tag, 32, 4>(sbuf + (size_t)r * row_bytes, ybase + (size_t)r * row_bytes,
-                                         nvec, mt.row0 + r, causal, lane, true);
+            row_in_registers<Tag, Checked, 32, 4>(sbuf + (size_t)r * row_bytes,
+                                                  ybase + (size_t)r * row_bytes, nvec, mt.row0 + r,
+                                                  causal, lane, true, bd);
     } else {
         for (int r = warp; r < nrows; r += kConsumerWarps)
-            row_in_smem<Tag>(sbuf + (size_t)r * row_bytes, ybase + (size_t)r * row_bytes, nvec,
-                             mt.row0 + r, causal, lane);
+            row_in_smem<Tag, Checked>(sbuf + (size_t)r * row_bytes, ybase + (size_t)r * row_bytes,
+                                      nvec, mt.row0 + r, causal, lane, bd);
     }
 }
 
@@ -427,7 +489,7 @@ struct Puller {
     }
 };
 
-template <typename Tag>
+template <typename Tag, bool Checked>
 __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelArgs a)
 {
     using E = Elem<Tag>;
@@ -493,10 +555,24 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                 mt.row0 = item.row0;
                 mt.kind = KIND_DATA;
                 const uint32_t bytes = static_cast<uint32_t>((int64_t)item.nrows * item.C * E::kSize);
+                unsigned char *dst = stages + (size_t)s * a.stage_bytes;
+                const unsigned char *src = static_cast<const unsigned char *>(a.x) + item.off * E::kSize;
+                if (Checked) {
+                    const unsigned char *x0 = static_cast<const unsigned char *>(a.x);
+                    const bool bad = s < 0 || s >= S || S > kMaxStages ||
+                                     src < x0 || src + bytes > x0 + a.total_elems * E::kSize ||
+                                     (reinterpret_cast<uintptr_t>(src) & 15) ||
+                                     (smem_addr(dst) & 15) || (bytes & 15) || bytes == 0 ||
+                                     dst + bytes > smem + kSmemHeader + (size_t)S * a.stage_bytes;
+                    if (bad) {
+                        check_fail(a.status, 3, static_cast<uint64_t>(idx), bytes);
+                        mt.kind = KIND_SKIP;
+                        mbar_arrive(&h.full[s]);
+                        continue;
+                    }
+                }
                 mbar_arrive_expect_tx(&h.full[s], bytes);
-                bulk_load(stages + (size_t)s * a.stage_bytes,
-                          static_cast<const unsigned char *>(a.x) + item.off * E::kSize, bytes,
-                          &h.full[s]);
+                bulk_load(dst, src, bytes, &h.full[s]);
                 issued[s] = true;
                 issued_phase[s] = ph;
             }
@@ -538,8 +614,17 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
         const StageMeta mt = h.meta[s];
         if (mt.kind == KIND_DONE)
             break;
-        if (mt.kind == KIND_DATA)
-            consume_stage<Tag>(stages + (size_t)s * a.stage_bytes, mt, y, causal, warp, lane);
+        if (mt.kind == KIND_DATA) {
+            Bounds bd{nullptr, nullptr, y, y + a.total_elems * E::kSize, a.status};
+            if (Checked && (mt.nrows <= 0 || mt.C <= 0 ||
+                            (int64_t)mt.nrows * mt.C * E::kSize > a.stage_bytes)) {
+                if (lane == 0)
+                    check_fail(a.status, 4, static_cast<uint64_t>(mt.nrows), static_cast<uint64_t>(mt.C));
+            } else {
+                consume_stage<Tag, Checked>(stages + (size_t)s * a.stage_bytes, mt, y, causal, warp,
+                                            lane, bd);
+            }
+        }
         __syncwarp();
         if (lane == 0)
             mbar_arrive(&h.empty[s]);
@@ -550,23 +635,33 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
 
 int kernel_set_smem_limit(int bytes)
 {
-    cudaError_t e = cudaFuncSetAttribute(softmax_persistent<F32>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-    if (e != cudaSuccess)
-        return static_cast<int>(e);
-    e = cudaFuncSetAttribute(softmax_persistent<BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             bytes);
-    return static_cast<int>(e);
+    const void *fns[] = {reinterpret_cast<const void *>(softmax_persistent<F32, false>),
+                         reinterpret_cast<const void *>(softmax_persistent<BF16, false>),
+                         reinterpret_cast<const void *>(softmax_persistent<F32, true>),
+                         reinterpret_cast<const void *>(softmax_persistent<BF16, true>)};
+    for (const void *f : fns) {
+        cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+        if (e != cudaSuccess)
+            return static_cast<int>(e);
+    }
+    return 0;
 }
 
-int launch_softmax(const KernelArgs &a, int dtype, int grid, void *stream)
+int launch_softmax(const KernelArgs &a, int dtype, int grid, void *stream, bool checked)
 {
     const size_t smem = kSmemHeader + (size_t)a.n_stages * a.stage_bytes;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    if (dtype == BSM_F32)
-        softmax_persistent<F32><<<grid, kThreads, smem, st>>>(a);
-    else
-        softmax_persistent<BF16><<<grid, kThreads, smem, st>>>(a);
+    if (dtype == BSM_F32) {
+        if (checked)
+            softmax_persistent<F32, true><<<grid, kThreads, smem, st>>>(a);
+        else
+            softmax_persistent<F32, false><<<grid, kThreads, smem, st>>>(a);
+    } else {
+        if (checked)
+            softmax_persistent<BF16, true><<<grid, kThreads, smem, st>>>(a);
+        else
+            softmax_persistent<BF16, false><<<grid, kThreads, smem, st>>>(a);
+    }
     return static_cast<int>(cudaGetLastError());
 }
 

@@ -4,9 +4,10 @@
 //
 // On GB300 each die owns half of the L2 and of the HBM stacks; an SM reading
 // a line homed on the other die crosses the die-to-die link.  Both kernels
-// time chains of dependent L2-only loads (ld.global.cg, the loaded value -- 0
-// -- feeds the next address) from one lane per SM, so the figure is the
-// round-trip latency of an L2 hit from that SM to that line's home slice.
+// time chains of dependent L2-only loads (ld.global.cg; each address waits
+// for the previous load through an "and 0", so it never depends on the data
+// read) from one lane per SM, so the figure is the round-trip latency of an
+// L2 hit from that SM to that line's home slice.
 // Every loop has a fixed trip count; every address is checked against the
 // buffer on the host before launch.
 
@@ -39,24 +40,35 @@ __device__ __forceinline__ long long clk()
     return t;
 }
 
-// Mean cycles of `reps` dependent L2-hit loads of the line at p.
+// Zero that the hardware can only produce after v has arrived: the next
+// load's address depends on the previous load without depending on the
+// (arbitrary) bytes it returned.
+__device__ __forceinline__ uint32_t zero_after(uint32_t v)
+{
+    uint32_t z;
+    asm volatile("and.b32 %0, %1, 0;" : "=r"(z) : "r"(v));
+    return z;
+}
+
+// Mean cycles of `reps` dependent L2-hit loads of the 4 bytes at p (every
+// load reads p itself).
 __device__ __forceinline__ float time_line(const unsigned char *p, int reps)
 {
     const uint32_t *q = reinterpret_cast<const uint32_t *>(p);
     uint32_t v = ld_l2(q);          // brings the line into L2
-    v = ld_l2(q + v);
+    v = ld_l2(q + zero_after(v));
     const long long t0 = clk();
     for (int r = 0; r < reps; ++r)
-        v = ld_l2(q + v);
-    asm volatile("add.u32 %0, %0, 0;" : "+r"(v));   // issue waits for the last load
+        v = ld_l2(q + zero_after(v));
+    const uint32_t z = zero_after(v);   // issue waits for the last load
     const long long t1 = clk();
-    return static_cast<float>(t1 - t0) / reps + (v == 0xFFFFFFFFu ? 1.0f : 0.0f);
+    return static_cast<float>(t1 - t0) / reps + static_cast<float>(z);
 }
 
 // One CTA of 32 threads per SM does the work: the first CTA that lands on an
 // SM claims it; the others return at once.
-__global__ void probe_latency_kernel(const unsigned char *buf, const int64_t *line_off, int n_lines,
-                                     int reps, float *lat, uint32_t *claim)
+__global__ void probe_latency_kernel(const unsigned char *buf, int64_t buf_bytes, const int64_t *line_off,
+                                     int n_lines, int reps, float *lat, uint32_t *claim)
 {
     if (threadIdx.x != 0)
         return;
@@ -65,13 +77,18 @@ __global__ void probe_latency_kernel(const unsigned char *buf, const int64_t *li
         return;
     for (int k = 0; k < n_lines; ++k) {
         const int i = static_cast<int>((k + 7ull * sm) % static_cast<unsigned>(n_lines));
-        lat[(size_t)sm * n_lines + i] = time_line(buf + line_off[i], reps);
+        const int64_t o = line_off[i];
+        if (o < 0 || o + 4 > buf_bytes || (o & 3)) {   // never true for host-checked offsets
+            lat[(size_t)sm * n_lines + i] = -1.0f;
+            continue;
+        }
+        lat[(size_t)sm * n_lines + i] = time_line(buf + o, reps);
     }
 }
 
 // Die of every `chunk`-byte chunk: an SM of known die times the chunk's
 // first line; below the threshold the line is near (same die), else far.
-__global__ void probe_map_kernel(const unsigned char *buf, int64_t n_chunks, int64_t chunk, int reps,
+__global__ void probe_map_kernel(const unsigned char *buf, int64_t buf_bytes, int64_t n_chunks, int64_t chunk, int reps,
                                  const int8_t *sm_die, float threshold, uint32_t *counter,
                                  int8_t *die_out)
 {
@@ -84,6 +101,8 @@ __global__ void probe_map_kernel(const unsigned char *buf, int64_t n_chunks, int
         const uint32_t c = atomicAdd(counter, 1u);
         if (c >= n_chunks)
             break;
+        if ((int64_t)c * chunk + 4 > buf_bytes)          // never true for host-checked sizes
+            break;
         const float t = time_line(buf + (int64_t)c * chunk, reps);
         die_out[c] = static_cast<int8_t>(t < threshold ? my : 1 - my);
     }
@@ -94,8 +113,8 @@ __global__ void probe_map_kernel(const unsigned char *buf, int64_t n_chunks, int
 int probe_latency_run(const void *buf, const int64_t *line_off_dev, int n_lines, int reps, int grid,
                       float *lat_dev, uint32_t *claim_dev)
 {
-    probe_latency_kernel<<<grid, 32>>>(static_cast<const unsigned char *>(buf), line_off_dev, n_lines,
-                                       reps, lat_dev, claim_dev);
+    probe_latency_kernel<<<grid, 32>>>(static_cast<const unsigned char *>(buf), 32ll << 20, line_off_dev,
+                                       n_lines, reps, lat_dev, claim_dev);
     cudaError_t e = cudaGetLastError();
     if (e == cudaSuccess)
         e = cudaDeviceSynchronize();
@@ -107,7 +126,7 @@ int probe_map_run(const void *buf, int64_t bytes, int64_t chunk, int reps, const
 {
     const int64_t n_chunks = (bytes + chunk - 1) / chunk;
     // the chunk's first line must lie inside the buffer: (n_chunks-1)*chunk < bytes
-    probe_map_kernel<<<n_sm, 32>>>(static_cast<const unsigned char *>(buf), n_chunks, chunk, reps,
+    probe_map_kernel<<<n_sm, 32>>>(static_cast<const unsigned char *>(buf), bytes, n_chunks, chunk, reps,
                                    sm_die_dev, threshold, counter_dev, die_dev);
     cudaError_t e = cudaGetLastError();
     if (e == cudaSuccess)

@@ -35,7 +35,7 @@ std::mutex g_topo_mu;
 bsm_topology g_topo[64];
 bool g_topo_valid[64];
 
-int cuda_fail(cudaError_t e) { return e == cudaSuccess ? BSM_OK : BSM_ERR_CUDA; }
+int cuda_fail(cudaError_t e) { return e == cudaSuccess ? BSM_OK : record_cuda_error(e, "topology probe"); }
 
 std::vector<int64_t> default_lines()
 {
