@@ -119,7 +119,7 @@ struct bsm_plan {
         int32_t begin, end, grid;
     };
     std::vector<Launch> whole_gpu;   // WHOLE_GPU: one launch per slice
-    void *blob = nullptr;            // device tables (items, queue, slices, sm_die, heads)
+    void *blob = nullptr;            // device tables (patches, slice index, sm_die, heads)
     bsm_plan_stats stats{};
     // identity of the plan for the cache
     const void *x = nullptr;
@@ -241,27 +241,44 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     if (n_stages < 2)
         return BSM_ERR_UNSUPPORTED;
 
-    // ---- patches: consecutive rows of one slice filling (at most) one stage
+    // ---- patches: consecutive rows filling (at most) one stage.  Under the
+    // queue policies a patch may run on into the next slices when they have
+    // the same shape and follow back to back (a "segment"); under RR and
+    // WHOLE_GPU a patch stays inside its slice, the unit those policies place.
+    const bool spanning = d->policy == BSM_POLICY_DYNAMIC || d->policy == BSM_POLICY_CBMF ||
+                          d->policy == BSM_POLICY_CBMF_LB;
     std::vector<Item> items;
     std::vector<int32_t> slice_first(slices.size() + 1, 0);
-    for (size_t s = 0; s < slices.size(); ++s) {
+    size_t s = 0;
+    while (s < slices.size()) {
         slice_first[s] = static_cast<int32_t>(items.size());
         const SliceView &v = slices[s];
-        if (v.R == 0)
-            continue;
-        const int64_t row_bytes = int64_t(v.C) * es;
-        int64_t rpi = std::max<int64_t>(1, stage / row_bytes);
-        if (d->rows_per_item > 0)
-            rpi = std::min<int64_t>(rpi, d->rows_per_item);
-        if (d->policy == BSM_POLICY_WHOLE_GPU)
-            rpi = std::min<int64_t>(rpi, (v.R + c->n_sm - 1) / c->n_sm);
-        rpi = std::max<int64_t>(1, std::min<int64_t>(rpi, v.R));
-        for (int64_t r0 = 0; r0 < v.R; r0 += rpi) {
-            if (items.size() >= static_cast<size_t>(INT32_MAX))
-                return BSM_ERR_UNSUPPORTED;
-            const int64_t nr = std::min<int64_t>(rpi, v.R - r0);
-            items.push_back({v.off + r0 * v.C, v.C, static_cast<int32_t>(nr), static_cast<int32_t>(r0), 0});
+        size_t e = s + 1;
+        if (spanning && v.R > 0) {
+            while (e < slices.size() && slices[e].R == v.R && slices[e].C == v.C &&
+                   slices[e].off == slices[e - 1].off + int64_t(v.R) * v.C) {
+                slice_first[e] = static_cast<int32_t>(items.size());
+                ++e;
+            }
         }
+        if (v.R > 0) {
+            const int64_t seg_rows = int64_t(v.R) * static_cast<int64_t>(e - s);
+            const int64_t row_bytes = int64_t(v.C) * es;
+            int64_t rpi = std::max<int64_t>(1, stage / row_bytes);
+            if (d->rows_per_item > 0)
+                rpi = std::min<int64_t>(rpi, d->rows_per_item);
+            if (d->policy == BSM_POLICY_WHOLE_GPU)
+                rpi = std::min<int64_t>(rpi, (v.R + c->n_sm - 1) / c->n_sm);
+            rpi = std::max<int64_t>(1, std::min<int64_t>(rpi, seg_rows));
+            for (int64_t g0 = 0; g0 < seg_rows; g0 += rpi) {
+                if (items.size() >= static_cast<size_t>(INT32_MAX))
+                    return BSM_ERR_UNSUPPORTED;
+                const int64_t nr = std::min<int64_t>(rpi, seg_rows - g0);
+                items.push_back({v.off + g0 * v.C, v.C, static_cast<int32_t>(nr),
+                                 static_cast<int32_t>(g0 % v.R), v.R});
+            }
+        }
+        s = e;
     }
     slice_first[slices.size()] = static_cast<int32_t>(items.size());
     const int64_t n_items = static_cast<int64_t>(items.size());
@@ -282,7 +299,7 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     st.n_stages = n_stages;
 
     // ---- the schedule
-    std::vector<int32_t> queue;
+    std::vector<int32_t> queue;      // schedule order of the patches (queue policies)
     int32_t qbeg[BSM_MAX_DIES] = {0}, qlen[BSM_MAX_DIES] = {0};
     int n_queues = 1;
     int8_t sm_die_tab[BSM_MAX_SM];
@@ -416,18 +433,24 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
         }
     }
 
+    // ---- queue policies store the patches in queue order (die 0's queue,
+    // then die 1's, ...), so a claimed queue slot is the patch record itself
+    if (!queue.empty()) {
+        std::vector<Item> ordered(items.size());
+        for (size_t k = 0; k < queue.size(); ++k)
+            ordered[k] = items[static_cast<size_t>(queue[k])];
+        items.swap(ordered);
+    }
+
     // ---- upload the tables in one allocation
     const size_t items_b = sizeof(Item) * static_cast<size_t>(n_items);
-    const size_t queue_b = sizeof(int32_t) * queue.size();
     const size_t slices_b = sizeof(int32_t) * slice_first.size();
     auto up = [](size_t v) { return (v + 255) & ~size_t(255); };
-    const size_t o_items = 0, o_queue = up(items_b), o_slices = o_queue + up(queue_b),
-                 o_smdie = o_slices + up(slices_b), o_heads = o_smdie + 256, blob_b = o_heads + 256;
+    const size_t o_items = 0, o_slices = up(items_b), o_smdie = o_slices + up(slices_b),
+                 o_heads = o_smdie + 256, blob_b = o_heads + 256;
     std::vector<unsigned char> host(blob_b, 0);
     if (items_b)
         std::memcpy(&host[o_items], items.data(), items_b);
-    if (queue_b)
-        std::memcpy(&host[o_queue], queue.data(), queue_b);
     std::memcpy(&host[o_slices], slice_first.data(), slices_b);
     std::memcpy(&host[o_smdie], sm_die_tab, BSM_MAX_SM);
     int prev = -1;
@@ -459,7 +482,6 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     a.slice_first_item = reinterpret_cast<const int32_t *>(b + o_slices);
     a.n_slices = static_cast<int32_t>(std::min<size_t>(slices.size(), INT32_MAX));
     a.n_queues = n_queues;
-    a.queue = reinterpret_cast<const int32_t *>(b + o_queue);
     for (int q = 0; q < BSM_MAX_DIES; ++q) {
         a.queue_begin[q] = qbeg[q];
         a.queue_len[q] = qlen[q];

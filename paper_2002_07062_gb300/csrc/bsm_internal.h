@@ -9,14 +9,18 @@
 namespace bsm {
 
 // One patch ("batch or patch", Sec. 4: the unit of work the scheduler places):
-// rows [row0, row0 + nrows) of one slice.  The patch's elements are contiguous:
-// they start at element `off` of x and y and span nrows * C elements.
+// nrows consecutive rows of C elements, contiguous in x and y from element
+// `off`.  Under the RR and WHOLE_GPU policies a patch stays inside one slice;
+// under the queue policies it may run on into following slices of the same
+// shape (R x C, packed back to back).  The first row is row `row0` of its
+// slice and every slice of the patch has R rows, so row r of the patch is row
+// (row0 + r) mod R of its slice (the causal mask needs it).
 struct Item {
     int64_t off;
     int32_t C;
     int32_t nrows;
-    int32_t row0;   // row index inside the slice of the first row (causal mask)
-    int32_t pad;
+    int32_t row0;
+    int32_t R;
 };
 static_assert(sizeof(Item) == 24, "Item layout");
 
@@ -26,6 +30,9 @@ enum PullMode : int32_t {
     PULL_RR_SLICE = 1,  // CTA b takes every patch of slices b, b + G, ... (Sec. 3 RR)
     PULL_QUEUE = 2      // CTA pulls from its die's queue, then (steal) the others'
 };
+
+// Patches fetched per producer round trip.
+constexpr int kFetch = 4;
 
 constexpr int kMaxStages = 8;
 constexpr int kConsumerWarps = 16;
@@ -43,9 +50,8 @@ struct KernelArgs {
     int32_t item_begin, item_end;           // PULL_STATIC
     const int32_t *slice_first_item;        // PULL_RR_SLICE: n_slices + 1 entries
     int32_t n_slices;
-    int32_t n_queues;                       // PULL_QUEUE
-    const int32_t *queue;                   // concatenated per-die queues
-    int32_t queue_begin[BSM_MAX_DIES];
+    int32_t n_queues;                       // PULL_QUEUE: items are stored in queue
+    int32_t queue_begin[BSM_MAX_DIES];      // order; queue d is items[begin, begin+len)
     int32_t queue_len[BSM_MAX_DIES];
     int32_t steal;
     uint32_t *heads;            // BSM_MAX_DIES queue heads + 1 exit counter; self-resetting

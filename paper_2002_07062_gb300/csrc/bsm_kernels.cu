@@ -44,7 +44,8 @@ struct alignas(16) StageMeta {
     int32_t nrows;
     int32_t row0;
     int32_t kind;
-    int32_t pad[2];
+    int32_t R;
+    int32_t pad;
 };
 static_assert(sizeof(StageMeta) == 32, "StageMeta layout");
 
@@ -407,34 +408,36 @@ __device__ __forceinline__ void consume_stage(const unsigned char *sbuf, const S
     unsigned char *ybase = y + mt.off * E::kSize;
     bd.s_lo = sbuf;
     bd.s_hi = sbuf + (size_t)nrows * row_bytes;
+    // row of the slice that patch row r belongs to (only the causal mask reads it)
+    auto row_of = [&](int r) { return causal ? (mt.row0 + r) % mt.R : 0; };
     if (nvec <= 16) {
         const int half = lane >> 4, l = lane & 15;
         for (int rb = 2 * warp; rb < nrows; rb += 2 * kConsumerWarps) {
             const int r = rb + half;
             const bool valid = r < nrows;
             row_in_registers<Tag, Checked, 16, 1>(sbuf + (size_t)r * row_bytes,
-                                                  ybase + (size_t)r * row_bytes, nvec, mt.row0 + r,
+                                                  ybase + (size_t)r * row_bytes, nvec, row_of(r),
                                                   causal, l, valid, bd);
         }
     } else if (nvec <= 32) {
         for (int r = warp; r < nrows; r += kConsumerWarps)
             row_in_registers<Tag, Checked, 32, 1>(sbuf + (size_t)r * row_bytes,
-                                                  ybase + (size_t)r * row_bytes, nvec, mt.row0 + r,
+                                                  ybase + (size_t)r * row_bytes, nvec, row_of(r),
                                                   causal, lane, true, bd);
     } else if (nvec <= 64) {
         for (int r = warp; r < nrows; r += kConsumerWarps)
             row_in_registers<Tag, Checked, 32, 2>(sbuf + (size_t)r * row_bytes,
-                                                  ybase + (size_t)r * row_bytes, nvec, mt.row0 + r,
+                                                  ybase + (size_t)r * row_bytes, nvec, row_of(r),
                                                   causal, lane, true, bd);
     } else if (nvec <= 128) {
         for (int r = warp; r < nrows; r += kConsumerWarps)
             row_in_registers<Tag, Checked, 32, 4>(sbuf + (size_t)r * row_bytes,
-                                                  ybase + (size_t)r * row_bytes, nvec, mt.row0 + r,
+                                                  ybase + (size_t)r * row_bytes, nvec, row_of(r),
                                                   causal, lane, true, bd);
     } else {
         for (int r = warp; r < nrows; r += kConsumerWarps)
             row_in_smem<Tag, Checked>(sbuf + (size_t)r * row_bytes, ybase + (size_t)r * row_bytes,
-                                      nvec, mt.row0 + r, causal, lane, bd);
+                                      nvec, row_of(r), causal, lane, bd);
     }
 }
 
@@ -458,34 +461,52 @@ struct Puller {
             slice = static_cast<int32_t>(blockIdx.x) - static_cast<int32_t>(gridDim.x);
     }
 
-    // Next patch index, or -1 when this CTA has no more work.
-    __device__ int32_t next()
+    // Positions in a.items of this CTA's next patches (up to kFetch); returns
+    // how many (0 when the CTA has no more work).
+    __device__ int next_batch(int32_t (&pos)[kFetch])
     {
+        int n = 0;
         if (a.mode == PULL_STATIC) {
-            const int64_t idx = (int64_t)a.item_begin + blockIdx.x + (int64_t)k * gridDim.x;
-            ++k;
-            return idx < a.item_end ? static_cast<int32_t>(idx) : -1;
+#pragma unroll
+            for (int j = 0; j < kFetch; ++j) {
+                const int64_t idx = (int64_t)a.item_begin + blockIdx.x + (int64_t)(k + j) * gridDim.x;
+                if (idx < a.item_end)
+                    pos[n++] = static_cast<int32_t>(idx);
+            }
+            k += kFetch;
+            return n;
         }
         if (a.mode == PULL_RR_SLICE) {
             while (cur >= end) {
                 slice += gridDim.x;
                 if (slice >= a.n_slices)
-                    return -1;
+                    return 0;
                 cur = a.slice_first_item[slice];
                 end = a.slice_first_item[slice + 1];
             }
-            return cur++;
+#pragma unroll
+            for (int j = 0; j < kFetch; ++j)
+                if (cur < end)
+                    pos[n++] = cur++;
+            return n;
         }
-        // PULL_QUEUE: own die first, then (steal) the other dies in order.
+        // PULL_QUEUE: claim kFetch consecutive slots of the own die's queue,
+        // then (steal) of the other dies' queues in order.
         const int tries = a.steal ? a.n_queues : 1;
         while (q < tries) {
             const int qq = (die + q) % a.n_queues;
-            const uint32_t t = atomicAdd(&a.heads[qq], 1u);
-            if (t < static_cast<uint32_t>(a.queue_len[qq]))
-                return a.queue[a.queue_begin[qq] + t];
+            const uint32_t t = atomicAdd(&a.heads[qq], static_cast<uint32_t>(kFetch));
+            const uint32_t len = static_cast<uint32_t>(a.queue_len[qq]);
+            if (t < len) {
+#pragma unroll
+                for (int j = 0; j < kFetch; ++j)
+                    if (t + j < len)
+                        pos[n++] = a.queue_begin[qq] + static_cast<int32_t>(t + j);
+                return n;
+            }
             ++q;
         }
-        return -1;
+        return 0;
     }
 };
 
@@ -517,64 +538,86 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
             bool issued[kMaxStages];
             for (int s = 0; s < kMaxStages; ++s)
                 issued[s] = false;
-            bool aborted = false;
-            for (uint32_t it = 0;; ++it) {
-                const int s = it % S;
-                const uint32_t ph = (it / S) & 1u;
-                if (!mbar_wait_bounded(&h.empty[s], ph ^ 1u, &h.abort_flag)) {
-                    aborted = true;
+            bool aborted = false, done = false;
+            uint32_t it = 0;
+            while (!done && !aborted) {
+                // fetch the next patches: their records load in parallel
+                int32_t pos[kFetch];
+                const int n = pull.next_batch(pos);
+                Item batch[kFetch];
+#pragma unroll
+                for (int j = 0; j < kFetch; ++j)
+                    if (j < n && pos[j] >= 0 && pos[j] < a.n_items)
+                        batch[j] = a.items[pos[j]];
+                if (n == 0) {
+                    // no more work: tell the consumers through the next stage
+                    const int s = it % S;
+                    const uint32_t ph = (it / S) & 1u;
+                    if (!mbar_wait_bounded(&h.empty[s], ph ^ 1u, &h.abort_flag)) {
+                        aborted = true;
+                        break;
+                    }
+                    issued[s] = false;
+                    h.meta[s].kind = KIND_DONE;
+                    mbar_arrive(&h.full[s]);
+                    done = true;
                     break;
                 }
-                issued[s] = false;                 // the consumers released it
-                StageMeta &mt = h.meta[s];
-                const int32_t idx = pull.next();
-                if (idx < 0) {
-                    mt.kind = KIND_DONE;
-                    mbar_arrive(&h.full[s]);
-                    break;
-                }
-                bool ok = idx < a.n_items;
-                Item item{};
-                if (ok) {
-                    item = a.items[idx];
-                    const int64_t n = (int64_t)item.nrows * item.C;
-                    const int64_t bytes = n * E::kSize;
-                    ok = item.off >= 0 && item.C > 0 && item.nrows > 0 && item.row0 >= 0 &&
-                         item.off + n <= a.total_elems && bytes <= a.stage_bytes &&
-                         (bytes & 15) == 0 && ((item.off * E::kSize) & 15) == 0;
-                }
-                if (!ok) {
-                    atomicOr(a.status, BSM_DEV_BOUNDS);
-                    mt.kind = KIND_SKIP;
-                    mbar_arrive(&h.full[s]);
-                    continue;
-                }
-                mt.off = item.off;
-                mt.C = item.C;
-                mt.nrows = item.nrows;
-                mt.row0 = item.row0;
-                mt.kind = KIND_DATA;
-                const uint32_t bytes = static_cast<uint32_t>((int64_t)item.nrows * item.C * E::kSize);
-                unsigned char *dst = stages + (size_t)s * a.stage_bytes;
-                const unsigned char *src = static_cast<const unsigned char *>(a.x) + item.off * E::kSize;
-                if (Checked) {
-                    const unsigned char *x0 = static_cast<const unsigned char *>(a.x);
-                    const bool bad = s < 0 || s >= S || S > kMaxStages ||
-                                     src < x0 || src + bytes > x0 + a.total_elems * E::kSize ||
-                                     (reinterpret_cast<uintptr_t>(src) & 15) ||
-                                     (smem_addr(dst) & 15) || (bytes & 15) || bytes == 0 ||
-                                     dst + bytes > smem + kSmemHeader + (size_t)S * a.stage_bytes;
-                    if (bad) {
-                        check_fail(a.status, 3, static_cast<uint64_t>(idx), bytes);
+#pragma unroll
+                for (int j = 0; j < kFetch; ++j) {
+                    if (j >= n)
+                        break;
+                    const int s = it % S;
+                    const uint32_t ph = (it / S) & 1u;
+                    if (!mbar_wait_bounded(&h.empty[s], ph ^ 1u, &h.abort_flag)) {
+                        aborted = true;
+                        break;
+                    }
+                    issued[s] = false;                 // the consumers released it
+                    ++it;
+                    StageMeta &mt = h.meta[s];
+                    const Item item = batch[j];
+                    const int64_t ne = (int64_t)item.nrows * item.C;
+                    const int64_t nbytes = ne * E::kSize;
+                    const bool ok = pos[j] >= 0 && pos[j] < a.n_items && item.off >= 0 && item.C > 0 &&
+                                    item.nrows > 0 && item.R > 0 && item.row0 >= 0 &&
+                                    item.row0 < item.R && item.off + ne <= a.total_elems &&
+                                    nbytes <= a.stage_bytes && (nbytes & 15) == 0 &&
+                                    ((item.off * E::kSize) & 15) == 0;
+                    if (!ok) {
+                        atomicOr(a.status, BSM_DEV_BOUNDS);
                         mt.kind = KIND_SKIP;
                         mbar_arrive(&h.full[s]);
                         continue;
                     }
+                    mt.off = item.off;
+                    mt.C = item.C;
+                    mt.nrows = item.nrows;
+                    mt.row0 = item.row0;
+                    mt.R = item.R;
+                    mt.kind = KIND_DATA;
+                    const uint32_t bytes = static_cast<uint32_t>(nbytes);
+                    unsigned char *dst = stages + (size_t)s * a.stage_bytes;
+                    const unsigned char *src = static_cast<const unsigned char *>(a.x) + item.off * E::kSize;
+                    if (Checked) {
+                        const unsigned char *x0 = static_cast<const unsigned char *>(a.x);
+                        const bool bad = s < 0 || s >= S || S > kMaxStages ||
+                                         src < x0 || src + bytes > x0 + a.total_elems * E::kSize ||
+                                         (reinterpret_cast<uintptr_t>(src) & 15) ||
+                                         (smem_addr(dst) & 15) || (bytes & 15) || bytes == 0 ||
+                                         dst + bytes > smem + kSmemHeader + (size_t)S * a.stage_bytes;
+                        if (bad) {
+                            check_fail(a.status, 3, static_cast<uint64_t>(pos[j]), bytes);
+                            mt.kind = KIND_SKIP;
+                            mbar_arrive(&h.full[s]);
+                            continue;
+                        }
+                    }
+                    mbar_arrive_expect_tx(&h.full[s], bytes);
+                    bulk_load(dst, src, bytes, &h.full[s]);
+                    issued[s] = true;
+                    issued_phase[s] = ph;
                 }
-                mbar_arrive_expect_tx(&h.full[s], bytes);
-                bulk_load(dst, src, bytes, &h.full[s]);
-                issued[s] = true;
-                issued_phase[s] = ph;
             }
             if (aborted) {
                 atomicOr(a.status, BSM_DEV_TIMEOUT);

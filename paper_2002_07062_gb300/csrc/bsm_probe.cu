@@ -5,8 +5,8 @@
 // On GB300 each die owns half of the L2 and of the HBM stacks; an SM reading
 // a line homed on the other die crosses the die-to-die link.  Both kernels
 // time chains of dependent L2-only loads (ld.global.cg; each address waits
-// for the previous load through an "and 0", so it never depends on the data
-// read) from one lane per SM, so the figure is the round-trip latency of an
+// for the previous load through an AND with a runtime zero, so it never
+// depends on the data read) from one lane per SM, so the figure is the round-trip latency of an
 // L2 hit from that SM to that line's home slice.
 // Every loop has a fixed trip count; every address is checked against the
 // buffer on the host before launch.
@@ -40,35 +40,28 @@ __device__ __forceinline__ long long clk()
     return t;
 }
 
-// Zero that the hardware can only produce after v has arrived: the next
-// load's address depends on the previous load without depending on the
-// (arbitrary) bytes it returned.
-__device__ __forceinline__ uint32_t zero_after(uint32_t v)
-{
-    uint32_t z;
-    asm volatile("and.b32 %0, %1, 0;" : "=r"(z) : "r"(v));
-    return z;
-}
-
-// Mean cycles of `reps` dependent L2-hit loads of the 4 bytes at p (every
-// load reads p itself).
-__device__ __forceinline__ float time_line(const unsigned char *p, int reps)
+// Mean cycles of `reps` dependent L2-hit loads of the 4 bytes at p: every
+// load reads p itself; its address waits for the previous load through
+// "value AND zero", where zero is a kernel argument (0) the compiler cannot
+// fold, so the chain never depends on the bytes read.
+__device__ __forceinline__ float time_line(const unsigned char *p, int reps, uint32_t zero)
 {
     const uint32_t *q = reinterpret_cast<const uint32_t *>(p);
     uint32_t v = ld_l2(q);          // brings the line into L2
-    v = ld_l2(q + zero_after(v));
+    v = ld_l2(q + (v & zero));
     const long long t0 = clk();
     for (int r = 0; r < reps; ++r)
-        v = ld_l2(q + zero_after(v));
-    const uint32_t z = zero_after(v);   // issue waits for the last load
-    const long long t1 = clk();
-    return static_cast<float>(t1 - t0) / reps + static_cast<float>(z);
+        v = ld_l2(q + (v & zero));
+    const uint32_t z = v & zero;    // the clock read waits for the last load
+    asm volatile("" ::"r"(z));
+    const long long t1 = clk() + z;
+    return static_cast<float>(t1 - t0) / reps;
 }
 
 // One CTA of 32 threads per SM does the work: the first CTA that lands on an
 // SM claims it; the others return at once.
 __global__ void probe_latency_kernel(const unsigned char *buf, int64_t buf_bytes, const int64_t *line_off,
-                                     int n_lines, int reps, float *lat, uint32_t *claim)
+                                     int n_lines, int reps, float *lat, uint32_t *claim, uint32_t zero)
 {
     if (threadIdx.x != 0)
         return;
@@ -82,7 +75,7 @@ __global__ void probe_latency_kernel(const unsigned char *buf, int64_t buf_bytes
             lat[(size_t)sm * n_lines + i] = -1.0f;
             continue;
         }
-        lat[(size_t)sm * n_lines + i] = time_line(buf + o, reps);
+        lat[(size_t)sm * n_lines + i] = time_line(buf + o, reps, zero);
     }
 }
 
@@ -90,7 +83,7 @@ __global__ void probe_latency_kernel(const unsigned char *buf, int64_t buf_bytes
 // first line; below the threshold the line is near (same die), else far.
 __global__ void probe_map_kernel(const unsigned char *buf, int64_t buf_bytes, int64_t n_chunks, int64_t chunk, int reps,
                                  const int8_t *sm_die, float threshold, uint32_t *counter,
-                                 int8_t *die_out)
+                                 int8_t *die_out, uint32_t zero)
 {
     if (threadIdx.x != 0)
         return;
@@ -103,7 +96,7 @@ __global__ void probe_map_kernel(const unsigned char *buf, int64_t buf_bytes, in
             break;
         if ((int64_t)c * chunk + 4 > buf_bytes)          // never true for host-checked sizes
             break;
-        const float t = time_line(buf + (int64_t)c * chunk, reps);
+        const float t = time_line(buf + (int64_t)c * chunk, reps, zero);
         die_out[c] = static_cast<int8_t>(t < threshold ? my : 1 - my);
     }
 }
@@ -114,7 +107,7 @@ int probe_latency_run(const void *buf, const int64_t *line_off_dev, int n_lines,
                       float *lat_dev, uint32_t *claim_dev)
 {
     probe_latency_kernel<<<grid, 32>>>(static_cast<const unsigned char *>(buf), 32ll << 20, line_off_dev,
-                                       n_lines, reps, lat_dev, claim_dev);
+                                       n_lines, reps, lat_dev, claim_dev, 0u);
     cudaError_t e = cudaGetLastError();
     if (e == cudaSuccess)
         e = cudaDeviceSynchronize();
@@ -127,7 +120,7 @@ int probe_map_run(const void *buf, int64_t bytes, int64_t chunk, int reps, const
     const int64_t n_chunks = (bytes + chunk - 1) / chunk;
     // the chunk's first line must lie inside the buffer: (n_chunks-1)*chunk < bytes
     probe_map_kernel<<<n_sm, 32>>>(static_cast<const unsigned char *>(buf), bytes, n_chunks, chunk, reps,
-                                   sm_die_dev, threshold, counter_dev, die_dev);
+                                   sm_die_dev, threshold, counter_dev, die_dev, 0u);
     cudaError_t e = cudaGetLastError();
     if (e == cudaSuccess)
         e = cudaDeviceSynchronize();
