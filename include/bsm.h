@@ -70,7 +70,8 @@ typedef enum {
     BSM_ERR_DEVICE_BOUNDS = 5, /* a kernel met a patch outside the buffers */
     BSM_ERR_TIMEOUT = 6,       /* a kernel wait gave up after its time limit */
     BSM_ERR_NO_DEVICE = 7,     /* no usable CUDA device */
-    BSM_ERR_NOMEM = 8          /* host or device allocation failed */
+    BSM_ERR_NOMEM = 8,         /* host or device allocation failed */
+    BSM_ERR_TOO_LARGE = 9      /* more patches than bsm_softmax_noalloc's fixed scratch holds */
 } bsm_status;
 
 typedef enum { BSM_F32 = 0, BSM_BF16 = 1 } bsm_dtype;   /* input type == output type */
@@ -121,6 +122,36 @@ int bsm_softmax_ex(const void *x, void *y, int64_t B, int64_t R, int64_t C, int 
 int bsm_softmax_ragged(const void *x, void *y, int64_t num_slices, const int64_t *offsets,
                        const int32_t *rows, const int32_t *cols, int dtype, int policy,
                        uint32_t flags, bsm_stream_t stream);
+
+/*
+ * bsm_softmax_ex without any allocation -- for callers that cannot allocate
+ * device memory: code living inside a pre-reserved memory pool or arena (a
+ * server that sized the whole device up front, a framework whose allocator
+ * must account for every byte), or a latency-critical path that must not
+ * pick up the device-wide synchronisation of cudaMalloc/cudaFree.  The paper
+ * has no counterpart; this is a deployment variant of the dynamic schedule.
+ *
+ * Same computation and the same kernel as bsm_softmax_ex with
+ * BSM_POLICY_DYNAMIC (results are identical), for B slices of R x C packed
+ * back to back.  Instead of a plan, the patch table and queue counters live
+ * in one fixed device array inside the library: every GPU that loads the
+ * library holds it (about 1.5 MiB) until the process exits.  The first call
+ * on a device, with that device current, looks the array's address up
+ * (cudaGetSymbolAddress): make that first call before any stream capture.
+ * Every call shares the array and it keeps the last call's contents; each
+ * call rewrites the patch table and zeroes the counters on `stream` first,
+ * so calls that overlap on the GPU (other streams, unordered threads) race.
+ * Device-side error bits of this entry point stay in the array and are not
+ * reported.  Nothing is allocated and nothing synchronises.
+ *   x, y, B, R, C, dtype, flags, stream: as bsm_softmax_ex.
+ * Errors: as bsm_softmax_ex, plus BSM_ERR_TOO_LARGE when the batch needs more
+ * than BSM_NOALLOC_MAX_PATCHES patches (a patch is the rows that fill one
+ * 32 KiB shared-memory stage: for 2 KiB rows, 16 rows; 65536 patches cover
+ * 2 GiB of input).
+ */
+#define BSM_NOALLOC_MAX_PATCHES 65536
+int bsm_softmax_noalloc(const void *x, void *y, int64_t B, int64_t R, int64_t C, int dtype,
+                        uint32_t flags, bsm_stream_t stream);
 
 /* ---- plans: build the schedule once ("upfront", Sec. 5), run it many times ---- */
 

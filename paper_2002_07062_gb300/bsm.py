@@ -30,7 +30,8 @@ MAX_SM = 256
 DEV_BOUNDS, DEV_TIMEOUT, DEV_CHECK = 1, 2, 4
 
 (OK, ERR_INVALID_ARG, ERR_MISALIGNED, ERR_UNSUPPORTED, ERR_CUDA, ERR_DEVICE_BOUNDS,
- ERR_TIMEOUT, ERR_NO_DEVICE, ERR_NOMEM) = range(9)
+ ERR_TIMEOUT, ERR_NO_DEVICE, ERR_NOMEM, ERR_TOO_LARGE) = range(10)
+NOALLOC_MAX_PATCHES = 65536
 
 c_i64p = ctypes.POINTER(ctypes.c_int64)
 c_i32p = ctypes.POINTER(ctypes.c_int32)
@@ -109,6 +110,7 @@ def lib():
         "bsm_softmax_ex": ([vp, vp, i64, i64, i64, ctypes.c_int, ctypes.c_int, u32, vp], ctypes.c_int),
         "bsm_softmax_ragged": ([vp, vp, i64, c_i64p, c_i32p, c_i32p, ctypes.c_int, ctypes.c_int, u32,
                                 vp], ctypes.c_int),
+        "bsm_softmax_noalloc": ([vp, vp, i64, i64, i64, ctypes.c_int, u32, vp], ctypes.c_int),
         "bsm_plan_desc_init": ([ctypes.POINTER(PlanDesc)], ctypes.c_int),
         "bsm_plan_create": ([ctypes.POINTER(vp), ctypes.POINTER(PlanDesc)], ctypes.c_int),
         "bsm_plan_execute": ([vp, vp], ctypes.c_int),
@@ -184,6 +186,12 @@ def bsm_softmax_ex(x, y, B: int, R: int, C: int, dtype: int, policy: int, flags:
                    stream=None):
     _check(lib().bsm_softmax_ex(_dptr(x), _dptr(y), B, R, C, dtype, policy, flags,
                                 _stream(stream)), "bsm_softmax_ex")
+
+
+def bsm_softmax_noalloc(x, y, B: int, R: int, C: int, dtype: int, flags: int = 0, stream=None):
+    """The allocation-free entry point (fixed scratch inside the library)."""
+    _check(lib().bsm_softmax_noalloc(_dptr(x), _dptr(y), B, R, C, dtype, flags, _stream(stream)),
+           "bsm_softmax_noalloc")
 
 
 def bsm_softmax_ragged(x, y, offsets, rows, cols, dtype: int, policy: int, flags: int = 0,

@@ -873,6 +873,9 @@ const char *bsm_status_string(int status)
         return "no usable CUDA device";
     case BSM_ERR_NOMEM:
         return "out of memory";
+    case BSM_ERR_TOO_LARGE:
+        return "batch needs more patches than bsm_softmax_noalloc's fixed scratch holds "
+               "(BSM_NOALLOC_MAX_PATCHES)";
     default:
         return "unknown status";
     }
