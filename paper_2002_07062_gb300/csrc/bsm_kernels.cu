@@ -279,6 +279,42 @@ template <int T> __device__ __forceinline__ float group_sum(float s)
     return s;
 }
 
+// Maximum / sum of the N elements of one vector as a balanced tree (fixed
+// order: the sum's rounding is the same wherever the row runs).
+template <int N> __device__ __forceinline__ float tree_max(const float *v)
+{
+    if constexpr (N == 1)
+        return v[0];
+    else
+        return fmaxf(tree_max<N / 2>(v), tree_max<N / 2>(v + N / 2));
+}
+
+template <int N> __device__ __forceinline__ float tree_sum(const float *v)
+{
+    if constexpr (N == 1)
+        return v[0];
+    else
+        return tree_sum<N / 2>(v) + tree_sum<N / 2>(v + N / 2);
+}
+
+// p = exp(v - m) for one vector, as 2^(v*log2e - m*log2e).  A vector lying
+// wholly above the causal diagonal has v = x + (-inf): -inf gives p = 0
+// without the exponential; NaN (x was NaN or +inf) stays NaN, as the formula
+// says.
+template <int EPV>
+__device__ __forceinline__ void vec_exp(float (&v)[EPV], float mL, bool masked)
+{
+    if (masked) {
+#pragma unroll
+        for (int e = 0; e < EPV; ++e)
+            v[e] = v[e] == -INFINITY ? 0.0f : __int_as_float(0x7FC00000);
+    } else {
+#pragma unroll
+        for (int e = 0; e < EPV; ++e)
+            v[e] = ex2(fmaf(v[e], kLog2e, -mL));
+    }
+}
+
 // Additive causal mask of one 16-byte vector: element c of the row gets -inf
 // when c > row.
 template <int EPV>
@@ -305,11 +341,10 @@ __device__ __forceinline__ void row_in_registers(const unsigned char *srow, unsi
         uint4 raw;
         if (valid && vi < nvec && load_vec<Checked>(srow + 16 * vi, bd, raw)) {
             E::unpack(raw, v[j]);
-            if (causal)
+            // the mask is needed only where some column of the group passes the diagonal
+            if (causal && (j + 1) * T * EPV - 1 > row)
                 apply_causal<EPV>(v[j], vi * EPV, row);
-#pragma unroll
-            for (int e = 0; e < EPV; ++e)
-                m = fmaxf(m, v[j][e]);
+            m = fmaxf(m, tree_max<EPV>(v[j]));
         } else {
 #pragma unroll
             for (int e = 0; e < EPV; ++e)
@@ -321,17 +356,13 @@ __device__ __forceinline__ void row_in_registers(const unsigned char *srow, unsi
     float s = 0.0f;
 #pragma unroll
     for (int j = 0; j < V; ++j) {
-        float ps = 0.0f;
-#pragma unroll
-        for (int e = 0; e < EPV; ++e) {
-            v[j][e] = ex2(fmaf(v[j][e], kLog2e, -mL));
-            ps += v[j][e];
-        }
-        if (j * T + l < nvec)
-            s += ps;
+        const int vi = j * T + l;
+        vec_exp<EPV>(v[j], mL, (causal && vi * EPV > row) || vi >= nvec);
+        if (vi < nvec)
+            s += tree_sum<EPV>(v[j]);
     }
     s = group_sum<T>(s);
-    const float inv = 1.0f / s;
+    const float inv = __frcp_rn(s);
 #pragma unroll
     for (int j = 0; j < V; ++j) {
         const int vi = j * T + l;
@@ -344,7 +375,8 @@ __device__ __forceinline__ void row_in_registers(const unsigned char *srow, unsi
     }
 }
 
-// Shared-memory-resident row of any length: one warp, three sweeps.
+// Shared-memory-resident row of any length: one warp, three sweeps (max;
+// exponentials and their sum; exponentials again, scaled, stored).
 template <typename Tag, bool Checked>
 __device__ __forceinline__ void row_in_smem(const unsigned char *srow, unsigned char *yrow, int nvec,
                                             int row, bool causal, int lane, const Bounds &bd)
@@ -360,9 +392,7 @@ __device__ __forceinline__ void row_in_smem(const unsigned char *srow, unsigned 
         E::unpack(raw, v);
         if (causal)
             apply_causal<EPV>(v, vi * EPV, row);
-#pragma unroll
-        for (int e = 0; e < EPV; ++e)
-            m = fmaxf(m, v[e]);
+        m = fmaxf(m, tree_max<EPV>(v));
     }
     m = group_max<32>(m);
     const float mL = m * kLog2e;
@@ -373,25 +403,71 @@ __device__ __forceinline__ void row_in_smem(const unsigned char *srow, unsigned 
         E::unpack(raw, v);
         if (causal)
             apply_causal<EPV>(v, vi * EPV, row);
-        float ps = 0.0f;
-#pragma unroll
-        for (int e = 0; e < EPV; ++e)
-            ps += ex2(fmaf(v[e], kLog2e, -mL));
-        s += ps;
+        vec_exp<EPV>(v, mL, causal && vi * EPV > row);
+        s += tree_sum<EPV>(v);
     }
     s = group_sum<32>(s);
-    const float inv = 1.0f / s;
+    const float inv = __frcp_rn(s);
     for (int vi = lane; vi < nvec; vi += 32) {
         if (!load_vec<Checked>(srow + 16 * vi, bd, raw))
             continue;
         E::unpack(raw, v);
         if (causal)
             apply_causal<EPV>(v, vi * EPV, row);
+        vec_exp<EPV>(v, mL, causal && vi * EPV > row);
 #pragma unroll
         for (int e = 0; e < EPV; ++e)
-            v[e] = ex2(fmaf(v[e], kLog2e, -mL)) * inv;
+            v[e] *= inv;
         store_vec<Checked>(yrow + 16 * vi, bd, E::pack(v));
     }
+}
+
+// fp32 rows of any length, two exponential-free sweeps: the second sweep
+// writes p = exp(v - m) back over the row in shared memory (same size as x),
+// the third scales it.  One exponential per element.  The proxy fence orders
+// these generic writes before the bulk copy that later refills the stage.
+template <bool Checked>
+__device__ __forceinline__ void row_in_smem_inplace(unsigned char *srow, unsigned char *yrow, int nvec,
+                                                    int row, bool causal, int lane, const Bounds &bd)
+{
+    using E = Elem<F32>;
+    constexpr int EPV = E::kPerVec;
+    float v[EPV];
+    uint4 raw;
+    float m = -INFINITY;
+    for (int vi = lane; vi < nvec; vi += 32) {
+        if (!load_vec<Checked>(srow + 16 * vi, bd, raw))
+            continue;
+        E::unpack(raw, v);
+        if (causal)
+            apply_causal<EPV>(v, vi * EPV, row);
+        m = fmaxf(m, tree_max<EPV>(v));
+    }
+    m = group_max<32>(m);
+    const float mL = m * kLog2e;
+    float s = 0.0f;
+    for (int vi = lane; vi < nvec; vi += 32) {
+        if (!load_vec<Checked>(srow + 16 * vi, bd, raw))
+            continue;
+        E::unpack(raw, v);
+        if (causal)
+            apply_causal<EPV>(v, vi * EPV, row);
+        vec_exp<EPV>(v, mL, causal && vi * EPV > row);
+        s += tree_sum<EPV>(v);
+        *reinterpret_cast<uint4 *>(srow + 16 * vi) = E::pack(v);
+    }
+    s = group_sum<32>(s);
+    const float inv = __frcp_rn(s);
+    for (int vi = lane; vi < nvec; vi += 32) {
+        if (!load_vec<Checked>(srow + 16 * vi, bd, raw))
+            continue;
+        E::unpack(raw, v);
+#pragma unroll
+        for (int e = 0; e < EPV; ++e)
+            v[e] *= inv;
+        store_vec<Checked>(yrow + 16 * vi, bd, E::pack(v));
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
 // All rows of one stage that belong to this consumer warp.
@@ -419,21 +495,42 @@ __device__ __forceinline__ void consume_stage(const unsigned char *sbuf, const S
                                                   ybase + (size_t)r * row_bytes, nvec, row_of(r),
                                                   causal, l, valid, bd);
         }
-    } else if (nvec <= 32) {
+        return;
+    }
+    if (nvec <= 32) {
         for (int r = warp; r < nrows; r += kConsumerWarps)
             row_in_registers<Tag, Checked, 32, 1>(sbuf + (size_t)r * row_bytes,
                                                   ybase + (size_t)r * row_bytes, nvec, row_of(r),
                                                   causal, lane, true, bd);
-    } else if (nvec <= 64) {
+        return;
+    }
+    if (nvec <= 64) {
         for (int r = warp; r < nrows; r += kConsumerWarps)
             row_in_registers<Tag, Checked, 32, 2>(sbuf + (size_t)r * row_bytes,
                                                   ybase + (size_t)r * row_bytes, nvec, row_of(r),
                                                   causal, lane, true, bd);
-    } else if (nvec <= 128) {
+        return;
+    }
+    if (nvec <= 128) {
         for (int r = warp; r < nrows; r += kConsumerWarps)
             row_in_registers<Tag, Checked, 32, 4>(sbuf + (size_t)r * row_bytes,
                                                   ybase + (size_t)r * row_bytes, nvec, row_of(r),
                                                   causal, lane, true, bd);
+        return;
+    }
+    if constexpr (E::kSize == 4) {
+        // fp32: rows up to 4 KiB in registers, longer ones in place in the stage
+        if (nvec <= 256) {
+            for (int r = warp; r < nrows; r += kConsumerWarps)
+                row_in_registers<Tag, Checked, 32, 8>(sbuf + (size_t)r * row_bytes,
+                                                      ybase + (size_t)r * row_bytes, nvec, row_of(r),
+                                                      causal, lane, true, bd);
+        } else {
+            for (int r = warp; r < nrows; r += kConsumerWarps)
+                row_in_smem_inplace<Checked>(const_cast<unsigned char *>(sbuf) + (size_t)r * row_bytes,
+                                             ybase + (size_t)r * row_bytes, nvec, row_of(r), causal,
+                                             lane, bd);
+        }
     } else {
         for (int r = warp; r < nrows; r += kConsumerWarps)
             row_in_smem<Tag, Checked>(sbuf + (size_t)r * row_bytes, ybase + (size_t)r * row_bytes,

@@ -38,17 +38,19 @@ def _all_policies_identical(w, x, policies=ALL):
     return ys[0]
 
 
-def _ragged_all_classes(dtype, flags, seed, nslices=24):
-    # C from one 16-byte vector to 2.5x the register-resident limit; R 1..60
+def _ragged_all_classes(dtype, flags, seed, nslices=24, col_steps=160):
+    # C in 16-byte vectors: 1..col_steps (160: up to 2.5 KiB rows, the register
+    # routines; 768: up to 12 KiB rows, the shared-memory routines); R 1..60
     unit = 4 if dtype == workload.F32 else 8
     return workload.ragged("classes", dtype, nslices, 2.0, seed, flags, row_unit=1,
-                           row_steps=60, col_unit=unit, col_steps=160).materialize()
+                           row_steps=60, col_unit=unit, col_steps=col_steps).materialize()
 
 
 @pytest.mark.parametrize("dtype", [workload.F32, workload.BF16])
 @pytest.mark.parametrize("flags", [0, bsm.FLAG_CAUSAL])
-def test_ragged_every_row_routine_full_parity(dtype, flags):
-    w = _ragged_all_classes(dtype, flags, 100 + 2 * dtype + flags)
+@pytest.mark.parametrize("col_steps", [160, 768])
+def test_ragged_every_row_routine_full_parity(dtype, flags, col_steps):
+    w = _ragged_all_classes(dtype, flags, 100 + 2 * dtype + flags + col_steps, col_steps=col_steps)
     x = to_device(w.x)
     y = _all_policies_identical(w, x)
     check_all_against_oracle(w, to_host(y))
