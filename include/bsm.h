@@ -214,6 +214,24 @@ typedef struct {
 int bsm_plan_get_stats(const bsm_plan *plan, bsm_plan_stats *out);
 void bsm_plan_destroy(bsm_plan *plan);
 
+/* Fault injection on one plan, for the library's failure-detection tests
+ * (nothing here faults, traps or hangs the GPU):
+ *   BSM_DEBUG_WITHHOLD_STAGE  later executes never fill the first shared-memory
+ *                             stage of each CTA, so the consumers' bounded waits
+ *                             run out; arg = the wait limit in ns (> 0).  The
+ *                             kernel sets BSM_DEV_TIMEOUT and every CTA exits.
+ *   BSM_DEBUG_CORRUPT_PATCH   the device patch table entry at position arg is
+ *                             rewritten to start past the end of the buffers; the
+ *                             kernel's bounds check skips it and sets
+ *                             BSM_DEV_BOUNDS (its rows are not written).
+ *   BSM_DEBUG_NONE            restore the normal wait limit and switch the
+ *                             withheld stage off (a corrupted entry stays).
+ * Synchronous.  Returns BSM_ERR_INVALID_ARG for an unknown `what` or arg. */
+#define BSM_DEBUG_NONE 0
+#define BSM_DEBUG_WITHHOLD_STAGE 1
+#define BSM_DEBUG_CORRUPT_PATCH 2
+int bsm_plan_debug(bsm_plan *plan, int what, int64_t arg);
+
 /* Drop every cached plan of bsm_softmax / bsm_softmax_ex / bsm_softmax_ragged. */
 void bsm_cache_clear(void);
 

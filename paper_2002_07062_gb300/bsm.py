@@ -116,6 +116,7 @@ def lib():
         "bsm_plan_execute": ([vp, vp], ctypes.c_int),
         "bsm_plan_get_stats": ([vp, ctypes.POINTER(PlanStats)], ctypes.c_int),
         "bsm_plan_destroy": ([vp], None),
+        "bsm_plan_debug": ([vp, ctypes.c_int, i64], ctypes.c_int),
         "bsm_cache_clear": ([], None),
         "bsm_topology_probe": ([ctypes.c_int, ctypes.c_int, ctypes.POINTER(Topology)], ctypes.c_int),
         "bsm_addr_die_map": ([ctypes.c_int, vp, i64, i64, ctypes.POINTER(ctypes.c_int8)], ctypes.c_int),
@@ -274,6 +275,14 @@ def bsm_plan_get_stats(plan: Plan) -> dict:
         v = getattr(s, name)
         out[name] = list(v) if not isinstance(v, (int, float)) else v
     return out
+
+
+DEBUG_NONE, DEBUG_WITHHOLD_STAGE, DEBUG_CORRUPT_PATCH = 0, 1, 2
+
+
+def bsm_plan_debug(plan: Plan, what: int, arg: int = 0):
+    """Test-only fault injection (see include/bsm.h)."""
+    _check(lib().bsm_plan_debug(plan.handle, what, arg), "bsm_plan_debug")
 
 
 def bsm_plan_destroy(plan: Plan):

@@ -9,6 +9,7 @@
 #include <atomic>
 #include <chrono>
 #include <cmath>
+#include <cstddef>
 #include <cstring>
 #include <list>
 #include <mutex>
@@ -676,6 +677,40 @@ int bsm_plan_get_stats(const bsm_plan *plan, bsm_plan_stats *out)
         return BSM_ERR_INVALID_ARG;
     *out = plan->stats;
     return BSM_OK;
+}
+
+int bsm_plan_debug(bsm_plan *plan, int what, int64_t arg)
+{
+    if (!plan)
+        return BSM_ERR_INVALID_ARG;
+    switch (what) {
+    case BSM_DEBUG_NONE:
+        plan->args.debug = 0;
+        plan->args.wait_limit_ns = 0;
+        return BSM_OK;
+    case BSM_DEBUG_WITHHOLD_STAGE:
+        if (arg <= 0)
+            return BSM_ERR_INVALID_ARG;
+        plan->args.debug |= KDEBUG_WITHHOLD_STAGE0;
+        plan->args.wait_limit_ns = static_cast<uint64_t>(arg);
+        return BSM_OK;
+    case BSM_DEBUG_CORRUPT_PATCH: {
+        if (arg < 0 || arg >= plan->args.n_items)
+            return BSM_ERR_INVALID_ARG;
+        const int64_t past_end = plan->args.total_elems;
+        unsigned char *entry = static_cast<unsigned char *>(plan->blob) + sizeof(Item) * static_cast<size_t>(arg);
+        int prev = -1;
+        cudaGetDevice(&prev);
+        cudaSetDevice(plan->device);
+        cudaError_t e = cudaMemcpy(entry + offsetof(Item, off), &past_end, sizeof past_end,
+                                   cudaMemcpyHostToDevice);
+        if (prev >= 0)
+            cudaSetDevice(prev);
+        return e == cudaSuccess ? BSM_OK : cuda_error(e, "cudaMemcpy(patch entry)");
+    }
+    default:
+        return BSM_ERR_INVALID_ARG;
+    }
 }
 
 void bsm_plan_destroy(bsm_plan *plan)

@@ -60,7 +60,12 @@ struct KernelArgs {
     int32_t n_stages;
     uint32_t flags;
     uint32_t *status;           // sticky device status word
+    uint64_t wait_limit_ns;     // bound of every pipeline wait (0 = the 2 s default)
+    uint32_t debug;             // fault injection for tests: KDEBUG_* bits
 };
+
+// Test-only fault injection (bsm_plan_debug).
+constexpr uint32_t KDEBUG_WITHHOLD_STAGE0 = 1u;   // producer never fills stage 0 of its first round
 
 // Launch the persistent softmax kernel (bsm_kernels.cu).  Returns a
 // cudaError_t value (0 = success).

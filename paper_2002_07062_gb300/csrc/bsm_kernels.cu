@@ -21,7 +21,8 @@
 // the exponent formed by one fused multiply-add, v*log2e - m*log2e, and the
 // power of two from the PTX ex2.approx instruction; y = p * (1/sum).
 //
-// Every wait is bounded (kWaitLimitNs, 2 s of wall time): on expiry the CTA
+// Every wait is bounded (2 s of wall time unless the launch asks for less):
+// on expiry the CTA
 // records BSM_DEV_TIMEOUT in the status word, lets its copies in flight land,
 // and returns.
 
@@ -101,24 +102,29 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t by
                  : "memory");
 }
 
+// One potentially blocking test of the phase: a waiting thread is suspended
+// in hardware (it issues nothing) until the phase completes or kSuspendNs
+// pass, so idle warps do not take issue slots from the working ones.
+constexpr uint32_t kSuspendNs = 50000;
+
 __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity)
 {
     uint32_t ok;
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
         "selp.u32 %0, 1, 0, p;\n\t}"
         : "=r"(ok)
-        : "r"(smem_addr(bar)), "r"(parity)
+        : "r"(smem_addr(bar)), "r"(parity), "r"(kSuspendNs)
         : "memory");
     return ok != 0;
 }
 
 // Wait until the phase with the given parity of `bar` has completed.  Gives
 // up (returns false) when *abort becomes non-zero (if abort != nullptr) or
-// after kWaitLimitNs.
+// after limit_ns.
 __device__ __noinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity,
-                                               const volatile int32_t *abort)
+                                               const volatile int32_t *abort, uint64_t limit_ns)
 {
     if (mbar_try_wait(bar, parity))
         return true;
@@ -126,10 +132,10 @@ __device__ __noinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity,
     for (uint32_t it = 0; it < (1u << 28); ++it) {
         if (mbar_try_wait(bar, parity))
             return true;
-        if ((it & 7u) == 7u) {
+        {
             if (abort && *abort)
                 return false;
-            if (global_timer_ns() - t0 > kWaitLimitNs)
+            if (global_timer_ns() - t0 > limit_ns)
                 return false;
         }
     }
@@ -616,6 +622,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
     unsigned char *stages = smem + kSmemHeader;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int S = a.n_stages;
+    const uint64_t wait_limit = a.wait_limit_ns ? a.wait_limit_ns : kWaitLimitNs;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
@@ -650,7 +657,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                     // no more work: tell the consumers through the next stage
                     const int s = it % S;
                     const uint32_t ph = (it / S) & 1u;
-                    if (!mbar_wait_bounded(&h.empty[s], ph ^ 1u, &h.abort_flag)) {
+                    if (!mbar_wait_bounded(&h.empty[s], ph ^ 1u, &h.abort_flag, wait_limit)) {
                         aborted = true;
                         break;
                     }
@@ -666,13 +673,15 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                         break;
                     const int s = it % S;
                     const uint32_t ph = (it / S) & 1u;
-                    if (!mbar_wait_bounded(&h.empty[s], ph ^ 1u, &h.abort_flag)) {
+                    if (!mbar_wait_bounded(&h.empty[s], ph ^ 1u, &h.abort_flag, wait_limit)) {
                         aborted = true;
                         break;
                     }
                     issued[s] = false;                 // the consumers released it
                     ++it;
                     StageMeta &mt = h.meta[s];
+                    if ((a.debug & KDEBUG_WITHHOLD_STAGE0) && it == 1)
+                        continue;                      // test hook: stage 0 is never filled
                     const Item item = batch[j];
                     const int64_t ne = (int64_t)item.nrows * item.C;
                     const int64_t nbytes = ne * E::kSize;
@@ -719,11 +728,12 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
             if (aborted) {
                 atomicOr(a.status, BSM_DEV_TIMEOUT);
                 h.abort_flag = 1;
-                // let every copy still in flight land before the CTA exits
-                for (int s = 0; s < S; ++s)
-                    if (issued[s])
-                        mbar_wait_bounded(&h.full[s], issued_phase[s], nullptr);
             }
+            // every copy this lane issued has landed before it leaves (normally
+            // they have: the consumers waited for them; after an abort they may not)
+            for (int s = 0; s < S; ++s)
+                if (issued[s])
+                    mbar_wait_bounded(&h.full[s], issued_phase[s], nullptr, wait_limit);
             if (a.mode == PULL_QUEUE) {
                 // the last CTA to finish pulling rewinds the queue heads
                 __threadfence();
@@ -744,7 +754,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
     for (uint32_t it = 0;; ++it) {
         const int s = it % S;
         const uint32_t ph = (it / S) & 1u;
-        if (!mbar_wait_bounded(&h.full[s], ph, &h.abort_flag)) {
+        if (!mbar_wait_bounded(&h.full[s], ph, &h.abort_flag, wait_limit)) {
             if (lane == 0) {
                 atomicOr(a.status, BSM_DEV_TIMEOUT);
                 h.abort_flag = 1;
