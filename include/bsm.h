@@ -114,6 +114,25 @@ int bsm_softmax_ex(const void *x, void *y, int64_t B, int64_t R, int64_t C, int 
                    int policy, uint32_t flags, bsm_stream_t stream);
 
 /*
+ * bsm_softmax_ex on HOST buffers: x_host is read and y_host written by copies
+ * that the call queues itself.  The batch is cut into chunks of whole slices
+ * (about 48 MiB of input each); each chunk is copied to a device staging
+ * buffer, processed, and copied back, on three streams of the library with
+ * two staging buffers, so that copying in, computing and copying out of
+ * consecutive chunks overlap.  Asynchronous with respect to `stream`: the work
+ * starts after what is already queued on `stream`, and `stream` waits for
+ * its end; synchronise `stream` before reading y_host.  Pinned (page-locked)
+ * host memory is needed for the copies to overlap.  The staging buffers
+ * (2 x 2 x chunk bytes) are allocated on first use and kept per device; calls
+ * on one device share them and are serialised on the host.
+ *   x_host, y_host  host pointers, B*R*C elements each; may be equal.
+ *   B, R, C, dtype, policy, flags  as bsm_softmax_ex.
+ * Errors: as bsm_softmax_ex.
+ */
+int bsm_softmax_host(const void *x_host, void *y_host, int64_t B, int64_t R, int64_t C, int dtype,
+                     int policy, uint32_t flags, bsm_stream_t stream);
+
+/*
  * Ragged batch: slice s has rows[s] x cols[s] elements at element offset
  * offsets[s] of x (and of y).  offsets/rows/cols are HOST arrays of
  * num_slices entries, copied.  Slices must not overlap each other; they need

@@ -111,6 +111,7 @@ def lib():
         "bsm_softmax_ragged": ([vp, vp, i64, c_i64p, c_i32p, c_i32p, ctypes.c_int, ctypes.c_int, u32,
                                 vp], ctypes.c_int),
         "bsm_softmax_noalloc": ([vp, vp, i64, i64, i64, ctypes.c_int, u32, vp], ctypes.c_int),
+        "bsm_softmax_host": ([vp, vp, i64, i64, i64, ctypes.c_int, ctypes.c_int, u32, vp], ctypes.c_int),
         "bsm_plan_desc_init": ([ctypes.POINTER(PlanDesc)], ctypes.c_int),
         "bsm_plan_create": ([ctypes.POINTER(vp), ctypes.POINTER(PlanDesc)], ctypes.c_int),
         "bsm_plan_execute": ([vp, vp], ctypes.c_int),
@@ -187,6 +188,20 @@ def bsm_softmax_ex(x, y, B: int, R: int, C: int, dtype: int, policy: int, flags:
                    stream=None):
     _check(lib().bsm_softmax_ex(_dptr(x), _dptr(y), B, R, C, dtype, policy, flags,
                                 _stream(stream)), "bsm_softmax_ex")
+
+
+def bsm_softmax_host(x_host, y_host, B: int, R: int, C: int, dtype: int, policy: int,
+                     flags: int = 0, stream=None):
+    """Softmax of host buffers (pinned torch CPU tensors, numpy arrays or host
+    addresses); copies in, computes and copies out in overlapping chunks."""
+    def hptr(a):
+        if isinstance(a, int):
+            return a
+        if isinstance(a, np.ndarray):
+            return a.ctypes.data
+        return int(a.data_ptr())
+    _check(lib().bsm_softmax_host(hptr(x_host), hptr(y_host), B, R, C, dtype, policy, flags,
+                                  _stream(stream)), "bsm_softmax_host")
 
 
 def bsm_softmax_noalloc(x, y, B: int, R: int, C: int, dtype: int, flags: int = 0, stream=None):

@@ -1,0 +1,41 @@
+"""The multi-rank timing path of bench.py on CPU with gloo, world size 2:
+the job time is the slowest rank's, and the job throughput counts every
+rank's batches (independent slices, no data-path collective)."""
+import os
+import socket
+
+import pytest
+
+
+def _free_port():
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    port = s.getsockname()[1]
+    s.close()
+    return port
+
+
+def _worker(rank, world, port, out):
+    import torch.distributed as dist
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    import bench
+    local_ms = [10.0, 25.0][rank]
+    mx = bench.reduce_max_ms(local_ms)
+    out[rank] = (mx, bench.job_gbs(world, 805306368, 100, mx))
+    dist.barrier()
+    dist.destroy_process_group()
+
+
+def test_two_rank_max_time_and_job_throughput():
+    import torch.multiprocessing as mp
+    port = _free_port()
+    with mp.Manager() as m:
+        out = m.dict()
+        mp.spawn(_worker, args=(2, port, out), nprocs=2, join=True)
+        res = dict(out)
+    assert res[0] == res[1]
+    mx, gbs = res[0]
+    assert mx == 25.0
+    assert gbs == pytest.approx(2 * 805306368 * 100 / 0.025 / 1e9)
