@@ -13,11 +13,14 @@
 // queue" of Sec. 5).
 //
 // Row routine (the arithmetic, identical under every policy): a row is owned
-// by a group of T lanes (T = 16 for rows of <= 256 bytes, else 32); lane l owns
-// the 16-byte vectors l, l + T, l + 2T, ...; the maximum and the sum are
-// per-lane in vector order, then a butterfly (xor) shuffle tree.  Rows of up
-// to 2 KiB are held in registers; longer rows are swept three times out of
-// shared memory (max, sum, write).  exp(t) is evaluated as 2^(t*log2 e) with
+// by a group of T lanes; lane l owns the 16-byte vectors l, l + T, l + 2T, ...
+// The maximum and the sum are per vector (a balanced tree), per lane in vector
+// order, then a butterfly (xor) shuffle tree over the group.  By row length in
+// 16-byte vectors: <= 8: T = 8, 1 vector per lane; <= 16: T = 8, 2; <= 32:
+// T = 8, 4; <= 64: T = 16, 4; <= 128: T = 32, 4; fp32 <= 256: T = 32, 8 -- all
+// in registers (at most 32 elements per lane); longer fp32 rows: one warp,
+// exponentials written back in place in shared memory; longer bf16 rows: one
+// warp, three sweeps over shared memory (max, sum, write).  exp(t) is evaluated as 2^(t*log2 e) with
 // the exponent formed by one fused multiply-add, v*log2e - m*log2e, and the
 // power of two from the PTX ex2.approx instruction; y = p * (1/sum).
 //
@@ -303,17 +306,17 @@ template <int N> __device__ __forceinline__ float tree_sum(const float *v)
         return tree_sum<N / 2>(v) + tree_sum<N / 2>(v + N / 2);
 }
 
-// p = exp(v - m) for one vector, as 2^(v*log2e - m*log2e).  A vector lying
-// wholly above the causal diagonal has v = x + (-inf): -inf gives p = 0
-// without the exponential; NaN (x was NaN or +inf) stays NaN, as the formula
-// says.
+// p = exp(v - m) for one vector, as 2^(v*log2e - m*log2e).  For a vector
+// lying wholly above the causal diagonal (v is x, or x + (-inf)) the formula
+// gives 0 where x is finite or -inf and NaN where x is NaN or +inf; that is
+// computed without the exponential.
 template <int EPV>
 __device__ __forceinline__ void vec_exp(float (&v)[EPV], float mL, bool masked)
 {
     if (masked) {
 #pragma unroll
         for (int e = 0; e < EPV; ++e)
-            v[e] = v[e] == -INFINITY ? 0.0f : __int_as_float(0x7FC00000);
+            v[e] = v[e] < INFINITY ? 0.0f : __int_as_float(0x7FC00000);
     } else {
 #pragma unroll
         for (int e = 0; e < EPV; ++e)
@@ -331,7 +334,10 @@ __device__ __forceinline__ void apply_causal(float (&v)[EPV], int col0, int row)
         v[e] += (col0 + e > row) ? -INFINITY : 0.0f;
 }
 
-// Register-resident row: T lanes, up to V vectors per lane.
+// Register-resident row: T lanes, up to V vectors per lane.  Under the
+// causal mask a vector is unmasked (all its columns <= row), on the diagonal
+// (masked element by element) or wholly masked (it adds nothing to the max;
+// its p is 0 or NaN, see vec_exp).
 template <typename Tag, bool Checked, int T, int V>
 __device__ __forceinline__ void row_in_registers(const unsigned char *srow, unsigned char *yrow,
                                                  int nvec, int row, bool causal, int l, bool valid,
@@ -344,13 +350,15 @@ __device__ __forceinline__ void row_in_registers(const unsigned char *srow, unsi
 #pragma unroll
     for (int j = 0; j < V; ++j) {
         const int vi = j * T + l;
+        const bool masked = causal && vi * EPV > row;
         uint4 raw;
         if (valid && vi < nvec && load_vec<Checked>(srow + 16 * vi, bd, raw)) {
             E::unpack(raw, v[j]);
-            // the mask is needed only where some column of the group passes the diagonal
-            if (causal && (j + 1) * T * EPV - 1 > row)
-                apply_causal<EPV>(v[j], vi * EPV, row);
-            m = fmaxf(m, tree_max<EPV>(v[j]));
+            if (!masked) {
+                if (causal && vi * EPV + EPV - 1 > row)
+                    apply_causal<EPV>(v[j], vi * EPV, row);
+                m = fmaxf(m, tree_max<EPV>(v[j]));
+            }
         } else {
 #pragma unroll
             for (int e = 0; e < EPV; ++e)
@@ -476,71 +484,77 @@ __device__ __forceinline__ void row_in_smem_inplace(unsigned char *srow, unsigne
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-// All rows of one stage that belong to this consumer warp.
+// The rows of a stage handled by one register routine: groups of T lanes,
+// 32/T rows per warp at a time; q tracks each group's row inside its slice
+// ((row0 + r) mod R) without a division per row.
+template <typename Tag, bool Checked, int T, int V>
+__device__ __forceinline__ void rows_in_registers(const unsigned char *sbuf, const StageMeta &mt,
+                                                  unsigned char *ybase, int row_bytes, int nvec,
+                                                  bool causal, int warp, int lane, const Bounds &bd)
+{
+    constexpr int G = 32 / T;
+    const int g = lane / T, l = lane % T;
+    const int step = G * kConsumerWarps;
+    int q = 0, qstep = 0;
+    if (causal) {
+        q = (mt.row0 + warp * G + g) % mt.R;
+        qstep = step % mt.R;
+    }
+    for (int rb = warp * G; rb < mt.nrows; rb += step) {
+        const int r = rb + g;
+        row_in_registers<Tag, Checked, T, V>(sbuf + (size_t)r * row_bytes, ybase + (size_t)r * row_bytes,
+                                             nvec, q, causal, l, r < mt.nrows, bd);
+        q += qstep;
+        if (q >= mt.R)
+            q -= mt.R;
+    }
+}
+
+// All rows of one stage that belong to this consumer warp.  The routine
+// depends on the row length only (see the table at the top of the file).
 template <typename Tag, bool Checked>
 __device__ __forceinline__ void consume_stage(const unsigned char *sbuf, const StageMeta &mt,
                                               unsigned char *y, bool causal, int warp, int lane,
                                               Bounds bd)
 {
     using E = Elem<Tag>;
-    const int C = mt.C;
-    const int nrows = mt.nrows;
-    const int row_bytes = C * E::kSize;
+    const int row_bytes = mt.C * E::kSize;
     const int nvec = row_bytes >> 4;
     unsigned char *ybase = y + mt.off * E::kSize;
     bd.s_lo = sbuf;
-    bd.s_hi = sbuf + (size_t)nrows * row_bytes;
-    // row of the slice that patch row r belongs to (only the causal mask reads it)
-    auto row_of = [&](int r) { return causal ? (mt.row0 + r) % mt.R : 0; };
-    if (nvec <= 16) {
-        const int half = lane >> 4, l = lane & 15;
-        for (int rb = 2 * warp; rb < nrows; rb += 2 * kConsumerWarps) {
-            const int r = rb + half;
-            const bool valid = r < nrows;
-            row_in_registers<Tag, Checked, 16, 1>(sbuf + (size_t)r * row_bytes,
-                                                  ybase + (size_t)r * row_bytes, nvec, row_of(r),
-                                                  causal, l, valid, bd);
-        }
-        return;
+    bd.s_hi = sbuf + (size_t)mt.nrows * row_bytes;
+    if (nvec <= 8)
+        return rows_in_registers<Tag, Checked, 8, 1>(sbuf, mt, ybase, row_bytes, nvec, causal, warp, lane, bd);
+    if (nvec <= 16)
+        return rows_in_registers<Tag, Checked, 8, 2>(sbuf, mt, ybase, row_bytes, nvec, causal, warp, lane, bd);
+    if (nvec <= 32)
+        return rows_in_registers<Tag, Checked, 8, 4>(sbuf, mt, ybase, row_bytes, nvec, causal, warp, lane, bd);
+    if (nvec <= 64)
+        return rows_in_registers<Tag, Checked, 16, 4>(sbuf, mt, ybase, row_bytes, nvec, causal, warp, lane, bd);
+    if (nvec <= 128)
+        return rows_in_registers<Tag, Checked, 32, 4>(sbuf, mt, ybase, row_bytes, nvec, causal, warp, lane, bd);
+    // one warp per row from here on
+    int q = 0, qstep = 0;
+    if (causal) {
+        q = (mt.row0 + warp) % mt.R;
+        qstep = kConsumerWarps % mt.R;
     }
-    if (nvec <= 32) {
-        for (int r = warp; r < nrows; r += kConsumerWarps)
-            row_in_registers<Tag, Checked, 32, 1>(sbuf + (size_t)r * row_bytes,
-                                                  ybase + (size_t)r * row_bytes, nvec, row_of(r),
-                                                  causal, lane, true, bd);
-        return;
-    }
-    if (nvec <= 64) {
-        for (int r = warp; r < nrows; r += kConsumerWarps)
-            row_in_registers<Tag, Checked, 32, 2>(sbuf + (size_t)r * row_bytes,
-                                                  ybase + (size_t)r * row_bytes, nvec, row_of(r),
-                                                  causal, lane, true, bd);
-        return;
-    }
-    if (nvec <= 128) {
-        for (int r = warp; r < nrows; r += kConsumerWarps)
-            row_in_registers<Tag, Checked, 32, 4>(sbuf + (size_t)r * row_bytes,
-                                                  ybase + (size_t)r * row_bytes, nvec, row_of(r),
-                                                  causal, lane, true, bd);
-        return;
-    }
-    if constexpr (E::kSize == 4) {
-        // fp32: rows up to 4 KiB in registers, longer ones in place in the stage
-        if (nvec <= 256) {
-            for (int r = warp; r < nrows; r += kConsumerWarps)
-                row_in_registers<Tag, Checked, 32, 8>(sbuf + (size_t)r * row_bytes,
-                                                      ybase + (size_t)r * row_bytes, nvec, row_of(r),
-                                                      causal, lane, true, bd);
+    for (int r = warp; r < mt.nrows; r += kConsumerWarps) {
+        const unsigned char *srow = sbuf + (size_t)r * row_bytes;
+        unsigned char *yrow = ybase + (size_t)r * row_bytes;
+        if constexpr (E::kSize == 4) {
+            // fp32: rows up to 4 KiB in registers, longer ones in place in the stage
+            if (nvec <= 256)
+                row_in_registers<Tag, Checked, 32, 8>(srow, yrow, nvec, q, causal, lane, true, bd);
+            else
+                row_in_smem_inplace<Checked>(const_cast<unsigned char *>(srow), yrow, nvec, q, causal, lane,
+                                             bd);
         } else {
-            for (int r = warp; r < nrows; r += kConsumerWarps)
-                row_in_smem_inplace<Checked>(const_cast<unsigned char *>(sbuf) + (size_t)r * row_bytes,
-                                             ybase + (size_t)r * row_bytes, nvec, row_of(r), causal,
-                                             lane, bd);
+            row_in_smem<Tag, Checked>(srow, yrow, nvec, q, causal, lane, bd);
         }
-    } else {
-        for (int r = warp; r < nrows; r += kConsumerWarps)
-            row_in_smem<Tag, Checked>(sbuf + (size_t)r * row_bytes, ybase + (size_t)r * row_bytes,
-                                      nvec, row_of(r), causal, lane, bd);
+        q += qstep;
+        if (q >= mt.R)
+            q -= mt.R;
     }
 }
 
