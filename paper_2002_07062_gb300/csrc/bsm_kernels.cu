@@ -155,14 +155,27 @@ __device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t b
         : "memory");
 }
 
-// Plain C++ accesses: the compiler sees them as memory operations, so the
-// "memory" clobber of the barrier waits orders them, and it may still
-// schedule them freely inside a row.
+// Stage reads and in-place writes are explicit shared-space accesses (a
+// 32-bit shared address), so they are issued as shared loads/stores whatever
+// the compiler can infer about the pointer; volatile keeps them on their side
+// of the barrier waits.
 __device__ __forceinline__ uint4 lds128(const unsigned char *p)
 {
-    return *reinterpret_cast<const uint4 *>(p);
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "r"(smem_addr(p)));
+    return v;
 }
 
+__device__ __forceinline__ void sts128(unsigned char *p, uint4 v)
+{
+    asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(smem_addr(p)), "r"(v.x), "r"(v.y),
+                 "r"(v.z), "r"(v.w)
+                 : "memory");
+}
+
+// Output stores: plain 128-bit global stores.
 __device__ __forceinline__ void stg128(void *p, uint4 v)
 {
     *reinterpret_cast<uint4 *>(p) = v;
@@ -468,7 +481,7 @@ __device__ __forceinline__ void row_in_smem_inplace(unsigned char *srow, unsigne
             apply_causal<EPV>(v, vi * EPV, row);
         vec_exp<EPV>(v, mL, causal && vi * EPV > row);
         s += tree_sum<EPV>(v);
-        *reinterpret_cast<uint4 *>(srow + 16 * vi) = E::pack(v);
+        sts128(srow + 16 * vi, E::pack(v));
     }
     s = group_sum<32>(s);
     const float inv = __frcp_rn(s);
@@ -485,22 +498,24 @@ __device__ __forceinline__ void row_in_smem_inplace(unsigned char *srow, unsigne
 }
 
 // The rows of a stage handled by one register routine: groups of T lanes,
-// 32/T rows per warp at a time; q tracks each group's row inside its slice
-// ((row0 + r) mod R) without a division per row.
+// G = 32/T rows per group of a warp.  Row groups are dealt to the consumer
+// warps round robin, starting at warp `first` (see consume_stage); q tracks
+// each lane group's row inside its slice ((row0 + r) mod R) without a
+// division per row.  Returns the number of row groups of the stage.
 template <typename Tag, bool Checked, int T, int V>
-__device__ __forceinline__ void rows_in_registers(const unsigned char *sbuf, const StageMeta &mt,
-                                                  unsigned char *ybase, int row_bytes, int nvec,
-                                                  bool causal, int warp, int lane, const Bounds &bd)
+__device__ __forceinline__ int rows_in_registers(const unsigned char *sbuf, const StageMeta &mt,
+                                                 unsigned char *ybase, int row_bytes, int nvec,
+                                                 bool causal, int first, int lane, const Bounds &bd)
 {
     constexpr int G = 32 / T;
     const int g = lane / T, l = lane % T;
     const int step = G * kConsumerWarps;
     int q = 0, qstep = 0;
     if (causal) {
-        q = (mt.row0 + warp * G + g) % mt.R;
+        q = (mt.row0 + first * G + g) % mt.R;
         qstep = step % mt.R;
     }
-    for (int rb = warp * G; rb < mt.nrows; rb += step) {
+    for (int rb = first * G; rb < mt.nrows; rb += step) {
         const int r = rb + g;
         row_in_registers<Tag, Checked, T, V>(sbuf + (size_t)r * row_bytes, ybase + (size_t)r * row_bytes,
                                              nvec, q, causal, l, r < mt.nrows, bd);
@@ -508,14 +523,18 @@ __device__ __forceinline__ void rows_in_registers(const unsigned char *sbuf, con
         if (q >= mt.R)
             q -= mt.R;
     }
+    return (mt.nrows + G - 1) / G;
 }
 
 // All rows of one stage that belong to this consumer warp.  The routine
 // depends on the row length only (see the table at the top of the file).
+// Row groups are dealt round robin over the consumer warps starting at warp
+// `first`; the caller advances `first` by the returned group count, so a
+// stage with fewer groups than warps does not always land on the same warps.
 template <typename Tag, bool Checked>
-__device__ __forceinline__ void consume_stage(const unsigned char *sbuf, const StageMeta &mt,
-                                              unsigned char *y, bool causal, int warp, int lane,
-                                              Bounds bd)
+__device__ __forceinline__ int consume_stage(const unsigned char *sbuf, const StageMeta &mt,
+                                             unsigned char *y, bool causal, int first, int lane,
+                                             Bounds bd)
 {
     using E = Elem<Tag>;
     const int row_bytes = mt.C * E::kSize;
@@ -524,22 +543,24 @@ __device__ __forceinline__ void consume_stage(const unsigned char *sbuf, const S
     bd.s_lo = sbuf;
     bd.s_hi = sbuf + (size_t)mt.nrows * row_bytes;
     if (nvec <= 8)
-        return rows_in_registers<Tag, Checked, 8, 1>(sbuf, mt, ybase, row_bytes, nvec, causal, warp, lane, bd);
+        return rows_in_registers<Tag, Checked, 8, 1>(sbuf, mt, ybase, row_bytes, nvec, causal, first, lane, bd);
     if (nvec <= 16)
-        return rows_in_registers<Tag, Checked, 8, 2>(sbuf, mt, ybase, row_bytes, nvec, causal, warp, lane, bd);
+        return rows_in_registers<Tag, Checked, 8, 2>(sbuf, mt, ybase, row_bytes, nvec, causal, first, lane, bd);
     if (nvec <= 32)
-        return rows_in_registers<Tag, Checked, 8, 4>(sbuf, mt, ybase, row_bytes, nvec, causal, warp, lane, bd);
+        return rows_in_registers<Tag, Checked, 8, 4>(sbuf, mt, ybase, row_bytes, nvec, causal, first, lane, bd);
     if (nvec <= 64)
-        return rows_in_registers<Tag, Checked, 16, 4>(sbuf, mt, ybase, row_bytes, nvec, causal, warp, lane, bd);
+        return rows_in_registers<Tag, Checked, 16, 4>(sbuf, mt, ybase, row_bytes, nvec, causal, first, lane,
+                                                      bd);
     if (nvec <= 128)
-        return rows_in_registers<Tag, Checked, 32, 4>(sbuf, mt, ybase, row_bytes, nvec, causal, warp, lane, bd);
+        return rows_in_registers<Tag, Checked, 32, 4>(sbuf, mt, ybase, row_bytes, nvec, causal, first, lane,
+                                                      bd);
     // one warp per row from here on
     int q = 0, qstep = 0;
     if (causal) {
-        q = (mt.row0 + warp) % mt.R;
+        q = (mt.row0 + first) % mt.R;
         qstep = kConsumerWarps % mt.R;
     }
-    for (int r = warp; r < mt.nrows; r += kConsumerWarps) {
+    for (int r = first; r < mt.nrows; r += kConsumerWarps) {
         const unsigned char *srow = sbuf + (size_t)r * row_bytes;
         unsigned char *yrow = ybase + (size_t)r * row_bytes;
         if constexpr (E::kSize == 4) {
@@ -556,6 +577,7 @@ __device__ __forceinline__ void consume_stage(const unsigned char *sbuf, const S
         if (q >= mt.R)
             q -= mt.R;
     }
+    return mt.nrows;
 }
 
 // -------------------------------------------------------------- the schedule
@@ -765,6 +787,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
     // ----------------------------------------------------------- consumers
     const bool causal = (a.flags & BSM_FLAG_CAUSAL) != 0;
     unsigned char *y = static_cast<unsigned char *>(a.y);
+    uint32_t groups_seen = 0;   // row groups dealt so far (the same count in every warp)
     for (uint32_t it = 0;; ++it) {
         const int s = it % S;
         const uint32_t ph = (it / S) & 1u;
@@ -785,8 +808,10 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                 if (lane == 0)
                     check_fail(a.status, 4, static_cast<uint64_t>(mt.nrows), static_cast<uint64_t>(mt.C));
             } else {
-                consume_stage<Tag, Checked>(stages + (size_t)s * a.stage_bytes, mt, y, causal, warp,
-                                            lane, bd);
+                const int first = static_cast<int>((warp + kConsumerWarps - groups_seen % kConsumerWarps) %
+                                                   kConsumerWarps);
+                groups_seen += consume_stage<Tag, Checked>(stages + (size_t)s * a.stage_bytes, mt, y, causal,
+                                                           first, lane, bd);
             }
         }
         __syncwarp();
