@@ -389,7 +389,7 @@ def main():
         nb = x.numel() * x.element_size()
         out["e2e"] = {"value": round(ws * bytes_step / (e_ms * 1e-3) / 1e9, 2), "unit": "GB/s",
                       "h2d_bytes_per_step": nb, "d2h_bytes_per_step": nb,
-                      "ms_per_step": round(e_ms, 4), "api": "bsm_softmax_host (pinned host buffers)"}
+                      "ms_per_step": round(e_ms, 4), "api": "bsm_softmax_host, pinned host buffers read and written by the kernel over the host link"}
     if not args.no_cpu_baseline and rank == 0 and ws == 1:
         out["cpu_baseline"] = cpu_baseline(w)
 

@@ -114,17 +114,19 @@ int bsm_softmax_ex(const void *x, void *y, int64_t B, int64_t R, int64_t C, int 
                    int policy, uint32_t flags, bsm_stream_t stream);
 
 /*
- * bsm_softmax_ex on HOST buffers: x_host is read and y_host written by copies
- * that the call queues itself.  The batch is cut into chunks of whole slices
- * (about 48 MiB of input each); each chunk is copied to a device staging
- * buffer, processed, and copied back, on three streams of the library with
- * two staging buffers, so that copying in, computing and copying out of
- * consecutive chunks overlap.  Asynchronous with respect to `stream`: the work
- * starts after what is already queued on `stream`, and `stream` waits for
- * its end; synchronise `stream` before reading y_host.  Pinned (page-locked)
- * host memory is needed for the copies to overlap.  The staging buffers
- * (2 x 2 x chunk bytes) are allocated on first use and kept per device; calls
- * on one device share them and are serialised on the host.
+ * bsm_softmax_ex on HOST buffers.  Page-locked (pinned, e.g. cudaHostAlloc or
+ * cudaHostRegister) buffers are read and written by the kernel directly over
+ * the CPU-GPU link (NVLink-C2C on Grace-Blackwell): no device memory, both
+ * link directions in use at once.  Pageable buffers go through a staged
+ * pipeline: the batch is cut into chunks of whole slices (about 48 MiB of
+ * input each); each chunk is copied to a device staging buffer, processed and
+ * copied back, on three streams of the library with two staging buffers, so
+ * that copying in, computing and copying out of consecutive chunks overlap;
+ * the staging buffers (2 x 2 x chunk bytes) are allocated on first use and
+ * kept per device, and such calls on one device are serialised on the host.
+ * Asynchronous with respect to `stream`: the work starts after what is
+ * already queued on `stream`, and `stream` waits for its end; synchronise
+ * `stream` before reading y_host.
  *   x_host, y_host  host pointers, B*R*C elements each; may be equal.
  *   B, R, C, dtype, policy, flags  as bsm_softmax_ex.
  * Errors: as bsm_softmax_ex.

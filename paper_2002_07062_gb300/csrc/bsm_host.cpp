@@ -1,6 +1,12 @@
 // bsm_host.cpp -- bsm_softmax_host: the batched softmax on HOST buffers.
 //
-// The batch is cut into chunks of whole slices; every chunk goes through
+// Page-locked (pinned) buffers are read and written by the kernel itself:
+// on Grace-Blackwell the GPU reaches host memory over NVLink-C2C, so the
+// bulk copies of the patches come straight from x_host and the stores go
+// straight to y_host -- no staging memory, both link directions busy at once.
+//
+// Pageable buffers go through a staged pipeline: the batch is cut into
+// chunks of whole slices; every chunk goes through
 // three stages on three streams of the library -- copy in (host to device),
 // the softmax kernel (the plan-cached bsm_softmax_ex path on a device staging
 // buffer), copy out (device to host) -- with two staging buffers, so chunk i
@@ -100,6 +106,14 @@ int softmax_host(const void *x_host, void *y_host, int64_t B, int64_t R, int64_t
     const uintptr_t len = static_cast<uintptr_t>(B * slice_bytes);
     if (xa != ya && xa < ya + len && ya < xa + len)
         return BSM_ERR_INVALID_ARG;
+    // pinned host memory: the kernel accesses it directly
+    cudaPointerAttributes ax{}, ay{};
+    if (cudaPointerGetAttributes(&ax, x_host) == cudaSuccess &&
+        cudaPointerGetAttributes(&ay, y_host) == cudaSuccess && ax.type == cudaMemoryTypeHost &&
+        ay.type == cudaMemoryTypeHost && ax.devicePointer && ay.devicePointer)
+        return bsm_softmax_ex(ax.devicePointer, ay.devicePointer, B, R, C, dtype, policy, flags, stream);
+    cudaGetLastError();   // a pageable pointer is not an error here
+
     const int64_t per_chunk = std::max<int64_t>(1, std::min<int64_t>(B, kChunkBytes / slice_bytes));
     const int64_t chunk_bytes = per_chunk * slice_bytes;
 
