@@ -37,6 +37,14 @@ def lib():
                                           ctypes.c_uint32, ctypes.c_void_p, ctypes.c_void_p,
                                           ctypes.c_int]
         L.orc_softmax_batched.restype = ctypes.c_int
+        L.orc_softmax_backward_row.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
+                                               ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]
+        L.orc_softmax_backward_row.restype = ctypes.c_int
+        L.orc_softmax_backward_batched.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
+                                                   ctypes.c_int64, ctypes.c_void_p,
+                                                   ctypes.c_void_p, ctypes.c_void_p,
+                                                   ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int]
+        L.orc_softmax_backward_batched.restype = ctypes.c_int
         L.orc_double_to_bf16.argtypes = [ctypes.c_double]
         L.orc_double_to_bf16.restype = ctypes.c_uint16
         _lib = L
@@ -89,6 +97,42 @@ def softmax_batched(x: np.ndarray, offsets: Sequence[int], rows: Sequence[int],
     if rc:
         raise RuntimeError("orc_softmax_batched failed: %d" % rc)
     return y64, yout
+
+
+def softmax_backward_row(yrow: np.ndarray, dyrow: np.ndarray):
+    """dx of one row (float64, rounded to the input type)."""
+    yrow = np.ascontiguousarray(yrow)
+    dyrow = np.ascontiguousarray(dyrow)
+    dt = _dtype_code(yrow)
+    assert dyrow.dtype == yrow.dtype and dyrow.shape == yrow.shape
+    C = yrow.shape[-1]
+    d64 = np.empty(C, np.float64)
+    dout = np.empty(C, yrow.dtype)
+    rc = lib().orc_softmax_backward_row(_ptr(yrow), _ptr(dyrow), dt, C, _ptr(d64), _ptr(dout))
+    if rc:
+        raise RuntimeError("orc_softmax_backward_row failed: %d" % rc)
+    return d64, dout
+
+
+def softmax_backward_batched(y: np.ndarray, dy: np.ndarray, offsets, rows, cols,
+                             want_f64: bool = True, want_rounded: bool = True,
+                             nthreads: Optional[int] = None):
+    """dx = y * (dy - rowsum(y * dy)) for every slice; arrays flat, like x."""
+    y = np.ascontiguousarray(y).reshape(-1)
+    dy = np.ascontiguousarray(dy).reshape(-1)
+    dt = _dtype_code(y)
+    assert dy.dtype == y.dtype and dy.size == y.size
+    off = np.ascontiguousarray(offsets, dtype=np.int64)
+    R = np.ascontiguousarray(rows, dtype=np.int32)
+    C = np.ascontiguousarray(cols, dtype=np.int32)
+    d64 = np.full(y.shape, np.nan, np.float64) if want_f64 else None
+    dout = np.zeros(y.shape, y.dtype) if want_rounded else None
+    rc = lib().orc_softmax_backward_batched(_ptr(y), _ptr(dy), dt, len(off), _ptr(off), _ptr(R),
+                                            _ptr(C), _ptr(d64), _ptr(dout),
+                                            nthreads or os.cpu_count() or 1)
+    if rc:
+        raise RuntimeError("orc_softmax_backward_batched failed: %d" % rc)
+    return d64, dout
 
 
 def double_to_bf16(d: float) -> int:

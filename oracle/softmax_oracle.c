@@ -21,6 +21,13 @@
  * same formula: a NaN or +inf anywhere in v, or a row that is all -inf, makes
  * the whole row NaN (0/0 or inf-inf).
  *
+ * The backward pass (the paper's batch algorithms run "in the forward pass or
+ * the backward pass", Sec. 1) is the vector-Jacobian product of the same
+ * softmax: given y = softmax(v) and an upstream gradient dy of one row,
+ *     dx[c] = y[c] * (dy[c] - sum_c' y[c'] * dy[c'])
+ * in double, y and dy exactly converted, the dot product summed left to
+ * right, rounded once to the output type.
+ *
  * Only tests/, __graft_entry__.smoke() and bench.py's cpu_baseline leg (and its
  * reference arm) may load this library.  It shares no code, header or constant
  * with the CUDA library: it has its own bf16 conversions, its own types and
@@ -119,11 +126,35 @@ int orc_softmax_row(const void *xrow, int dtype, int64_t C, int64_t row_in_slice
     return 0;
 }
 
+/* Backward of one row: y and dy point at the row's first elements. */
+int orc_softmax_backward_row(const void *yrow, const void *dyrow, int dtype, int64_t C,
+                             double *dx64, void *dxout)
+{
+    if (C <= 0 || (dtype != ORC_F32 && dtype != ORC_BF16))
+        return -1;
+    double dot = 0.0;
+    for (int64_t c = 0; c < C; ++c)
+        dot += orc_load(yrow, dtype, c) * orc_load(dyrow, dtype, c);
+    for (int64_t c = 0; c < C; ++c) {
+        double d = orc_load(yrow, dtype, c) * (orc_load(dyrow, dtype, c) - dot);
+        if (dx64)
+            dx64[c] = d;
+        if (dxout) {
+            if (dtype == ORC_F32)
+                ((float *)dxout)[c] = (float)d;
+            else
+                ((uint16_t *)dxout)[c] = orc_double_to_bf16(d);
+        }
+    }
+    return 0;
+}
+
 /* ---- batched form: slices s = 0..B-1, slice s has rows[s] x cols[s] elements
  *      starting at element offsets[s] of x (and of y64 / yout). ---- */
 
 typedef struct {
     const void *x;
+    const void *dy;            /* backward: upstream gradient (x is y) */
     int dtype;
     int64_t nslices;
     const int64_t *offsets;
@@ -166,7 +197,13 @@ static void *orc_worker(void *arg)
         int64_t r = g - j->row_base[s];
         int64_t C = j->cols[s];
         int64_t e = j->offsets[s] + r * C;
-        int rc = orc_softmax_row((const char *)j->x + e * es, j->dtype, C, r, j->flags,
+        int rc;
+        if (j->dy)
+            rc = orc_softmax_backward_row((const char *)j->x + e * es, (const char *)j->dy + e * es,
+                                          j->dtype, C, j->y64 ? j->y64 + e : NULL,
+                                          j->yout ? (void *)((char *)j->yout + e * es) : NULL);
+        else
+            rc = orc_softmax_row((const char *)j->x + e * es, j->dtype, C, r, j->flags,
                                  j->y64 ? j->y64 + e : NULL,
                                  j->yout ? (void *)((char *)j->yout + e * es) : NULL);
         if (rc) {
@@ -177,9 +214,9 @@ static void *orc_worker(void *arg)
     return NULL;
 }
 
-int orc_softmax_batched(const void *x, int dtype, int64_t nslices, const int64_t *offsets,
-                        const int32_t *rows, const int32_t *cols, uint32_t flags,
-                        double *y64, void *yout, int nthreads)
+static int orc_run_batched(const void *x, const void *dy, int dtype, int64_t nslices,
+                           const int64_t *offsets, const int32_t *rows, const int32_t *cols,
+                           uint32_t flags, double *y64, void *yout, int nthreads)
 {
     if (nslices < 0 || (nslices > 0 && (!x || !offsets || !rows || !cols)))
         return -1;
@@ -210,7 +247,7 @@ int orc_softmax_batched(const void *x, int dtype, int64_t nslices, const int64_t
         return -2;
     }
     for (int t = 0; t < nthreads; ++t) {
-        orc_job j = {x, dtype, nslices, offsets, rows, cols, flags, y64, yout,
+        orc_job j = {x, dy, dtype, nslices, offsets, rows, cols, flags, y64, yout,
                      total, row_base, nthreads, t, 0};
         jobs[t] = j;
     }
@@ -229,4 +266,21 @@ int orc_softmax_batched(const void *x, int dtype, int64_t nslices, const int64_t
     free(jobs);
     free(th);
     return status;
+}
+
+int orc_softmax_batched(const void *x, int dtype, int64_t nslices, const int64_t *offsets,
+                        const int32_t *rows, const int32_t *cols, uint32_t flags,
+                        double *y64, void *yout, int nthreads)
+{
+    return orc_run_batched(x, NULL, dtype, nslices, offsets, rows, cols, flags, y64, yout, nthreads);
+}
+
+/* Backward over every slice: y and dy laid out like the forward's x. */
+int orc_softmax_backward_batched(const void *y, const void *dy, int dtype, int64_t nslices,
+                                 const int64_t *offsets, const int32_t *rows, const int32_t *cols,
+                                 double *dx64, void *dxout, int nthreads)
+{
+    if (nslices > 0 && !dy)
+        return -1;
+    return orc_run_batched(y, dy, dtype, nslices, offsets, rows, cols, 0u, dx64, dxout, nthreads);
 }
