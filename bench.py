@@ -430,6 +430,27 @@ def sweep(args, bsm, workload, stream):
                               "ms": round(med, 4),
                               "GBps": round(w.algorithmic_bytes / (med * 1e-3) / 1e9, 2),
                               "slices_per_s": round(w.nslices / (med * 1e-3), 1)}), flush=True)
+        if k in (2, 3, 5):
+            # backward pass on the same slices: read y and dy, write dx
+            dy = torch.empty_like(x).normal_() if w.dtype == workload.F32 else \
+                torch.empty_like(x).normal_()
+            dx = torch.empty_like(x)
+            bsm.bsm_softmax_ragged(x, y, w.offsets, w.rows, w.cols, w.dtype, bsm.POLICY_DYNAMIC,
+                                   w.flags, stream)
+
+            def bstep():
+                bsm.bsm_softmax_backward_ragged(y, dy, dx, w.offsets, w.rows, w.cols, w.dtype,
+                                                bsm.POLICY_DYNAMIC, stream)
+            for _ in range(3):
+                bstep()
+            stream.synchronize()
+            _, per = time_steps(bstep, 20, stream, per_launch=True)
+            med = float(np.median(per))
+            nbytes = 3 * w.numel * w.esize
+            print(json.dumps({"sweep": True, "op": "backward", "workload": w.name,
+                              "policy": "dynamic", "ms": round(med, 4),
+                              "GBps": round(nbytes / (med * 1e-3) / 1e9, 2)}), flush=True)
+            del dy, dx
         del x, y
         torch.cuda.empty_cache()
 

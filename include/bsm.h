@@ -174,6 +174,26 @@ int bsm_softmax_ragged(const void *x, void *y, int64_t num_slices, const int64_t
 int bsm_softmax_noalloc(const void *x, void *y, int64_t B, int64_t R, int64_t C, int dtype,
                         uint32_t flags, bsm_stream_t stream);
 
+/*
+ * Backward pass of the batched softmax (Sec. 1: the batch algorithms run in
+ * the forward or the backward pass) over the same slices and the same
+ * scheduler: for every row, given the forward output y and the upstream
+ * gradient dy,
+ *     dx[c] = y[c] * (dy[c] - sum_c' y[c'] * dy[c'])
+ * (the vector-Jacobian product of the row softmax; with a causal forward the
+ * masked y are 0 and so are their dx).  y, dy, dx: device pointers, B*R*C
+ * elements of `dtype`; dx may equal y or dy; other overlaps are rejected.
+ * Rows may be at most half of bsm_max_row_bytes() (y and dy share a stage).
+ * Same scheduling policies, errors and alignment rules as bsm_softmax.
+ */
+int bsm_softmax_backward(const void *y, const void *dy, void *dx, int64_t B, int64_t R, int64_t C,
+                         int dtype, int policy, bsm_stream_t stream);
+
+/* Ragged form of bsm_softmax_backward (slices as in bsm_softmax_ragged). */
+int bsm_softmax_backward_ragged(const void *y, const void *dy, void *dx, int64_t num_slices,
+                                const int64_t *offsets, const int32_t *rows, const int32_t *cols,
+                                int dtype, int policy, bsm_stream_t stream);
+
 /* ---- plans: build the schedule once ("upfront", Sec. 5), run it many times ---- */
 
 typedef struct bsm_plan bsm_plan;
@@ -193,7 +213,12 @@ typedef struct {
     int32_t lb_weighted;        /* CBMF_LB: 1 = weights from measured latency, 0 = equal */
     int32_t count_output_bytes; /* CBMF: 1 = a patch's bytes on a die count x and y */
     int32_t device;             /* -1 = the current device */
+    int32_t op;                 /* BSM_OP_FORWARD (default) or BSM_OP_BACKWARD */
+    const void *x2;             /* BSM_OP_BACKWARD: the upstream gradient dy (x holds y) */
 } bsm_plan_desc;
+
+#define BSM_OP_FORWARD 0        /* y = softmax(x) */
+#define BSM_OP_BACKWARD 1       /* y = x * (x2 - rowsum(x * x2)): dx from y = x and dy = x2 */
 
 /* Fill a descriptor with the defaults (rows_per_item 0, tie_seed 0x2002070600,
  * lb_weighted 1, count_output_bytes 1, device -1, offsets NULL). */

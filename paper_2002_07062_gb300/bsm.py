@@ -25,6 +25,7 @@ POLICIES = {"whole_gpu": POLICY_WHOLE_GPU, "rr": POLICY_RR, "cbmf": POLICY_CBMF,
             "cbmf_lb": POLICY_CBMF_LB, "dynamic": POLICY_DYNAMIC}
 POLICY_NAMES = {v: k for k, v in POLICIES.items()}
 FLAG_CAUSAL = 1
+OP_FORWARD, OP_BACKWARD = 0, 1
 MAX_DIES = 4
 MAX_SM = 256
 DEV_BOUNDS, DEV_TIMEOUT, DEV_CHECK = 1, 2, 4
@@ -52,7 +53,7 @@ class PlanDesc(ctypes.Structure):
                 ("dtype", ctypes.c_int32), ("policy", ctypes.c_int32), ("flags", ctypes.c_uint32),
                 ("rows_per_item", ctypes.c_int32), ("tie_seed", ctypes.c_uint64),
                 ("lb_weighted", ctypes.c_int32), ("count_output_bytes", ctypes.c_int32),
-                ("device", ctypes.c_int32)]
+                ("device", ctypes.c_int32), ("op", ctypes.c_int32), ("x2", ctypes.c_void_p)]
 
 
 class PlanStats(ctypes.Structure):
@@ -112,6 +113,9 @@ def lib():
                                 vp], ctypes.c_int),
         "bsm_softmax_noalloc": ([vp, vp, i64, i64, i64, ctypes.c_int, u32, vp], ctypes.c_int),
         "bsm_softmax_host": ([vp, vp, i64, i64, i64, ctypes.c_int, ctypes.c_int, u32, vp], ctypes.c_int),
+        "bsm_softmax_backward": ([vp, vp, vp, i64, i64, i64, ctypes.c_int, ctypes.c_int, vp], ctypes.c_int),
+        "bsm_softmax_backward_ragged": ([vp, vp, vp, i64, c_i64p, c_i32p, c_i32p, ctypes.c_int,
+                                         ctypes.c_int, vp], ctypes.c_int),
         "bsm_plan_desc_init": ([ctypes.POINTER(PlanDesc)], ctypes.c_int),
         "bsm_plan_create": ([ctypes.POINTER(vp), ctypes.POINTER(PlanDesc)], ctypes.c_int),
         "bsm_plan_execute": ([vp, vp], ctypes.c_int),
@@ -210,6 +214,24 @@ def bsm_softmax_noalloc(x, y, B: int, R: int, C: int, dtype: int, flags: int = 0
            "bsm_softmax_noalloc")
 
 
+def bsm_softmax_backward(y, dy, dx, B: int, R: int, C: int, dtype: int, policy: int, stream=None):
+    _check(lib().bsm_softmax_backward(_dptr(y), _dptr(dy), _dptr(dx), B, R, C, dtype, policy,
+                                      _stream(stream)), "bsm_softmax_backward")
+
+
+def bsm_softmax_backward_ragged(y, dy, dx, offsets, rows, cols, dtype: int, policy: int,
+                                stream=None):
+    off = _np(offsets, np.int64)
+    r = _np(rows, np.int32)
+    c = _np(cols, np.int32)
+    if not (len(off) == len(r) == len(c)):
+        raise ValueError("offsets, rows and cols must have the same length")
+    _check(lib().bsm_softmax_backward_ragged(_dptr(y), _dptr(dy), _dptr(dx), len(off),
+                                             off.ctypes.data_as(c_i64p), r.ctypes.data_as(c_i32p),
+                                             c.ctypes.data_as(c_i32p), dtype, policy,
+                                             _stream(stream)), "bsm_softmax_backward_ragged")
+
+
 def bsm_softmax_ragged(x, y, offsets, rows, cols, dtype: int, policy: int, flags: int = 0,
                        stream=None):
     off = _np(offsets, np.int64)
@@ -251,7 +273,7 @@ class Plan:
 def bsm_plan_create(x, y, rows, cols, dtype: int, policy: int, offsets=None, flags: int = 0,
                     rows_per_item: int = 0, tie_seed: Optional[int] = None,
                     lb_weighted: bool = True, count_output_bytes: bool = True,
-                    device: int = -1) -> Plan:
+                    device: int = -1, op: int = 0, x2=None) -> Plan:
     d = PlanDesc()
     _check(lib().bsm_plan_desc_init(ctypes.byref(d)), "bsm_plan_desc_init")
     r = _np(rows, np.int32)
@@ -273,9 +295,11 @@ def bsm_plan_create(x, y, rows, cols, dtype: int, policy: int, offsets=None, fla
     d.lb_weighted = 1 if lb_weighted else 0
     d.count_output_bytes = 1 if count_output_bytes else 0
     d.device = device
+    d.op = op
+    d.x2 = _dptr(x2)
     h = ctypes.c_void_p()
     _check(lib().bsm_plan_create(ctypes.byref(h), ctypes.byref(d)), "bsm_plan_create")
-    return Plan(h.value, (x, y))
+    return Plan(h.value, (x, y, x2))
 
 
 def bsm_plan_execute(plan: Plan, stream=None):

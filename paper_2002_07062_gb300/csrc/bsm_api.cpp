@@ -114,6 +114,7 @@ struct bsm_plan {
     int device = 0;
     int policy = 0;
     int dtype = 0;
+    int op = 0;
     bsm::KernelArgs args{};
     int grid = 0;
     struct Launch {
@@ -149,12 +150,16 @@ int validate(const bsm_plan_desc *d, const DeviceCtx &c, std::vector<SliceView> 
         return BSM_ERR_INVALID_ARG;
     if (d->flags & ~BSM_FLAG_CAUSAL)
         return BSM_ERR_INVALID_ARG;
+    if (d->op != BSM_OP_FORWARD && d->op != BSM_OP_BACKWARD)
+        return BSM_ERR_INVALID_ARG;
+    if (d->op == BSM_OP_BACKWARD && d->flags)
+        return BSM_ERR_INVALID_ARG;
     if (d->num_slices < 0 || d->rows_per_item < 0)
         return BSM_ERR_INVALID_ARG;
     if (d->num_slices > 0 && (!d->rows || !d->cols))
         return BSM_ERR_INVALID_ARG;
     const int es = esize(d->dtype);
-    const int64_t row_limit = max_row_bytes_for(c);
+    const int64_t row_limit = max_row_bytes_for(c) / (d->op == BSM_OP_BACKWARD ? 2 : 1);
     slices.clear();
     slices.reserve(static_cast<size_t>(d->num_slices));
     total_elems = 0;
@@ -193,6 +198,15 @@ int validate(const bsm_plan_desc *d, const DeviceCtx &c, std::vector<SliceView> 
             return BSM_ERR_INVALID_ARG;   // partial overlap
         if ((xa & 15) || (ya & 15))
             misaligned = true;
+        if (d->op == BSM_OP_BACKWARD) {
+            if (!d->x2)
+                return BSM_ERR_INVALID_ARG;
+            const uintptr_t ga = reinterpret_cast<uintptr_t>(d->x2);
+            if (ga != ya && ga < ya + len && ya < ga + len)
+                return BSM_ERR_INVALID_ARG;
+            if (ga & 15)
+                misaligned = true;
+        }
     }
     if (misaligned)
         return BSM_ERR_MISALIGNED;
@@ -237,7 +251,8 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
 
     // ---- stages: one CTA per SM, as many stages as fit the shared memory
     const int64_t avail = c->smem_optin - kSmemHeader;
-    const int64_t stage = std::max<int64_t>(kMinStageBytes, (max_row + 127) & ~int64_t(127));
+    const int in_arrays = d->op == BSM_OP_BACKWARD ? 2 : 1;   // inputs sharing a stage
+    const int64_t stage = std::max<int64_t>(kMinStageBytes, in_arrays * ((max_row + 127) & ~int64_t(127)));
     const int n_stages = static_cast<int>(std::min<int64_t>(kMaxStages, avail / stage));
     if (n_stages < 2)
         return BSM_ERR_UNSUPPORTED;
@@ -265,7 +280,7 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
         if (v.R > 0) {
             const int64_t seg_rows = int64_t(v.R) * static_cast<int64_t>(e - s);
             const int64_t row_bytes = int64_t(v.C) * es;
-            int64_t rpi = std::max<int64_t>(1, stage / row_bytes);
+            int64_t rpi = std::max<int64_t>(1, stage / in_arrays / row_bytes);
             if (d->rows_per_item > 0)
                 rpi = std::min<int64_t>(rpi, d->rows_per_item);
             if (d->policy == BSM_POLICY_WHOLE_GPU)
@@ -288,6 +303,7 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     p->device = device;
     p->policy = d->policy;
     p->dtype = d->dtype;
+    p->op = d->op;
     p->x = d->x;
     p->y = d->y;
     p->flags = d->flags;
@@ -476,6 +492,7 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
 
     KernelArgs &a = p->args;
     a.x = d->x;
+    a.x2 = d->op == BSM_OP_BACKWARD ? d->x2 : nullptr;
     a.y = d->y;
     a.total_elems = total;
     a.items = reinterpret_cast<const Item *>(b + o_items);
@@ -540,11 +557,11 @@ int plan_execute_impl(const bsm_plan *p, bsm_stream_t stream)
         for (const auto &l : p->whole_gpu) {
             a.item_begin = l.begin;
             a.item_end = l.end;
-            if ((err = launch_softmax(a, p->dtype, l.grid, stream, checked)))
+            if ((err = launch_softmax(a, p->dtype, p->op, l.grid, stream, checked)))
                 break;
         }
     } else {
-        err = launch_softmax(p->args, p->dtype, p->grid, stream, checked);
+        err = launch_softmax(p->args, p->dtype, p->op, p->grid, stream, checked);
     }
     if (prev >= 0 && prev != p->device)
         cudaSetDevice(prev);
@@ -559,6 +576,8 @@ struct CacheKey {
     void *y;
     int dtype, policy;
     uint32_t flags;
+    int op;
+    const void *x2;
 };
 
 std::mutex g_cache_mu;
@@ -568,7 +587,7 @@ constexpr size_t kCacheMax = 32;
 bool same_key(const bsm_plan *p, const CacheKey &k)
 {
     return p->device == k.device && p->x == k.x && p->y == k.y && p->dtype == k.dtype &&
-           p->policy == k.policy && p->flags == k.flags;
+           p->policy == k.policy && p->flags == k.flags && p->op == k.op && p->args.x2 == k.x2;
 }
 
 int cached_run(const CacheKey &k, int64_t B, int64_t R, int64_t C, int64_t n, const int64_t *off,
@@ -601,6 +620,8 @@ int cached_run(const CacheKey &k, int64_t B, int64_t R, int64_t C, int64_t n, co
     d.policy = k.policy;
     d.flags = k.flags;
     d.device = k.device;
+    d.op = k.op;
+    d.x2 = k.x2;
     std::vector<int32_t> r, c;
     if (B >= 0) {
         if (B > INT32_MAX || R > INT32_MAX || C > INT32_MAX)
@@ -732,7 +753,8 @@ void bsm_cache_clear(void)
 }
 
 static int softmax_uniform(const void *x, void *y, int64_t B, int64_t R, int64_t C, int dtype, int policy,
-                           uint32_t flags, bsm_stream_t stream)
+                           uint32_t flags, bsm_stream_t stream, int op = BSM_OP_FORWARD,
+                           const void *x2 = nullptr)
 {
     if (B < 0 || R < 0 || C < 1)
         return BSM_ERR_INVALID_ARG;
@@ -747,7 +769,7 @@ static int softmax_uniform(const void *x, void *y, int64_t B, int64_t R, int64_t
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess)
         return BSM_ERR_NO_DEVICE;
-    CacheKey k{dev, x, y, dtype, policy, flags};
+    CacheKey k{dev, x, y, dtype, policy, flags, op, x2};
     return cached_run(k, B, R, C, 0, nullptr, nullptr, nullptr, stream);
 }
 
@@ -764,7 +786,8 @@ int bsm_softmax_ex(const void *x, void *y, int64_t B, int64_t R, int64_t C, int 
 }
 
 static int softmax_ragged(const void *x, void *y, int64_t n, const int64_t *off, const int32_t *rows,
-                          const int32_t *cols, int dtype, int policy, uint32_t flags, bsm_stream_t stream)
+                          const int32_t *cols, int dtype, int policy, uint32_t flags, bsm_stream_t stream,
+                          int op = BSM_OP_FORWARD, const void *x2 = nullptr)
 {
     if (n < 0 || (n > 0 && (!off || !rows || !cols)))
         return BSM_ERR_INVALID_ARG;
@@ -777,7 +800,7 @@ static int softmax_ragged(const void *x, void *y, int64_t n, const int64_t *off,
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess)
         return BSM_ERR_NO_DEVICE;
-    CacheKey k{dev, x, y, dtype, policy, flags};
+    CacheKey k{dev, x, y, dtype, policy, flags, op, x2};
     return cached_run(k, -1, 0, 0, n, off, rows, cols, stream);
 }
 
@@ -786,6 +809,24 @@ int bsm_softmax_ragged(const void *x, void *y, int64_t num_slices, const int64_t
                        bsm_stream_t stream)
 {
     BSM_GUARD(softmax_ragged(x, y, num_slices, offsets, rows, cols, dtype, policy, flags, stream))
+}
+
+int bsm_softmax_backward(const void *y, const void *dy, void *dx, int64_t B, int64_t R, int64_t C,
+                         int dtype, int policy, bsm_stream_t stream)
+{
+    if (!dy && B > 0 && R > 0)
+        return BSM_ERR_INVALID_ARG;
+    BSM_GUARD(softmax_uniform(y, dx, B, R, C, dtype, policy, 0u, stream, BSM_OP_BACKWARD, dy))
+}
+
+int bsm_softmax_backward_ragged(const void *y, const void *dy, void *dx, int64_t num_slices,
+                                const int64_t *offsets, const int32_t *rows, const int32_t *cols,
+                                int dtype, int policy, bsm_stream_t stream)
+{
+    if (!dy && num_slices > 0)
+        return BSM_ERR_INVALID_ARG;
+    BSM_GUARD(softmax_ragged(y, dx, num_slices, offsets, rows, cols, dtype, policy, 0u, stream,
+                             BSM_OP_BACKWARD, dy))
 }
 
 int bsm_topology_probe(int device, int force, bsm_topology *out)

@@ -40,8 +40,15 @@ constexpr int kThreads = (kConsumerWarps + 1) * 32;  // + one producer warp
 constexpr int kSmemHeader = 1024;                     // barriers + stage metadata
 constexpr int kMinStageBytes = 32 * 1024;
 
+// What the kernel computes on every row.
+enum Op : int32_t {
+    OP_FORWARD = 0,     // y = softmax(x [+ causal mask])
+    OP_BACKWARD = 1     // y = x * (x2 - rowsum(x * x2)): x = softmax output, x2 = its gradient
+};
+
 struct KernelArgs {
     const void *x;
+    const void *x2;             // OP_BACKWARD: the upstream gradient
     void *y;
     int64_t total_elems;        // extent of x and y, elements (bounds checks)
     const Item *items;
@@ -69,7 +76,7 @@ constexpr uint32_t KDEBUG_WITHHOLD_STAGE0 = 1u;   // producer never fills stage 
 
 // Launch the persistent softmax kernel (bsm_kernels.cu).  Returns a
 // cudaError_t value (0 = success).
-int launch_softmax(const KernelArgs &a, int dtype, int grid, void *stream, bool checked);
+int launch_softmax(const KernelArgs &a, int dtype, int op, int grid, void *stream, bool checked);
 // Raise the dynamic shared-memory limit of both kernel instances.
 int kernel_set_smem_limit(int bytes);
 

@@ -497,6 +497,137 @@ __device__ __forceinline__ void row_in_smem_inplace(unsigned char *srow, unsigne
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
+// ------------------------------------------------ backward row routines
+// dx = y * (dy - <y, dy>) of one row; y and dy sit in the two halves of the
+// stage.  The dot product: per vector a balanced tree of y*dy, per lane in
+// vector order, then the butterfly over the lane group.
+
+template <typename Tag, bool Checked, int T, int V>
+__device__ __forceinline__ void row_bwd_registers(const unsigned char *sy, const unsigned char *sdy,
+                                                  unsigned char *dxrow, int nvec, int l, bool valid,
+                                                  const Bounds &by, const Bounds &bdy)
+{
+    using E = Elem<Tag>;
+    constexpr int EPV = E::kPerVec;
+    float yv[V][EPV], dv[V][EPV];
+    float dot = 0.0f;
+#pragma unroll
+    for (int j = 0; j < V; ++j) {
+        const int vi = j * T + l;
+        uint4 ry, rd;
+        if (valid && vi < nvec && load_vec<Checked>(sy + 16 * vi, by, ry) &&
+            load_vec<Checked>(sdy + 16 * vi, bdy, rd)) {
+            E::unpack(ry, yv[j]);
+            E::unpack(rd, dv[j]);
+            float pr[EPV];
+#pragma unroll
+            for (int e = 0; e < EPV; ++e)
+                pr[e] = yv[j][e] * dv[j][e];
+            dot += tree_sum<EPV>(pr);
+        } else {
+#pragma unroll
+            for (int e = 0; e < EPV; ++e)
+                yv[j][e] = dv[j][e] = 0.0f;
+        }
+    }
+    dot = group_sum<T>(dot);
+#pragma unroll
+    for (int j = 0; j < V; ++j) {
+        const int vi = j * T + l;
+        if (valid && vi < nvec) {
+#pragma unroll
+            for (int e = 0; e < EPV; ++e)
+                yv[j][e] = yv[j][e] * (dv[j][e] - dot);
+            store_vec<Checked>(dxrow + 16 * vi, by, E::pack(yv[j]));
+        }
+    }
+}
+
+template <typename Tag, bool Checked>
+__device__ __forceinline__ void row_bwd_smem(const unsigned char *sy, const unsigned char *sdy,
+                                             unsigned char *dxrow, int nvec, int lane, const Bounds &by,
+                                             const Bounds &bdy)
+{
+    using E = Elem<Tag>;
+    constexpr int EPV = E::kPerVec;
+    float yv[EPV], dv[EPV], pr[EPV];
+    uint4 ry, rd;
+    float dot = 0.0f;
+    for (int vi = lane; vi < nvec; vi += 32) {
+        if (!load_vec<Checked>(sy + 16 * vi, by, ry) || !load_vec<Checked>(sdy + 16 * vi, bdy, rd))
+            continue;
+        E::unpack(ry, yv);
+        E::unpack(rd, dv);
+#pragma unroll
+        for (int e = 0; e < EPV; ++e)
+            pr[e] = yv[e] * dv[e];
+        dot += tree_sum<EPV>(pr);
+    }
+    dot = group_sum<32>(dot);
+    for (int vi = lane; vi < nvec; vi += 32) {
+        if (!load_vec<Checked>(sy + 16 * vi, by, ry) || !load_vec<Checked>(sdy + 16 * vi, bdy, rd))
+            continue;
+        E::unpack(ry, yv);
+        E::unpack(rd, dv);
+#pragma unroll
+        for (int e = 0; e < EPV; ++e)
+            yv[e] = yv[e] * (dv[e] - dot);
+        store_vec<Checked>(dxrow + 16 * vi, by, E::pack(yv));
+    }
+}
+
+// Backward rows of a stage, dealt like consume_stage's: groups of G = 32/T
+// rows round robin over the consumer warps from warp `first`.
+template <typename Tag, bool Checked, int T, int V>
+__device__ __forceinline__ int rows_bwd_registers(const unsigned char *sbuf, int half, const StageMeta &mt,
+                                                  unsigned char *ybase, int row_bytes, int nvec, int first,
+                                                  int lane, const Bounds &by, const Bounds &bdy)
+{
+    constexpr int G = 32 / T;
+    const int g = lane / T, l = lane % T;
+    for (int rb = first * G; rb < mt.nrows; rb += G * kConsumerWarps) {
+        const int r = rb + g;
+        row_bwd_registers<Tag, Checked, T, V>(sbuf + (size_t)r * row_bytes, sbuf + half + (size_t)r * row_bytes,
+                                              ybase + (size_t)r * row_bytes, nvec, l, r < mt.nrows, by, bdy);
+    }
+    return (mt.nrows + G - 1) / G;
+}
+
+template <typename Tag, bool Checked>
+__device__ __forceinline__ int consume_stage_bwd(const unsigned char *sbuf, int half, const StageMeta &mt,
+                                                 unsigned char *y, int first, int lane, Bounds by)
+{
+    using E = Elem<Tag>;
+    const int row_bytes = mt.C * E::kSize;
+    const int nvec = row_bytes >> 4;
+    unsigned char *ybase = y + mt.off * E::kSize;
+    by.s_lo = sbuf;
+    by.s_hi = sbuf + (size_t)mt.nrows * row_bytes;
+    Bounds bdy = by;
+    bdy.s_lo = sbuf + half;
+    bdy.s_hi = sbuf + half + (size_t)mt.nrows * row_bytes;
+    constexpr int VMAX = 16 / E::kPerVec;   // y and dy: at most 32 floats per lane
+    if (nvec <= 8)
+        return rows_bwd_registers<Tag, Checked, 8, 1>(sbuf, half, mt, ybase, row_bytes, nvec, first, lane, by,
+                                                      bdy);
+    if (nvec <= 16)
+        return rows_bwd_registers<Tag, Checked, 8, 2>(sbuf, half, mt, ybase, row_bytes, nvec, first, lane, by,
+                                                      bdy);
+    if (nvec <= 32)
+        return rows_bwd_registers<Tag, Checked, 16, 2>(sbuf, half, mt, ybase, row_bytes, nvec, first, lane, by,
+                                                       bdy);
+    if (nvec <= 64)
+        return rows_bwd_registers<Tag, Checked, 32, 2>(sbuf, half, mt, ybase, row_bytes, nvec, first, lane, by,
+                                                       bdy);
+    if (VMAX >= 4 && nvec <= 128)
+        return rows_bwd_registers<Tag, Checked, 32, (VMAX >= 4 ? 4 : 2)>(sbuf, half, mt, ybase, row_bytes, nvec,
+                                                                         first, lane, by, bdy);
+    for (int r = first; r < mt.nrows; r += kConsumerWarps)
+        row_bwd_smem<Tag, Checked>(sbuf + (size_t)r * row_bytes, sbuf + half + (size_t)r * row_bytes,
+                                   ybase + (size_t)r * row_bytes, nvec, lane, by, bdy);
+    return mt.nrows;
+}
+
 // The rows of a stage handled by one register routine: groups of T lanes,
 // G = 32/T rows per group of a warp.  Row groups are dealt to the consumer
 // warps round robin, starting at warp `first` (see consume_stage); q tracks
@@ -649,7 +780,7 @@ struct Puller {
     }
 };
 
-template <typename Tag, bool Checked>
+template <typename Tag, int Op, bool Checked>
 __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelArgs a)
 {
     using E = Elem<Tag>;
@@ -721,10 +852,11 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                     const Item item = batch[j];
                     const int64_t ne = (int64_t)item.nrows * item.C;
                     const int64_t nbytes = ne * E::kSize;
+                    const int64_t cap = Op == OP_BACKWARD ? a.stage_bytes / 2 : a.stage_bytes;
                     const bool ok = pos[j] >= 0 && pos[j] < a.n_items && item.off >= 0 && item.C > 0 &&
                                     item.nrows > 0 && item.R > 0 && item.row0 >= 0 &&
                                     item.row0 < item.R && item.off + ne <= a.total_elems &&
-                                    nbytes <= a.stage_bytes && (nbytes & 15) == 0 &&
+                                    nbytes <= cap && (nbytes & 15) == 0 &&
                                     ((item.off * E::kSize) & 15) == 0;
                     if (!ok) {
                         atomicOr(a.status, BSM_DEV_BOUNDS);
@@ -741,13 +873,22 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                     const uint32_t bytes = static_cast<uint32_t>(nbytes);
                     unsigned char *dst = stages + (size_t)s * a.stage_bytes;
                     const unsigned char *src = static_cast<const unsigned char *>(a.x) + item.off * E::kSize;
+                    const int half = a.stage_bytes / 2;
+                    const unsigned char *src2 =
+                        Op == OP_BACKWARD ? static_cast<const unsigned char *>(a.x2) + item.off * E::kSize : nullptr;
                     if (Checked) {
                         const unsigned char *x0 = static_cast<const unsigned char *>(a.x);
-                        const bool bad = s < 0 || s >= S || S > kMaxStages ||
-                                         src < x0 || src + bytes > x0 + a.total_elems * E::kSize ||
-                                         (reinterpret_cast<uintptr_t>(src) & 15) ||
-                                         (smem_addr(dst) & 15) || (bytes & 15) || bytes == 0 ||
-                                         dst + bytes > smem + kSmemHeader + (size_t)S * a.stage_bytes;
+                        bool bad = s < 0 || s >= S || S > kMaxStages ||
+                                   src < x0 || src + bytes > x0 + a.total_elems * E::kSize ||
+                                   (reinterpret_cast<uintptr_t>(src) & 15) ||
+                                   (smem_addr(dst) & 15) || (bytes & 15) || bytes == 0 ||
+                                   dst + bytes > smem + kSmemHeader + (size_t)S * a.stage_bytes;
+                        if (Op == OP_BACKWARD) {
+                            const unsigned char *g0 = static_cast<const unsigned char *>(a.x2);
+                            bad = bad || bytes > (uint32_t)half || src2 < g0 ||
+                                  src2 + bytes > g0 + a.total_elems * E::kSize ||
+                                  (reinterpret_cast<uintptr_t>(src2) & 15) || (half & 15);
+                        }
                         if (bad) {
                             check_fail(a.status, 3, static_cast<uint64_t>(pos[j]), bytes);
                             mt.kind = KIND_SKIP;
@@ -755,8 +896,14 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                             continue;
                         }
                     }
-                    mbar_arrive_expect_tx(&h.full[s], bytes);
-                    bulk_load(dst, src, bytes, &h.full[s]);
+                    if (Op == OP_BACKWARD) {
+                        mbar_arrive_expect_tx(&h.full[s], 2 * bytes);
+                        bulk_load(dst, src, bytes, &h.full[s]);
+                        bulk_load(dst + half, src2, bytes, &h.full[s]);
+                    } else {
+                        mbar_arrive_expect_tx(&h.full[s], bytes);
+                        bulk_load(dst, src, bytes, &h.full[s]);
+                    }
                     issued[s] = true;
                     issued_phase[s] = ph;
                 }
@@ -803,15 +950,19 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
             break;
         if (mt.kind == KIND_DATA) {
             Bounds bd{nullptr, nullptr, y, y + a.total_elems * E::kSize, a.status};
-            if (Checked && (mt.nrows <= 0 || mt.C <= 0 ||
-                            (int64_t)mt.nrows * mt.C * E::kSize > a.stage_bytes)) {
+            const int64_t cap = Op == OP_BACKWARD ? a.stage_bytes / 2 : a.stage_bytes;
+            if (Checked && (mt.nrows <= 0 || mt.C <= 0 || (int64_t)mt.nrows * mt.C * E::kSize > cap)) {
                 if (lane == 0)
                     check_fail(a.status, 4, static_cast<uint64_t>(mt.nrows), static_cast<uint64_t>(mt.C));
             } else {
                 const int first = static_cast<int>((warp + kConsumerWarps - groups_seen % kConsumerWarps) %
                                                    kConsumerWarps);
-                groups_seen += consume_stage<Tag, Checked>(stages + (size_t)s * a.stage_bytes, mt, y, causal,
-                                                           first, lane, bd);
+                if constexpr (Op == OP_BACKWARD)
+                    groups_seen += consume_stage_bwd<Tag, Checked>(stages + (size_t)s * a.stage_bytes,
+                                                                   a.stage_bytes / 2, mt, y, first, lane, bd);
+                else
+                    groups_seen += consume_stage<Tag, Checked>(stages + (size_t)s * a.stage_bytes, mt, y,
+                                                               causal, first, lane, bd);
             }
         }
         __syncwarp();
@@ -824,10 +975,15 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
 
 int kernel_set_smem_limit(int bytes)
 {
-    const void *fns[] = {reinterpret_cast<const void *>(softmax_persistent<F32, false>),
-                         reinterpret_cast<const void *>(softmax_persistent<BF16, false>),
-                         reinterpret_cast<const void *>(softmax_persistent<F32, true>),
-                         reinterpret_cast<const void *>(softmax_persistent<BF16, true>)};
+    const void *fns[] = {
+        reinterpret_cast<const void *>(softmax_persistent<F32, OP_FORWARD, false>),
+        reinterpret_cast<const void *>(softmax_persistent<BF16, OP_FORWARD, false>),
+        reinterpret_cast<const void *>(softmax_persistent<F32, OP_FORWARD, true>),
+        reinterpret_cast<const void *>(softmax_persistent<BF16, OP_FORWARD, true>),
+        reinterpret_cast<const void *>(softmax_persistent<F32, OP_BACKWARD, false>),
+        reinterpret_cast<const void *>(softmax_persistent<BF16, OP_BACKWARD, false>),
+        reinterpret_cast<const void *>(softmax_persistent<F32, OP_BACKWARD, true>),
+        reinterpret_cast<const void *>(softmax_persistent<BF16, OP_BACKWARD, true>)};
     for (const void *f : fns) {
         cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
         if (e != cudaSuccess)
@@ -836,20 +992,31 @@ int kernel_set_smem_limit(int bytes)
     return 0;
 }
 
-int launch_softmax(const KernelArgs &a, int dtype, int grid, void *stream, bool checked)
+namespace {
+template <typename Tag, int Op>
+void launch_one(const KernelArgs &a, int grid, size_t smem, cudaStream_t st, bool checked)
+{
+    if (checked)
+        softmax_persistent<Tag, Op, true><<<grid, kThreads, smem, st>>>(a);
+    else
+        softmax_persistent<Tag, Op, false><<<grid, kThreads, smem, st>>>(a);
+}
+}  // namespace
+
+int launch_softmax(const KernelArgs &a, int dtype, int op, int grid, void *stream, bool checked)
 {
     const size_t smem = kSmemHeader + (size_t)a.n_stages * a.stage_bytes;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    if (dtype == BSM_F32) {
-        if (checked)
-            softmax_persistent<F32, true><<<grid, kThreads, smem, st>>>(a);
+    if (op == OP_BACKWARD) {
+        if (dtype == BSM_F32)
+            launch_one<F32, OP_BACKWARD>(a, grid, smem, st, checked);
         else
-            softmax_persistent<F32, false><<<grid, kThreads, smem, st>>>(a);
+            launch_one<BF16, OP_BACKWARD>(a, grid, smem, st, checked);
     } else {
-        if (checked)
-            softmax_persistent<BF16, true><<<grid, kThreads, smem, st>>>(a);
+        if (dtype == BSM_F32)
+            launch_one<F32, OP_FORWARD>(a, grid, smem, st, checked);
         else
-            softmax_persistent<BF16, false><<<grid, kThreads, smem, st>>>(a);
+            launch_one<BF16, OP_FORWARD>(a, grid, smem, st, checked);
     }
     return static_cast<int>(cudaGetLastError());
 }

@@ -160,7 +160,7 @@ int softmax_noalloc(const void *x, void *y, int64_t B, int64_t R, int64_t C, int
     a.n_stages = n_stages;
     a.flags = flags;
     a.status = status;
-    if (int e = launch_softmax(a, dtype, nd->n_sm, stream, false))
+    if (int e = launch_softmax(a, dtype, OP_FORWARD, nd->n_sm, stream, false))
         return record_cuda_error(e, "noalloc kernel launch");
     return BSM_OK;
 }
