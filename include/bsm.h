@@ -45,8 +45,11 @@
  *     BSM_ERR_MISALIGNED.
  *   - In place (x == y) is allowed; partially overlapping x and y are not
  *     (BSM_ERR_INVALID_ARG).
- *   - Row length limit: C * element size <= bsm_max_row_bytes() (a row must
- *     fit one shared-memory stage), else BSM_ERR_UNSUPPORTED.
+ *   - Row length: a row of up to bsm_max_row_bytes() is read once from one
+ *     shared-memory stage.  Longer rows (forward only) stream through the
+ *     stages in chunks twice -- a running maximum and rescaled sum, then the
+ *     output -- so they cost one extra read; the backward pass rejects rows
+ *     over half of bsm_max_row_bytes() with BSM_ERR_UNSUPPORTED.
  */
 #ifndef BSM_H
 #define BSM_H
@@ -65,7 +68,7 @@ typedef enum {
     BSM_OK = 0,
     BSM_ERR_INVALID_ARG = 1,   /* null / negative / inconsistent arguments */
     BSM_ERR_MISALIGNED = 2,    /* 16-byte alignment rule broken */
-    BSM_ERR_UNSUPPORTED = 3,   /* row too long for a stage, too many patches */
+    BSM_ERR_UNSUPPORTED = 3,   /* backward row too long for a stage, too many patches */
     BSM_ERR_CUDA = 4,          /* a CUDA runtime call failed */
     BSM_ERR_DEVICE_BOUNDS = 5, /* a kernel met a patch outside the buffers */
     BSM_ERR_TIMEOUT = 6,       /* a kernel wait gave up after its time limit */
@@ -255,6 +258,7 @@ typedef struct {
     int32_t steal;              /* 1 if CTAs steal from other dies' queues */
     int64_t map_chunk_bytes;    /* granularity of the address->die map used */
     double plan_ms;             /* host time spent in bsm_plan_create */
+    int64_t long_items;         /* rows longer than a stage (streamed in two passes) */
 } bsm_plan_stats;
 
 int bsm_plan_get_stats(const bsm_plan *plan, bsm_plan_stats *out);
@@ -380,7 +384,8 @@ void bsm_set_device_checks(int on);
  * the same thread. */
 const char *bsm_last_cuda_error(void);
 
-/* Largest row (C * element size) a plan accepts on this device, bytes. */
+/* Largest row (C * element size) processed from a single shared-memory stage
+ * on this device, bytes; longer forward rows take two passes. */
 int64_t bsm_max_row_bytes(int device);
 
 /* Static description of a status code. */

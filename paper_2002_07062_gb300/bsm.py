@@ -66,7 +66,8 @@ class PlanStats(ctypes.Structure):
                 ("est_finish_after", ctypes.c_double * MAX_DIES),
                 ("stage_bytes", ctypes.c_int32), ("n_stages", ctypes.c_int32),
                 ("grid", ctypes.c_int32), ("launches", ctypes.c_int32), ("steal", ctypes.c_int32),
-                ("map_chunk_bytes", ctypes.c_int64), ("plan_ms", ctypes.c_double)]
+                ("map_chunk_bytes", ctypes.c_int64), ("plan_ms", ctypes.c_double),
+                ("long_items", ctypes.c_int64)]
 
 
 class Topology(ctypes.Structure):

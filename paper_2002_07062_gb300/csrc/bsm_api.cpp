@@ -182,8 +182,8 @@ int validate(const bsm_plan_desc *d, const DeviceCtx &c, std::vector<SliceView> 
         if (R > 0) {
             if ((C * es) % 16 != 0 || (off * es) % 16 != 0)
                 misaligned = true;
-            if (C * es > row_limit)
-                too_long = true;
+            if (d->op == BSM_OP_BACKWARD && C * es > row_limit)
+                too_long = true;   // forward rows of any length stream in two passes
             max_row_bytes = std::max(max_row_bytes, C * es);
             total_elems = std::max(total_elems, off + n);
         }
@@ -252,7 +252,10 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     // ---- stages: one CTA per SM, as many stages as fit the shared memory
     const int64_t avail = c->smem_optin - kSmemHeader;
     const int in_arrays = d->op == BSM_OP_BACKWARD ? 2 : 1;   // inputs sharing a stage
-    const int64_t stage = std::max<int64_t>(kMinStageBytes, in_arrays * ((max_row + 127) & ~int64_t(127)));
+    // a stage holds the longest row, up to half the shared memory; longer
+    // (forward) rows go through the stages in chunks, twice
+    const int64_t row_cap = std::min<int64_t>((max_row + 127) & ~int64_t(127), max_row_bytes_for(*c));
+    const int64_t stage = std::max<int64_t>(kMinStageBytes, in_arrays * row_cap);
     const int n_stages = static_cast<int>(std::min<int64_t>(kMaxStages, avail / stage));
     if (n_stages < 2)
         return BSM_ERR_UNSUPPORTED;
@@ -265,11 +268,14 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
                           d->policy == BSM_POLICY_CBMF_LB;
     std::vector<Item> items;
     std::vector<int32_t> slice_first(slices.size() + 1, 0);
+    int64_t long_rows = 0;
     size_t s = 0;
     while (s < slices.size()) {
         slice_first[s] = static_cast<int32_t>(items.size());
         const SliceView &v = slices[s];
         size_t e = s + 1;
+        if (int64_t(v.C) * es > stage / in_arrays)
+            long_rows += v.R;
         if (spanning && v.R > 0) {
             while (e < slices.size() && slices[e].R == v.R && slices[e].C == v.C &&
                    slices[e].off == slices[e - 1].off + int64_t(v.R) * v.C) {
@@ -314,6 +320,7 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     st.n_items = n_items;
     st.stage_bytes = static_cast<int32_t>(stage);
     st.n_stages = n_stages;
+    st.long_items = long_rows;
 
     // ---- the schedule
     std::vector<int32_t> queue;      // schedule order of the patches (queue policies)
@@ -938,7 +945,7 @@ const char *bsm_status_string(int status)
     case BSM_ERR_MISALIGNED:
         return "misaligned: pointers, slice offsets and row lengths must be multiples of 16 bytes";
     case BSM_ERR_UNSUPPORTED:
-        return "unsupported: row longer than a shared-memory stage, or too many patches";
+        return "unsupported: backward row longer than half a shared-memory stage, or too many patches";
     case BSM_ERR_CUDA:
         return "CUDA runtime error";
     case BSM_ERR_DEVICE_BOUNDS:

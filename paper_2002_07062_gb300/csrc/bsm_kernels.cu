@@ -40,23 +40,28 @@ namespace {
 constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s
 constexpr float kLog2e = 1.4426950408889634f;
 
-enum : int32_t { KIND_DATA = 0, KIND_SKIP = 1, KIND_DONE = 2 };
+enum : int32_t { KIND_DATA = 0, KIND_SKIP = 1, KIND_DONE = 2, KIND_LONG = 3 };
 
 struct alignas(16) StageMeta {
     int64_t off;
-    int32_t C;
+    int32_t C;          // KIND_LONG: elements of this chunk of the row
     int32_t nrows;
     int32_t row0;
     int32_t kind;
     int32_t R;
-    int32_t pad;
+    int32_t col0;       // KIND_LONG: column of the chunk's first element
+    int32_t pass;       // KIND_LONG: 0 = max and sum, 1 = write
+    int32_t last;       // KIND_LONG: last chunk of its pass
+    int32_t pad[2];
 };
-static_assert(sizeof(StageMeta) == 32, "StageMeta layout");
+static_assert(sizeof(StageMeta) == 48, "StageMeta layout");
 
 struct SmemHeader {
     uint64_t full[kMaxStages];
     uint64_t empty[kMaxStages];
+    uint64_t xwarp;                 // long rows: the consumer warps' partials are in
     StageMeta meta[kMaxStages];
+    float2 partial[2][kConsumerWarps];   // long rows: (max, sum) per warp, two rows deep
     int32_t abort_flag;
 };
 static_assert(sizeof(SmemHeader) <= kSmemHeader, "header too large");
@@ -628,6 +633,66 @@ __device__ __forceinline__ int consume_stage_bwd(const unsigned char *sbuf, int 
     return mt.nrows;
 }
 
+// ------------------------------------------------------------ long rows
+// A row longer than a stage is streamed through the stages twice, in
+// chunks; all consumer warps share every chunk (warp w takes the vectors
+// w*32 + lane, + 512, ...).  Pass 0 keeps a running (max m, sum s of
+// exp(v - m)) per lane -- when the max grows, s is rescaled by exp(m_old -
+// m_new) -- then the lanes, the warps (through shared memory) combine their
+// pairs in a fixed order; pass 1 writes exp(v - m) / s.
+
+// (m, s) of two partials; a -inf maximum contributes nothing.
+__device__ __forceinline__ void combine_ms(float &m, float &s, float mo, float so)
+{
+    const float mn = fmaxf(m, mo);
+    const float fa = m == mn ? 1.0f : ex2((m - mn) * kLog2e);
+    const float fb = mo == mn ? 1.0f : ex2((mo - mn) * kLog2e);
+    s = s * fa + so * fb;
+    m = mn;
+}
+
+template <typename Tag, bool Checked>
+__device__ __forceinline__ void long_chunk(const unsigned char *sbuf, const StageMeta &mt, unsigned char *y,
+                                           bool causal, int warp, int lane, Bounds bd, float &m_l,
+                                           float &s_l, float mL, float inv)
+{
+    using E = Elem<Tag>;
+    constexpr int EPV = E::kPerVec;
+    const int nvec = (mt.C * E::kSize) >> 4;
+    bd.s_lo = sbuf;
+    bd.s_hi = sbuf + (size_t)mt.C * E::kSize;
+    unsigned char *ybase = y + mt.off * E::kSize;
+    const int row = mt.row0;
+    for (int vi = warp * 32 + lane; vi < nvec; vi += kConsumerWarps * 32) {
+        uint4 raw;
+        if (!load_vec<Checked>(sbuf + 16 * vi, bd, raw))
+            continue;
+        float v[EPV];
+        E::unpack(raw, v);
+        const int col = mt.col0 + vi * EPV;
+        const bool masked = causal && col > row;
+        if (causal && !masked && col + EPV - 1 > row)
+            apply_causal<EPV>(v, col, row);
+        if (mt.pass == 0) {
+            if (!masked) {
+                const float vm = tree_max<EPV>(v);
+                if (vm > m_l) {
+                    s_l *= ex2((m_l - vm) * kLog2e);
+                    m_l = vm;
+                }
+            }
+            vec_exp<EPV>(v, m_l * kLog2e, masked);
+            s_l += tree_sum<EPV>(v);
+        } else {
+            vec_exp<EPV>(v, mL, masked);
+#pragma unroll
+            for (int e = 0; e < EPV; ++e)
+                v[e] *= inv;
+            store_vec<Checked>(ybase + 16 * vi, bd, E::pack(v));
+        }
+    }
+}
+
 // The rows of a stage handled by one register routine: groups of T lanes,
 // G = 32/T rows per group of a warp.  Row groups are dealt to the consumer
 // warps round robin, starting at warp `first` (see consume_stage); q tracks
@@ -781,7 +846,7 @@ struct Puller {
 };
 
 template <typename Tag, int Op, bool Checked>
-__global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelArgs a)
+__global__ void __maxnreg__(120) softmax_persistent(const KernelArgs a)
 {
     using E = Elem<Tag>;
     extern __shared__ __align__(1024) unsigned char smem[];
@@ -796,6 +861,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
             mbar_init(&h.full[s], 1);
             mbar_init(&h.empty[s], kConsumerWarps);
         }
+        mbar_init(&h.xwarp, kConsumerWarps);
         h.abort_flag = 0;
         mbar_init_fence();
     }
@@ -811,6 +877,18 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                 issued[s] = false;
             bool aborted = false, done = false;
             uint32_t it = 0;
+            // take the next stage of the ring once the consumers released it
+            auto next_stage = [&](int &s, uint32_t &ph) -> bool {
+                s = static_cast<int>(it % S);
+                ph = (it / S) & 1u;
+                if (!mbar_wait_bounded(&h.empty[s], ph ^ 1u, &h.abort_flag, wait_limit)) {
+                    aborted = true;
+                    return false;
+                }
+                issued[s] = false;
+                ++it;
+                return true;
+            };
             while (!done && !aborted) {
                 // fetch the next patches: their records load in parallel
                 int32_t pos[kFetch];
@@ -822,30 +900,20 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                         batch[j] = a.items[pos[j]];
                 if (n == 0) {
                     // no more work: tell the consumers through the next stage
-                    const int s = it % S;
-                    const uint32_t ph = (it / S) & 1u;
-                    if (!mbar_wait_bounded(&h.empty[s], ph ^ 1u, &h.abort_flag, wait_limit)) {
-                        aborted = true;
+                    int s = 0;
+                    uint32_t ph = 0;
+                    if (!next_stage(s, ph))
                         break;
-                    }
-                    issued[s] = false;
                     h.meta[s].kind = KIND_DONE;
                     mbar_arrive(&h.full[s]);
                     done = true;
                     break;
                 }
-#pragma unroll
-                for (int j = 0; j < kFetch; ++j) {
-                    if (j >= n)
+                for (int j = 0; j < n && !aborted; ++j) {
+                    int s = 0;
+                    uint32_t ph = 0;
+                    if (!next_stage(s, ph))
                         break;
-                    const int s = it % S;
-                    const uint32_t ph = (it / S) & 1u;
-                    if (!mbar_wait_bounded(&h.empty[s], ph ^ 1u, &h.abort_flag, wait_limit)) {
-                        aborted = true;
-                        break;
-                    }
-                    issued[s] = false;                 // the consumers released it
-                    ++it;
                     StageMeta &mt = h.meta[s];
                     if ((a.debug & KDEBUG_WITHHOLD_STAGE0) && it == 1)
                         continue;                      // test hook: stage 0 is never filled
@@ -853,15 +921,48 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                     const int64_t ne = (int64_t)item.nrows * item.C;
                     const int64_t nbytes = ne * E::kSize;
                     const int64_t cap = Op == OP_BACKWARD ? a.stage_bytes / 2 : a.stage_bytes;
+                    const bool is_long = Op == OP_FORWARD && nbytes > cap && item.nrows == 1;
                     const bool ok = pos[j] >= 0 && pos[j] < a.n_items && item.off >= 0 && item.C > 0 &&
                                     item.nrows > 0 && item.R > 0 && item.row0 >= 0 &&
                                     item.row0 < item.R && item.off + ne <= a.total_elems &&
-                                    nbytes <= cap && (nbytes & 15) == 0 &&
+                                    (nbytes <= cap || is_long) && (nbytes & 15) == 0 &&
                                     ((item.off * E::kSize) & 15) == 0;
                     if (!ok) {
                         atomicOr(a.status, BSM_DEV_BOUNDS);
                         mt.kind = KIND_SKIP;
                         mbar_arrive(&h.full[s]);
+                        continue;
+                    }
+                    if (is_long) {
+                        // the row in chunks of one stage, twice
+                        const int64_t chunk = cap / E::kSize;
+                        const int64_t nch = (item.C + chunk - 1) / chunk;
+                        bool first = true;
+                        for (int pass = 0; pass < 2 && !aborted; ++pass)
+                            for (int64_t k = 0; k < nch; ++k) {
+                                if (!first && !next_stage(s, ph))
+                                    break;
+                                first = false;
+                                StageMeta &lm = h.meta[s];
+                                const int64_t c0 = k * chunk;
+                                const int64_t cn = item.C - c0 < chunk ? item.C - c0 : chunk;
+                                lm.off = item.off + c0;
+                                lm.C = static_cast<int32_t>(cn);
+                                lm.nrows = 1;
+                                lm.row0 = item.row0;
+                                lm.R = item.R;
+                                lm.col0 = static_cast<int32_t>(c0);
+                                lm.pass = pass;
+                                lm.last = k == nch - 1;
+                                lm.kind = KIND_LONG;
+                                const uint32_t cb = static_cast<uint32_t>(cn * E::kSize);
+                                mbar_arrive_expect_tx(&h.full[s], cb);
+                                bulk_load(stages + (size_t)s * a.stage_bytes,
+                                          static_cast<const unsigned char *>(a.x) + (item.off + c0) * E::kSize,
+                                          cb, &h.full[s]);
+                                issued[s] = true;
+                                issued_phase[s] = ph;
+                            }
                         continue;
                     }
                     mt.off = item.off;
@@ -935,6 +1036,10 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
     const bool causal = (a.flags & BSM_FLAG_CAUSAL) != 0;
     unsigned char *y = static_cast<unsigned char *>(a.y);
     uint32_t groups_seen = 0;   // row groups dealt so far (the same count in every warp)
+    // long rows: this lane's running (max, sum); the row's final exponent
+    // offset and reciprocal; which partial buffer and barrier phase is next
+    float m_l = -INFINITY, s_l = 0.0f, long_mL = 0.0f, long_inv = 0.0f;
+    uint32_t long_rows = 0;
     for (uint32_t it = 0;; ++it) {
         const int s = it % S;
         const uint32_t ph = (it / S) & 1u;
@@ -948,6 +1053,46 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
         const StageMeta mt = h.meta[s];
         if (mt.kind == KIND_DONE)
             break;
+        if (Op == OP_FORWARD && mt.kind == KIND_LONG) {
+            Bounds bd{nullptr, nullptr, y, y + a.total_elems * E::kSize, a.status};
+            long_chunk<Tag, Checked>(stages + (size_t)s * a.stage_bytes, mt, y, causal, warp, lane, bd, m_l,
+                                     s_l, long_mL, long_inv);
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(&h.empty[s]);
+            if (mt.pass == 0 && mt.last) {
+                // lanes, then warps: every warp ends with the same (m, s)
+#pragma unroll
+                for (int o = 16; o >= 1; o >>= 1) {
+                    const float mo = __shfl_xor_sync(0xFFFFFFFFu, m_l, o);
+                    const float so = __shfl_xor_sync(0xFFFFFFFFu, s_l, o);
+                    combine_ms(m_l, s_l, mo, so);
+                }
+                const int par = long_rows & 1;
+                if (lane == 0) {
+                    h.partial[par][warp] = make_float2(m_l, s_l);
+                    mbar_arrive(&h.xwarp);
+                }
+                if (!mbar_wait_bounded(&h.xwarp, long_rows & 1u, &h.abort_flag, wait_limit)) {
+                    if (lane == 0) {
+                        atomicOr(a.status, BSM_DEV_TIMEOUT);
+                        h.abort_flag = 1;
+                    }
+                    break;
+                }
+                float m = -INFINITY, sum = 0.0f;
+                for (int w = 0; w < kConsumerWarps; ++w) {
+                    const float2 pw = h.partial[par][w];
+                    combine_ms(m, sum, pw.x, pw.y);
+                }
+                long_mL = m * kLog2e;
+                long_inv = __frcp_rn(sum);
+                m_l = -INFINITY;
+                s_l = 0.0f;
+                ++long_rows;
+            }
+            continue;
+        }
         if (mt.kind == KIND_DATA) {
             Bounds bd{nullptr, nullptr, y, y + a.total_elems * E::kSize, a.status};
             const int64_t cap = Op == OP_BACKWARD ? a.stage_bytes / 2 : a.stage_bytes;

@@ -1,0 +1,84 @@
+"""Rows longer than one shared-memory stage (streamed twice in chunks: a
+running max and rescaled sum, then the output) against the oracle, under
+every policy, bit-identical across policies."""
+import numpy as np
+import pytest
+
+from gpu_util import bits, check_all_against_oracle, run, to_device, to_host
+from paper_2002_07062_gb300 import bsm, workload
+
+pytestmark = pytest.mark.gpu
+
+ALL = [bsm.POLICY_WHOLE_GPU, bsm.POLICY_RR, bsm.POLICY_DYNAMIC, bsm.POLICY_CBMF,
+       bsm.POLICY_CBMF_LB]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def setup():
+    import torch
+    import __graft_entry__ as g
+    g.build()
+    torch.cuda.set_device(0)
+    bsm.bsm_device_status_clear()
+
+
+def _all(w, x):
+    import torch
+    ys = [run(w, x, p) for p in ALL]
+    torch.cuda.synchronize()
+    for y in ys[1:]:
+        assert torch.equal(bits(y), bits(ys[0]))
+    return ys[0]
+
+
+@pytest.mark.parametrize("dtype", [workload.F32, workload.BF16])
+def test_rows_just_over_and_far_over_a_stage(dtype):
+    es = 4 if dtype == workload.F32 else 2
+    limit = bsm.bsm_max_row_bytes() // es
+    for B, R, C, flags in [(2, 3, limit + 16 // es, 0), (1, 2, 262144, 0),
+                           (1, 1, 1 << 21, 0), (2, 5, 65536, workload.CAUSAL)]:
+        w = workload.uniform("long", dtype, B, R, C, 4.0, 0x1046 + C + flags, flags).materialize()
+        x = to_device(w.x)
+        p = bsm.bsm_plan_create(x, x, w.rows, w.cols, dtype, bsm.POLICY_DYNAMIC, flags=flags)
+        assert p.stats()["long_items"] == B * R
+        p.close()
+        y = _all(w, x)
+        check_all_against_oracle(w, to_host(y))
+    assert bsm.bsm_device_status() == 0
+
+
+def test_mixed_short_and_long_rows_in_one_batch():
+    # ragged: 256 B .. 1.6 MB rows interleaved, some slices with one row
+    rows = np.array([4, 1, 3, 2, 5, 1, 2], np.int32)
+    cols = np.array([64, 400000, 2048, 120000, 512, 16, 70000], np.int32)
+    sizes = rows.astype(np.int64) * cols
+    off = np.concatenate([[0], np.cumsum(sizes)[:-1]]).astype(np.int64)
+    w = workload.Workload("mixed long", workload.F32, rows, cols, off, 0, 0x4D17, 3.0)
+    w.materialize()
+    x = to_device(w.x)
+    y = _all(w, x)
+    check_all_against_oracle(w, to_host(y))
+
+
+def test_non_finite_long_rows():
+    C = 100000
+    rows = []
+    rng = np.random.default_rng(3)
+    for kind in range(4):
+        r = rng.normal(0, 3, C).astype(np.float32)
+        if kind == 1:
+            r[77777] = np.nan
+        elif kind == 2:
+            r[5] = np.inf
+        elif kind == 3:
+            r[:] = -np.inf
+            r[99999] = 1.0
+        rows.append(r)
+    w = workload.uniform("long nonfinite", workload.F32, 1, 4, C, 1.0, 0)
+    w.x = np.stack(rows).reshape(-1)
+    x = to_device(w.x)
+    y = _all(w, x)
+    yh = to_host(y).reshape(4, C)
+    assert np.isnan(yh[1]).all() and np.isnan(yh[2]).all()
+    assert yh[3, 99999] == 1.0 and np.count_nonzero(yh[3]) == 1
+    check_all_against_oracle(w, to_host(y))

@@ -177,10 +177,10 @@ def test_argument_errors_on_device():
     with pytest.raises(bsm.BsmError) as e:
         bsm.bsm_softmax(x, x.data_ptr() + 16, 4, 1, 64, bsm.F32, bsm.POLICY_RR)
     assert e.value.status == bsm.ERR_INVALID_ARG                        # partial overlap
-    big = bsm.bsm_max_row_bytes() // 4 + 4
+    big = bsm.bsm_max_row_bytes() // 8 + 4          # backward: half a stage per row
     xb = torch.zeros(big, device="cuda")
     with pytest.raises(bsm.BsmError) as e:
-        bsm.bsm_softmax(xb, xb, 1, 1, big, bsm.F32, bsm.POLICY_RR)
+        bsm.bsm_softmax_backward(xb, xb, xb, 1, 1, big, bsm.F32, bsm.POLICY_RR)
     assert e.value.status == bsm.ERR_UNSUPPORTED
     with pytest.raises(bsm.BsmError) as e:                              # overlapping slices
         bsm.bsm_softmax_ragged(x, y, [0, 32], [1, 1], [64, 64], bsm.F32, bsm.POLICY_RR)
