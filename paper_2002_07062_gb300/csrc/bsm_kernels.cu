@@ -846,7 +846,7 @@ struct Puller {
 };
 
 template <typename Tag, int Op, bool Checked>
-__global__ void __maxnreg__(120) softmax_persistent(const KernelArgs a)
+__global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelArgs a)
 {
     using E = Elem<Tag>;
     extern __shared__ __align__(1024) unsigned char smem[];
