@@ -274,8 +274,6 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
         slice_first[s] = static_cast<int32_t>(items.size());
         const SliceView &v = slices[s];
         size_t e = s + 1;
-        if (int64_t(v.C) * es > stage / in_arrays)
-            long_rows += v.R;
         if (spanning && v.R > 0) {
             while (e < slices.size() && slices[e].R == v.R && slices[e].C == v.C &&
                    slices[e].off == slices[e - 1].off + int64_t(v.R) * v.C) {
@@ -285,6 +283,8 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
         }
         if (v.R > 0) {
             const int64_t seg_rows = int64_t(v.R) * static_cast<int64_t>(e - s);
+            if (int64_t(v.C) * es > stage / in_arrays)
+                long_rows += seg_rows;
             const int64_t row_bytes = int64_t(v.C) * es;
             int64_t rpi = std::max<int64_t>(1, stage / in_arrays / row_bytes);
             if (d->rows_per_item > 0)
