@@ -681,7 +681,9 @@ __device__ __forceinline__ void long_chunk(const unsigned char *sbuf, const Stag
                     m_l = vm;
                 }
             }
-            vec_exp<EPV>(v, m_l * kLog2e, masked);
+            // while the running max is still -inf every value seen is -inf (or
+            // NaN): it adds 0 (NaN), as a masked vector does
+            vec_exp<EPV>(v, m_l * kLog2e, masked || m_l == -INFINITY);
             s_l += tree_sum<EPV>(v);
         } else {
             vec_exp<EPV>(v, mL, masked);
