@@ -114,7 +114,8 @@ struct bsm_plan {
     int device = 0;
     int policy = 0;
     int dtype = 0;
-    int op = 0;
+    int op = 0;          // BSM_OP_* of the plan
+    int kernel_op = 0;   // the kernel instance it launches (bsm::Op)
     bsm::KernelArgs args{};
     int grid = 0;
     struct Launch {
@@ -321,6 +322,7 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     st.stage_bytes = static_cast<int32_t>(stage);
     st.n_stages = n_stages;
     st.long_items = long_rows;
+    p->kernel_op = d->op == BSM_OP_BACKWARD ? OP_BACKWARD : (long_rows > 0 ? OP_FORWARD_LONG : OP_FORWARD);
 
     // ---- the schedule
     std::vector<int32_t> queue;      // schedule order of the patches (queue policies)
@@ -564,11 +566,11 @@ int plan_execute_impl(const bsm_plan *p, bsm_stream_t stream)
         for (const auto &l : p->whole_gpu) {
             a.item_begin = l.begin;
             a.item_end = l.end;
-            if ((err = launch_softmax(a, p->dtype, p->op, l.grid, stream, checked)))
+            if ((err = launch_softmax(a, p->dtype, p->kernel_op, l.grid, stream, checked)))
                 break;
         }
     } else {
-        err = launch_softmax(p->args, p->dtype, p->op, p->grid, stream, checked);
+        err = launch_softmax(p->args, p->dtype, p->kernel_op, p->grid, stream, checked);
     }
     if (prev >= 0 && prev != p->device)
         cudaSetDevice(prev);

@@ -43,7 +43,8 @@ constexpr int kMinStageBytes = 32 * 1024;
 // What the kernel computes on every row.
 enum Op : int32_t {
     OP_FORWARD = 0,     // y = softmax(x [+ causal mask])
-    OP_BACKWARD = 1     // y = x * (x2 - rowsum(x * x2)): x = softmax output, x2 = its gradient
+    OP_BACKWARD = 1,    // y = x * (x2 - rowsum(x * x2)): x = softmax output, x2 = its gradient
+    OP_FORWARD_LONG = 2 // OP_FORWARD for plans with rows longer than a stage (two passes)
 };
 
 struct KernelArgs {

@@ -851,6 +851,9 @@ template <typename Tag, int Op, bool Checked>
 __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelArgs a)
 {
     using E = Elem<Tag>;
+    // the long-row machinery is compiled into its own instance, so plans
+    // without long rows do not pay its registers
+    constexpr bool kLong = Op == OP_FORWARD_LONG;
     extern __shared__ __align__(1024) unsigned char smem[];
     SmemHeader &h = *reinterpret_cast<SmemHeader *>(smem);
     unsigned char *stages = smem + kSmemHeader;
@@ -923,7 +926,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                     const int64_t ne = (int64_t)item.nrows * item.C;
                     const int64_t nbytes = ne * E::kSize;
                     const int64_t cap = Op == OP_BACKWARD ? a.stage_bytes / 2 : a.stage_bytes;
-                    const bool is_long = Op == OP_FORWARD && nbytes > cap && item.nrows == 1;
+                    const bool is_long = kLong && nbytes > cap && item.nrows == 1;
                     const bool ok = pos[j] >= 0 && pos[j] < a.n_items && item.off >= 0 && item.C > 0 &&
                                     item.nrows > 0 && item.R > 0 && item.row0 >= 0 &&
                                     item.row0 < item.R && item.off + ne <= a.total_elems &&
@@ -935,7 +938,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                         mbar_arrive(&h.full[s]);
                         continue;
                     }
-                    if (is_long) {
+                    if (kLong && is_long) {
                         // the row in chunks of one stage, twice
                         const int64_t chunk = cap / E::kSize;
                         const int64_t nch = (item.C + chunk - 1) / chunk;
@@ -1042,6 +1045,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
     // offset and reciprocal; which partial buffer and barrier phase is next
     float m_l = -INFINITY, s_l = 0.0f, long_mL = 0.0f, long_inv = 0.0f;
     uint32_t long_rows = 0;
+    (void)m_l, (void)s_l, (void)long_mL, (void)long_inv, (void)long_rows;
     for (uint32_t it = 0;; ++it) {
         const int s = it % S;
         const uint32_t ph = (it / S) & 1u;
@@ -1055,7 +1059,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
         const StageMeta mt = h.meta[s];
         if (mt.kind == KIND_DONE)
             break;
-        if (Op == OP_FORWARD && mt.kind == KIND_LONG) {
+        if (kLong && mt.kind == KIND_LONG) {
             Bounds bd{nullptr, nullptr, y, y + a.total_elems * E::kSize, a.status};
             long_chunk<Tag, Checked>(stages + (size_t)s * a.stage_bytes, mt, y, causal, warp, lane, bd, m_l,
                                      s_l, long_mL, long_inv);
@@ -1130,7 +1134,11 @@ int kernel_set_smem_limit(int bytes)
         reinterpret_cast<const void *>(softmax_persistent<F32, OP_BACKWARD, false>),
         reinterpret_cast<const void *>(softmax_persistent<BF16, OP_BACKWARD, false>),
         reinterpret_cast<const void *>(softmax_persistent<F32, OP_BACKWARD, true>),
-        reinterpret_cast<const void *>(softmax_persistent<BF16, OP_BACKWARD, true>)};
+        reinterpret_cast<const void *>(softmax_persistent<BF16, OP_BACKWARD, true>),
+        reinterpret_cast<const void *>(softmax_persistent<F32, OP_FORWARD_LONG, false>),
+        reinterpret_cast<const void *>(softmax_persistent<BF16, OP_FORWARD_LONG, false>),
+        reinterpret_cast<const void *>(softmax_persistent<F32, OP_FORWARD_LONG, true>),
+        reinterpret_cast<const void *>(softmax_persistent<BF16, OP_FORWARD_LONG, true>)};
     for (const void *f : fns) {
         cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
         if (e != cudaSuccess)
@@ -1159,6 +1167,11 @@ int launch_softmax(const KernelArgs &a, int dtype, int op, int grid, void *strea
             launch_one<F32, OP_BACKWARD>(a, grid, smem, st, checked);
         else
             launch_one<BF16, OP_BACKWARD>(a, grid, smem, st, checked);
+    } else if (op == OP_FORWARD_LONG) {
+        if (dtype == BSM_F32)
+            launch_one<F32, OP_FORWARD_LONG>(a, grid, smem, st, checked);
+        else
+            launch_one<BF16, OP_FORWARD_LONG>(a, grid, smem, st, checked);
     } else {
         if (dtype == BSM_F32)
             launch_one<F32, OP_FORWARD>(a, grid, smem, st, checked);
