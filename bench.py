@@ -17,7 +17,7 @@ output element written once) per step; also % of the measured HBM copy
 peak and of the 8 TB/s nominal, and slices/s.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 2]
-                  [--policy cbmf_lb|dynamic|rr|cbmf|whole_gpu] [--sweep]
+                  [--policy dynamic|cbmf_lb|minimax|rr|cbmf|whole_gpu] [--sweep]
                   [--impl reference]
 
 --impl reference times the double-precision CPU oracle (the only other
@@ -414,7 +414,7 @@ def sweep(args, bsm, workload, stream):
         if w.dtype == workload.BF16:
             x = x.view(torch.bfloat16)
         y = torch.empty_like(x)
-        for name in ("whole_gpu", "rr", "dynamic", "cbmf", "cbmf_lb"):
+        for name in ("whole_gpu", "rr", "dynamic", "cbmf", "cbmf_lb", "minimax"):
             pol = bsm.POLICIES[name]
             reps = 3 if name == "whole_gpu" and k == 5 else 20
 

@@ -29,6 +29,11 @@
  *   BSM_POLICY_DYNAMIC    Not in the paper: one device-wide queue of patches,
  *                         every SM pulls the next one (the locality-blind
  *                         dynamic schedule CBMF is measured against).
+ *   BSM_POLICY_MINIMAX    Sec. 4.2, general form: patches assigned to dies to
+ *                         minimise the largest per-SM finish time, a patch's
+ *                         cost depending on its distance to the die (near /
+ *                         far latency); solved by longest-patch-first, the
+ *                         queues then run longest first, with stealing.
  * Every policy computes every row with the same device routine, chosen only
  * by the row length, so y is bit-identical across policies.
  *
@@ -84,7 +89,8 @@ typedef enum {
     BSM_POLICY_RR = 1,
     BSM_POLICY_CBMF = 2,
     BSM_POLICY_CBMF_LB = 3,
-    BSM_POLICY_DYNAMIC = 4
+    BSM_POLICY_DYNAMIC = 4,
+    BSM_POLICY_MINIMAX = 5
 } bsm_policy;
 
 #define BSM_FLAG_CAUSAL 1u     /* additive -inf mask above each slice's diagonal */
@@ -341,6 +347,8 @@ typedef struct {
     const int32_t *units;       /* compute units near each bank */
     int64_t l_near, l_far;      /* latency weights (equal = unweighted) */
     const int64_t *cost;        /* work of each patch (bytes it moves) */
+    int32_t method;             /* 0: Sec. 4.1 (+ 4.2 balance); 1: MINIMAX by longest
+                                   patch first (uses the table, units, l_near, l_far) */
 } bsm_schedule_desc;
 
 typedef struct {
@@ -354,7 +362,7 @@ typedef struct {
     int32_t *moved;             /* n_patches: patch ids in the order moved */
     int64_t n_moved;
     int64_t *work_before;       /* n_banks: l_near*native + l_far*moved-in bytes */
-    int64_t *work_after;        /* n_banks */
+    int64_t *work_after;        /* n_banks (MINIMAX: the cost assigned to each bank) */
 } bsm_schedule_out;
 
 int bsm_schedule_host(const bsm_schedule_desc *d, bsm_schedule_out *out);

@@ -209,3 +209,48 @@ def brute_force_minimax(home: Sequence[int], cost: Sequence[int], units: Sequenc
             best = ms
     assert best is not None
     return best
+
+
+def minimax_lpt(table: BankTable, units: Sequence[int], l_near: int, l_far: int):
+    """Sec. 4.2 MINIMAX (minimise the largest per-unit finish time) by the
+    longest-processing-time rule: the cost of patch i on bank b is
+    sum over banks b' of bytes_on_bank[i][b'] * (l_near if b' == b else
+    l_far); patches go in decreasing order of their smallest cost (ties:
+    lower index first), each to the bank whose finish time after taking it,
+    (W_b + cost) / units[b], is smallest (ties: lower bank).  Returns the
+    per-bank queues in assignment order and the final W."""
+    nb = len(units)
+    rows = table.bytes_on_bank
+
+    def cost(i, b):
+        return sum(v * (l_near if bb == b else l_far) for bb, v in enumerate(rows[i]))
+
+    order = sorted(range(len(rows)), key=lambda i: (-min(cost(i, b) for b in range(nb)), i))
+    W = [0] * nb
+    queues: List[List[int]] = [[] for _ in range(nb)]
+    for i in order:
+        best = 0
+        for b in range(1, nb):
+            # (W_b + c_b) / u_b < (W_best + c_best) / u_best
+            if _finish_less(W[b] + cost(i, b), units[b], W[best] + cost(i, best), units[best]):
+                best = b
+        W[best] += cost(i, best)
+        queues[best].append(i)
+    return queues, W
+
+
+def brute_force_minimax_table(table: BankTable, units: Sequence[int], l_near: int,
+                              l_far: int) -> Tuple[int, int]:
+    """Exact optimum of the same problem (every assignment tried)."""
+    nb = len(units)
+    rows = table.bytes_on_bank
+    best: Optional[Tuple[int, int]] = None
+    for assign in product(range(nb), repeat=len(rows)):
+        W = [0] * nb
+        for i, b in enumerate(assign):
+            W[b] += sum(v * (l_near if bb == b else l_far) for bb, v in enumerate(rows[i]))
+        ms = makespan_num_den(W, units)
+        if best is None or _finish_less(ms[0], ms[1], best[0], best[1]):
+            best = ms
+    assert best is not None
+    return best

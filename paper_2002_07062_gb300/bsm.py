@@ -20,9 +20,9 @@ LIB_PATH = os.path.join(PKG, "_lib", "libbsm.so")
 HEADER = os.path.join(os.path.dirname(PKG), "include", "bsm.h")
 
 F32, BF16 = 0, 1
-POLICY_WHOLE_GPU, POLICY_RR, POLICY_CBMF, POLICY_CBMF_LB, POLICY_DYNAMIC = range(5)
+POLICY_WHOLE_GPU, POLICY_RR, POLICY_CBMF, POLICY_CBMF_LB, POLICY_DYNAMIC, POLICY_MINIMAX = range(6)
 POLICIES = {"whole_gpu": POLICY_WHOLE_GPU, "rr": POLICY_RR, "cbmf": POLICY_CBMF,
-            "cbmf_lb": POLICY_CBMF_LB, "dynamic": POLICY_DYNAMIC}
+            "cbmf_lb": POLICY_CBMF_LB, "dynamic": POLICY_DYNAMIC, "minimax": POLICY_MINIMAX}
 POLICY_NAMES = {v: k for k, v in POLICIES.items()}
 FLAG_CAUSAL = 1
 OP_FORWARD, OP_BACKWARD = 0, 1
@@ -84,7 +84,8 @@ class ScheduleDesc(ctypes.Structure):
                 ("chunk", ctypes.c_int64 * 2), ("n_chunks", ctypes.c_int64 * 2),
                 ("bank_of_chunk", ctypes.POINTER(ctypes.c_int8) * 2),
                 ("tie_seed", ctypes.c_uint64), ("balance", ctypes.c_int32), ("units", c_i32p),
-                ("l_near", ctypes.c_int64), ("l_far", ctypes.c_int64), ("cost", c_i64p)]
+                ("l_near", ctypes.c_int64), ("l_far", ctypes.c_int64), ("cost", c_i64p),
+                ("method", ctypes.c_int32)]
 
 
 class ScheduleOut(ctypes.Structure):
@@ -364,7 +365,7 @@ def bsm_probe_latency(line_off, reps: int = 8, device: int = -1):
 
 def bsm_schedule_host(patches: Sequence, maps: Sequence, n_banks: int, tie_seed: int,
                       balance: bool = False, units=None, l_near: int = 1, l_far: int = 1,
-                      cost=None) -> dict:
+                      cost=None, minimax: bool = False) -> dict:
     """patches: (begin, end) byte ranges; maps: (chunk, bank_of_chunk) pairs."""
     n = len(patches)
     pb = _np([p[0] for p in patches], np.int64)
@@ -390,6 +391,7 @@ def bsm_schedule_host(patches: Sequence, maps: Sequence, n_banks: int, tie_seed:
     d.l_far = l_far
     cst = _np(cost if cost is not None else [p[1] - p[0] for p in patches], np.int64)
     d.cost = cst.ctypes.data_as(c_i64p)
+    d.method = 1 if minimax else 0
     bob = np.zeros((max(n, 1), n_banks), np.int64)
     ov = np.zeros(max(n, 1), np.uint8)
     N = np.zeros(n_banks, np.int64)

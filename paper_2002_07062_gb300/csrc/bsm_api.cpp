@@ -147,7 +147,7 @@ int validate(const bsm_plan_desc *d, const DeviceCtx &c, std::vector<SliceView> 
 {
     if (d->dtype != BSM_F32 && d->dtype != BSM_BF16)
         return BSM_ERR_INVALID_ARG;
-    if (d->policy < BSM_POLICY_WHOLE_GPU || d->policy > BSM_POLICY_DYNAMIC)
+    if (d->policy < BSM_POLICY_WHOLE_GPU || d->policy > BSM_POLICY_MINIMAX)
         return BSM_ERR_INVALID_ARG;
     if (d->flags & ~BSM_FLAG_CAUSAL)
         return BSM_ERR_INVALID_ARG;
@@ -266,7 +266,7 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     // the same shape and follow back to back (a "segment"); under RR and
     // WHOLE_GPU a patch stays inside its slice, the unit those policies place.
     const bool spanning = d->policy == BSM_POLICY_DYNAMIC || d->policy == BSM_POLICY_CBMF ||
-                          d->policy == BSM_POLICY_CBMF_LB;
+                          d->policy == BSM_POLICY_CBMF_LB || d->policy == BSM_POLICY_MINIMAX;
     std::vector<Item> items;
     std::vector<int32_t> slice_first(slices.size() + 1, 0);
     int64_t long_rows = 0;
@@ -338,13 +338,15 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
         st.queue_items[0] = n_items;
         st.queue_bytes[0] = total * es * 2;
         st.L[0] = st.N[0] = n_items;
-    } else if (d->policy == BSM_POLICY_CBMF || d->policy == BSM_POLICY_CBMF_LB) {
+    } else if (d->policy == BSM_POLICY_CBMF || d->policy == BSM_POLICY_CBMF_LB ||
+               d->policy == BSM_POLICY_MINIMAX) {
         bsm_topology topo;
         if ((rc = topology_get(device, 0, &topo))) {
             delete p;
             return rc;
         }
         const bool lb = d->policy == BSM_POLICY_CBMF_LB;
+        const bool minimax = d->policy == BSM_POLICY_MINIMAX;
         if (!topo.separable || n_items == 0) {
             // one die: CBMF degenerates to a single queue
             queue.resize(static_cast<size_t>(n_items));
@@ -398,6 +400,7 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
             sd.bank_of_chunk[1] = count_y ? ymap.data() : nullptr;
             sd.tie_seed = d->tie_seed;
             sd.balance = lb ? 1 : 0;
+            sd.method = minimax ? 1 : 0;
             sd.units = units;
             sd.l_near = d->lb_weighted ? std::max<int64_t>(1, llround(topo.l_near)) : 1;
             sd.l_far = d->lb_weighted ? std::max<int64_t>(1, llround(topo.l_far)) : 1;
@@ -440,6 +443,8 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
                 if (lb) {
                     st.est_finish_before[b] = double(wb[b]) / units[b];
                     st.est_finish_after[b] = double(wa[b]) / units[b];
+                } else if (minimax) {
+                    st.est_finish_after[b] = double(wa[b]) / units[b];
                 }
             }
             for (int64_t i = 0; i < n_items; ++i) {
@@ -455,7 +460,7 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
                 if (sm_die_tab[s] < 0)
                     sm_die_tab[s] = 0;
             use_sm_die = true;
-            p->args.steal = lb ? 1 : 0;
+            p->args.steal = (lb || minimax) ? 1 : 0;
         }
     }
 
@@ -769,7 +774,7 @@ static int softmax_uniform(const void *x, void *y, int64_t B, int64_t R, int64_t
         return BSM_ERR_INVALID_ARG;
     if (dtype != BSM_F32 && dtype != BSM_BF16)
         return BSM_ERR_INVALID_ARG;
-    if (policy < BSM_POLICY_WHOLE_GPU || policy > BSM_POLICY_DYNAMIC || (flags & ~BSM_FLAG_CAUSAL))
+    if (policy < BSM_POLICY_WHOLE_GPU || policy > BSM_POLICY_MINIMAX || (flags & ~BSM_FLAG_CAUSAL))
         return BSM_ERR_INVALID_ARG;
     if (R > 0 && (B > (int64_t(1) << 62) / R || C > (int64_t(1) << 62) / std::max<int64_t>(1, B * R)))
         return BSM_ERR_INVALID_ARG;
@@ -802,7 +807,7 @@ static int softmax_ragged(const void *x, void *y, int64_t n, const int64_t *off,
         return BSM_ERR_INVALID_ARG;
     if (dtype != BSM_F32 && dtype != BSM_BF16)
         return BSM_ERR_INVALID_ARG;
-    if (policy < BSM_POLICY_WHOLE_GPU || policy > BSM_POLICY_DYNAMIC || (flags & ~BSM_FLAG_CAUSAL))
+    if (policy < BSM_POLICY_WHOLE_GPU || policy > BSM_POLICY_MINIMAX || (flags & ~BSM_FLAG_CAUSAL))
         return BSM_ERR_INVALID_ARG;
     if (n == 0)
         return BSM_OK;

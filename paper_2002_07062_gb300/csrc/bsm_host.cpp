@@ -88,7 +88,7 @@ int softmax_host(const void *x_host, void *y_host, int64_t B, int64_t R, int64_t
                  uint32_t flags, bsm_stream_t stream)
 {
     if (B < 0 || R < 0 || C < 1 || (dtype != BSM_F32 && dtype != BSM_BF16) || (flags & ~BSM_FLAG_CAUSAL) ||
-        policy < BSM_POLICY_WHOLE_GPU || policy > BSM_POLICY_DYNAMIC)
+        policy < BSM_POLICY_WHOLE_GPU || policy > BSM_POLICY_MINIMAX)
         return BSM_ERR_INVALID_ARG;
     if (R > INT32_MAX || C > INT32_MAX || (R > 0 && B > (int64_t(1) << 40) / R))
         return BSM_ERR_INVALID_ARG;

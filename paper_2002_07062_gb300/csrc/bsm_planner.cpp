@@ -17,6 +17,13 @@
 //   strictly lowers the larger of the two finish times; a moved patch costs
 //   l_far per byte on its new bank, a native one l_near.  Moves are "virtual":
 //   only the queue changes, the data stays where it is.
+// Sec. 4.2, general form (MINIMAX: minimise the largest per-unit finish
+// time; the cost of a patch depends on its distance to the unit): here the
+// cost of patch i on bank b is sum_b' bytes(i, b') * (l_near if b' == b else
+// l_far); patches are taken in decreasing order of their smallest cost
+// (ties: lower index), each to the bank with the smallest (W_b + cost) /
+// units_b (ties: lower bank) -- the longest-processing-time rule.  The
+// queues keep that order, so every bank runs its longest patches first.
 // All quantities are integers, so the result is exact and reproducible.
 
 #include <algorithm>
@@ -162,6 +169,49 @@ int schedule_host(const bsm_schedule_desc *d, bsm_schedule_out *o)
         }
         for (int b = 0; b < nb; ++b)
             o->work_after[b] = W[b];
+    }
+
+    if (d->method == 1) {
+        // MINIMAX by longest patch first (replaces the queues built above)
+        if (!d->units || d->l_near <= 0 || d->l_far <= 0 || !o->work_after)
+            return BSM_ERR_INVALID_ARG;
+        for (int b = 0; b < nb; ++b)
+            if (d->units[b] <= 0)
+                return BSM_ERR_INVALID_ARG;
+        auto cost = [&](int64_t i, int b) {
+            const int64_t *row = o->bytes_on_bank + i * nb;
+            int64_t c = 0;
+            for (int bb = 0; bb < nb; ++bb)
+                c += row[bb] * (bb == b ? d->l_near : d->l_far);
+            return c;
+        };
+        std::vector<int64_t> key(static_cast<size_t>(np));
+        std::vector<int32_t> order(static_cast<size_t>(np));
+        for (int64_t i = 0; i < np; ++i) {
+            int64_t mn = cost(i, 0);
+            for (int b = 1; b < nb; ++b)
+                mn = std::min(mn, cost(i, b));
+            key[i] = mn;
+            order[i] = static_cast<int32_t>(i);
+        }
+        std::stable_sort(order.begin(), order.end(),
+                         [&](int32_t u, int32_t v) { return key[u] > key[v]; });
+        std::vector<int64_t> W(nb, 0);
+        for (int b = 0; b < nb; ++b)
+            q[b].clear();
+        for (int32_t i : order) {
+            int best = 0;
+            for (int b = 1; b < nb; ++b)
+                if (ratio_less(W[b] + cost(i, b), d->units[b], W[best] + cost(i, best), d->units[best]))
+                    best = b;
+            W[best] += cost(i, best);
+            q[best].push_back(i);
+        }
+        for (int b = 0; b < nb; ++b) {
+            o->work_after[b] = W[b];
+            if (o->work_before)
+                o->work_before[b] = 0;
+        }
     }
 
     int64_t pos = 0;

@@ -17,7 +17,7 @@ from paper_2002_07062_gb300 import bsm, workload
 pytestmark = pytest.mark.gpu
 
 ALL = [bsm.POLICY_WHOLE_GPU, bsm.POLICY_RR, bsm.POLICY_DYNAMIC, bsm.POLICY_CBMF,
-       bsm.POLICY_CBMF_LB]
+       bsm.POLICY_CBMF_LB, bsm.POLICY_MINIMAX]
 U = 2.0 ** -24
 
 

@@ -135,3 +135,43 @@ def test_load_balance_against_brute_force_minimax(trial):
         lhs = got[0] * opt[1] * total_units
         rhs = opt[0] * got[1] * total_units + max(cost) * got[1] * opt[1]
         assert lhs <= rhs
+
+
+def _rand_table(rng, n, nb, chunk=256):
+    nch = n * 4 + 8
+    m = S.BankMap(chunk, [rng.randrange(nb) for _ in range(nch)])
+    patches, pos = [], 0
+    for _ in range(n):
+        size = rng.choice([256, 512, 768, 1024])
+        patches.append((pos, pos + size))
+        pos += size
+    return S.bank_table(patches, [m], nb)
+
+
+@pytest.mark.parametrize("trial", range(40))
+def test_minimax_lpt_against_brute_force(trial):
+    rng = random.Random(5000 + trial)
+    n = rng.randrange(1, 8)
+    t = _rand_table(rng, n, 2)
+    identical = trial % 2 == 0
+    units = [2, 2] if identical else [rng.randrange(1, 4), rng.randrange(1, 4)]
+    ln, lf = (1, 1) if identical else (3, 4)
+    queues, W = S.minimax_lpt(t, units, ln, lf)
+    assert sorted(queues[0] + queues[1]) == list(range(n))
+    got = S.makespan_num_den(W, units)
+    opt = S.brute_force_minimax_table(t, units, ln, lf)
+    assert got[0] * opt[1] >= opt[0] * got[1]            # never better than the optimum
+    if identical:
+        # two identical machines: Graham's LPT bound, makespan <= (4/3 - 1/6) * OPT
+        assert 6 * got[0] * opt[1] <= 7 * opt[0] * got[1]
+
+
+def test_minimax_queues_are_longest_first():
+    m = S.BankMap(256, [0, 1] * 40)
+    patches = [(0, 256), (256, 1280), (1280, 1536), (1536, 3584), (3584, 3840)]
+    t = S.bank_table(patches, [m], 2)
+    queues, _ = S.minimax_lpt(t, [1, 1], 1, 1)
+    sizes = {i: p[1] - p[0] for i, p in enumerate(patches)}
+    assert queues[0][0] == 3 and queues[1][0] == 1          # the two largest first
+    for q in queues:
+        assert [sizes[i] for i in q] == sorted((sizes[i] for i in q), reverse=True)

@@ -99,3 +99,26 @@ def test_degenerate_first_portion_map_balances():
     assert [len(q) for q in got["queues"]] == [100, 100]
     want = _oracle(patches, maps, 2, 0, True, [76, 76], 1, 1, [8192] * n)
     _compare(got, want, True)
+
+
+@pytest.mark.parametrize("trial", range(30))
+def test_minimax_matches_oracle(trial):
+    rng = random.Random(900 + trial)
+    nb = rng.choice([2, 2, 3])
+    chunk = rng.choice([128, 1024])
+    n = rng.randrange(0, 200)
+    sizes = [rng.choice([256, 1024, 4096, 32768, 8192]) for _ in range(n)]
+    patches, pos = [], 0
+    for sz in sizes:
+        patches.append((pos, pos + sz))
+        pos += sz
+    nch = pos // chunk + 1
+    maps = [(chunk, [rng.randrange(nb) for _ in range(nch)])]
+    units = [rng.randrange(1, 80) for _ in range(nb)]
+    ln = rng.randrange(1, 500)
+    lf = ln + rng.randrange(0, 300)
+    got = bsm.bsm_schedule_host(patches, maps, nb, 0, False, units, ln, lf, minimax=True)
+    t = S.bank_table(patches, [S.BankMap(c, b) for c, b in maps], nb)
+    queues, W = S.minimax_lpt(t, units, ln, lf)
+    assert got["queues"] == queues
+    assert got["work_after"] == W

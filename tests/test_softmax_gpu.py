@@ -15,7 +15,7 @@ from paper_2002_07062_gb300 import bsm, workload
 pytestmark = pytest.mark.gpu
 
 ALL = [bsm.POLICY_WHOLE_GPU, bsm.POLICY_RR, bsm.POLICY_DYNAMIC, bsm.POLICY_CBMF,
-       bsm.POLICY_CBMF_LB]
+       bsm.POLICY_CBMF_LB, bsm.POLICY_MINIMAX]
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -91,7 +91,8 @@ def test_ragged_workload4_full_size():
     w = workload.config(4).materialize()
     x = to_device(w.x)
     y = _all_policies_identical(w, x, [bsm.POLICY_RR, bsm.POLICY_DYNAMIC, bsm.POLICY_CBMF,
-                                       bsm.POLICY_CBMF_LB, bsm.POLICY_WHOLE_GPU])
+                                       bsm.POLICY_CBMF_LB, bsm.POLICY_MINIMAX,
+                                       bsm.POLICY_WHOLE_GPU])
     yh = to_host(y)
     check_rows_against_oracle(w, yh, sample_rows(w, 3000, 44))
     assert not torch.isnan(y).any()
@@ -200,7 +201,7 @@ def test_topology_and_plan_stats():
     w = workload.config(2)
     x = torch.empty(w.numel, device="cuda")
     y = torch.empty_like(x)
-    for pol in (bsm.POLICY_CBMF, bsm.POLICY_CBMF_LB):
+    for pol in (bsm.POLICY_CBMF, bsm.POLICY_CBMF_LB, bsm.POLICY_MINIMAX):
         p = bsm.bsm_plan_create(x, y, w.rows, w.cols, w.dtype, pol)
         st = p.stats()
         n = st["n_items"]
