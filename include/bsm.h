@@ -203,6 +203,25 @@ int bsm_softmax_backward_ragged(const void *y, const void *dy, void *dx, int64_t
                                 const int64_t *offsets, const int32_t *rows, const int32_t *cols,
                                 int dtype, int policy, bsm_stream_t stream);
 
+/*
+ * Batched matrix product, the paper's other batch algorithm (Sec. 6: batch
+ * 384 of (512 x 64) x (64 x 512) and of (512 x 512) x (512 x 64)), on the
+ * tensor cores, with the output tiles (128 x 64/128/256 of one slice) as the
+ * patches of the same scheduling policies:
+ *     C_s[m, n] = sum_k A_s[m, k] * Bt_s[n, k]        (C_s = A_s Bt_s^T)
+ *   a   device, B x M x K bf16, row-major (slice s at s*M*K)
+ *   bt  device, B x N x K bf16, row-major: the second factor TRANSPOSED, i.e.
+ *       with the reduction dimension contiguous (attention's K matrix as it
+ *       is; for P*V pass V^T)
+ *   c   device, B x M x N, out_dtype BSM_F32 or BSM_BF16 (fp32 accumulation,
+ *       rounded to nearest even for bf16)
+ *   M a multiple of 128, N of 64, K of 64 (else BSM_ERR_UNSUPPORTED);
+ *   pointers 16-byte aligned; c must not overlap a or bt.
+ * Plans are cached like bsm_softmax's.  Errors as bsm_softmax.
+ */
+int bsm_bmm(const void *a, const void *bt, void *c, int64_t B, int64_t M, int64_t N, int64_t K,
+            int out_dtype, int policy, bsm_stream_t stream);
+
 /* ---- plans: build the schedule once ("upfront", Sec. 5), run it many times ---- */
 
 typedef struct bsm_plan bsm_plan;

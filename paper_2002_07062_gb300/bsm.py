@@ -115,6 +115,7 @@ def lib():
                                 vp], ctypes.c_int),
         "bsm_softmax_noalloc": ([vp, vp, i64, i64, i64, ctypes.c_int, u32, vp], ctypes.c_int),
         "bsm_softmax_host": ([vp, vp, i64, i64, i64, ctypes.c_int, ctypes.c_int, u32, vp], ctypes.c_int),
+        "bsm_bmm": ([vp, vp, vp, i64, i64, i64, i64, ctypes.c_int, ctypes.c_int, vp], ctypes.c_int),
         "bsm_softmax_backward": ([vp, vp, vp, i64, i64, i64, ctypes.c_int, ctypes.c_int, vp], ctypes.c_int),
         "bsm_softmax_backward_ragged": ([vp, vp, vp, i64, c_i64p, c_i32p, c_i32p, ctypes.c_int,
                                          ctypes.c_int, vp], ctypes.c_int),
@@ -214,6 +215,12 @@ def bsm_softmax_noalloc(x, y, B: int, R: int, C: int, dtype: int, flags: int = 0
     """The allocation-free entry point (fixed scratch inside the library)."""
     _check(lib().bsm_softmax_noalloc(_dptr(x), _dptr(y), B, R, C, dtype, flags, _stream(stream)),
            "bsm_softmax_noalloc")
+
+
+def bsm_bmm(a, bt, c, B: int, M: int, N: int, K: int, out_dtype: int, policy: int, stream=None):
+    """C_s = A_s Bt_s^T for every slice (bf16 inputs, fp32 or bf16 output)."""
+    _check(lib().bsm_bmm(_dptr(a), _dptr(bt), _dptr(c), B, M, N, K, out_dtype, policy,
+                         _stream(stream)), "bsm_bmm")
 
 
 def bsm_softmax_backward(y, dy, dx, B: int, R: int, C: int, dtype: int, policy: int, stream=None):

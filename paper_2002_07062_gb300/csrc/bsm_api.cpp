@@ -100,6 +100,20 @@ int device_ctx(int device, DeviceCtx **out)
     return BSM_OK;
 }
 
+}  // namespace
+
+// The sticky status word of a device, shared by every kernel of the library.
+int device_status_word(int device, uint32_t **out)
+{
+    DeviceCtx *c = nullptr;
+    if (int rc = device_ctx(device, &c))
+        return rc;
+    *out = c->status;
+    return BSM_OK;
+}
+
+namespace {
+
 int64_t max_row_bytes_for(const DeviceCtx &c)
 {
     return ((static_cast<int64_t>(c.smem_optin) - kSmemHeader) / 2) & ~int64_t(127);

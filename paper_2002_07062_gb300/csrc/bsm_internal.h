@@ -75,6 +75,41 @@ struct KernelArgs {
 // Test-only fault injection (bsm_plan_debug).
 constexpr uint32_t KDEBUG_WITHHOLD_STAGE0 = 1u;   // producer never fills stage 0 of its first round
 
+// One output tile of the batched matrix product: rows [m0, m0 + 128) and
+// columns [n0, n0 + BN) of slice `slice`.
+struct GemmItem {
+    int32_t slice, m0, n0, pad;
+};
+
+struct GemmArgs {
+    void *c;                    // B x M x N output (bf16 or fp32)
+    int32_t B, M, N, K;
+    const GemmItem *items;
+    int32_t n_items;
+    int32_t mode;               // PullMode
+    int32_t item_begin, item_end;
+    const int32_t *slice_first_item;
+    int32_t n_slices;
+    int32_t n_queues;
+    int32_t queue_begin[BSM_MAX_DIES];
+    int32_t queue_len[BSM_MAX_DIES];
+    int32_t steal;
+    uint32_t *heads;
+    const int8_t *sm_die;
+    int32_t n_stages;
+    uint32_t *status;
+};
+
+// Batched matrix product kernel (bsm_bmm.cu).  tmap_a / tmap_b / tmap_c point
+// at host CUtensorMap objects (C: boxes of 32 rows x 128 bytes, 128-byte
+// swizzle).  Return cudaError_t values.
+int launch_bmm(const void *tmap_a, const void *tmap_b, const void *tmap_c, const GemmArgs &a, int bn,
+               bool out_bf16, int grid, void *stream);
+int gemm_set_smem_limit(int bytes);
+int gemm_stage_bytes(int bn);
+// shared memory of one launch besides the stages (header, slack, epilogue buffers)
+int gemm_fixed_smem();
+
 // Launch the persistent softmax kernel (bsm_kernels.cu).  Returns a
 // cudaError_t value (0 = success).
 int launch_softmax(const KernelArgs &a, int dtype, int op, int grid, void *stream, bool checked);

@@ -195,3 +195,68 @@ def slice_sample(w: Workload, slices) -> Workload:
             fill_normal(n, w.dtype, w.seed, w.sigma, index_base=int(w.offsets[s]), out=seg)
     return Workload(w.name + " [sample of %d slices]" % len(slices), w.dtype, rows, cols,
                     offsets, w.flags, w.seed, w.sigma, x)
+
+
+# ---------------------------------------------------------------------------
+# Batched matrix product operands (Sec. 6 matrix-multiplication table).
+
+@dataclass
+class BmmWorkload:
+    """B slices of A_s (M x K) and Bt_s (N x K), bf16, row-major, packed; the
+    product is written as out_dtype (F32 or BF16).  kind "normal": N(0, sigma)
+    draws; kind "int": the same draws rounded to integers in [-6, 6], so that
+    every product and partial sum is exact in fp32."""
+    name: str
+    B: int
+    M: int
+    N: int
+    K: int
+    out_dtype: int
+    seed: int
+    sigma: float = 1.0
+    kind: str = "normal"
+
+    @property
+    def flops(self) -> int:
+        return 2 * self.B * self.M * self.N * self.K
+
+    @property
+    def algorithmic_bytes(self) -> int:
+        """Both operands read once, the product written once."""
+        out_es = 4 if self.out_dtype == F32 else 2
+        return 2 * self.B * (self.M + self.N) * self.K + out_es * self.B * self.M * self.N
+
+    def _draw(self, which: int, n: int, base: int, out=None) -> np.ndarray:
+        seed = (self.seed * 2 + which) & ((1 << 64) - 1)
+        if self.kind == "int":
+            v = fill_normal(n, F32, seed, 2.0, index_base=base)
+            v = np.clip(np.rint(v), -6, 6).astype(np.float32)
+            bits16 = (v.view(np.uint32) >> 16).astype(np.uint16)
+            if out is not None:
+                out[:] = bits16
+                return out
+            return bits16
+        return fill_normal(n, BF16, seed, self.sigma, index_base=base, out=out)
+
+    def operands(self, slices=None):
+        """(a_bits, bt_bits) as uint16 bf16 patterns, for all slices or for
+        the listed ones (packed, same values as in the full tensors)."""
+        mk, nk = self.M * self.K, self.N * self.K
+        if slices is None:
+            return self._draw(0, self.B * mk, 0), self._draw(1, self.B * nk, 0)
+        slices = list(slices)
+        a = np.empty(len(slices) * mk, np.uint16)
+        bt = np.empty(len(slices) * nk, np.uint16)
+        for j, s in enumerate(slices):
+            self._draw(0, mk, s * mk, out=a[j * mk:(j + 1) * mk])
+            self._draw(1, nk, s * nk, out=bt[j * nk:(j + 1) * nk])
+        return a, bt
+
+
+def bmm_config(k: int) -> BmmWorkload:
+    """The paper's two batched products (Sec. 6), bf16 in, bf16 out."""
+    if k == 1:
+        return BmmWorkload("bf16 384 x (512x64)(64x512)", 384, 512, 512, 64, BF16, SEED_BASE + 101)
+    if k == 2:
+        return BmmWorkload("bf16 384 x (512x512)(512x64)", 384, 512, 64, 512, BF16, SEED_BASE + 102)
+    raise ValueError("batched product %d does not exist (1..2)" % k)

@@ -73,3 +73,31 @@ def test_schedule_host_rejects_bad_maps():
         bsm.bsm_schedule_host([(0, 1024)], [(256, [0, 1])], 2, 0)     # past the map
     with pytest.raises(bsm.BsmError):
         bsm.bsm_schedule_host([(0, 512)], [(256, [0, 1])], 2, 0, balance=True, units=[0, 1])
+
+
+@pytest.mark.parametrize("args,code", [
+    ((1, 128, 64, 64, bsm.F32, bsm.POLICY_DYNAMIC), bsm.OK),            # placeholder row
+    ((-1, 128, 64, 64, bsm.F32, bsm.POLICY_DYNAMIC), bsm.ERR_INVALID_ARG),
+    ((1, 128, 64, 64, 7, bsm.POLICY_DYNAMIC), bsm.ERR_INVALID_ARG),     # output dtype
+    ((1, 128, 64, 64, bsm.F32, 9), bsm.ERR_INVALID_ARG),                # policy
+    ((1, 64, 64, 64, bsm.F32, bsm.POLICY_DYNAMIC), bsm.ERR_UNSUPPORTED),   # M % 128
+    ((1, 128, 96, 64, bsm.F32, bsm.POLICY_DYNAMIC), bsm.ERR_UNSUPPORTED),  # N % 64
+    ((1, 128, 64, 80, bsm.F32, bsm.POLICY_DYNAMIC), bsm.ERR_UNSUPPORTED),  # K % 64
+    ((1, 128, 64, 0, bsm.F32, bsm.POLICY_DYNAMIC), bsm.ERR_UNSUPPORTED),   # K = 0
+])
+def test_bmm_argument_errors_without_gpu(args, code):
+    B, M, N, K, out, pol = args
+    if code == bsm.OK:
+        # well-formed but misaligned pointers: rejected before any CUDA call
+        rc = bsm.lib().bsm_bmm(0x1008, 0x20000, 0x40000, B, M, N, K, out, pol, None)
+        assert rc == bsm.ERR_MISALIGNED
+        # output overlapping the first operand
+        rc = bsm.lib().bsm_bmm(0x10000, 0x80000, 0x10100, B, M, N, K, out, pol, None)
+        assert rc == bsm.ERR_INVALID_ARG
+        return
+    assert bsm.lib().bsm_bmm(0x10000, 0x80000, 0x100000, B, M, N, K, out, pol, None) == code
+
+
+def test_bmm_empty_batch_is_a_no_op():
+    for B, M, N in [(0, 128, 64), (3, 0, 64), (3, 128, 0)]:
+        assert bsm.lib().bsm_bmm(None, None, None, B, M, N, 64, bsm.BF16, bsm.POLICY_RR, None) == bsm.OK
