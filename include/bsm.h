@@ -222,6 +222,20 @@ int bsm_softmax_backward_ragged(const void *y, const void *dy, void *dx, int64_t
 int bsm_bmm(const void *a, const void *bt, void *c, int64_t B, int64_t M, int64_t N, int64_t K,
             int out_dtype, int policy, bsm_stream_t stream);
 
+/*
+ * bsm_bmm with the shared-memory split chosen by the caller (0 = automatic,
+ * as bsm_bmm): n_stages operand stages in flight per SM (2..8), each holding
+ * k_blocks_per_stage (1, 2 or 4; must divide K/64) blocks of 64 columns of
+ * K of the 128-row A tile and of the N_tile-row Bt tile, fetched with one
+ * copy per operand; epi_bufs 4 KiB output store buffers per epilogue warp
+ * (2..4).  A split that does not fit in one SM's shared memory, or a block
+ * count that does not divide K/64, returns BSM_ERR_UNSUPPORTED; out-of-range
+ * values BSM_ERR_INVALID_ARG.  Results do not depend on the split.
+ */
+int bsm_bmm_ex(const void *a, const void *bt, void *c, int64_t B, int64_t M, int64_t N, int64_t K,
+               int out_dtype, int policy, int n_stages, int epi_bufs, int k_blocks_per_stage,
+               bsm_stream_t stream);
+
 /* ---- plans: build the schedule once ("upfront", Sec. 5), run it many times ---- */
 
 typedef struct bsm_plan bsm_plan;

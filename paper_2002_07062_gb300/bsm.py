@@ -116,6 +116,8 @@ def lib():
         "bsm_softmax_noalloc": ([vp, vp, i64, i64, i64, ctypes.c_int, u32, vp], ctypes.c_int),
         "bsm_softmax_host": ([vp, vp, i64, i64, i64, ctypes.c_int, ctypes.c_int, u32, vp], ctypes.c_int),
         "bsm_bmm": ([vp, vp, vp, i64, i64, i64, i64, ctypes.c_int, ctypes.c_int, vp], ctypes.c_int),
+        "bsm_bmm_ex": ([vp, vp, vp, i64, i64, i64, i64, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                        ctypes.c_int, ctypes.c_int, vp], ctypes.c_int),
         "bsm_softmax_backward": ([vp, vp, vp, i64, i64, i64, ctypes.c_int, ctypes.c_int, vp], ctypes.c_int),
         "bsm_softmax_backward_ragged": ([vp, vp, vp, i64, c_i64p, c_i32p, c_i32p, ctypes.c_int,
                                          ctypes.c_int, vp], ctypes.c_int),
@@ -221,6 +223,14 @@ def bsm_bmm(a, bt, c, B: int, M: int, N: int, K: int, out_dtype: int, policy: in
     """C_s = A_s Bt_s^T for every slice (bf16 inputs, fp32 or bf16 output)."""
     _check(lib().bsm_bmm(_dptr(a), _dptr(bt), _dptr(c), B, M, N, K, out_dtype, policy,
                          _stream(stream)), "bsm_bmm")
+
+
+def bsm_bmm_ex(a, bt, c, B: int, M: int, N: int, K: int, out_dtype: int, policy: int,
+               n_stages: int = 0, epi_bufs: int = 0, k_blocks_per_stage: int = 0, stream=None):
+    """bsm_bmm with the shared-memory split (stages, store buffers, K blocks
+    per stage) chosen."""
+    _check(lib().bsm_bmm_ex(_dptr(a), _dptr(bt), _dptr(c), B, M, N, K, out_dtype, policy,
+                            n_stages, epi_bufs, k_blocks_per_stage, _stream(stream)), "bsm_bmm_ex")
 
 
 def bsm_softmax_backward(y, dy, dx, B: int, R: int, C: int, dtype: int, policy: int, stream=None):

@@ -39,7 +39,13 @@ constexpr int kBK = 64;                 // bf16 columns per stage: one 128-byte 
 constexpr int kEpiWarps = 8;
 constexpr int kGemmThreads = (2 + kEpiWarps) * 32;
 constexpr int kEpiBuf = 32 * 128;       // one store unit: 32 rows x 128 bytes
-constexpr int kEpiBytes = kEpiWarps * 2 * kEpiBuf;
+
+// Epilogue warps with work: two per TMEM lane quarter when a tile row block
+// has at least two 128-byte store units, else one.
+__host__ __device__ constexpr int epi_active(int bn, bool out_bf16)
+{
+    return (bn * (out_bf16 ? 2 : 4)) / 128 >= 2 ? 8 : 4;
+}
 constexpr int kGemmMaxStages = 8;
 constexpr uint64_t kGemmWaitNs = 2000000000ull;
 
@@ -127,14 +133,14 @@ __device__ __noinline__ bool bar_wait(uint64_t *b, uint32_t parity, const volati
     return false;
 }
 
-// 2-D TMA tile load: box of the tensor map at (c0 = column, c1 = row).
-__device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, int32_t c0, int32_t c1,
+// 3-D TMA tile load: box at (c0 = column in the K block, c1 = row, c2 = K block).
+__device__ __forceinline__ void tma_load_3d(void *dst, const CUtensorMap *map, int32_t c0, int32_t c1, int32_t c2,
                                             uint64_t *bar)
 {
     asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, "
-        "%3}], [%4];" ::"r"(saddr(dst)),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(saddr(bar))
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, "
+        "%3, %4}], [%5];" ::"r"(saddr(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(saddr(bar))
         : "memory");
 }
 
@@ -143,6 +149,19 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, i
 // address (16-byte units), leading-dimension offset (unused for this
 // layout: 1), stride between 8-row groups = 1024 bytes, descriptor version 1,
 // base offset 0 (tiles are 1024-byte aligned), swizzle mode 2 = 128 bytes.
+// Tile record of queue entry idx: read from the plan, or computed when the
+// plan keeps tiles in their natural order (slice, row block, column block).
+template <int BN> __device__ __forceinline__ GemmItem tile_at(const GemmArgs &a, int32_t idx)
+{
+    if (idx < 0 || idx >= a.n_items)
+        return GemmItem{-1, 0, 0, 0};
+    if (!a.identity)
+        return a.items[idx];
+    const int32_t per = a.tiles_m * a.tiles_n;
+    const int32_t s = idx / per, r = idx - s * per;
+    return GemmItem{s, (r / a.tiles_n) * 128, (r % a.tiles_n) * BN, 0};
+}
+
 __device__ __forceinline__ uint64_t smem_desc(const void *tile)
 {
     const uint64_t a = (saddr(tile) & 0x3FFFFu) >> 4;
@@ -208,6 +227,14 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t x, uint32_t
                  : "memory");
 }
 
+// Programmatic dependent launch: the kernel may start while the previous
+// kernel of the stream is finishing; this waits until that kernel has
+// completed and its writes are visible (a no-op without such a predecessor).
+__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// Let the next kernel of the stream start its launch (it still waits on its own
+// grid_dependency_wait before touching memory).
+__device__ __forceinline__ void grid_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 __device__ __forceinline__ uint32_t bf16x2(float lo, float hi)
 {
     uint32_t r;
@@ -220,6 +247,7 @@ __device__ __forceinline__ uint32_t bf16x2(float lo, float hi)
 struct GemmPuller {
     const GemmArgs &a;
     int32_t k = 0, slice = -1, cur = 0, end = 0, q = 0, die = 0;
+    bool first = true;
 
     __device__ explicit GemmPuller(const GemmArgs &args) : a(args)
     {
@@ -248,6 +276,13 @@ struct GemmPuller {
             }
             return cur++;
         }
+        if (a.n_queues == 1) {
+            // one queue: CTA i starts with tile i without touching the
+            // counter; later claims are counter + gridDim.x
+            const uint32_t t = first ? blockIdx.x : atomicAdd(&a.heads[0], 1u) + gridDim.x;
+            first = false;
+            return t < static_cast<uint32_t>(a.queue_len[0]) ? a.queue_begin[0] + static_cast<int32_t>(t) : -1;
+        }
         const int tries = a.steal ? a.n_queues : 1;
         while (q < tries) {
             const int qq = (die + q) % a.n_queues;
@@ -272,57 +307,67 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     GemmSmem &h = *reinterpret_cast<GemmSmem *>(smem);
     constexpr uint32_t kABytes = kBM * kBK * 2;
     constexpr uint32_t kBBytes = BN * kBK * 2;
-    constexpr uint32_t kStage = kABytes + kBBytes;
+    const int G = a.kbs;                                   // K blocks per stage (one 3-D copy each)
+    const uint32_t stage_bytes = static_cast<uint32_t>(G) * (kABytes + kBBytes);
     constexpr uint32_t kTmemCols = 2 * BN;
-    unsigned char *epi = smem + 1024;                      // kEpiBytes of store buffers
-    unsigned char *stages = smem + 1024 + kEpiBytes;
+    constexpr int kActive = epi_active(BN, kOutBf16);
+    const int bufs = a.epi_bufs;                           // store buffers per active warp
+    unsigned char *epi = smem + 1024;
+    unsigned char *stages = smem + 1024 + kActive * bufs * kEpiBuf;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int S = a.n_stages;
-    const int KB = a.K / kBK;
-
-    if (threadIdx.x == 0) {
-        for (int s = 0; s < S; ++s) {
-            bar_init(&h.full[s], 1);
-            bar_init(&h.empty[s], 1);
-        }
-        for (int b = 0; b < 2; ++b) {
-            bar_init(&h.tfull[b], 1);
-            bar_init(&h.tempty[b], kEpiWarps);
-        }
-        bar_init(&h.drain, 1);
-        h.abort_flag = 0;
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    }
-    if (warp == 1) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(saddr(&h.tmem_base)),
-                     "r"(kTmemCols)
-                     : "memory");
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tmem = h.tmem_base;
+    const int NS = a.K / (kBK * G);                        // stages per tile
 
     if (warp == 0) {
         // ------------------------------------------------------- producer
+        // The first claim and the tensor-map fetches are issued before the
+        // barriers are set up; the producer streams as soon as they exist,
+        // without waiting for the tensor-memory allocation.
+        GemmPuller pull(a);
+        int32_t idx = -1;
         if (lane == 0) {
-            GemmPuller pull(a);
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmC)) : "memory");
+            const bool static_first = a.mode != PULL_QUEUE || a.n_queues == 1;
+            if (static_first)
+                idx = pull.next();                 // no memory access: before the wait
+            for (int s = 0; s < S; ++s) {
+                bar_init(&h.full[s], 1);
+                bar_init(&h.empty[s], 1);
+            }
+            for (int b = 0; b < 2; ++b) {
+                bar_init(&h.tfull[b], 1);
+                bar_init(&h.tempty[b], kActive);
+            }
+            bar_init(&h.drain, 1);
+            h.abort_flag = 0;
+            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+            // launched early behind the previous kernel of the stream: from
+            // here on memory is touched, so wait until that kernel is done
+            grid_dependency_wait();
+            if (!static_first)
+                idx = pull.next();
+        }
+        __syncwarp();
+        asm volatile("barrier.cta.arrive 1, %0;" ::"r"(kGemmThreads) : "memory");   // barriers ready
+        grid_launch_dependents();
+        if (lane == 0) {
             uint32_t it = 0;
             bool ok = true;
+            // the next tile is claimed (and its record fetched) while the
+            // current one streams, so the ring never waits on the queue
+            GemmItem item = tile_at<BN>(a, idx);
             for (;;) {
-                const int32_t idx = pull.next();
-                GemmItem item{};
+                const int32_t nidx = idx >= 0 ? pull.next() : -1;
                 const bool have = idx >= 0 && idx < a.n_items;
-                if (have)
-                    item = a.items[idx];
                 const bool valid = have && item.slice >= 0 && item.slice < a.B && item.m0 >= 0 &&
                                    item.m0 + kBM <= a.M && item.n0 >= 0 && item.n0 + BN <= a.N;
-                if (have && !valid)
-                    atomicOr(a.status, BSM_DEV_BOUNDS);
                 if (idx >= 0 && !valid)
-                    continue;                       // skip a bad tile, keep going
-                for (int kb = 0; kb < (idx < 0 ? 1 : KB); ++kb) {
+                    atomicOr(a.status, BSM_DEV_BOUNDS);     // skip a bad tile, keep going
+                GemmItem nitem{};
+                const int nks = idx < 0 ? 1 : (valid ? NS : 0);
+                for (int kb = 0; kb < nks; ++kb) {
                     const int s = static_cast<int>(it % S);
                     const uint32_t ph = (it / S) & 1u;
                     if (!bar_wait(&h.empty[s], ph ^ 1u, &h.abort_flag)) {
@@ -337,13 +382,19 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     }
                     if (kb == 0)
                         h.smeta[s] = GemmMeta{item.slice, item.m0, item.n0, GK_DATA};
-                    unsigned char *st = stages + (size_t)s * kStage;
-                    bar_expect(&h.full[s], kStage);
-                    tma_load_2d(st, &tmA, kb * kBK, item.slice * a.M + item.m0, &h.full[s]);
-                    tma_load_2d(st + kABytes, &tmB, kb * kBK, item.slice * a.N + item.n0, &h.full[s]);
+                    unsigned char *st = stages + (size_t)s * stage_bytes;
+                    bar_expect(&h.full[s], stage_bytes);
+                    tma_load_3d(st, &tmA, 0, item.slice * a.M + item.m0, kb * G, &h.full[s]);
+                    tma_load_3d(st + G * kABytes, &tmB, 0, item.slice * a.N + item.n0, kb * G, &h.full[s]);
+                    if (kb == 0)
+                        nitem = tile_at<BN>(a, nidx);
                 }
                 if (!ok || idx < 0)
                     break;
+                if (nks == 0)
+                    nitem = tile_at<BN>(a, nidx);
+                idx = nidx;
+                item = nitem;
             }
             if (!ok) {
                 atomicOr(a.status, BSM_DEV_TIMEOUT);
@@ -363,134 +414,160 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 }
             }
         }
-    } else if (warp == 1) {
-        // ------------------------------------------------------- MMA issuer
-        if (lane == 0) {
-            const uint32_t idesc = mma_idesc<BN>();
-            uint32_t it = 0, t = 0;
-            bool ok = true;
-            for (;;) {
-                int s = static_cast<int>(it % S);
-                uint32_t ph = (it / S) & 1u;
-                if (!bar_wait(&h.full[s], ph, &h.abort_flag)) {
-                    ok = false;
-                    break;
-                }
-                const GemmMeta m = h.smeta[s];
-                const int buf = static_cast<int>(t & 1u);
-                const uint32_t tph = (t >> 1) & 1u;
-                if (!bar_wait(&h.tempty[buf], tph ^ 1u, &h.abort_flag)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                h.tmeta[buf] = m;
-                __threadfence_block();              // visible before the MMAs (and their commit)
-                if (m.kind == GK_DONE) {
-                    bar_arrive(&h.tfull[buf]);
-                    break;
-                }
-                const uint32_t d = tmem + static_cast<uint32_t>(buf * BN);
-                for (int kb = 0; kb < KB; ++kb) {
-                    if (kb > 0) {
-                        s = static_cast<int>(it % S);
-                        ph = (it / S) & 1u;
-                        if (!bar_wait(&h.full[s], ph, &h.abort_flag)) {
-                            ok = false;
-                            break;
-                        }
+    } else {
+        asm volatile("barrier.cta.sync 1, %0;" ::"r"(kGemmThreads) : "memory");          // barriers ready
+        if (warp == 1) {
+            asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(saddr(&h.tmem_base)),
+                         "r"(kTmemCols)
+                         : "memory");
+            asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+        }
+        tc_fence_before();
+        asm volatile("barrier.cta.sync 2, %0;" ::"r"(kGemmThreads - 32) : "memory");     // TMEM address ready
+        tc_fence_after();
+        const uint32_t tmem = h.tmem_base;
+        if (warp == 1) {
+            // ------------------------------------------------------- MMA issuer
+            if (lane == 0) {
+                // no bounded wait may start before the previous kernel is done
+                grid_dependency_wait();
+                const uint32_t idesc = mma_idesc<BN>();
+                uint32_t it = 0, t = 0;
+                bool ok = true;
+                for (;;) {
+                    int s = static_cast<int>(it % S);
+                    uint32_t ph = (it / S) & 1u;
+                    if (!bar_wait(&h.full[s], ph, &h.abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    const GemmMeta m = h.smeta[s];
+                    const int buf = static_cast<int>(t & 1u);
+                    const uint32_t tph = (t >> 1) & 1u;
+                    if (!bar_wait(&h.tempty[buf], tph ^ 1u, &h.abort_flag)) {
+                        ok = false;
+                        break;
                     }
                     tc_fence_after();
-                    unsigned char *st = stages + (size_t)s * kStage;
-                    const uint64_t ad = smem_desc(st), bd = smem_desc(st + kABytes);
-#pragma unroll
-                    for (int k = 0; k < kBK / 16; ++k)
-                        mma_bf16(d, ad + 2 * k, bd + 2 * k, idesc, (kb | k) != 0);
-                    mma_commit(&h.empty[s]);        // the stage is free once these are done
-                    ++it;
+                    h.tmeta[buf] = m;
+                    __threadfence_block();              // visible before the MMAs (and their commit)
+                    if (m.kind == GK_DONE) {
+                        bar_arrive(&h.tfull[buf]);
+                        break;
+                    }
+                    const uint32_t d = tmem + static_cast<uint32_t>(buf * BN);
+                    for (int kb = 0; kb < NS; ++kb) {
+                        if (kb > 0) {
+                            s = static_cast<int>(it % S);
+                            ph = (it / S) & 1u;
+                            if (!bar_wait(&h.full[s], ph, &h.abort_flag)) {
+                                ok = false;
+                                break;
+                            }
+                        }
+                        tc_fence_after();
+                        unsigned char *st = stages + (size_t)s * stage_bytes;
+                        for (int j = 0; j < G; ++j) {
+                            const uint64_t ad = smem_desc(st + j * kABytes);
+                            const uint64_t bd = smem_desc(st + G * kABytes + j * kBBytes);
+    #pragma unroll
+                            for (int k = 0; k < kBK / 16; ++k)
+                                mma_bf16(d, ad + 2 * k, bd + 2 * k, idesc, (kb | j | k) != 0);
+                        }
+                        mma_commit(&h.empty[s]);        // the stage is free once these are done
+                        ++it;
+                    }
+                    if (!ok)
+                        break;
+                    mma_commit(&h.tfull[buf]);          // the accumulator is ready
+                    ++t;
                 }
-                if (!ok)
-                    break;
-                mma_commit(&h.tfull[buf]);          // the accumulator is ready
-                ++t;
-            }
-            if (!ok) {
-                atomicOr(a.status, BSM_DEV_TIMEOUT);
-                h.abort_flag = 1;
-            }
-            // every MMA issued has finished before the tensor memory is freed
-            mma_commit(&h.drain);
-            bar_wait(&h.drain, 0, nullptr);
-        }
-    } else {
-        // ------------------------------------------------------- epilogue
-        constexpr int kEs = kOutBf16 ? 2 : 4;
-        constexpr int kUnitCols = 128 / kEs;                  // output columns per store unit
-        constexpr int kUnits = BN / kUnitCols;                // store units per tile row block
-        const int ew = warp - 2;
-        const int quarter = warp & 3;                         // TMEM lanes this warp may read
-        const int half = ew >> 2;                             // which units of the quarter
-        const uint32_t buf0 = saddr(epi + ew * 2 * kEpiBuf);
-        uint32_t nst = 0;                                     // units stored by this warp
-        for (uint32_t t = 0;; ++t) {
-            const int buf = static_cast<int>(t & 1u);
-            // lane 0 waits; the warp follows its verdict (tcgen05.ld is warp-wide)
-            int ok = 0;
-            if (lane == 0) {
-                ok = bar_wait(&h.tfull[buf], (t >> 1) & 1u, &h.abort_flag);
                 if (!ok) {
                     atomicOr(a.status, BSM_DEV_TIMEOUT);
                     h.abort_flag = 1;
                 }
+                // every MMA issued has finished before the tensor memory is freed
+                mma_commit(&h.drain);
+                bar_wait(&h.drain, 0, nullptr);
             }
-            ok = __shfl_sync(0xffffffffu, ok, 0);
-            __syncwarp();
-            if (!ok)
-                break;
-            tc_fence_after();
-            const GemmMeta m = h.tmeta[buf];
-            if (m.kind == GK_DONE)
-                break;
-            const uint32_t tbase =
-                tmem + (static_cast<uint32_t>(quarter * 32) << 16) + static_cast<uint32_t>(buf * BN);
-            const int32_t crow = m.slice * a.M + m.m0 + quarter * 32;
-#pragma unroll 1
-            for (int u = half; u < kUnits; u += 2, ++nst) {
-                uint32_t r[64];
-                tmem_ld32_nowait(tbase + static_cast<uint32_t>(u * kUnitCols), r);
-                if (kOutBf16)
-                    tmem_ld32_nowait(tbase + static_cast<uint32_t>(u * kUnitCols + 32), r + 32);
-                tmem_wait_ld();
-                // the buffer written two units ago must have been read by its store
-                if (lane == 0)
-                    asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
-                __syncwarp();
-                const uint32_t sb = buf0 + (nst & 1u) * kEpiBuf + static_cast<uint32_t>(lane * 128);
-#pragma unroll
-                for (int c = 0; c < 8; ++c) {
-                    const uint32_t dst = sb + (static_cast<uint32_t>(c ^ (lane & 7)) << 4);
-                    if (kOutBf16) {
-                        const float *f = reinterpret_cast<const float *>(r + 8 * c);
-                        st_shared_v4(dst, bf16x2(f[0], f[1]), bf16x2(f[2], f[3]), bf16x2(f[4], f[5]),
-                                     bf16x2(f[6], f[7]));
-                    } else {
-                        st_shared_v4(dst, r[4 * c], r[4 * c + 1], r[4 * c + 2], r[4 * c + 3]);
+        } else {
+            // ------------------------------------------------------- epilogue
+            constexpr int kEs = kOutBf16 ? 2 : 4;
+            constexpr int kUnitCols = 128 / kEs;                  // output columns per store unit
+            constexpr int kUnits = BN / kUnitCols;                // store units per tile row block
+            const int ew = warp - 2;
+            const int quarter = warp & 3;                         // TMEM lanes this warp may read
+            const int half = ew >> 2;                             // which units of the quarter
+            unsigned char *mybuf = epi + ew * bufs * kEpiBuf;
+            uint32_t nst = 0;                                     // units stored by this warp
+            grid_dependency_wait();                       // before any wait or store
+            for (uint32_t t = 0; ew < kActive; ++t) {
+                const int buf = static_cast<int>(t & 1u);
+                // lane 0 waits; the warp follows its verdict (tcgen05.ld is warp-wide)
+                int ok = 0;
+                if (lane == 0) {
+                    ok = bar_wait(&h.tfull[buf], (t >> 1) & 1u, &h.abort_flag);
+                    if (!ok) {
+                        atomicOr(a.status, BSM_DEV_TIMEOUT);
+                        h.abort_flag = 1;
                     }
                 }
-                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                ok = __shfl_sync(0xffffffffu, ok, 0);
+                __syncwarp();
+                if (!ok)
+                    break;
+                tc_fence_after();
+                const GemmMeta m = h.tmeta[buf];
+                if (m.kind == GK_DONE)
+                    break;
+                const uint32_t tbase =
+                    tmem + (static_cast<uint32_t>(quarter * 32) << 16) + static_cast<uint32_t>(buf * BN);
+                const int32_t crow = m.slice * a.M + m.m0 + quarter * 32;
+    #pragma unroll 1
+                for (int u = half; u < kUnits; u += kActive / 4, ++nst) {
+                    uint32_t r[64];
+                    tmem_ld32_nowait(tbase + static_cast<uint32_t>(u * kUnitCols), r);
+                    if (kOutBf16)
+                        tmem_ld32_nowait(tbase + static_cast<uint32_t>(u * kUnitCols + 32), r + 32);
+                    tmem_wait_ld();
+                    // the buffer about to be rewritten must have been read by its store
+                    if (lane == 0) {
+                        if (bufs >= 4)
+                            asm volatile("cp.async.bulk.wait_group.read 3;" ::: "memory");
+                        else if (bufs == 3)
+                            asm volatile("cp.async.bulk.wait_group.read 2;" ::: "memory");
+                        else
+                            asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+                    }
+                    __syncwarp();
+                    unsigned char *ub = mybuf + (nst % static_cast<uint32_t>(bufs)) * kEpiBuf;
+                    const uint32_t sb = saddr(ub) + static_cast<uint32_t>(lane * 128);
+    #pragma unroll
+                    for (int c = 0; c < 8; ++c) {
+                        const uint32_t dst = sb + (static_cast<uint32_t>(c ^ (lane & 7)) << 4);
+                        if (kOutBf16) {
+                            const float *f = reinterpret_cast<const float *>(r + 8 * c);
+                            st_shared_v4(dst, bf16x2(f[0], f[1]), bf16x2(f[2], f[3]), bf16x2(f[4], f[5]),
+                                         bf16x2(f[6], f[7]));
+                        } else {
+                            st_shared_v4(dst, r[4 * c], r[4 * c + 1], r[4 * c + 2], r[4 * c + 3]);
+                        }
+                    }
+                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                    __syncwarp();
+                    if (lane == 0)
+                        tma_store_2d(&tmC, m.n0 + u * kUnitCols, crow, ub);
+                }
+                tc_fence_before();
                 __syncwarp();
                 if (lane == 0)
-                    tma_store_2d(&tmC, m.n0 + u * kUnitCols, crow, epi + ew * 2 * kEpiBuf + (nst & 1u) * kEpiBuf);
+                    bar_arrive(&h.tempty[buf]);
             }
-            tc_fence_before();
-            __syncwarp();
+            // stores complete before the CTA leaves
             if (lane == 0)
-                bar_arrive(&h.tempty[buf]);
+                asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+            __syncwarp();
         }
-        // stores complete before the CTA leaves
-        if (lane == 0)
-            asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
-        __syncwarp();
     }
 
     // every thread gets here (all waits are bounded); then the owner frees TMEM
@@ -499,7 +576,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     if (warp == 1) {
         __syncwarp();
         tc_fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(h.tmem_base), "r"(kTmemCols)
                      : "memory");
     }
 }
@@ -508,16 +585,34 @@ template <int BN, bool kOutBf16>
 int launch_bn(const CUtensorMap &ta, const CUtensorMap &tb, const CUtensorMap &tc, const GemmArgs &a, int grid,
               cudaStream_t st)
 {
-    const size_t smem = 2048 + kEpiBytes + (size_t)a.n_stages * (kBM * kBK * 2 + BN * kBK * 2);
+    const size_t smem = static_cast<size_t>(gemm_fixed_smem(BN, kOutBf16, a.epi_bufs)) +
+                        (size_t)a.n_stages * a.kbs * (kBM * kBK * 2 + BN * kBK * 2);
+#ifndef BSM_NO_PDL
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(grid));
+    cfg.blockDim = dim3(kGemmThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return static_cast<int>(cudaLaunchKernelEx(&cfg, bmm_persistent<BN, kOutBf16>, ta, tb, tc, a));
+#else
     bmm_persistent<BN, kOutBf16><<<grid, kGemmThreads, smem, st>>>(ta, tb, tc, a);
     return static_cast<int>(cudaGetLastError());
+#endif
 }
 
 }  // namespace
 
 int gemm_stage_bytes(int bn) { return kBM * kBK * 2 + bn * kBK * 2; }
 int gemm_threads() { return kGemmThreads; }
-int gemm_fixed_smem() { return 2048 + kEpiBytes; }
+int gemm_fixed_smem(int bn, bool out_bf16, int epi_bufs)
+{
+    return 2048 + epi_active(bn, out_bf16) * epi_bufs * kEpiBuf;
+}
 
 int gemm_set_smem_limit(int bytes)
 {

@@ -66,6 +66,22 @@ int gemm_device(int device, GemmDev **out)
     return BSM_OK;
 }
 
+// Operand view of a (rows_total x K) bf16 row-major matrix as K/64 blocks of
+// 64 columns: dims (64, rows, K/64), one box = box_rows rows x kbs blocks,
+// 128-byte swizzle; in shared memory the blocks follow one another, each
+// box_rows x 128 bytes -- the K-major layout the MMA descriptors read.
+int make_operand_map(CUtensorMap *m, const void *base, int64_t rows_total, int64_t K, int box_rows, int kbs)
+{
+    const cuuint64_t dims[3] = {64u, static_cast<cuuint64_t>(rows_total), static_cast<cuuint64_t>(K / 64)};
+    const cuuint64_t strides[2] = {static_cast<cuuint64_t>(K * 2), 128u};
+    const cuuint32_t box[3] = {64u, static_cast<cuuint32_t>(box_rows), static_cast<cuuint32_t>(kbs)};
+    const cuuint32_t estr[3] = {1u, 1u, 1u};
+    const CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box,
+                                estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? BSM_OK : BSM_ERR_INVALID_ARG;
+}
+
 // box_rows x (128 bytes) boxes of a (rows_total x cols) row-major matrix, 128-byte swizzle
 int make_map(CUtensorMap *m, const void *base, int64_t rows_total, int64_t cols, int box_rows, bool f32 = false)
 {
@@ -83,6 +99,7 @@ int make_map(CUtensorMap *m, const void *base, int64_t rows_total, int64_t cols,
 
 struct GemmPlan {
     int device = 0, policy = 0, bn = 0, grid = 0;
+    int want_stages = 0, want_bufs = 0, want_kbs = 0;   // caller's choices (0 = automatic)
     bool out_bf16 = false;
     const void *a = nullptr, *bt = nullptr;
     void *c = nullptr;
@@ -234,7 +251,38 @@ int build_plan(GemmPlan *p, const GemmDev &dev)
     a.steal = steal;
     a.heads = reinterpret_cast<uint32_t *>(b + o_heads);
     a.sm_die = use_die ? reinterpret_cast<const int8_t *>(b + o_smdie) : nullptr;
-    a.n_stages = std::min(8, (dev.smem_optin - gemm_fixed_smem()) / gemm_stage_bytes(bn));
+    // shared memory split: with few K blocks per tile the output dominates,
+    // so favour store buffers; with many, favour stages in flight
+    // and fetch several K blocks per copy when the tile has them (longer
+    // runs of each operand row per request), keeping two stages or more
+    const int64_t kb = p->K / 64;
+    int kbs = p->want_kbs;
+    if (!kbs) {
+        kbs = 1;
+        for (int g : {4, 2})
+            if (kb % g == 0 &&
+                (dev.smem_optin - gemm_fixed_smem(bn, p->out_bf16, 2)) / (g * gemm_stage_bytes(bn)) >= 2) {
+                kbs = g;
+                break;
+            }
+    }
+    if (kb % kbs)
+        return BSM_ERR_UNSUPPORTED;
+    int bufs = p->want_bufs ? p->want_bufs : (kb <= 2 ? 4 : 2);
+    int fit = 0;
+    for (;; --bufs) {
+        fit = (dev.smem_optin - gemm_fixed_smem(bn, p->out_bf16, bufs)) / (kbs * gemm_stage_bytes(bn));
+        if (fit >= 2 || bufs <= 2 || p->want_bufs)
+            break;
+    }
+    a.epi_bufs = bufs;
+    a.kbs = kbs;
+    a.identity = use_die ? 0 : 1;
+    a.tiles_m = static_cast<int32_t>(mt);
+    a.tiles_n = static_cast<int32_t>(nt);
+    a.n_stages = std::min(8, fit);
+    if (p->want_stages)
+        a.n_stages = p->want_stages <= fit ? p->want_stages : 0;
     a.status = dev.status;
     if (a.n_stages < 2)
         return BSM_ERR_UNSUPPORTED;
@@ -253,9 +301,9 @@ int build_plan(GemmPlan *p, const GemmDev &dev)
         p->grid = dev.n_sm;
         break;
     }
-    if (int rc = make_map(&p->ta, p->a, p->B * p->M, p->K, 128))
+    if (int rc = make_operand_map(&p->ta, p->a, p->B * p->M, p->K, 128, kbs))
         return rc;
-    if (int rc = make_map(&p->tb, p->bt, p->B * p->N, p->K, bn))
+    if (int rc = make_operand_map(&p->tb, p->bt, p->B * p->N, p->K, bn, kbs))
         return rc;
     if (int rc = make_map(&p->tc, p->c, p->B * p->M, p->N, 32, !p->out_bf16))
         return rc;
@@ -280,10 +328,12 @@ int run_plan(GemmPlan *p, bsm_stream_t stream)
 }
 
 int bmm_impl(const void *a, const void *bt, void *c, int64_t B, int64_t M, int64_t N, int64_t K, int out_dtype,
-             int policy, bsm_stream_t stream)
+             int policy, int n_stages, int epi_bufs, int kbs, bsm_stream_t stream)
 {
     if (B < 0 || M < 0 || N < 0 || K < 0 || (out_dtype != BSM_F32 && out_dtype != BSM_BF16) ||
-        policy < BSM_POLICY_WHOLE_GPU || policy > BSM_POLICY_MINIMAX)
+        policy < BSM_POLICY_WHOLE_GPU || policy > BSM_POLICY_MINIMAX || n_stages < 0 || n_stages == 1 ||
+        n_stages > 8 || epi_bufs < 0 || epi_bufs == 1 || epi_bufs > 4 || (kbs != 0 && kbs != 1 && kbs != 2 &&
+                                                                           kbs != 4))
         return BSM_ERR_INVALID_ARG;
     if (B == 0 || M == 0 || N == 0)
         return BSM_OK;
@@ -312,7 +362,8 @@ int bmm_impl(const void *a, const void *bt, void *c, int64_t B, int64_t M, int64
     for (auto it = g_gcache.begin(); it != g_gcache.end(); ++it) {
         GemmPlan *p = *it;
         if (p->device == device && p->a == a && p->bt == bt && p->c == c && p->B == B && p->M == M && p->N == N &&
-            p->K == K && p->out_bf16 == (out_dtype == BSM_BF16) && p->policy == policy) {
+            p->K == K && p->out_bf16 == (out_dtype == BSM_BF16) && p->policy == policy &&
+            p->want_stages == n_stages && p->want_bufs == epi_bufs && p->want_kbs == kbs) {
             g_gcache.splice(g_gcache.begin(), g_gcache, it);
             return run_plan(p, stream);
         }
@@ -320,6 +371,9 @@ int bmm_impl(const void *a, const void *bt, void *c, int64_t B, int64_t M, int64
     GemmPlan *p = new GemmPlan();
     p->device = device;
     p->policy = policy;
+    p->want_stages = n_stages;
+    p->want_bufs = epi_bufs;
+    p->want_kbs = kbs;
     p->bn = N % 256 == 0 ? 256 : (N % 128 == 0 ? 128 : 64);
     p->out_bf16 = out_dtype == BSM_BF16;
     p->a = a;
@@ -348,7 +402,19 @@ extern "C" int bsm_bmm(const void *a, const void *bt, void *c, int64_t B, int64_
                        int out_dtype, int policy, bsm_stream_t stream)
 {
     try {
-        return bsm::bmm_impl(a, bt, c, B, M, N, K, out_dtype, policy, stream);
+        return bsm::bmm_impl(a, bt, c, B, M, N, K, out_dtype, policy, 0, 0, 0, stream);
+    } catch (const std::bad_alloc &) {
+        return BSM_ERR_NOMEM;
+    }
+}
+
+extern "C" int bsm_bmm_ex(const void *a, const void *bt, void *c, int64_t B, int64_t M, int64_t N, int64_t K,
+                          int out_dtype, int policy, int n_stages, int epi_bufs, int k_blocks_per_stage,
+                          bsm_stream_t stream)
+{
+    try {
+        return bsm::bmm_impl(a, bt, c, B, M, N, K, out_dtype, policy, n_stages, epi_bufs, k_blocks_per_stage,
+                             stream);
     } catch (const std::bad_alloc &) {
         return BSM_ERR_NOMEM;
     }

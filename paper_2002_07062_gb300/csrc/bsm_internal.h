@@ -97,6 +97,10 @@ struct GemmArgs {
     uint32_t *heads;
     const int8_t *sm_die;
     int32_t n_stages;
+    int32_t epi_bufs;               // 2..4 store buffers per epilogue warp
+    int32_t kbs;                    // K blocks of 64 per stage (1, 2 or 4)
+    int32_t identity;               // items in natural order: computed, not read
+    int32_t tiles_m, tiles_n;       // row / column blocks per slice
     uint32_t *status;
 };
 
@@ -107,8 +111,9 @@ int launch_bmm(const void *tmap_a, const void *tmap_b, const void *tmap_c, const
                bool out_bf16, int grid, void *stream);
 int gemm_set_smem_limit(int bytes);
 int gemm_stage_bytes(int bn);
-// shared memory of one launch besides the stages (header, slack, epilogue buffers)
-int gemm_fixed_smem();
+// shared memory of one launch besides the stages (header, slack, epilogue
+// store buffers: epi_bufs of 4 KiB per epilogue warp with work)
+int gemm_fixed_smem(int bn, bool out_bf16, int epi_bufs);
 
 // Launch the persistent softmax kernel (bsm_kernels.cu).  Returns a
 // cudaError_t value (0 = success).
