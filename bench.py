@@ -235,8 +235,11 @@ def cpu_baseline(w, seconds: float = 10.0):
                       "%d threads)" % (n_sl, w.nslices, passes, per, cores)}
 
 
-def time_steps(fn, steps, stream, per_launch=True):
-    """Run fn() `steps` times on `stream`; returns (total ms, per-step ms list)."""
+def time_steps(fn, steps, stream, per_launch=False):
+    """Run fn() `steps` times on `stream`; returns (total ms, per-step ms list).
+    With per_launch, an event pair brackets every step -- which also keeps
+    consecutive launches from overlapping, so the timed region uses one event
+    pair around all steps."""
     import torch
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(steps)] if per_launch else []
@@ -265,6 +268,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--sweep", action="store_true",
                     help="also time every policy on workloads 2-5 (extra JSON lines)")
+    ap.add_argument("--bmm", type=int, default=0, choices=[0, 1, 2],
+                    help="time the Sec. 6 batched product 1 or 2 instead of the softmax")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=20)
@@ -293,6 +298,9 @@ def main():
         dist.barrier()
         g.build()
     dev = torch.cuda.current_device()
+
+    if args.bmm:
+        return run_bmm(args, bsm, workload, ws, rank, dev)
 
     w = workload.config(args.workload).materialize()
     pol = policy_code(args.policy)
@@ -328,7 +336,7 @@ def main():
         dist.barrier()
     torch.cuda.synchronize()
     with ClockSampler(dev) as clk:
-        total_ms, per = time_steps(step, args.steps, stream, per_launch=launches_per_step == 1)
+        total_ms, _ = time_steps(step, args.steps, stream)
     torch.cuda.synchronize()
     if ws > 1:
         dist.barrier()
@@ -338,8 +346,10 @@ def main():
     bytes_step = w.algorithmic_bytes
     value = job_gbs(ws, bytes_step, args.steps, total_ms)
     peak, peak_src = measured_peak()
-    launch_ms = float(np.mean(per)) if per else ms
-    achieved = bytes_step / (launch_ms * 1e-3) / 1e9
+    # average duration of one launch of the kernel over the timed region (the
+    # step is nothing but its launches)
+    launch_ms = total_ms / (args.steps * launches_per_step)
+    achieved = bytes_step / launches_per_step / (launch_ms * 1e-3) / 1e9
     traffic = profiled_traffic(args.workload, "f32")
 
     out = {
@@ -424,8 +434,7 @@ def sweep(args, bsm, workload, stream):
             for _ in range(3):
                 step()
             stream.synchronize()
-            _, per = time_steps(step, reps, stream, per_launch=True)
-            med = float(np.median(per))
+            med = _median_ms(step, reps, stream)
             print(json.dumps({"sweep": True, "workload": w.name, "policy": name,
                               "ms": round(med, 4),
                               "GBps": round(w.algorithmic_bytes / (med * 1e-3) / 1e9, 2),
@@ -444,8 +453,7 @@ def sweep(args, bsm, workload, stream):
             for _ in range(3):
                 bstep()
             stream.synchronize()
-            _, per = time_steps(bstep, 20, stream, per_launch=True)
-            med = float(np.median(per))
+            med = _median_ms(bstep, 20, stream)
             nbytes = 3 * w.numel * w.esize
             print(json.dumps({"sweep": True, "op": "backward", "workload": w.name,
                               "policy": "dynamic", "ms": round(med, 4),
@@ -453,6 +461,96 @@ def sweep(args, bsm, workload, stream):
             del dy, dx
         del x, y
         torch.cuda.empty_cache()
+    bmm_sweep(bsm, workload, stream)
+
+
+def run_bmm(args, bsm, workload, ws, rank, dev):
+    """One JSON line for a Sec. 6 batched product on the tensor cores
+    (operands resident, back-to-back launches, one event pair)."""
+    import numpy as np
+    import torch
+    w = workload.bmm_config(args.bmm)
+    a_bits, bt_bits = w.operands()
+    a = torch.from_numpy(a_bits.view(np.int16)).cuda()
+    bt = torch.from_numpy(bt_bits.view(np.int16)).cuda()
+    c = torch.empty(w.B * w.M * w.N, dtype=torch.int16, device="cuda")
+    stream = torch.cuda.Stream()
+    pol = policy_code(args.policy)
+
+    def step():
+        bsm.bsm_bmm(a, bt, c, w.B, w.M, w.N, w.K, w.out_dtype, pol, stream)
+    for _ in range(max(3, args.warmup)):
+        step()
+    stream.synchronize()
+    launches = w.B if pol == bsm.POLICY_WHOLE_GPU else 1
+    with ClockSampler(dev) as clk:
+        total_ms, _ = time_steps(step, args.steps, stream)
+    torch.cuda.synchronize()
+    ms = total_ms / args.steps
+    gbs = w.algorithmic_bytes / (ms * 1e-3) / 1e9
+    peak, peak_src = measured_peak()
+    out = {"metric": "batched matmul GB/s (operands read + product written)", "value": round(gbs, 2),
+           "unit": "GB/s", "n_gpus": 1, "steps": args.steps, "warmup": max(3, args.warmup),
+           "ms_per_step": round(ms, 5), "higher_is_better": True, "scaling": "weak",
+           "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+           "config": {"workload": w.name, "policy": args.policy, "bytes_per_step": w.algorithmic_bytes,
+                      "flops_per_step": w.flops,
+                      "l2": "operands + product %d MB vs 129 MB L2, no flush" % (w.algorithmic_bytes >> 20)},
+           "tflops": round(w.flops / (ms * 1e-3) / 1e12, 2),
+           "gpu_launches": launches * args.steps,
+           "roofline": {"bound": "hbm", "achieved": round(gbs, 2), "peak": peak, "unit": "GB/s",
+                        "frac": round(gbs / peak, 4), "traffic": None, "peak_source": peak_src,
+                        "kernel": "bmm_persistent", "launch_ms": round(ms / launches, 5)},
+           "clocks": clk.summary(), "device_status": bsm.bsm_device_status()}
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    return 0
+
+
+def _median_ms(fn, reps, stream, rounds=5):
+    """Median over `rounds` of the mean time of `reps` back-to-back calls."""
+    import numpy as np
+    return float(np.median([time_steps(fn, reps, stream)[0] / reps for _ in range(rounds)]))
+
+
+def bmm_sweep(bsm, workload, stream):
+    """The batched products of Sec. 6 on the tensor cores under every policy,
+    with torch.bmm (cuBLAS) on the same operands as context."""
+    import torch
+    for k in (1, 2):
+        w = workload.bmm_config(k)
+        a_bits, bt_bits = w.operands()
+        import numpy as np
+        a = torch.from_numpy(a_bits.view(np.int16)).cuda()
+        bt = torch.from_numpy(bt_bits.view(np.int16)).cuda()
+        c = torch.empty(w.B * w.M * w.N, dtype=torch.int16, device="cuda")
+        for name in ("whole_gpu", "rr", "dynamic", "cbmf", "cbmf_lb", "minimax"):
+            pol = bsm.POLICIES[name]
+
+            def step():
+                bsm.bsm_bmm(a, bt, c, w.B, w.M, w.N, w.K, w.out_dtype, pol, stream)
+            for _ in range(3):
+                step()
+            stream.synchronize()
+            med = _median_ms(step, 5 if name == "whole_gpu" else 50, stream)
+            print(json.dumps({"sweep": True, "op": "bmm", "workload": w.name, "policy": name,
+                              "ms": round(med, 5),
+                              "GBps": round(w.algorithmic_bytes / (med * 1e-3) / 1e9, 2),
+                              "TFLOPs": round(w.flops / (med * 1e-3) / 1e12, 2)}), flush=True)
+        A3 = a.view(torch.bfloat16).view(w.B, w.M, w.K)
+        B3 = bt.view(torch.bfloat16).view(w.B, w.N, w.K)
+        with torch.cuda.stream(stream):
+            def lib_step():
+                torch.bmm(A3, B3.transpose(1, 2))
+            for _ in range(3):
+                lib_step()
+            stream.synchronize()
+            med = _median_ms(lib_step, 50, stream)
+        print(json.dumps({"sweep": True, "op": "bmm", "workload": w.name,
+                          "policy": "torch.bmm (cuBLAS), context only", "ms": round(med, 5),
+                          "GBps": round(w.algorithmic_bytes / (med * 1e-3) / 1e9, 2),
+                          "TFLOPs": round(w.flops / (med * 1e-3) / 1e12, 2)}), flush=True)
+        del a, bt, c
 
 
 if __name__ == "__main__":

@@ -871,6 +871,12 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
         mbar_init_fence();
     }
     __syncthreads();
+    // Programmatic dependent launch: this kernel may have started while the
+    // previous kernel of the stream was finishing.  No role touches memory or
+    // starts a bounded wait before that kernel is done (a no-op without such
+    // a predecessor); then the next kernel may begin its own launch.
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
     if (warp == kConsumerWarps) {
         // ------------------------------------------------------- producer
@@ -1151,10 +1157,25 @@ namespace {
 template <typename Tag, int Op>
 void launch_one(const KernelArgs &a, int grid, size_t smem, cudaStream_t st, bool checked)
 {
+    // launched with programmatic stream serialisation: the kernel's prologue
+    // overlaps the tail of the previous kernel (see griddepcontrol.wait)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(grid));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+#ifdef BSM_NO_PDL
+    cfg.numAttrs = 0;
+#endif
     if (checked)
-        softmax_persistent<Tag, Op, true><<<grid, kThreads, smem, st>>>(a);
+        cudaLaunchKernelEx(&cfg, softmax_persistent<Tag, Op, true>, a);
     else
-        softmax_persistent<Tag, Op, false><<<grid, kThreads, smem, st>>>(a);
+        cudaLaunchKernelEx(&cfg, softmax_persistent<Tag, Op, false>, a);
 }
 }  // namespace
 
