@@ -229,10 +229,63 @@ def cpu_baseline(w, seconds: float = 10.0):
         dt += time.perf_counter() - t0
         passes += 1
     per = dt / passes
+    # and on one core: the first slice(s), about a second
+    n1 = int(max(1, min(n_sl, 1.0 / (t_one * cores))))
+    samp1 = workload.slice_sample(w, list(range(n1)))
+    t0 = time.perf_counter()
+    O.softmax_batched(samp1.x, samp1.offsets, samp1.rows, samp1.cols, samp1.flags,
+                      want_f64=False, nthreads=1)
+    t1 = time.perf_counter() - t0
     return {"value": round(samp.algorithmic_bytes / per / 1e9, 4), "unit": "GB/s",
             "cores": cores, "kind": "oracle",
             "sample": "first %d of %d slices, %d passes, %.3f s per pass (double precision, "
-                      "%d threads)" % (n_sl, w.nslices, passes, per, cores)}
+                      "%d threads)" % (n_sl, w.nslices, passes, per, cores),
+            "single_thread_value": round(samp1.algorithmic_bytes / t1 / 1e9, 4),
+            "single_thread_sample": "first %d slices, one pass, 1 thread" % n1}
+
+
+def bmm_cpu_baseline(w, seconds: float = 10.0):
+    """The batched-product oracle (double-precision matrix product of the
+    exactly converted bf16 operands) on a bounded sample of slices."""
+    from oracle import bmm_oracle as O
+    cores = os.cpu_count() or 1
+    a1, b1 = w.operands([0])
+    t0 = time.perf_counter()
+    O.bmm_f64(a1, b1, 1, w.M, w.N, w.K)
+    t_one = max(time.perf_counter() - t0, 1e-4)
+    n_sl = int(max(1, min(w.B, seconds / 4 / t_one)))
+    sl = list(range(n_sl))
+    a, b = w.operands(sl)
+    passes, dt = 0, 0.0
+    while dt < 2.0 and passes < 20:
+        t0 = time.perf_counter()
+        O.bmm_f64(a, b, n_sl, w.M, w.N, w.K)
+        dt += time.perf_counter() - t0
+        passes += 1
+    per = dt / passes
+    frac = n_sl / w.B
+    return {"value": round(w.algorithmic_bytes * frac / per / 1e9, 4), "unit": "GB/s",
+            "cores": cores, "kind": "oracle",
+            "tflops": round(w.flops * frac / per / 1e12, 5),
+            "sample": "first %d of %d slices, %d passes, %.3f s per pass (float64 product, "
+                      "numpy's BLAS threads; bf16 rounding of the result not timed)"
+                      % (n_sl, w.B, passes, per)}
+
+
+def profiled_bmm_traffic(k: int):
+    """DRAM bytes per launch of the batched-product kernel for Sec. 6 shape k
+    from the committed ncu summary, if it was taken on the current source."""
+    path = os.path.join(PROFILE_DIR, "bmm_persistent_sec6_shapes.md")
+    if not os.path.exists(path):
+        return None
+    text = open(path).read()
+    m_hash = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]{16})", text)
+    m_traf = re.search(r"dram_bytes_per_launch_E%d:\s*([0-9]+)" % k, text)
+    src = os.path.join(ROOT, "paper_2002_07062_gb300", "csrc", "bsm_bmm.cu")
+    if not m_hash or not m_traf or \
+            m_hash.group(1) != hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]:
+        return None
+    return int(m_traf.group(1))
 
 
 def time_steps(fn, steps, stream, per_launch=False):
@@ -499,9 +552,12 @@ def run_bmm(args, bsm, workload, ws, rank, dev):
            "tflops": round(w.flops / (ms * 1e-3) / 1e12, 2),
            "gpu_launches": launches * args.steps,
            "roofline": {"bound": "hbm", "achieved": round(gbs, 2), "peak": peak, "unit": "GB/s",
-                        "frac": round(gbs / peak, 4), "traffic": None, "peak_source": peak_src,
+                        "frac": round(gbs / peak, 4), "traffic": profiled_bmm_traffic(args.bmm),
+                        "peak_source": peak_src,
                         "kernel": "bmm_persistent", "launch_ms": round(ms / launches, 5)},
            "clocks": clk.summary(), "device_status": bsm.bsm_device_status()}
+    if not args.no_cpu_baseline and rank == 0 and ws == 1:
+        out["cpu_baseline"] = bmm_cpu_baseline(w)
     if rank == 0:
         print(json.dumps(out), flush=True)
     return 0
