@@ -174,13 +174,12 @@ int validate(const bsm_plan_desc *d, const DeviceCtx &c, std::vector<SliceView> 
     if (d->num_slices > 0 && (!d->rows || !d->cols))
         return BSM_ERR_INVALID_ARG;
     const int es = esize(d->dtype);
-    const int64_t row_limit = max_row_bytes_for(c) / (d->op == BSM_OP_BACKWARD ? 2 : 1);
     slices.clear();
     slices.reserve(static_cast<size_t>(d->num_slices));
     total_elems = 0;
     max_row_bytes = 0;
     int64_t packed = 0;
-    bool misaligned = false, too_long = false;
+    bool misaligned = false;
     for (int64_t s = 0; s < d->num_slices; ++s) {
         const int64_t R = d->rows[s], C = d->cols[s];
         if (R < 0 || C < 1)
@@ -197,8 +196,6 @@ int validate(const bsm_plan_desc *d, const DeviceCtx &c, std::vector<SliceView> 
         if (R > 0) {
             if ((C * es) % 16 != 0 || (off * es) % 16 != 0)
                 misaligned = true;
-            if (d->op == BSM_OP_BACKWARD && C * es > row_limit)
-                too_long = true;   // forward rows of any length stream in two passes
             max_row_bytes = std::max(max_row_bytes, C * es);
             total_elems = std::max(total_elems, off + n);
         }
@@ -225,8 +222,6 @@ int validate(const bsm_plan_desc *d, const DeviceCtx &c, std::vector<SliceView> 
     }
     if (misaligned)
         return BSM_ERR_MISALIGNED;
-    if (too_long)
-        return BSM_ERR_UNSUPPORTED;
     // slices must not overlap one another
     if (d->offsets && slices.size() > 1) {
         std::vector<size_t> order;
@@ -267,9 +262,11 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     // ---- stages: one CTA per SM, as many stages as fit the shared memory
     const int64_t avail = c->smem_optin - kSmemHeader;
     const int in_arrays = d->op == BSM_OP_BACKWARD ? 2 : 1;   // inputs sharing a stage
-    // a stage holds the longest row, up to half the shared memory; longer
-    // (forward) rows go through the stages in chunks, twice
-    const int64_t row_cap = std::min<int64_t>((max_row + 127) & ~int64_t(127), max_row_bytes_for(*c));
+    // a stage holds the longest row (for the backward pass: the row of y and
+    // the row of dy), up to half the shared memory; longer rows go through
+    // the stages in chunks, twice
+    const int64_t row_cap =
+        std::min<int64_t>((max_row + 127) & ~int64_t(127), (max_row_bytes_for(*c) / in_arrays) & ~int64_t(127));
     const int64_t stage = std::max<int64_t>(kMinStageBytes, in_arrays * row_cap);
     const int n_stages = static_cast<int>(std::min<int64_t>(kMaxStages, avail / stage));
     if (n_stages < 2)
@@ -336,7 +333,8 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     st.stage_bytes = static_cast<int32_t>(stage);
     st.n_stages = n_stages;
     st.long_items = long_rows;
-    p->kernel_op = d->op == BSM_OP_BACKWARD ? OP_BACKWARD : (long_rows > 0 ? OP_FORWARD_LONG : OP_FORWARD);
+    p->kernel_op = d->op == BSM_OP_BACKWARD ? (long_rows > 0 ? OP_BACKWARD_LONG : OP_BACKWARD)
+                                            : (long_rows > 0 ? OP_FORWARD_LONG : OP_FORWARD);
 
     // ---- the schedule
     std::vector<int32_t> queue;      // schedule order of the patches (queue policies)
@@ -966,7 +964,7 @@ const char *bsm_status_string(int status)
     case BSM_ERR_MISALIGNED:
         return "misaligned: pointers, slice offsets and row lengths must be multiples of 16 bytes";
     case BSM_ERR_UNSUPPORTED:
-        return "unsupported: backward row longer than half a shared-memory stage, or too many patches";
+        return "unsupported: shape outside the kernel's limits, or too many patches";
     case BSM_ERR_CUDA:
         return "CUDA runtime error";
     case BSM_ERR_DEVICE_BOUNDS:

@@ -44,7 +44,8 @@ constexpr int kMinStageBytes = 32 * 1024;
 enum Op : int32_t {
     OP_FORWARD = 0,     // y = softmax(x [+ causal mask])
     OP_BACKWARD = 1,    // y = x * (x2 - rowsum(x * x2)): x = softmax output, x2 = its gradient
-    OP_FORWARD_LONG = 2 // OP_FORWARD for plans with rows longer than a stage (two passes)
+    OP_FORWARD_LONG = 2, // OP_FORWARD for plans with rows longer than a stage (two passes)
+    OP_BACKWARD_LONG = 3 // OP_BACKWARD for plans with rows longer than half a stage (two passes)
 };
 
 struct KernelArgs {
@@ -124,8 +125,8 @@ int kernel_set_smem_limit(int bytes);
 // Probe kernels (bsm_probe.cu).  All synchronous; return cudaError_t values.
 int probe_latency_run(const void *buf, const int64_t *line_off_dev, int n_lines, int reps,
                       int grid, float *lat_dev, uint32_t *claim_dev);
-int probe_map_run(const void *buf, int64_t bytes, int64_t chunk, int reps, const int8_t *sm_die_dev,
-                  float threshold, int n_sm, uint32_t *counter_dev, int8_t *die_dev);
+int probe_map_run(const void *buf, int64_t bytes, int64_t chunk, int reps, const int8_t *sm_die_dev, int want_die,
+                  int n_sm, uint32_t *counter_dev, float *lat_dev);
 
 // Remember a failing CUDA call for bsm_last_cuda_error (bsm_api.cpp);
 // returns BSM_ERR_CUDA.

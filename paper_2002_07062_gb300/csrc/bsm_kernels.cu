@@ -695,6 +695,44 @@ __device__ __forceinline__ void long_chunk(const unsigned char *sbuf, const Stag
     }
 }
 
+// Backward long rows: y and dy of a chunk sit in the two halves of a stage.
+// Pass 0 adds this lane's y*dy products to dot_l (its vectors in order, chunk
+// after chunk); pass 1 writes dx = y * (dy - dot).
+template <typename Tag, bool Checked>
+__device__ __forceinline__ void long_chunk_bwd(const unsigned char *sbuf, int half, const StageMeta &mt,
+                                               unsigned char *dx, int warp, int lane, Bounds by, float &dot_l,
+                                               float dot)
+{
+    using E = Elem<Tag>;
+    constexpr int EPV = E::kPerVec;
+    const int nvec = (mt.C * E::kSize) >> 4;
+    by.s_lo = sbuf;
+    by.s_hi = sbuf + (size_t)mt.C * E::kSize;
+    Bounds bdy = by;
+    bdy.s_lo = sbuf + half;
+    bdy.s_hi = sbuf + half + (size_t)mt.C * E::kSize;
+    unsigned char *base = dx + mt.off * E::kSize;
+    for (int vi = warp * 32 + lane; vi < nvec; vi += kConsumerWarps * 32) {
+        uint4 ry, rd;
+        if (!load_vec<Checked>(sbuf + 16 * vi, by, ry) || !load_vec<Checked>(sbuf + half + 16 * vi, bdy, rd))
+            continue;
+        float yv[EPV], dv[EPV];
+        E::unpack(ry, yv);
+        E::unpack(rd, dv);
+        if (mt.pass == 0) {
+#pragma unroll
+            for (int e = 0; e < EPV; ++e)
+                yv[e] *= dv[e];
+            dot_l += tree_sum<EPV>(yv);
+        } else {
+#pragma unroll
+            for (int e = 0; e < EPV; ++e)
+                yv[e] = yv[e] * (dv[e] - dot);
+            store_vec<Checked>(base + 16 * vi, by, E::pack(yv));
+        }
+    }
+}
+
 // The rows of a stage handled by one register routine: groups of T lanes,
 // G = 32/T rows per group of a warp.  Row groups are dealt to the consumer
 // warps round robin, starting at warp `first` (see consume_stage); q tracks
@@ -853,7 +891,8 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
     using E = Elem<Tag>;
     // the long-row machinery is compiled into its own instance, so plans
     // without long rows do not pay its registers
-    constexpr bool kLong = Op == OP_FORWARD_LONG;
+    constexpr bool kLong = Op == OP_FORWARD_LONG || Op == OP_BACKWARD_LONG;
+    constexpr bool kBwd = Op == OP_BACKWARD || Op == OP_BACKWARD_LONG;
     extern __shared__ __align__(1024) unsigned char smem[];
     SmemHeader &h = *reinterpret_cast<SmemHeader *>(smem);
     unsigned char *stages = smem + kSmemHeader;
@@ -931,7 +970,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                     const Item item = batch[j];
                     const int64_t ne = (int64_t)item.nrows * item.C;
                     const int64_t nbytes = ne * E::kSize;
-                    const int64_t cap = Op == OP_BACKWARD ? a.stage_bytes / 2 : a.stage_bytes;
+                    const int64_t cap = kBwd ? a.stage_bytes / 2 : a.stage_bytes;
                     const bool is_long = kLong && nbytes > cap && item.nrows == 1;
                     const bool ok = pos[j] >= 0 && pos[j] < a.n_items && item.off >= 0 && item.C > 0 &&
                                     item.nrows > 0 && item.R > 0 && item.row0 >= 0 &&
@@ -967,10 +1006,16 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                                 lm.last = k == nch - 1;
                                 lm.kind = KIND_LONG;
                                 const uint32_t cb = static_cast<uint32_t>(cn * E::kSize);
-                                mbar_arrive_expect_tx(&h.full[s], cb);
-                                bulk_load(stages + (size_t)s * a.stage_bytes,
+                                unsigned char *ldst = stages + (size_t)s * a.stage_bytes;
+                                mbar_arrive_expect_tx(&h.full[s], kBwd ? 2 * cb : cb);
+                                bulk_load(ldst,
                                           static_cast<const unsigned char *>(a.x) + (item.off + c0) * E::kSize,
                                           cb, &h.full[s]);
+                                if (kBwd)   // dy's chunk into the second half
+                                    bulk_load(ldst + a.stage_bytes / 2,
+                                              static_cast<const unsigned char *>(a.x2) +
+                                                  (item.off + c0) * E::kSize,
+                                              cb, &h.full[s]);
                                 issued[s] = true;
                                 issued_phase[s] = ph;
                             }
@@ -987,7 +1032,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                     const unsigned char *src = static_cast<const unsigned char *>(a.x) + item.off * E::kSize;
                     const int half = a.stage_bytes / 2;
                     const unsigned char *src2 =
-                        Op == OP_BACKWARD ? static_cast<const unsigned char *>(a.x2) + item.off * E::kSize : nullptr;
+                        kBwd ? static_cast<const unsigned char *>(a.x2) + item.off * E::kSize : nullptr;
                     if (Checked) {
                         const unsigned char *x0 = static_cast<const unsigned char *>(a.x);
                         bool bad = s < 0 || s >= S || S > kMaxStages ||
@@ -995,7 +1040,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                                    (reinterpret_cast<uintptr_t>(src) & 15) ||
                                    (smem_addr(dst) & 15) || (bytes & 15) || bytes == 0 ||
                                    dst + bytes > smem + kSmemHeader + (size_t)S * a.stage_bytes;
-                        if (Op == OP_BACKWARD) {
+                        if (kBwd) {
                             const unsigned char *g0 = static_cast<const unsigned char *>(a.x2);
                             bad = bad || bytes > (uint32_t)half || src2 < g0 ||
                                   src2 + bytes > g0 + a.total_elems * E::kSize ||
@@ -1008,7 +1053,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                             continue;
                         }
                     }
-                    if (Op == OP_BACKWARD) {
+                    if (kBwd) {
                         mbar_arrive_expect_tx(&h.full[s], 2 * bytes);
                         bulk_load(dst, src, bytes, &h.full[s]);
                         bulk_load(dst + half, src2, bytes, &h.full[s]);
@@ -1067,12 +1112,39 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
             break;
         if (kLong && mt.kind == KIND_LONG) {
             Bounds bd{nullptr, nullptr, y, y + a.total_elems * E::kSize, a.status};
-            long_chunk<Tag, Checked>(stages + (size_t)s * a.stage_bytes, mt, y, causal, warp, lane, bd, m_l,
-                                     s_l, long_mL, long_inv);
+            if constexpr (kBwd)
+                long_chunk_bwd<Tag, Checked>(stages + (size_t)s * a.stage_bytes, a.stage_bytes / 2, mt, y, warp,
+                                             lane, bd, s_l, long_mL);
+            else
+                long_chunk<Tag, Checked>(stages + (size_t)s * a.stage_bytes, mt, y, causal, warp, lane, bd, m_l,
+                                         s_l, long_mL, long_inv);
             __syncwarp();
             if (lane == 0)
                 mbar_arrive(&h.empty[s]);
-            if (mt.pass == 0 && mt.last) {
+            if (kBwd && mt.pass == 0 && mt.last) {
+                // the dot product: lanes, then warps in a fixed order
+#pragma unroll
+                for (int o = 16; o >= 1; o >>= 1)
+                    s_l += __shfl_xor_sync(0xFFFFFFFFu, s_l, o);
+                const int par = long_rows & 1;
+                if (lane == 0) {
+                    h.partial[par][warp] = make_float2(s_l, 0.0f);
+                    mbar_arrive(&h.xwarp);
+                }
+                if (!mbar_wait_bounded(&h.xwarp, long_rows & 1u, &h.abort_flag, wait_limit)) {
+                    if (lane == 0) {
+                        atomicOr(a.status, BSM_DEV_TIMEOUT);
+                        h.abort_flag = 1;
+                    }
+                    break;
+                }
+                float dot = 0.0f;
+                for (int w = 0; w < kConsumerWarps; ++w)
+                    dot += h.partial[par][w].x;
+                long_mL = dot;
+                s_l = 0.0f;
+                ++long_rows;
+            } else if (!kBwd && mt.pass == 0 && mt.last) {
                 // lanes, then warps: every warp ends with the same (m, s)
 #pragma unroll
                 for (int o = 16; o >= 1; o >>= 1) {
@@ -1107,14 +1179,14 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
         }
         if (mt.kind == KIND_DATA) {
             Bounds bd{nullptr, nullptr, y, y + a.total_elems * E::kSize, a.status};
-            const int64_t cap = Op == OP_BACKWARD ? a.stage_bytes / 2 : a.stage_bytes;
+            const int64_t cap = kBwd ? a.stage_bytes / 2 : a.stage_bytes;
             if (Checked && (mt.nrows <= 0 || mt.C <= 0 || (int64_t)mt.nrows * mt.C * E::kSize > cap)) {
                 if (lane == 0)
                     check_fail(a.status, 4, static_cast<uint64_t>(mt.nrows), static_cast<uint64_t>(mt.C));
             } else {
                 const int first = static_cast<int>((warp + kConsumerWarps - groups_seen % kConsumerWarps) %
                                                    kConsumerWarps);
-                if constexpr (Op == OP_BACKWARD)
+                if constexpr (kBwd)
                     groups_seen += consume_stage_bwd<Tag, Checked>(stages + (size_t)s * a.stage_bytes,
                                                                    a.stage_bytes / 2, mt, y, first, lane, bd);
                 else
@@ -1144,7 +1216,11 @@ int kernel_set_smem_limit(int bytes)
         reinterpret_cast<const void *>(softmax_persistent<F32, OP_FORWARD_LONG, false>),
         reinterpret_cast<const void *>(softmax_persistent<BF16, OP_FORWARD_LONG, false>),
         reinterpret_cast<const void *>(softmax_persistent<F32, OP_FORWARD_LONG, true>),
-        reinterpret_cast<const void *>(softmax_persistent<BF16, OP_FORWARD_LONG, true>)};
+        reinterpret_cast<const void *>(softmax_persistent<BF16, OP_FORWARD_LONG, true>),
+        reinterpret_cast<const void *>(softmax_persistent<F32, OP_BACKWARD_LONG, false>),
+        reinterpret_cast<const void *>(softmax_persistent<BF16, OP_BACKWARD_LONG, false>),
+        reinterpret_cast<const void *>(softmax_persistent<F32, OP_BACKWARD_LONG, true>),
+        reinterpret_cast<const void *>(softmax_persistent<BF16, OP_BACKWARD_LONG, true>)};
     for (const void *f : fns) {
         cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
         if (e != cudaSuccess)
@@ -1188,6 +1264,11 @@ int launch_softmax(const KernelArgs &a, int dtype, int op, int grid, void *strea
             launch_one<F32, OP_BACKWARD>(a, grid, smem, st, checked);
         else
             launch_one<BF16, OP_BACKWARD>(a, grid, smem, st, checked);
+    } else if (op == OP_BACKWARD_LONG) {
+        if (dtype == BSM_F32)
+            launch_one<F32, OP_BACKWARD_LONG>(a, grid, smem, st, checked);
+        else
+            launch_one<BF16, OP_BACKWARD_LONG>(a, grid, smem, st, checked);
     } else if (op == OP_FORWARD_LONG) {
         if (dtype == BSM_F32)
             launch_one<F32, OP_FORWARD_LONG>(a, grid, smem, st, checked);

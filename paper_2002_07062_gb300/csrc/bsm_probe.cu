@@ -79,16 +79,17 @@ __global__ void probe_latency_kernel(const unsigned char *buf, int64_t buf_bytes
     }
 }
 
-// Die of every `chunk`-byte chunk: an SM of known die times the chunk's
-// first line; below the threshold the line is near (same die), else far.
-__global__ void probe_map_kernel(const unsigned char *buf, int64_t buf_bytes, int64_t n_chunks, int64_t chunk, int reps,
-                                 const int8_t *sm_die, float threshold, uint32_t *counter,
-                                 int8_t *die_out, uint32_t zero)
+// Latency of every `chunk`-byte chunk's first line as seen from the SMs of
+// die `want_die` (the others return at once): the host compares the two
+// dies' figures for each chunk, so no absolute threshold is involved.
+__global__ void probe_map_kernel(const unsigned char *buf, int64_t buf_bytes, int64_t n_chunks, int64_t chunk,
+                                 int reps, const int8_t *sm_die, int want_die, uint32_t *counter, float *lat_out,
+                                 uint32_t zero)
 {
     if (threadIdx.x != 0)
         return;
     const int my = sm_die[probe_smid() & (BSM_MAX_SM - 1)];
-    if (my < 0 || my > 1)
+    if (my != want_die)
         return;
     for (int64_t guard = 0; guard < n_chunks; ++guard) {
         const uint32_t c = atomicAdd(counter, 1u);
@@ -96,8 +97,7 @@ __global__ void probe_map_kernel(const unsigned char *buf, int64_t buf_bytes, in
             break;
         if ((int64_t)c * chunk + 4 > buf_bytes)          // never true for host-checked sizes
             break;
-        const float t = time_line(buf + (int64_t)c * chunk, reps, zero);
-        die_out[c] = static_cast<int8_t>(t < threshold ? my : 1 - my);
+        lat_out[c] = time_line(buf + (int64_t)c * chunk, reps, zero);
     }
 }
 
@@ -114,13 +114,13 @@ int probe_latency_run(const void *buf, const int64_t *line_off_dev, int n_lines,
     return static_cast<int>(e);
 }
 
-int probe_map_run(const void *buf, int64_t bytes, int64_t chunk, int reps, const int8_t *sm_die_dev,
-                  float threshold, int n_sm, uint32_t *counter_dev, int8_t *die_dev)
+int probe_map_run(const void *buf, int64_t bytes, int64_t chunk, int reps, const int8_t *sm_die_dev, int want_die,
+                  int n_sm, uint32_t *counter_dev, float *lat_dev)
 {
     const int64_t n_chunks = (bytes + chunk - 1) / chunk;
     // the chunk's first line must lie inside the buffer: (n_chunks-1)*chunk < bytes
     probe_map_kernel<<<n_sm, 32>>>(static_cast<const unsigned char *>(buf), bytes, n_chunks, chunk, reps,
-                                   sm_die_dev, threshold, counter_dev, die_dev, 0u);
+                                   sm_die_dev, want_die, counter_dev, lat_dev, 0u);
     cudaError_t e = cudaGetLastError();
     if (e == cudaSuccess)
         e = cudaDeviceSynchronize();

@@ -265,10 +265,14 @@ int addr_die_map_host(int device, const void *ptr, int64_t bytes, int64_t chunk,
         return BSM_ERR_UNSUPPORTED;
     if (cudaSetDevice(device) != cudaSuccess)
         return BSM_ERR_NO_DEVICE;
-    int8_t *d_die = nullptr, *d_sm = nullptr;
+    // every chunk is timed once from an SM of die 0 and once from an SM of
+    // die 1; it belongs to the die that reached it faster (ties: alternate)
+    float *d_lat = nullptr;
+    int8_t *d_sm = nullptr;
     uint32_t *d_ctr = nullptr;
+    std::vector<float> lat0, lat1;
     do {
-        if ((rc = cuda_fail(cudaMalloc(&d_die, (size_t)n_chunks))))
+        if ((rc = cuda_fail(cudaMalloc(&d_lat, (size_t)n_chunks * sizeof(float)))))
             break;
         if ((rc = cuda_fail(cudaMalloc(&d_sm, BSM_MAX_SM))))
             break;
@@ -276,17 +280,24 @@ int addr_die_map_host(int device, const void *ptr, int64_t bytes, int64_t chunk,
             break;
         if ((rc = cuda_fail(cudaMalloc(&d_ctr, sizeof(uint32_t)))))
             break;
-        if ((rc = cuda_fail(cudaMemset(d_ctr, 0, sizeof(uint32_t)))))
+        for (int die = 0; die < 2 && !rc; ++die) {
+            std::vector<float> &lat = die == 0 ? lat0 : lat1;
+            lat.assign(static_cast<size_t>(n_chunks), 0.0f);
+            if ((rc = cuda_fail(cudaMemset(d_ctr, 0, sizeof(uint32_t)))))
+                break;
+            if ((rc = cuda_fail(cudaMemset(d_lat, 0, (size_t)n_chunks * sizeof(float)))))
+                break;
+            if ((rc = cuda_fail(static_cast<cudaError_t>(
+                     probe_map_run(ptr, bytes, chunk, 4, d_sm, die, t.n_sm, d_ctr, d_lat)))))
+                break;
+            rc = cuda_fail(cudaMemcpy(lat.data(), d_lat, (size_t)n_chunks * sizeof(float), cudaMemcpyDeviceToHost));
+        }
+        if (rc)
             break;
-        if ((rc = cuda_fail(cudaMemset(d_die, 0, (size_t)n_chunks))))
-            break;
-        const float thr = static_cast<float>(0.5 * (t.l_near + t.l_far));
-        if ((rc = cuda_fail(static_cast<cudaError_t>(
-                 probe_map_run(ptr, bytes, chunk, 4, d_sm, thr, t.n_sm, d_ctr, d_die)))))
-            break;
-        rc = cuda_fail(cudaMemcpy(die_out, d_die, (size_t)n_chunks, cudaMemcpyDeviceToHost));
+        for (int64_t c = 0; c < n_chunks; ++c)
+            die_out[c] = lat0[c] < lat1[c] ? 0 : (lat1[c] < lat0[c] ? 1 : static_cast<int8_t>(c & 1));
     } while (false);
-    cudaFree(d_die);
+    cudaFree(d_lat);
     cudaFree(d_sm);
     cudaFree(d_ctr);
     return rc;

@@ -109,3 +109,57 @@ def test_backward_full_size_uniform_and_in_place(k):
     torch.cuda.synchronize()
     assert torch.equal(bits(dyd), bits(dx))
     assert bsm.bsm_device_status() == 0
+
+
+@pytest.mark.parametrize("dtype", [workload.F32, workload.BF16])
+def test_backward_rows_longer_than_half_a_stage(dtype):
+    """Rows whose y and dy do not fit one stage are streamed twice in chunks
+    (the dot product, then dx); same tolerance, all policies bit-identical,
+    and in place into dy."""
+    import torch
+    es = 4 if dtype == workload.F32 else 2
+    half = bsm.bsm_max_row_bytes() // 2 // es          # elements in half a stage
+    for B, R, C in [(2, 3, half + 16 // es), (1, 2, 262144), (3, 1, 100000 // 8 * 8)]:
+        w = workload.uniform("bwd long", dtype, B, R, C, 3.0, 0xB10 + C).materialize()
+        y, dy = _inputs(w)
+        yd, dyd = to_device(y), to_device(dy)
+        p = bsm.bsm_plan_create(yd, torch.empty_like(yd), w.rows, w.cols, dtype,
+                                bsm.POLICY_DYNAMIC, op=bsm.OP_BACKWARD, x2=dyd)
+        assert p.stats()["long_items"] == B * R
+        p.close()
+        outs = []
+        for pol in ALL:
+            dx = torch.full_like(yd, float("nan"))
+            bsm.bsm_softmax_backward(yd, dyd, dx, B, R, C, dtype, pol)
+            outs.append(dx)
+        torch.cuda.synchronize()
+        for o in outs[1:]:
+            assert torch.equal(bits(o), bits(outs[0]))
+        _check(w, y, dy, to_host(outs[0]))
+        dyd2 = dyd.clone()
+        bsm.bsm_softmax_backward(yd, dyd2, dyd2, B, R, C, dtype, bsm.POLICY_DYNAMIC)
+        torch.cuda.synchronize()
+        assert torch.equal(bits(dyd2), bits(outs[0]))
+    assert bsm.bsm_device_status() == 0
+
+
+def test_backward_mixed_short_and_long_rows():
+    import torch
+    rows = np.array([4, 1, 3, 2, 5, 1], np.int32)
+    cols = np.array([64, 200000, 2048, 30000, 512, 16], np.int32)
+    sizes = rows.astype(np.int64) * cols
+    off = np.concatenate([[0], np.cumsum(sizes)[:-1]]).astype(np.int64)
+    w = workload.Workload("bwd mixed long", workload.F32, rows, cols, off, 0, 0x4D18, 2.0)
+    w.materialize()
+    y, dy = _inputs(w)
+    yd, dyd = to_device(y), to_device(dy)
+    outs = []
+    for pol in ALL:
+        dx = torch.full_like(yd, float("nan"))
+        bsm.bsm_softmax_backward_ragged(yd, dyd, dx, w.offsets, w.rows, w.cols, w.dtype, pol)
+        outs.append(dx)
+    torch.cuda.synchronize()
+    for o in outs[1:]:
+        assert torch.equal(bits(o), bits(outs[0]))
+    _check(w, y, dy, to_host(outs[0]))
+    assert bsm.bsm_device_status() == 0

@@ -178,11 +178,16 @@ def test_argument_errors_on_device():
     with pytest.raises(bsm.BsmError) as e:
         bsm.bsm_softmax(x, x.data_ptr() + 16, 4, 1, 64, bsm.F32, bsm.POLICY_RR)
     assert e.value.status == bsm.ERR_INVALID_ARG                        # partial overlap
-    big = bsm.bsm_max_row_bytes() // 8 + 4          # backward: half a stage per row
-    xb = torch.zeros(big, device="cuda")
-    with pytest.raises(bsm.BsmError) as e:
-        bsm.bsm_softmax_backward(xb, xb, xb, 1, 1, big, bsm.F32, bsm.POLICY_RR)
-    assert e.value.status == bsm.ERR_UNSUPPORTED
+    # a backward row longer than half a stage streams in chunks (no limit):
+    # y = 1/C everywhere and dy = 1 give dx = 1/C * (1 - 1) = 0 exactly
+    big = bsm.bsm_max_row_bytes() // 8 + 4
+    yb = torch.full((big,), 1.0 / 1024, device="cuda")
+    gb = torch.ones(big, device="cuda")
+    db = torch.full((big,), float("nan"), device="cuda")
+    bsm.bsm_softmax_backward(yb, gb, db, 1, 1, big, bsm.F32, bsm.POLICY_RR)
+    torch.cuda.synchronize()
+    dot = (big / 1024.0)
+    assert torch.all(db == torch.tensor(1.0 / 1024, device="cuda") * (1.0 - dot))
     with pytest.raises(bsm.BsmError) as e:                              # overlapping slices
         bsm.bsm_softmax_ragged(x, y, [0, 32], [1, 1], [64, 64], bsm.F32, bsm.POLICY_RR)
     assert e.value.status == bsm.ERR_INVALID_ARG
