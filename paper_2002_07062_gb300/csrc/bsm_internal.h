@@ -39,6 +39,11 @@ constexpr int kConsumerWarps = 16;
 constexpr int kThreads = (kConsumerWarps + 1) * 32;  // + one producer warp
 constexpr int kSmemHeader = 1024;                     // barriers + stage metadata
 constexpr int kMinStageBytes = 32 * 1024;
+// bf16 rows carry half the bytes per element, so a stage holds twice the
+// elements' work per fixed stage cost (wait, metadata, dispatch, release);
+// larger stages amortise that cost (measured: +11 % causal 512-wide rows,
+// +16 % 32 x 128 slices over 32 KiB stages; fp32 is unchanged).
+constexpr int kMinStageBytesBf16 = 64 * 1024;
 
 // What the kernel computes on every row.
 enum Op : int32_t {

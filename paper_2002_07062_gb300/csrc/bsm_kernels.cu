@@ -267,6 +267,8 @@ template <> struct Elem<F32> {
         return make_uint4(__float_as_uint(v[0]), __float_as_uint(v[1]), __float_as_uint(v[2]),
                           __float_as_uint(v[3]));
     }
+    // a vector of -inf (stands in for vectors past the end of a row)
+    __device__ static __forceinline__ uint4 neg_inf_vec() { return make_uint4(0xFF800000u, 0xFF800000u, 0xFF800000u, 0xFF800000u); }
 };
 
 template <> struct Elem<BF16> {
@@ -286,6 +288,7 @@ template <> struct Elem<BF16> {
         return make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]),
                           pack_bf16x2(v[6], v[7]));
     }
+    __device__ static __forceinline__ uint4 neg_inf_vec() { return make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u); }
 };
 
 // ------------------------------------------------------------- row routines
@@ -352,12 +355,13 @@ __device__ __forceinline__ void apply_causal(float (&v)[EPV], int col0, int row)
         v[e] += (col0 + e > row) ? -INFINITY : 0.0f;
 }
 
-// Register-resident row: T lanes, up to V vectors per lane.  Under the
-// causal mask a vector is unmasked (all its columns <= row), on the diagonal
-// (masked element by element) or wholly masked (it adds nothing to the max;
-// its p is 0 or NaN, see vec_exp).
+// Register-resident fp32 row: T lanes, up to V vectors per lane, scalar
+// arithmetic (fp32 rows move 8 bytes per element: memory, not instruction
+// issue, bounds them).  Under the causal mask a vector is unmasked (all its
+// columns <= row), on the diagonal (masked element by element) or wholly
+// masked (it adds nothing to the max; its p is 0 or NaN, see vec_exp).
 template <typename Tag, bool Checked, int T, int V>
-__device__ __forceinline__ void row_in_registers(const unsigned char *srow, unsigned char *yrow,
+__device__ __forceinline__ void row_in_registers_scalar(const unsigned char *srow, unsigned char *yrow,
                                                  int nvec, int row, bool causal, int l, bool valid,
                                                  const Bounds &bd)
 {
@@ -402,6 +406,199 @@ __device__ __forceinline__ void row_in_registers(const unsigned char *srow, unsi
 #pragma unroll
             for (int e = 0; e < EPV; ++e)
                 v[j][e] *= inv;
+            store_vec<Checked>(yrow + 16 * vi, bd, E::pack(v[j]));
+        }
+    }
+}
+
+// ------------------------------------------------ fp32 pair arithmetic
+// One instruction, two IEEE operations, each rounded like its scalar form.
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c)
+{
+    float2 d;
+    asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
+        "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+    return d;
+}
+
+__device__ __forceinline__ float2 add2(float2 a, float2 b)
+{
+    float2 d;
+    asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+        "add.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return d;
+}
+
+__device__ __forceinline__ float2 mul2(float2 a, float2 b)
+{
+    float2 d;
+    asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+        "mul.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return d;
+}
+
+// p = 2^(v*log2e - mL) for one vector, in pairs; returns the vector's sum as
+// a pair: ((p0,p1) + (p2,p3)) [+ ((p4,p5) + (p6,p7))].
+template <int EPV>
+__device__ __forceinline__ float2 vec_exp_pairs(float (&v)[EPV], float mL)
+{
+    const float2 l2 = make_float2(kLog2e, kLog2e), nm = make_float2(-mL, -mL);
+#pragma unroll
+    for (int e = 0; e < EPV; e += 2) {
+        const float2 t = fma2(make_float2(v[e], v[e + 1]), l2, nm);
+        v[e] = ex2(t.x);
+        v[e + 1] = ex2(t.y);
+    }
+    const float2 a = add2(make_float2(v[0], v[1]), make_float2(v[2], v[3]));
+    if constexpr (EPV == 4)
+        return a;
+    else
+        return add2(a, add2(make_float2(v[4], v[5]), make_float2(v[6], v[7])));
+}
+
+// Element-wise maximum of two bf16 pairs.
+__device__ __forceinline__ uint32_t bmax2(uint32_t a, uint32_t b)
+{
+    uint32_t d;
+    asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+    return d;
+}
+
+// True when one of the vector's elements is NaN or +inf (such an element
+// masked by the causal mask still turns its row into NaN: NaN + (-inf) and
+// +inf + (-inf) are NaN); a NaN-propagating maximum over the raw vector.
+template <typename Tag> __device__ __forceinline__ bool vec_poisons(uint4 r);
+template <> __device__ __forceinline__ bool vec_poisons<F32>(uint4 r)
+{
+    float m;
+    asm("{\n\t.reg .f32 a, b;\n\tmax.NaN.f32 a, %1, %2;\n\tmax.NaN.f32 b, %3, %4;\n\t"
+        "max.NaN.f32 %0, a, b;\n\t}"
+        : "=f"(m)
+        : "f"(__uint_as_float(r.x)), "f"(__uint_as_float(r.y)), "f"(__uint_as_float(r.z)),
+          "f"(__uint_as_float(r.w)));
+    return !(m < INFINITY);
+}
+template <> __device__ __forceinline__ bool vec_poisons<BF16>(uint4 r)
+{
+    uint32_t w;
+    asm("{\n\t.reg .b32 a, b;\n\tmax.NaN.bf16x2 a, %1, %2;\n\tmax.NaN.bf16x2 b, %3, %4;\n\t"
+        "max.NaN.bf16x2 %0, a, b;\n\t}"
+        : "=r"(w)
+        : "r"(r.x), "r"(r.y), "r"(r.z), "r"(r.w));
+    const float lo = __uint_as_float(w << 16), hi = __uint_as_float(w & 0xFFFF0000u);
+    return !(lo < INFINITY) || !(hi < INFINITY);
+}
+
+// Register-resident bf16 row (bf16 rows move 4 bytes per element, so
+// instruction issue matters): T lanes, V vectors per lane (vector j of lane l
+// is vector j*T + l of the row).  Arithmetic, the same in both variants and
+// under every policy: m = max over the lane's vectors (balanced tree per
+// vector, vectors in order), butterfly over the lane group; p = 2^(v*log2e
+// - m*log2e) in fp32 pairs; the lane's sum is a pair accumulated vector by
+// vector, then its two halves, then the butterfly; y = p * (1/sum).
+// Full = true: every lane holds V vectors of a valid row and nothing needs a
+// bound (no per-vector predicates).  Under the causal mask each vector is
+// classed for the whole warp: unmasked everywhere (no mask work), masked
+// everywhere (p = 0 without an exponential; a NaN or +inf among its inputs
+// still makes the row NaN), or mixed (the additive -inf mask element by
+// element).  Results do not depend on the class: the mask's sums are exact.
+template <typename Tag, bool Checked, int T, int V, bool Full>
+__device__ __forceinline__ void row_in_registers_pairs(const unsigned char *srow, unsigned char *yrow,
+                                                 int nvec, int row, bool causal, int l, bool valid,
+                                                 const Bounds &bd)
+{
+    using E = Elem<Tag>;
+    constexpr int EPV = E::kPerVec;
+    float v[V][EPV];
+    uint32_t skip = 0;          // bit j: vector j is masked for the whole warp
+    bool poison = false;
+    float m = -INFINITY;
+    uint32_t mw = 0xFF80FF80u;  // running maximum of the unmasked vectors, two bf16 halves
+#pragma unroll
+    for (int j = 0; j < V; ++j) {
+        const int vi = j * T + l;
+        const int col0 = vi * EPV;
+        const bool in = Full || (valid && vi < nvec);
+        // the vector's mask class depends on its position only (warp-wide)
+        bool mixed = false;
+        if (causal) {
+            const bool lane_un = !in || col0 + EPV - 1 <= row;
+            const bool lane_mk = !in || col0 > row;
+            if (!__all_sync(0xFFFFFFFFu, lane_un)) {
+                if (__all_sync(0xFFFFFFFFu, lane_mk))
+                    skip |= 1u << j;
+                else
+                    mixed = true;
+            }
+        }
+        uint4 raw = E::neg_inf_vec();
+        if (Full) {
+            raw = lds128(srow + 16 * vi);
+        } else if (in) {
+            uint4 r;
+            if (load_vec<Checked>(srow + 16 * vi, bd, r))
+                raw = r;
+        }
+        if (skip & (1u << j)) {
+            if (in)
+                poison |= vec_poisons<Tag>(raw);
+#pragma unroll
+            for (int e = 0; e < EPV; ++e)
+                v[j][e] = 0.0f;
+            continue;
+        }
+        E::unpack(raw, v[j]);
+        if (mixed) {
+#pragma unroll
+            for (int e = 0; e < EPV; ++e)
+                v[j][e] += (col0 + e > row) ? -INFINITY : 0.0f;
+            m = fmaxf(m, tree_max<EPV>(v[j]));
+        } else {
+            // the maximum of bf16 values is exact in bf16: take it on the
+            // packed words (non-NaN operand wins, as fmaxf), unpack once
+            mw = bmax2(mw, bmax2(bmax2(raw.x, raw.y), bmax2(raw.z, raw.w)));
+        }
+    }
+    m = fmaxf(m, fmaxf(__uint_as_float(mw << 16), __uint_as_float(mw & 0xFFFF0000u)));
+    m = group_max<T>(m);
+    const float mL = m * kLog2e;
+    float2 acc = make_float2(0.0f, 0.0f);
+#pragma unroll
+    for (int j = 0; j < V; ++j)
+        if (!(skip & (1u << j)))
+            acc = add2(acc, vec_exp_pairs<EPV>(v[j], mL));
+    float s = acc.x + acc.y;
+    if (poison)
+        s = __int_as_float(0x7FC00000);
+    s = group_sum<T>(s);
+    const float inv = __frcp_rn(s);
+    const float2 inv2 = make_float2(inv, inv);
+    const float zero_y = 0.0f * inv;   // the output of a masked element (0, or NaN in a NaN row)
+#pragma unroll
+    for (int j = 0; j < V; ++j) {
+        const int vi = j * T + l;
+        if (Full || (valid && vi < nvec)) {
+            if (skip & (1u << j)) {
+#pragma unroll
+                for (int e = 0; e < EPV; ++e)
+                    v[j][e] = zero_y;
+            } else {
+#pragma unroll
+                for (int e = 0; e < EPV; e += 2) {
+                    const float2 y2 = mul2(make_float2(v[j][e], v[j][e + 1]), inv2);
+                    v[j][e] = y2.x;
+                    v[j][e + 1] = y2.y;
+                }
+            }
             store_vec<Checked>(yrow + 16 * vi, bd, E::pack(v[j]));
         }
     }
@@ -751,10 +948,21 @@ __device__ __forceinline__ int rows_in_registers(const unsigned char *sbuf, cons
         q = (mt.row0 + first * G + g) % mt.R;
         qstep = step % mt.R;
     }
+    const bool full_rows = nvec == T * V;
     for (int rb = first * G; rb < mt.nrows; rb += step) {
         const int r = rb + g;
-        row_in_registers<Tag, Checked, T, V>(sbuf + (size_t)r * row_bytes, ybase + (size_t)r * row_bytes,
-                                             nvec, q, causal, l, r < mt.nrows, bd);
+        if constexpr (Elem<Tag>::kSize == 4)
+            row_in_registers_scalar<Tag, Checked, T, V>(sbuf + (size_t)r * row_bytes,
+                                                        ybase + (size_t)r * row_bytes, nvec, q, causal, l,
+                                                        r < mt.nrows, bd);
+        else if (full_rows && rb + G <= mt.nrows)   // warp-uniform
+            row_in_registers_pairs<Tag, Checked, T, V, true>(sbuf + (size_t)r * row_bytes,
+                                                             ybase + (size_t)r * row_bytes, nvec, q, causal, l,
+                                                             true, bd);
+        else
+            row_in_registers_pairs<Tag, Checked, T, V, false>(sbuf + (size_t)r * row_bytes,
+                                                              ybase + (size_t)r * row_bytes, nvec, q, causal, l,
+                                                              r < mt.nrows, bd);
         q += qstep;
         if (q >= mt.R)
             q -= mt.R;
@@ -802,7 +1010,7 @@ __device__ __forceinline__ int consume_stage(const unsigned char *sbuf, const St
         if constexpr (E::kSize == 4) {
             // fp32: rows up to 4 KiB in registers, longer ones in place in the stage
             if (nvec <= 256)
-                row_in_registers<Tag, Checked, 32, 8>(srow, yrow, nvec, q, causal, lane, true, bd);
+                row_in_registers_scalar<Tag, Checked, 32, 8>(srow, yrow, nvec, q, causal, lane, true, bd);
             else
                 row_in_smem_inplace<Checked>(const_cast<unsigned char *>(srow), yrow, nvec, q, causal, lane,
                                              bd);
