@@ -165,6 +165,45 @@ def test_non_finite_rows_match_oracle():
     check_all_against_oracle(w, to_host(y))
 
 
+@pytest.mark.parametrize("C", [512, 128])
+def test_causal_bf16_non_finite_in_masked_and_unmasked_positions(C):
+    """Causal bf16 rows: a NaN or +inf in a masked position turns the row into
+    NaN (NaN + (-inf), +inf + (-inf)), whether its vector is masked for every
+    lane of the warp (no exponential is taken there), straddles the diagonal,
+    or is unmasked; a -inf in a masked position changes nothing."""
+    from oracle import softmax as O
+    R = 8
+    rng = np.random.default_rng(C)
+    x = rng.normal(0, 3, (R, C)).astype(np.float32)
+    x[1, C - 12] = np.nan            # far right of row 1: warp-wide masked vector
+    x[2, 3] = np.inf                 # just past the diagonal of row 2
+    x[3, C // 2:C // 2 + 40] = -np.inf   # masked -inf: no effect
+    x[4, C // 3:C // 3 + 60] = -np.inf
+    x[4, 2] = np.inf                 # unmasked +inf
+    x[5, 5] = np.nan                 # on the diagonal (unmasked)
+    x[6, 7:] = np.nan                # everything masked is NaN
+    bits16 = (x.view(np.uint32) >> 16).astype(np.uint16)   # exact: the draws are re-read as bf16
+    bits16[np.isnan(x)] = 0x7FC0
+    w = workload.uniform("causal nonfinite", workload.BF16, 3, R, C, 1.0, 0, workload.CAUSAL)
+    w.x = np.tile(bits16.reshape(-1), 3)
+    xd = to_device(w.x)
+    y = _all_policies_identical(w, xd)
+    yh = to_host(y).reshape(3, R, C)
+    _, yr = O.softmax_batched(w.x, w.offsets, w.rows, w.cols, w.flags)
+    yr = yr.reshape(3, R, C)
+    nan_g = (yh & 0x7FFF) > 0x7F80
+    nan_o = (yr & 0x7FFF) > 0x7F80
+    assert np.array_equal(nan_g, nan_o)
+    for s in range(3):
+        for r in (1, 2, 4, 5, 6):
+            assert nan_g[s, r].all(), (s, r)
+        for r in (0, 3, 7):
+            assert not nan_g[s, r].any(), (s, r)
+    ok = ~nan_o
+    assert np.max(np.abs(yh[ok].astype(np.int32) - yr[ok].astype(np.int32))) <= 1
+    assert bsm.bsm_device_status() == 0
+
+
 def test_argument_errors_on_device():
     import torch
     x = torch.zeros(4 * 64 + 8, device="cuda")
