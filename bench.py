@@ -514,7 +514,51 @@ def sweep(args, bsm, workload, stream):
             del dy, dx
         del x, y
         torch.cuda.empty_cache()
+    long_row_sweep(bsm, workload, stream)
     bmm_sweep(bsm, workload, stream)
+
+
+def long_row_sweep(bsm, workload, stream):
+    """Rows longer than a shared-memory stage (streamed twice in chunks):
+    GB/s of algorithmic traffic and of the bytes actually moved (the row is
+    read twice: 1.5x the algorithmic bytes forward, 5/3x backward)."""
+    import torch
+    for dtype, name in ((workload.F32, "fp32"), (workload.BF16, "bf16")):
+        tdt = torch.float32 if dtype == workload.F32 else torch.bfloat16
+        es = 4 if dtype == workload.F32 else 2
+        for C in (65536, 262144, 1048576):
+            R = max(1, (256 << 20) // (C * es))        # 256 MiB of input
+            x = torch.randn(R * C, device="cuda").to(tdt)
+            y = torch.empty_like(x)
+
+            def step():
+                bsm.bsm_softmax(x, y, 1, R, C, dtype, bsm.POLICY_DYNAMIC, stream)
+            for _ in range(3):
+                step()
+            stream.synchronize()
+            med = _median_ms(step, 10, stream)
+            alg = 2 * R * C * es
+            print(json.dumps({"sweep": True, "op": "forward long rows", "workload":
+                              "%s %d rows x %d (%d KiB rows)" % (name, R, C, C * es >> 10),
+                              "policy": "dynamic", "ms": round(med, 4),
+                              "GBps": round(alg / (med * 1e-3) / 1e9, 2),
+                              "moved_GBps": round(1.5 * alg / (med * 1e-3) / 1e9, 2)}), flush=True)
+            dy = torch.randn(R * C, device="cuda").to(tdt)
+
+            def bstep():
+                bsm.bsm_softmax_backward(y, dy, x, 1, R, C, dtype, bsm.POLICY_DYNAMIC, stream)
+            for _ in range(3):
+                bstep()
+            stream.synchronize()
+            med = _median_ms(bstep, 10, stream)
+            alg = 3 * R * C * es
+            print(json.dumps({"sweep": True, "op": "backward long rows", "workload":
+                              "%s %d rows x %d (%d KiB rows)" % (name, R, C, C * es >> 10),
+                              "policy": "dynamic", "ms": round(med, 4),
+                              "GBps": round(alg / (med * 1e-3) / 1e9, 2),
+                              "moved_GBps": round(5 / 3 * alg / (med * 1e-3) / 1e9, 2)}), flush=True)
+            del x, y, dy
+            torch.cuda.empty_cache()
 
 
 def run_bmm(args, bsm, workload, ws, rank, dev):

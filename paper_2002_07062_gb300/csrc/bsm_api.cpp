@@ -133,8 +133,10 @@ struct bsm_plan {
     bsm::KernelArgs args{};
     int grid = 0;
     struct Launch {
-        int32_t begin, end, grid;
+        int32_t begin, end, grid, phase;
     };
+    bsm::KernelArgs args1{};         // phase 1 of plans with rows longer than a stage
+    int64_t n_phase1 = 0;
     std::vector<Launch> whole_gpu;   // WHOLE_GPU: one launch per slice
     void *blob = nullptr;            // device tables (patches, slice index, sm_die, heads)
     bsm_plan_stats stats{};
@@ -281,23 +283,72 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
                           d->policy == BSM_POLICY_CBMF_LB || d->policy == BSM_POLICY_MINIMAX;
     std::vector<Item> items;
     std::vector<int32_t> slice_first(slices.size() + 1, 0);
+    // rows longer than a stage: when they are too few to fill two waves of
+    // the SMs, cut into segments of whole chunks, about four per SM over the
+    // batch, so that a few long rows still spread over the device (two
+    // launches, see LongSeg); otherwise each row is one segment that one CTA
+    // streams twice within the launch (its second read mostly hits L2)
+    int64_t n_long_rows = 0;
+    for (const SliceView &v : slices)
+        if (v.R > 0 && int64_t(v.C) * es > stage / in_arrays)
+            n_long_rows += v.R;
+    const int64_t chunk_elems = stage / in_arrays / es;
+    const int64_t want_segs = n_long_rows > 0 && n_long_rows < 2 * c->n_sm
+                                  ? std::max<int64_t>(1, (4 * c->n_sm + n_long_rows - 1) / n_long_rows)
+                                  : 1;
+    std::vector<LongSeg> segs;              // parallel to items when there are long rows
+    std::vector<Item> items1;               // phase 1: the long-row segments
+    std::vector<LongSeg> segs1;
+    std::vector<int32_t> slice_first1(slices.size() + 1, 0);
+    int64_t n_parts = 0;
     int64_t long_rows = 0;
     size_t s = 0;
     while (s < slices.size()) {
         slice_first[s] = static_cast<int32_t>(items.size());
+        slice_first1[s] = static_cast<int32_t>(items1.size());
         const SliceView &v = slices[s];
         size_t e = s + 1;
         if (spanning && v.R > 0) {
             while (e < slices.size() && slices[e].R == v.R && slices[e].C == v.C &&
                    slices[e].off == slices[e - 1].off + int64_t(v.R) * v.C) {
                 slice_first[e] = static_cast<int32_t>(items.size());
+                slice_first1[e] = static_cast<int32_t>(items1.size());
                 ++e;
             }
         }
-        if (v.R > 0) {
+        if (v.R > 0 && int64_t(v.C) * es > stage / in_arrays) {
             const int64_t seg_rows = int64_t(v.R) * static_cast<int64_t>(e - s);
-            if (int64_t(v.C) * es > stage / in_arrays)
-                long_rows += seg_rows;
+            long_rows += seg_rows;
+            const int64_t nch = (v.C + chunk_elems - 1) / chunk_elems;
+            const int64_t per_row = std::min<int64_t>(nch, want_segs);
+            const int64_t seg_elems = (nch + per_row - 1) / per_row * chunk_elems;
+            const int64_t n_seg = (v.C + seg_elems - 1) / seg_elems;
+            if (segs.size() < items.size())
+                segs.resize(items.size(), LongSeg{0, 0, 0, 0});
+            for (int64_t g = 0; g < seg_rows; ++g) {
+                if (items.size() + n_seg >= static_cast<size_t>(INT32_MAX) || n_parts + n_seg >= INT32_MAX)
+                    return BSM_ERR_UNSUPPORTED;
+                for (int64_t k = 0; k < n_seg; ++k) {
+                    const int64_t c0 = k * seg_elems;
+                    const Item it{v.off + g * v.C + c0, static_cast<int32_t>(std::min<int64_t>(seg_elems, v.C - c0)),
+                                  1, static_cast<int32_t>(g % v.R), v.R};
+                    if (n_seg == 1) {       // the whole row, both passes in one launch
+                        items.push_back(it);
+                        segs.push_back(LongSeg{0, 0, 0, 1});
+                        continue;
+                    }
+                    const LongSeg sg{static_cast<int32_t>(c0), static_cast<int32_t>(n_parts + k),
+                                     static_cast<int32_t>(n_parts), static_cast<int32_t>(n_seg)};
+                    items.push_back(it);
+                    segs.push_back(sg);
+                    items1.push_back(it);
+                    segs1.push_back(sg);
+                }
+                if (n_seg > 1)
+                    n_parts += n_seg;
+            }
+        } else if (v.R > 0) {
+            const int64_t seg_rows = int64_t(v.R) * static_cast<int64_t>(e - s);
             const int64_t row_bytes = int64_t(v.C) * es;
             int64_t rpi = std::max<int64_t>(1, stage / in_arrays / row_bytes);
             if (d->rows_per_item > 0)
@@ -316,6 +367,15 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
         s = e;
     }
     slice_first[slices.size()] = static_cast<int32_t>(items.size());
+    slice_first1[slices.size()] = static_cast<int32_t>(items1.size());
+    if (!segs.empty())
+        segs.resize(items.size(), LongSeg{0, 0, 0, 0});
+    if (spanning && !items1.empty()) {
+        // phase 1 takes the segments in reverse: it starts with those phase 0
+        // read last, which are most likely still in L2
+        std::reverse(items1.begin(), items1.end());
+        std::reverse(segs1.begin(), segs1.end());
+    }
     const int64_t n_items = static_cast<int64_t>(items.size());
 
     bsm_plan *p = new bsm_plan();
@@ -484,19 +544,38 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
         for (size_t k = 0; k < queue.size(); ++k)
             ordered[k] = items[static_cast<size_t>(queue[k])];
         items.swap(ordered);
+        if (!segs.empty()) {
+            std::vector<LongSeg> osegs(segs.size());
+            for (size_t k = 0; k < queue.size(); ++k)
+                osegs[k] = segs[static_cast<size_t>(queue[k])];
+            segs.swap(osegs);
+        }
     }
 
     // ---- upload the tables in one allocation
     const size_t items_b = sizeof(Item) * static_cast<size_t>(n_items);
     const size_t slices_b = sizeof(int32_t) * slice_first.size();
+    const int64_t n1 = static_cast<int64_t>(items1.size());
+    const size_t segs_b = sizeof(LongSeg) * segs.size(), items1_b = sizeof(Item) * items1.size(),
+                 segs1_b = sizeof(LongSeg) * segs1.size(), parts_b = 2 * sizeof(float) * size_t(n_parts);
     auto up = [](size_t v) { return (v + 255) & ~size_t(255); };
     const size_t o_items = 0, o_slices = up(items_b), o_smdie = o_slices + up(slices_b),
-                 o_heads = o_smdie + 256, blob_b = o_heads + 256;
+                 o_heads = o_smdie + 256, o_segs = o_heads + 256, o_items1 = o_segs + up(segs_b),
+                 o_segs1 = o_items1 + up(items1_b), o_slices1 = o_segs1 + up(segs1_b),
+                 o_heads1 = o_slices1 + (n1 ? up(slices_b) : 0), o_parts = o_heads1 + 256,
+                 blob_b = o_parts + up(parts_b);
     std::vector<unsigned char> host(blob_b, 0);
     if (items_b)
         std::memcpy(&host[o_items], items.data(), items_b);
     std::memcpy(&host[o_slices], slice_first.data(), slices_b);
     std::memcpy(&host[o_smdie], sm_die_tab, BSM_MAX_SM);
+    if (segs_b)
+        std::memcpy(&host[o_segs], segs.data(), segs_b);
+    if (n1) {
+        std::memcpy(&host[o_items1], items1.data(), items1_b);
+        std::memcpy(&host[o_segs1], segs1.data(), segs1_b);
+        std::memcpy(&host[o_slices1], slice_first1.data(), slices_b);
+    }
     int prev = -1;
     cudaGetDevice(&prev);
     cudaSetDevice(device);
@@ -537,6 +616,28 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     a.n_stages = n_stages;
     a.flags = d->flags;
     a.status = c->status;
+    a.segs = segs.empty() ? nullptr : reinterpret_cast<const LongSeg *>(b + o_segs);
+    a.partials = n_parts ? reinterpret_cast<float *>(b + o_parts) : nullptr;
+    a.phase = 0;
+    // phase 1 (rows longer than a stage): their segments again, one queue
+    // (or the same static / round-robin split as phase 0)
+    p->n_phase1 = n1;
+    if (n1) {
+        KernelArgs &a1 = p->args1;
+        a1 = a;
+        a1.items = reinterpret_cast<const Item *>(b + o_items1);
+        a1.segs = reinterpret_cast<const LongSeg *>(b + o_segs1);
+        a1.n_items = static_cast<int32_t>(n1);
+        a1.slice_first_item = reinterpret_cast<const int32_t *>(b + o_slices1);
+        a1.n_queues = 1;
+        for (int q = 0; q < BSM_MAX_DIES; ++q)
+            a1.queue_begin[q] = a1.queue_len[q] = 0;
+        a1.queue_len[0] = static_cast<int32_t>(n1);
+        a1.steal = 0;
+        a1.sm_die = nullptr;
+        a1.heads = reinterpret_cast<uint32_t *>(b + o_heads1);
+        a1.phase = 1;
+    }
 
     switch (d->policy) {
     case BSM_POLICY_WHOLE_GPU:
@@ -544,7 +645,10 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
         for (size_t s = 0; s < slices.size(); ++s) {
             const int32_t n = slice_first[s + 1] - slice_first[s];
             if (n > 0)
-                p->whole_gpu.push_back({slice_first[s], slice_first[s + 1], std::min(n, c->n_sm)});
+                p->whole_gpu.push_back({slice_first[s], slice_first[s + 1], std::min(n, c->n_sm), 0});
+            const int32_t n1s = slice_first1[s + 1] - slice_first1[s];
+            if (n1s > 0)
+                p->whole_gpu.push_back({slice_first1[s], slice_first1[s + 1], std::min(n1s, c->n_sm), 1});
         }
         p->grid = c->n_sm;
         st.launches = static_cast<int32_t>(p->whole_gpu.size());
@@ -552,14 +656,15 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     case BSM_POLICY_RR:
         a.mode = PULL_RR_SLICE;
         p->grid = static_cast<int>(std::min<int64_t>(c->n_sm, std::max<int64_t>(1, int64_t(slices.size()))));
-        st.launches = n_items > 0 ? 1 : 0;
+        st.launches = n_items > 0 ? (n1 ? 2 : 1) : 0;
         break;
     default:
         a.mode = PULL_QUEUE;
         p->grid = c->n_sm;
-        st.launches = n_items > 0 ? 1 : 0;
+        st.launches = n_items > 0 ? (n1 ? 2 : 1) : 0;
         break;
     }
+    p->args1.mode = a.mode;
     st.grid = p->grid;
     st.steal = a.steal;
     st.plan_ms = std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t0).count();
@@ -580,15 +685,18 @@ int plan_execute_impl(const bsm_plan *p, bsm_stream_t stream)
     int err = 0;
     const bool checked = g_checked.load(std::memory_order_relaxed) != 0;
     if (p->policy == BSM_POLICY_WHOLE_GPU) {
-        KernelArgs a = p->args;
+        KernelArgs a = p->args, a1 = p->args1;
         for (const auto &l : p->whole_gpu) {
-            a.item_begin = l.begin;
-            a.item_end = l.end;
-            if ((err = launch_softmax(a, p->dtype, p->kernel_op, l.grid, stream, checked)))
+            KernelArgs &al = l.phase ? a1 : a;
+            al.item_begin = l.begin;
+            al.item_end = l.end;
+            if ((err = launch_softmax(al, p->dtype, p->kernel_op, l.grid, stream, checked)))
                 break;
         }
     } else {
         err = launch_softmax(p->args, p->dtype, p->kernel_op, p->grid, stream, checked);
+        if (!err && p->n_phase1)
+            err = launch_softmax(p->args1, p->dtype, p->kernel_op, p->grid, stream, checked);
     }
     if (prev >= 0 && prev != p->device)
         cudaSetDevice(prev);
@@ -735,6 +843,8 @@ int bsm_plan_debug(bsm_plan *plan, int what, int64_t arg)
     case BSM_DEBUG_NONE:
         plan->args.debug = 0;
         plan->args.wait_limit_ns = 0;
+        plan->args1.debug = 0;
+        plan->args1.wait_limit_ns = 0;
         return BSM_OK;
     case BSM_DEBUG_WITHHOLD_STAGE:
         if (arg <= 0)

@@ -53,6 +53,21 @@ enum Op : int32_t {
     OP_BACKWARD_LONG = 3 // OP_BACKWARD for plans with rows longer than half a stage (two passes)
 };
 
+// A row longer than one stage is cut into segments of whole stage-sized
+// chunks, each its own patch (nrows = 1, off/C = the segment).  An execute
+// then takes two launches: in phase 0 every segment streams its chunks and
+// leaves a partial in partials[2*part] -- (max, sum of exp(v - max)) forward,
+// (<y, dy>, 0) backward -- while short rows are finished; in phase 1 every
+// segment combines its row's partials [part_first, part_first + part_count)
+// in that order (the same for every segment and every policy) and streams
+// its chunks again to write the output.  part_count = 0: a short-row patch.
+struct LongSeg {
+    int32_t col0;               // column of the segment's first element in its row
+    int32_t part;
+    int32_t part_first;
+    int32_t part_count;
+};
+
 struct KernelArgs {
     const void *x;
     const void *x2;             // OP_BACKWARD: the upstream gradient
@@ -76,6 +91,10 @@ struct KernelArgs {
     uint32_t *status;           // sticky device status word
     uint64_t wait_limit_ns;     // bound of every pipeline wait (0 = the 2 s default)
     uint32_t debug;             // fault injection for tests: KDEBUG_* bits
+    // rows longer than a stage (OP_*_LONG): see LongSeg
+    const LongSeg *segs;        // per patch, in the order of `items`; NULL: no long rows
+    float *partials;            // 2 floats per segment
+    int32_t phase;              // 0: segments leave their partials; 1: combine and write
 };
 
 // Test-only fault injection (bsm_plan_debug).

@@ -50,11 +50,15 @@ struct alignas(16) StageMeta {
     int32_t kind;
     int32_t R;
     int32_t col0;       // KIND_LONG: column of the chunk's first element
-    int32_t pass;       // KIND_LONG: 0 = max and sum, 1 = write
-    int32_t last;       // KIND_LONG: last chunk of its pass
+    int32_t pass;       // KIND_LONG: 0 = partial of the segment, 1 = combine and write
+    int32_t last;       // KIND_LONG: last chunk of the segment
+    int32_t first;      // KIND_LONG: first chunk of the segment
+    int32_t part;       // KIND_LONG: the segment's partial slot
+    int32_t part_first; // KIND_LONG: the row's first partial slot
+    int32_t part_count; // KIND_LONG: the row's number of segments
     int32_t pad[2];
 };
-static_assert(sizeof(StageMeta) == 48, "StageMeta layout");
+static_assert(sizeof(StageMeta) == 64, "StageMeta layout");
 
 struct SmemHeader {
     uint64_t full[kMaxStages];
@@ -1179,12 +1183,17 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                     const int64_t ne = (int64_t)item.nrows * item.C;
                     const int64_t nbytes = ne * E::kSize;
                     const int64_t cap = kBwd ? a.stage_bytes / 2 : a.stage_bytes;
-                    const bool is_long = kLong && nbytes > cap && item.nrows == 1;
+                    LongSeg sg{0, 0, 0, 0};
+                    if (kLong && a.segs && pos[j] >= 0 && pos[j] < a.n_items)
+                        sg = a.segs[pos[j]];
+                    const bool is_long = kLong && sg.part_count > 0;
                     const bool ok = pos[j] >= 0 && pos[j] < a.n_items && item.off >= 0 && item.C > 0 &&
                                     item.nrows > 0 && item.R > 0 && item.row0 >= 0 &&
                                     item.row0 < item.R && item.off + ne <= a.total_elems &&
                                     (nbytes <= cap || is_long) && (nbytes & 15) == 0 &&
-                                    ((item.off * E::kSize) & 15) == 0;
+                                    ((item.off * E::kSize) & 15) == 0 && (!is_long || item.nrows == 1) &&
+                                    (!is_long || (sg.part >= sg.part_first &&
+                                                  sg.part < sg.part_first + sg.part_count && sg.part_first >= 0));
                     if (!ok) {
                         atomicOr(a.status, BSM_DEV_BOUNDS);
                         mt.kind = KIND_SKIP;
@@ -1192,41 +1201,48 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                         continue;
                     }
                     if (kLong && is_long) {
-                        // the row in chunks of one stage, twice
+                        // the segment in chunks of one stage: a whole row (one
+                        // segment) streams twice in this launch; a segment of a
+                        // longer row streams once, for this launch's phase
                         const int64_t chunk = cap / E::kSize;
                         const int64_t nch = (item.C + chunk - 1) / chunk;
-                        bool first = true;
-                        for (int pass = 0; pass < 2 && !aborted; ++pass)
-                            for (int64_t k = 0; k < nch; ++k) {
-                                if (!first && !next_stage(s, ph))
-                                    break;
-                                first = false;
-                                StageMeta &lm = h.meta[s];
-                                const int64_t c0 = k * chunk;
-                                const int64_t cn = item.C - c0 < chunk ? item.C - c0 : chunk;
-                                lm.off = item.off + c0;
-                                lm.C = static_cast<int32_t>(cn);
-                                lm.nrows = 1;
-                                lm.row0 = item.row0;
-                                lm.R = item.R;
-                                lm.col0 = static_cast<int32_t>(c0);
-                                lm.pass = pass;
-                                lm.last = k == nch - 1;
-                                lm.kind = KIND_LONG;
-                                const uint32_t cb = static_cast<uint32_t>(cn * E::kSize);
-                                unsigned char *ldst = stages + (size_t)s * a.stage_bytes;
-                                mbar_arrive_expect_tx(&h.full[s], kBwd ? 2 * cb : cb);
-                                bulk_load(ldst,
-                                          static_cast<const unsigned char *>(a.x) + (item.off + c0) * E::kSize,
+                        const int p_lo = sg.part_count == 1 ? 0 : a.phase;
+                        const int p_hi = sg.part_count == 1 ? 1 : a.phase;
+                        bool first_stage = true;
+                        for (int pass = p_lo; pass <= p_hi && !aborted; ++pass)
+                        for (int64_t k = 0; k < nch && !aborted; ++k) {
+                            if (!first_stage && !next_stage(s, ph))
+                                break;
+                            first_stage = false;
+                            StageMeta &lm = h.meta[s];
+                            const int64_t c0 = k * chunk;
+                            const int64_t cn = item.C - c0 < chunk ? item.C - c0 : chunk;
+                            lm.off = item.off + c0;
+                            lm.C = static_cast<int32_t>(cn);
+                            lm.nrows = 1;
+                            lm.row0 = item.row0;
+                            lm.R = item.R;
+                            lm.col0 = static_cast<int32_t>(sg.col0 + c0);
+                            lm.pass = pass;
+                            lm.last = k == nch - 1;
+                            lm.first = k == 0;
+                            lm.part = sg.part;
+                            lm.part_first = sg.part_first;
+                            lm.part_count = sg.part_count;
+                            lm.kind = KIND_LONG;
+                            const uint32_t cb = static_cast<uint32_t>(cn * E::kSize);
+                            unsigned char *ldst = stages + (size_t)s * a.stage_bytes;
+                            mbar_arrive_expect_tx(&h.full[s], kBwd ? 2 * cb : cb);
+                            bulk_load(ldst,
+                                      static_cast<const unsigned char *>(a.x) + (item.off + c0) * E::kSize,
+                                      cb, &h.full[s]);
+                            if (kBwd)   // dy's chunk into the second half
+                                bulk_load(ldst + a.stage_bytes / 2,
+                                          static_cast<const unsigned char *>(a.x2) + (item.off + c0) * E::kSize,
                                           cb, &h.full[s]);
-                                if (kBwd)   // dy's chunk into the second half
-                                    bulk_load(ldst + a.stage_bytes / 2,
-                                              static_cast<const unsigned char *>(a.x2) +
-                                                  (item.off + c0) * E::kSize,
-                                              cb, &h.full[s]);
-                                issued[s] = true;
-                                issued_phase[s] = ph;
-                            }
+                            issued[s] = true;
+                            issued_phase[s] = ph;
+                        }
                         continue;
                     }
                     mt.off = item.off;
@@ -1320,6 +1336,23 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
             break;
         if (kLong && mt.kind == KIND_LONG) {
             Bounds bd{nullptr, nullptr, y, y + a.total_elems * E::kSize, a.status};
+            if (mt.pass == 1 && mt.first && mt.part_count > 1) {
+                // the row's partials, left by phase 0, combined in slot order
+                // (every segment of the row, on any SM, gets the same result)
+                const float *pp = a.partials + 2 * static_cast<int64_t>(mt.part_first);
+                if constexpr (kBwd) {
+                    float dot = 0.0f;
+                    for (int k = 0; k < mt.part_count; ++k)
+                        dot += pp[2 * k];
+                    long_mL = dot;
+                } else {
+                    float m = -INFINITY, sum = 0.0f;
+                    for (int k = 0; k < mt.part_count; ++k)
+                        combine_ms(m, sum, pp[2 * k], pp[2 * k + 1]);
+                    long_mL = m * kLog2e;
+                    long_inv = __frcp_rn(sum);
+                }
+            }
             if constexpr (kBwd)
                 long_chunk_bwd<Tag, Checked>(stages + (size_t)s * a.stage_bytes, a.stage_bytes / 2, mt, y, warp,
                                              lane, bd, s_l, long_mL);
@@ -1329,40 +1362,23 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
             __syncwarp();
             if (lane == 0)
                 mbar_arrive(&h.empty[s]);
-            if (kBwd && mt.pass == 0 && mt.last) {
-                // the dot product: lanes, then warps in a fixed order
+            if (mt.pass == 0 && mt.last) {
+                // the segment's partial: lanes, then warps in a fixed order
+                if constexpr (kBwd) {
 #pragma unroll
-                for (int o = 16; o >= 1; o >>= 1)
-                    s_l += __shfl_xor_sync(0xFFFFFFFFu, s_l, o);
-                const int par = long_rows & 1;
-                if (lane == 0) {
-                    h.partial[par][warp] = make_float2(s_l, 0.0f);
-                    mbar_arrive(&h.xwarp);
-                }
-                if (!mbar_wait_bounded(&h.xwarp, long_rows & 1u, &h.abort_flag, wait_limit)) {
-                    if (lane == 0) {
-                        atomicOr(a.status, BSM_DEV_TIMEOUT);
-                        h.abort_flag = 1;
+                    for (int o = 16; o >= 1; o >>= 1)
+                        s_l += __shfl_xor_sync(0xFFFFFFFFu, s_l, o);
+                } else {
+#pragma unroll
+                    for (int o = 16; o >= 1; o >>= 1) {
+                        const float mo = __shfl_xor_sync(0xFFFFFFFFu, m_l, o);
+                        const float so = __shfl_xor_sync(0xFFFFFFFFu, s_l, o);
+                        combine_ms(m_l, s_l, mo, so);
                     }
-                    break;
-                }
-                float dot = 0.0f;
-                for (int w = 0; w < kConsumerWarps; ++w)
-                    dot += h.partial[par][w].x;
-                long_mL = dot;
-                s_l = 0.0f;
-                ++long_rows;
-            } else if (!kBwd && mt.pass == 0 && mt.last) {
-                // lanes, then warps: every warp ends with the same (m, s)
-#pragma unroll
-                for (int o = 16; o >= 1; o >>= 1) {
-                    const float mo = __shfl_xor_sync(0xFFFFFFFFu, m_l, o);
-                    const float so = __shfl_xor_sync(0xFFFFFFFFu, s_l, o);
-                    combine_ms(m_l, s_l, mo, so);
                 }
                 const int par = long_rows & 1;
                 if (lane == 0) {
-                    h.partial[par][warp] = make_float2(m_l, s_l);
+                    h.partial[par][warp] = make_float2(kBwd ? s_l : m_l, kBwd ? 0.0f : s_l);
                     mbar_arrive(&h.xwarp);
                 }
                 if (!mbar_wait_bounded(&h.xwarp, long_rows & 1u, &h.abort_flag, wait_limit)) {
@@ -1375,10 +1391,23 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                 float m = -INFINITY, sum = 0.0f;
                 for (int w = 0; w < kConsumerWarps; ++w) {
                     const float2 pw = h.partial[par][w];
-                    combine_ms(m, sum, pw.x, pw.y);
+                    if constexpr (kBwd)
+                        m = w == 0 ? pw.x : m + pw.x;
+                    else
+                        combine_ms(m, sum, pw.x, pw.y);
                 }
-                long_mL = m * kLog2e;
-                long_inv = __frcp_rn(sum);
+                if (mt.part_count == 1) {
+                    // the whole row: its second pass follows in this launch
+                    if constexpr (kBwd) {
+                        long_mL = m;
+                    } else {
+                        long_mL = m * kLog2e;
+                        long_inv = __frcp_rn(sum);
+                    }
+                } else if (warp == 0 && lane == 0) {
+                    a.partials[2 * static_cast<int64_t>(mt.part)] = m;
+                    a.partials[2 * static_cast<int64_t>(mt.part) + 1] = sum;
+                }
                 m_l = -INFINITY;
                 s_l = 0.0f;
                 ++long_rows;

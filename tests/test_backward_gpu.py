@@ -163,3 +163,24 @@ def test_backward_mixed_short_and_long_rows():
         assert torch.equal(bits(o), bits(outs[0]))
     _check(w, y, dy, to_host(outs[0]))
     assert bsm.bsm_device_status() == 0
+
+
+def test_backward_many_long_rows_one_launch():
+    """Two waves of backward long rows: each row streams twice in one launch."""
+    import torch
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    half = bsm.bsm_max_row_bytes() // 2 // 4
+    R, C = 2 * n_sm + 8, half + 4
+    w = workload.uniform("bwd many long", workload.F32, 1, R, C, 3.0, 0xB77).materialize()
+    y, dy = _inputs(w)
+    yd, dyd = to_device(y), to_device(dy)
+    outs = []
+    for pol in ALL:
+        dx = torch.full_like(yd, float("nan"))
+        bsm.bsm_softmax_backward(yd, dyd, dx, 1, R, C, workload.F32, pol)
+        outs.append(dx)
+    torch.cuda.synchronize()
+    for o in outs[1:]:
+        assert torch.equal(bits(o), bits(outs[0]))
+    _check(w, y, dy, to_host(outs[0]))
+    assert bsm.bsm_device_status() == 0

@@ -82,3 +82,38 @@ def test_non_finite_long_rows():
     assert np.isnan(yh[1]).all() and np.isnan(yh[2]).all()
     assert yh[3, 99999] == 1.0 and np.count_nonzero(yh[3]) == 1
     check_all_against_oracle(w, to_host(y))
+
+
+@pytest.mark.parametrize("dtype", [workload.F32, workload.BF16])
+def test_many_long_rows_stream_whole_rows_in_one_launch(dtype):
+    """With at least two waves of long rows each row is one segment that one
+    CTA streams twice in a single launch (fewer rows are cut into segments
+    over two launches); both against the oracle, all policies bit-identical."""
+    import torch
+    es = 4 if dtype == workload.F32 else 2
+    limit = bsm.bsm_max_row_bytes() // es
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    R, C = 2 * n_sm + 8, limit + 16 // es
+    w = workload.uniform("many long", dtype, 1, R, C, 3.0, 0x10A6 + dtype).materialize()
+    x = to_device(w.x)
+    p = bsm.bsm_plan_create(x, x, w.rows, w.cols, dtype, bsm.POLICY_DYNAMIC)
+    st = p.stats()
+    assert st["long_items"] == R and st["launches"] == 1 and st["n_items"] == R
+    p.close()
+    y = _all(w, x)
+    check_all_against_oracle(w, to_host(y))
+    assert bsm.bsm_device_status() == 0
+
+
+def test_few_long_rows_are_segmented_over_two_launches():
+    import torch
+    es = 4
+    limit = bsm.bsm_max_row_bytes() // es
+    w = workload.uniform("few long", workload.F32, 1, 3, 8 * limit, 2.0, 0x5E6).materialize()
+    x = to_device(w.x)
+    p = bsm.bsm_plan_create(x, torch.empty_like(x), w.rows, w.cols, workload.F32, bsm.POLICY_DYNAMIC)
+    st = p.stats()
+    assert st["long_items"] == 3 and st["launches"] == 2 and st["n_items"] > 3
+    p.close()
+    y = _all(w, x)
+    check_all_against_oracle(w, to_host(y))
