@@ -1037,6 +1037,7 @@ struct Puller {
     int32_t cur = 0, end = 0;
     int32_t q = 0;           // PULL_QUEUE: index into the try order
     int32_t die = 0;
+    uint32_t fetch = kFetch; // PULL_QUEUE: patches per claim (1 near the end of a queue)
 
     __device__ explicit Puller(const KernelArgs &args) : a(args)
     {
@@ -1082,13 +1083,17 @@ struct Puller {
         const int tries = a.steal ? a.n_queues : 1;
         while (q < tries) {
             const int qq = (die + q) % a.n_queues;
-            const uint32_t t = atomicAdd(&a.heads[qq], static_cast<uint32_t>(kFetch));
+            const uint32_t t = atomicAdd(&a.heads[qq], fetch);
             const uint32_t len = static_cast<uint32_t>(a.queue_len[qq]);
             if (t < len) {
 #pragma unroll
                 for (int j = 0; j < kFetch; ++j)
-                    if (t + j < len)
+                    if (static_cast<uint32_t>(j) < fetch && t + j < len)
                         pos[n++] = a.queue_begin[qq] + static_cast<int32_t>(t + j);
+                // near the end of the queue, claim one patch at a time so the
+                // last patches spread over the SMs instead of queueing in fours
+                if (len - t < 2u * kFetch * gridDim.x)
+                    fetch = 1;
                 return n;
             }
             ++q;
