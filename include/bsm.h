@@ -28,7 +28,8 @@
  *                         run-time stealing once a die's own queue is empty.
  *   BSM_POLICY_DYNAMIC    Not in the paper: one device-wide queue of patches,
  *                         every SM pulls the next one (the locality-blind
- *                         dynamic schedule CBMF is measured against).
+ *                         dynamic schedule CBMF is measured against); under
+ *                         the causal mask the queue runs heaviest patch first.
  *   BSM_POLICY_MINIMAX    Sec. 4.2, general form: patches assigned to dies to
  *                         minimise the largest per-SM finish time, a patch's
  *                         cost depending on its distance to the die (near /
@@ -50,11 +51,15 @@
  *     BSM_ERR_MISALIGNED.
  *   - In place (x == y) is allowed; partially overlapping x and y are not
  *     (BSM_ERR_INVALID_ARG).
- *   - Row length: a row of up to bsm_max_row_bytes() is read once from one
- *     shared-memory stage.  Longer rows (forward only) stream through the
- *     stages in chunks twice -- a running maximum and rescaled sum, then the
- *     output -- so they cost one extra read; the backward pass rejects rows
- *     over half of bsm_max_row_bytes() with BSM_ERR_UNSUPPORTED.
+ *   - Row length: a row of up to bsm_max_row_bytes() (half of it for the
+ *     backward pass, where y and dy share a stage) is read once from one
+ *     shared-memory stage.  Longer rows stream through the stages in chunks
+ *     twice -- a running maximum and rescaled sum (backward: the dot
+ *     product), then the output -- so they cost one extra read.  When a
+ *     batch has fewer such rows than two per SM, each is cut into segments
+ *     spread over the SMs and the execute takes two launches (segment
+ *     partials, then combine and write); otherwise each row stays on one SM
+ *     within one launch.
  */
 #ifndef BSM_H
 #define BSM_H
@@ -73,7 +78,7 @@ typedef enum {
     BSM_OK = 0,
     BSM_ERR_INVALID_ARG = 1,   /* null / negative / inconsistent arguments */
     BSM_ERR_MISALIGNED = 2,    /* 16-byte alignment rule broken */
-    BSM_ERR_UNSUPPORTED = 3,   /* backward row too long for a stage, too many patches */
+    BSM_ERR_UNSUPPORTED = 3,   /* shape outside a kernel's limits, too many patches */
     BSM_ERR_CUDA = 4,          /* a CUDA runtime call failed */
     BSM_ERR_DEVICE_BOUNDS = 5, /* a kernel met a patch outside the buffers */
     BSM_ERR_TIMEOUT = 6,       /* a kernel wait gave up after its time limit */
@@ -192,7 +197,7 @@ int bsm_softmax_noalloc(const void *x, void *y, int64_t B, int64_t R, int64_t C,
  * (the vector-Jacobian product of the row softmax; with a causal forward the
  * masked y are 0 and so are their dx).  y, dy, dx: device pointers, B*R*C
  * elements of `dtype`; dx may equal y or dy; other overlaps are rejected.
- * Rows may be at most half of bsm_max_row_bytes() (y and dy share a stage).
+ * Rows of any length (see "Row length" above).
  * Same scheduling policies, errors and alignment rules as bsm_softmax.
  */
 int bsm_softmax_backward(const void *y, const void *dy, void *dx, int64_t B, int64_t R, int64_t C,
@@ -274,7 +279,8 @@ int bsm_plan_create(bsm_plan **plan, const bsm_plan_desc *d);
 
 /* Launch the plan on `stream` (async).  Allocates nothing and does not
  * synchronise.  Executions of one plan must not overlap in time (they share
- * the plan's queue counters): keep them on one stream, or order them. */
+ * the plan's queue counters and its long-row partials): keep them on one
+ * stream, or order them. */
 int bsm_plan_execute(const bsm_plan *plan, bsm_stream_t stream);
 
 typedef struct {
