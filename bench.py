@@ -478,20 +478,15 @@ def sweep(args, bsm, workload, stream):
             x = x.view(torch.bfloat16)
         y = torch.empty_like(x)
         for name in ("whole_gpu", "rr", "dynamic", "cbmf", "cbmf_lb", "minimax"):
-            pol = bsm.POLICIES[name]
             reps = 3 if name == "whole_gpu" and k == 5 else 20
-
-            def step():
-                bsm.bsm_softmax_ragged(x, y, w.offsets, w.rows, w.cols, w.dtype, pol, w.flags,
-                                       stream)
-            for _ in range(3):
-                step()
-            stream.synchronize()
-            med = _median_ms(step, reps, stream)
-            print(json.dumps({"sweep": True, "workload": w.name, "policy": name,
-                              "ms": round(med, 4),
-                              "GBps": round(w.algorithmic_bytes / (med * 1e-3) / 1e9, 2),
-                              "slices_per_s": round(w.nslices / (med * 1e-3), 1)}), flush=True)
+            # rows per patch: as many as fill a stage, or at most 64 / 16
+            for rpi in (0, 64, 16):
+                med = _sweep_cell(bsm, w, x, y, bsm.POLICIES[name], rpi, reps, stream)
+                print(json.dumps({"sweep": True, "workload": w.name, "policy": name,
+                                  "rows_per_patch": rpi or "stage", "ms": round(med, 4),
+                                  "GBps": round(w.algorithmic_bytes / (med * 1e-3) / 1e9, 2),
+                                  "slices_per_s": round(w.nslices / (med * 1e-3), 1)}),
+                      flush=True)
         if k in (2, 3, 5):
             # backward pass on the same slices: read y and dy, write dx
             dy = torch.empty_like(x).normal_() if w.dtype == workload.F32 else \
@@ -605,6 +600,28 @@ def run_bmm(args, bsm, workload, ws, rank, dev):
     if rank == 0:
         print(json.dumps(out), flush=True)
     return 0
+
+
+def _sweep_cell(bsm, w, x, y, pol, rpi, reps, stream):
+    """Median ms of one policy on one workload; rpi > 0 caps the rows per
+    patch (a plan of its own), 0 lets patches fill a stage."""
+    plan = None
+    if rpi:
+        plan = bsm.bsm_plan_create(x, y, w.rows, w.cols, w.dtype, pol, offsets=w.offsets,
+                                   flags=w.flags, rows_per_item=rpi)
+
+    def step():
+        if plan is not None:
+            plan.execute(stream)
+        else:
+            bsm.bsm_softmax_ragged(x, y, w.offsets, w.rows, w.cols, w.dtype, pol, w.flags, stream)
+    for _ in range(3):
+        step()
+    stream.synchronize()
+    med = _median_ms(step, reps, stream)
+    if plan is not None:
+        plan.close()
+    return med
 
 
 def _median_ms(fn, reps, stream, rounds=5):
