@@ -28,8 +28,7 @@
  *                         run-time stealing once a die's own queue is empty.
  *   BSM_POLICY_DYNAMIC    Not in the paper: one device-wide queue of patches,
  *                         every SM pulls the next one (the locality-blind
- *                         dynamic schedule CBMF is measured against); under
- *                         the causal mask the queue runs heaviest patch first.
+ *                         dynamic schedule CBMF is measured against).
  *   BSM_POLICY_MINIMAX    Sec. 4.2, general form: patches assigned to dies to
  *                         minimise the largest per-SM finish time, a patch's
  *                         cost depending on its distance to the die (near /

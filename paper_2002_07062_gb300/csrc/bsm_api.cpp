@@ -407,21 +407,6 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     if (d->policy == BSM_POLICY_DYNAMIC) {
         queue.resize(static_cast<size_t>(n_items));
         std::iota(queue.begin(), queue.end(), 0);
-        if ((d->flags & BSM_FLAG_CAUSAL) && d->op == BSM_OP_FORWARD) {
-            // under the causal mask a patch's work grows with its rows'
-            // index: take the heaviest first (longest processing time first,
-            // Sec. 4.2), so that the last patches of the queue are light
-            std::vector<int64_t> work(static_cast<size_t>(n_items));
-            for (int64_t i = 0; i < n_items; ++i) {
-                const Item &it = items[static_cast<size_t>(i)];
-                int64_t w = 0;
-                for (int32_t k = 0; k < it.nrows; ++k)
-                    w += std::min<int64_t>((int64_t(it.row0) + k) % it.R + 1, it.C);
-                work[static_cast<size_t>(i)] = w;
-            }
-            std::stable_sort(queue.begin(), queue.end(),
-                             [&](int32_t u, int32_t v) { return work[u] > work[v]; });
-        }
         qlen[0] = static_cast<int32_t>(n_items);
         st.queue_items[0] = n_items;
         st.queue_bytes[0] = total * es * 2;
