@@ -415,7 +415,8 @@ def main():
                    "causal": bool(w.flags & 1), "seed": hex(w.seed),
                    "bytes_per_step": bytes_step,
                    "l2": "inputs larger than L2 (%d MB vs 129 MB), no flush" % (bytes_step >> 20),
-                   "parallelism": "slices sharded by rank, no collective" if ws > 1 else "1 GPU"},
+                   "parallelism": ("%d ranks, each its own batch of %d slices (weak scaling), "
+                                   "no collective on the data path" % (ws, B)) if ws > 1 else "1 GPU"},
         "pct_of_measured_hbm": round(100 * value / ws / peak, 2),
         "pct_of_nominal_8tbs": round(100 * value / ws / NOMINAL_HBM_GBS, 2),
         "slices_per_s": round(ws * B / (ms * 1e-3), 1),
