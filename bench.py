@@ -323,6 +323,8 @@ def main():
                     help="also time every policy on workloads 2-5 (extra JSON lines)")
     ap.add_argument("--bmm", type=int, default=0, choices=[0, 1, 2],
                     help="time the Sec. 6 batched product 1 or 2 instead of the softmax")
+    ap.add_argument("--long-rows", type=int, default=0,
+                    help="time fp32 rows of this many elements (longer than a stage), 256 MiB in all")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=20)
@@ -354,6 +356,8 @@ def main():
 
     if args.bmm:
         return run_bmm(args, bsm, workload, ws, rank, dev)
+    if args.long_rows:
+        return run_long_rows(args, bsm, rank, dev)
 
     w = workload.config(args.workload).materialize()
     pol = policy_code(args.policy)
@@ -598,6 +602,46 @@ def run_bmm(args, bsm, workload, ws, rank, dev):
            "clocks": clk.summary(), "device_status": bsm.bsm_device_status()}
     if not args.no_cpu_baseline and rank == 0 and ws == 1:
         out["cpu_baseline"] = bmm_cpu_baseline(w)
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    return 0
+
+
+def run_long_rows(args, bsm, rank, dev):
+    """One JSON line for fp32 rows longer than a shared-memory stage (256 MiB
+    of input, dynamic policy): GB/s of algorithmic traffic (x read once, y
+    written once) and of the bytes the two passes move (x read twice)."""
+    import torch
+    C = args.long_rows
+    R = max(1, (256 << 20) // (4 * C))
+    g = torch.Generator(device="cuda").manual_seed(0x2002070600 + C)
+    x = torch.randn(R * C, device="cuda", generator=g)
+    y = torch.empty_like(x)
+    stream = torch.cuda.Stream()
+    plan = bsm.bsm_plan_create(x, y, [R], [C], bsm.F32, bsm.POLICY_DYNAMIC)
+    st = plan.stats()
+
+    def step():
+        plan.execute(stream)
+    for _ in range(max(3, args.warmup)):
+        step()
+    stream.synchronize()
+    with ClockSampler(dev) as clk:
+        total_ms, _ = time_steps(step, args.steps, stream)
+    torch.cuda.synchronize()
+    ms = total_ms / args.steps
+    alg = 2 * R * C * 4
+    out = {"metric": "softmax of rows longer than a stage, GB/s (read+write)",
+           "value": round(alg / (ms * 1e-3) / 1e9, 2), "unit": "GB/s", "n_gpus": 1,
+           "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": round(ms, 5),
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+           "data": "synthetic", "config": {"workload": "fp32 %d rows x %d" % (R, C),
+                                           "policy": "dynamic", "bytes_per_step": alg},
+           "moved_GBps": round(1.5 * alg / (ms * 1e-3) / 1e9, 2),
+           "gpu_launches": int(st["launches"]) * args.steps,
+           "plan": {k: st[k] for k in ("n_items", "long_items", "launches", "stage_bytes", "n_stages")},
+           "clocks": clk.summary(), "device_status": bsm.bsm_device_status()}
+    plan.close()
     if rank == 0:
         print(json.dumps(out), flush=True)
     return 0
