@@ -101,3 +101,28 @@ def test_bmm_argument_errors_without_gpu(args, code):
 def test_bmm_empty_batch_is_a_no_op():
     for B, M, N in [(0, 128, 64), (3, 0, 64), (3, 128, 0)]:
         assert bsm.lib().bsm_bmm(None, None, None, B, M, N, 64, bsm.BF16, bsm.POLICY_RR, None) == bsm.OK
+
+
+def test_header_is_plain_c_and_links_from_c(tmp_path):
+    """include/bsm.h compiles as C11 under -pedantic, and a C program links
+    against libbsm.so and gets argument errors back without a GPU."""
+    import os
+    import shutil
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("no C compiler")
+    inc = os.path.dirname(bsm.HEADER)
+    lib_dir = os.path.dirname(bsm.LIB_PATH)
+    src = tmp_path / "capi.c"
+    src.write_text(
+        "#include <stdio.h>\n#include \"bsm.h\"\n"
+        "int main(void) {\n"
+        "  int rc = bsm_softmax(NULL, NULL, -1, 4, 4, BSM_F32, BSM_POLICY_DYNAMIC, NULL);\n"
+        "  int rb = bsm_bmm(NULL, NULL, NULL, 1, 64, 64, 64, BSM_F32, BSM_POLICY_DYNAMIC, NULL);\n"
+        "  printf(\"%d %d %d\\n\", bsm_version(), rc, rb);\n"
+        "  return rc == BSM_ERR_INVALID_ARG && rb == BSM_ERR_UNSUPPORTED ? 0 : 1;\n}\n")
+    exe = tmp_path / "capi"
+    subprocess.run([gcc, "-std=c11", "-Wall", "-Wextra", "-pedantic", "-Werror", "-I", inc, str(src),
+                    "-L", lib_dir, "-lbsm", "-Wl,-rpath," + lib_dir, "-o", str(exe)], check=True)
+    out = subprocess.run([str(exe)], capture_output=True, text=True)
+    assert out.returncode == 0, out.stdout + out.stderr
