@@ -158,7 +158,7 @@ struct SliceView {
 };
 
 // Validate a descriptor; fills the slice list and the element extent.
-int validate(const bsm_plan_desc *d, const DeviceCtx &c, std::vector<SliceView> &slices,
+int validate(const bsm_plan_desc *d, std::vector<SliceView> &slices,
              int64_t &total_elems, int64_t &max_row_bytes)
 {
     if (d->dtype != BSM_F32 && d->dtype != BSM_BF16)
@@ -257,7 +257,7 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
         cudaGetDevice(&device);
     std::vector<SliceView> slices;
     int64_t total = 0, max_row = 0;
-    if ((rc = validate(d, *c, slices, total, max_row)))
+    if ((rc = validate(d, slices, total, max_row)))
         return rc;
     const int es = esize(d->dtype);
 

@@ -481,16 +481,6 @@ __device__ __forceinline__ uint32_t bmax2(uint32_t a, uint32_t b)
 // masked by the causal mask still turns its row into NaN: NaN + (-inf) and
 // +inf + (-inf) are NaN); a NaN-propagating maximum over the raw vector.
 template <typename Tag> __device__ __forceinline__ bool vec_poisons(uint4 r);
-template <> __device__ __forceinline__ bool vec_poisons<F32>(uint4 r)
-{
-    float m;
-    asm("{\n\t.reg .f32 a, b;\n\tmax.NaN.f32 a, %1, %2;\n\tmax.NaN.f32 b, %3, %4;\n\t"
-        "max.NaN.f32 %0, a, b;\n\t}"
-        : "=f"(m)
-        : "f"(__uint_as_float(r.x)), "f"(__uint_as_float(r.y)), "f"(__uint_as_float(r.z)),
-          "f"(__uint_as_float(r.w)));
-    return !(m < INFINITY);
-}
 template <> __device__ __forceinline__ bool vec_poisons<BF16>(uint4 r)
 {
     uint32_t w;
