@@ -1039,19 +1039,19 @@ struct Puller {
             slice = static_cast<int32_t>(blockIdx.x) - static_cast<int32_t>(gridDim.x);
     }
 
-    // Positions in a.items of this CTA's next patches (up to kFetch); returns
-    // how many (0 when the CTA has no more work).
-    __device__ int next_batch(int32_t (&pos)[kFetch])
+    // Positions in a.items of this CTA's next patches (up to `most`, at most
+    // kFetch); returns how many (0 when the CTA has no more work).
+    __device__ int next_batch(int32_t (&pos)[kFetch], int most = kFetch)
     {
         int n = 0;
         if (a.mode == PULL_STATIC) {
 #pragma unroll
             for (int j = 0; j < kFetch; ++j) {
                 const int64_t idx = (int64_t)a.item_begin + blockIdx.x + (int64_t)(k + j) * gridDim.x;
-                if (idx < a.item_end)
+                if (j < most && idx < a.item_end)
                     pos[n++] = static_cast<int32_t>(idx);
             }
-            k += kFetch;
+            k += most;
             return n;
         }
         if (a.mode == PULL_RR_SLICE) {
@@ -1064,7 +1064,7 @@ struct Puller {
             }
 #pragma unroll
             for (int j = 0; j < kFetch; ++j)
-                if (cur < end)
+                if (j < most && cur < end)
                     pos[n++] = cur++;
             return n;
         }
@@ -1073,12 +1073,13 @@ struct Puller {
         const int tries = a.steal ? a.n_queues : 1;
         while (q < tries) {
             const int qq = (die + q) % a.n_queues;
-            const uint32_t t = atomicAdd(&a.heads[qq], fetch);
+            const uint32_t take = fetch < static_cast<uint32_t>(most) ? fetch : static_cast<uint32_t>(most);
+            const uint32_t t = atomicAdd(&a.heads[qq], take);
             const uint32_t len = static_cast<uint32_t>(a.queue_len[qq]);
             if (t < len) {
 #pragma unroll
                 for (int j = 0; j < kFetch; ++j)
-                    if (static_cast<uint32_t>(j) < fetch && t + j < len)
+                    if (static_cast<uint32_t>(j) < take && t + j < len)
                         pos[n++] = a.queue_begin[qq] + static_cast<int32_t>(t + j);
                 // near the end of the queue, claim one patch at a time so the
                 // last patches spread over the SMs instead of queueing in fours
@@ -1146,15 +1147,45 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                 ++it;
                 return true;
             };
+            // Long-row instances claim one patch at a time, and the next one
+            // while a row streams: the queue atomic and the record loads
+            // behind it are round trips of microseconds under full load,
+            // which would otherwise stall the ring at every row start.
+            int nx_n = -1;              // patches claimed ahead (-1: none)
+            int32_t nx_pos = 0;
+            Item nx_item{0, 0, 0, 0, 0};
+            LongSeg nx_seg{0, 0, 0, 0};
+            auto claim_ahead = [&]() {
+                int32_t p1[kFetch];
+                nx_n = pull.next_batch(p1, 1);
+                nx_pos = p1[0];
+                if (nx_n > 0 && nx_pos >= 0 && nx_pos < a.n_items) {
+                    nx_item = a.items[nx_pos];
+                    nx_seg = a.segs ? a.segs[nx_pos] : LongSeg{0, 0, 0, 0};
+                }
+            };
             while (!done && !aborted) {
-                // fetch the next patches: their records load in parallel
+                // the next patches: their records load in parallel
                 int32_t pos[kFetch];
-                const int n = pull.next_batch(pos);
                 Item batch[kFetch];
+                LongSeg lseg[kFetch];   // long-row instances: the segment records
+                int n = 0;
+                if (kLong && nx_n >= 0) {
+                    n = nx_n;
+                    pos[0] = nx_pos;
+                    batch[0] = nx_item;
+                    lseg[0] = nx_seg;
+                    nx_n = -1;
+                } else {
+                    n = pull.next_batch(pos, kLong ? 1 : kFetch);
 #pragma unroll
-                for (int j = 0; j < kFetch; ++j)
-                    if (j < n && pos[j] >= 0 && pos[j] < a.n_items)
-                        batch[j] = a.items[pos[j]];
+                    for (int j = 0; j < kFetch; ++j)
+                        if (j < n && pos[j] >= 0 && pos[j] < a.n_items) {
+                            batch[j] = a.items[pos[j]];
+                            if (kLong && a.segs)
+                                lseg[j] = a.segs[pos[j]];
+                        }
+                }
                 if (n == 0) {
                     // no more work: tell the consumers through the next stage
                     int s = 0;
@@ -1167,20 +1198,20 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                     break;
                 }
                 for (int j = 0; j < n && !aborted; ++j) {
+                    // long-row instances check the patch (and cut a long one
+                    // into chunks) before the wait for its stage, the others
+                    // after it
                     int s = 0;
                     uint32_t ph = 0;
-                    if (!next_stage(s, ph))
+                    if (!kLong && !next_stage(s, ph))
                         break;
-                    StageMeta &mt = h.meta[s];
-                    if ((a.debug & KDEBUG_WITHHOLD_STAGE0) && it == 1)
-                        continue;                      // test hook: stage 0 is never filled
                     const Item item = batch[j];
                     const int64_t ne = (int64_t)item.nrows * item.C;
                     const int64_t nbytes = ne * E::kSize;
                     const int64_t cap = kBwd ? a.stage_bytes / 2 : a.stage_bytes;
                     LongSeg sg{0, 0, 0, 0};
                     if (kLong && a.segs && pos[j] >= 0 && pos[j] < a.n_items)
-                        sg = a.segs[pos[j]];
+                        sg = lseg[j];
                     const bool is_long = kLong && sg.part_count > 0;
                     const bool ok = pos[j] >= 0 && pos[j] < a.n_items && item.off >= 0 && item.C > 0 &&
                                     item.nrows > 0 && item.R > 0 && item.row0 >= 0 &&
@@ -1189,6 +1220,24 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                                     ((item.off * E::kSize) & 15) == 0 && (!is_long || item.nrows == 1) &&
                                     (!is_long || (sg.part >= sg.part_first &&
                                                   sg.part < sg.part_first + sg.part_count && sg.part_first >= 0));
+                    // a long segment: chunks of equal length in whole 16-byte
+                    // vectors (no short last chunk leaves the consumers waiting
+                    // on the next copy), every one non-empty; 32-bit arithmetic
+                    // (C < 2^31, a stage < 2^18 bytes)
+                    int64_t chunk = 1, nch = 0;
+                    if (kLong && is_long && ok) {
+                        const uint32_t cl = static_cast<uint32_t>(item.C);
+                        const uint32_t cmax = static_cast<uint32_t>(cap / E::kSize);
+                        const uint32_t n_min = (cl + cmax - 1) / cmax;
+                        const uint32_t c = ((cl + n_min - 1) / n_min + E::kPerVec - 1) & ~uint32_t(E::kPerVec - 1);
+                        chunk = c;
+                        nch = (cl + c - 1) / c;
+                    }
+                    if (kLong && !next_stage(s, ph))
+                        break;
+                    StageMeta &mt = h.meta[s];
+                    if ((a.debug & KDEBUG_WITHHOLD_STAGE0) && it == 1)
+                        continue;                      // test hook: stage 0 is never filled
                     if (!ok) {
                         atomicOr(a.status, BSM_DEV_BOUNDS);
                         mt.kind = KIND_SKIP;
@@ -1199,13 +1248,17 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                         // the segment in chunks of one stage: a whole row (one
                         // segment) streams twice in this launch; a segment of a
                         // longer row streams once, for this launch's phase
-                        const int64_t chunk = cap / E::kSize;
-                        const int64_t nch = (item.C + chunk - 1) / chunk;
                         const int p_lo = sg.part_count == 1 ? 0 : a.phase;
                         const int p_hi = sg.part_count == 1 ? 1 : a.phase;
                         bool first_stage = true;
-                        for (int pass = p_lo; pass <= p_hi && !aborted; ++pass)
-                        for (int64_t k = 0; k < nch && !aborted; ++k) {
+                        for (int pass = p_lo; pass <= p_hi && !aborted; ++pass) {
+                        // a whole row's second pass runs backwards from its
+                        // last chunk, which the consumers keep in its stage
+                        // and finish first (no copy); the others follow, the
+                        // most recently read (most likely still in L2) first
+                        const bool rev = pass == 1 && sg.part_count == 1;
+                        for (int64_t kk = 0; kk < (rev ? nch - 1 : nch) && !aborted; ++kk) {
+                            const int64_t k = rev ? nch - 2 - kk : kk;
                             if (!first_stage && !next_stage(s, ph))
                                 break;
                             first_stage = false;
@@ -1219,8 +1272,8 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                             lm.R = item.R;
                             lm.col0 = static_cast<int32_t>(sg.col0 + c0);
                             lm.pass = pass;
-                            lm.last = k == nch - 1;
-                            lm.first = k == 0;
+                            lm.last = rev ? k == 0 : k == nch - 1;
+                            lm.first = rev ? kk == 0 : k == 0;
                             lm.part = sg.part;
                             lm.part_first = sg.part_first;
                             lm.part_count = sg.part_count;
@@ -1237,6 +1290,11 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                                           cb, &h.full[s]);
                             issued[s] = true;
                             issued_phase[s] = ph;
+                            // the row's second chunk is on its way (or its only
+                            // one): claim the next patch now
+                            if (nx_n < 0 && j == n - 1 && pass == p_lo && (kk == 1 || nch == 1))
+                                claim_ahead();
+                        }
                         }
                         continue;
                     }
@@ -1355,7 +1413,9 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                 long_chunk<Tag, Checked>(stages + (size_t)s * a.stage_bytes, mt, y, causal, warp, lane, bd, m_l,
                                          s_l, long_mL, long_inv);
             __syncwarp();
-            if (lane == 0)
+            // a whole row keeps its last chunk staged for the second pass
+            const bool keep = mt.pass == 0 && mt.last && mt.part_count == 1;
+            if (lane == 0 && !keep)
                 mbar_arrive(&h.empty[s]);
             if (mt.pass == 0 && mt.last) {
                 // the segment's partial: lanes, then warps in a fixed order
@@ -1392,13 +1452,25 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                         combine_ms(m, sum, pw.x, pw.y);
                 }
                 if (mt.part_count == 1) {
-                    // the whole row: its second pass follows in this launch
+                    // the whole row: its second pass follows in this launch,
+                    // starting on the chunk still in this stage
                     if constexpr (kBwd) {
                         long_mL = m;
                     } else {
                         long_mL = m * kLog2e;
                         long_inv = __frcp_rn(sum);
                     }
+                    StageMeta m1 = mt;
+                    m1.pass = 1;
+                    if constexpr (kBwd)
+                        long_chunk_bwd<Tag, Checked>(stages + (size_t)s * a.stage_bytes, a.stage_bytes / 2, m1, y,
+                                                     warp, lane, bd, s_l, long_mL);
+                    else
+                        long_chunk<Tag, Checked>(stages + (size_t)s * a.stage_bytes, m1, y, causal, warp, lane, bd,
+                                                 m_l, s_l, long_mL, long_inv);
+                    __syncwarp();
+                    if (lane == 0)
+                        mbar_arrive(&h.empty[s]);
                 } else if (warp == 0 && lane == 0) {
                     a.partials[2 * static_cast<int64_t>(mt.part)] = m;
                     a.partials[2 * static_cast<int64_t>(mt.part) + 1] = sum;
