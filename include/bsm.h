@@ -180,8 +180,8 @@ int bsm_softmax_ragged(const void *x, void *y, int64_t num_slices, const int64_t
  *   x, y, B, R, C, dtype, flags, stream: as bsm_softmax_ex.
  * Errors: as bsm_softmax_ex, plus BSM_ERR_TOO_LARGE when the batch needs more
  * than BSM_NOALLOC_MAX_PATCHES patches (a patch is the rows that fill one
- * 32 KiB shared-memory stage: for 2 KiB rows, 16 rows; 65536 patches cover
- * 2 GiB of input).
+ * 64 KiB shared-memory stage: for 2 KiB rows, 32 rows; 65536 patches cover
+ * 4 GiB of input).
  */
 #define BSM_NOALLOC_MAX_PATCHES 65536
 int bsm_softmax_noalloc(const void *x, void *y, int64_t B, int64_t R, int64_t C, int dtype,

@@ -269,7 +269,7 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     // the stages in chunks, twice
     const int64_t row_cap =
         std::min<int64_t>((max_row + 127) & ~int64_t(127), (max_row_bytes_for(*c) / in_arrays) & ~int64_t(127));
-    const int64_t min_stage = d->dtype == BSM_BF16 ? kMinStageBytesBf16 : kMinStageBytes;
+    const int64_t min_stage = kMinStageBytes;
     const int64_t stage = std::max<int64_t>(min_stage, in_arrays * row_cap);
     const int n_stages = static_cast<int>(std::min<int64_t>(kMaxStages, avail / stage));
     if (n_stages < 2)

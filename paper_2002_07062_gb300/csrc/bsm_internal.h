@@ -38,12 +38,12 @@ constexpr int kMaxStages = 8;
 constexpr int kConsumerWarps = 16;
 constexpr int kThreads = (kConsumerWarps + 1) * 32;  // + one producer warp
 constexpr int kSmemHeader = 1024;                     // barriers + stage metadata
-constexpr int kMinStageBytes = 32 * 1024;
-// bf16 rows carry half the bytes per element, so a stage holds twice the
-// elements' work per fixed stage cost (wait, metadata, dispatch, release);
-// larger stages amortise that cost (measured: +11 % causal 512-wide rows,
-// +16 % 32 x 128 slices over 32 KiB stages; fp32 is unchanged).
-constexpr int kMinStageBytesBf16 = 64 * 1024;
+// Smallest stage (three fit the shared memory).  Each stage has a fixed cost
+// (wait, metadata, dispatch, release) that larger stages amortise; measured
+// over 32 KiB stages: bf16 +11 % causal 512-wide rows, +16 % 32 x 128 slices;
+// fp32 +2 % 512 x 512 slices (+4 % with die queues), backward +2 %; 72 KiB
+// and more (two or three stages) is slower again.
+constexpr int kMinStageBytes = 64 * 1024;
 
 // What the kernel computes on every row.
 enum Op : int32_t {

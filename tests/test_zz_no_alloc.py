@@ -21,8 +21,9 @@ def built():
 
 
 def test_oversized_batch_is_rejected_before_any_device_work():
-    # 65537 patches of 16 fp32 rows of 512 elements: one more than the scratch holds
-    rows = 16 * (bsm.NOALLOC_MAX_PATCHES + 1)
+    # 65537 patches of 32 fp32 rows of 512 elements (one 64 KiB stage each):
+    # one more than the scratch holds
+    rows = 32 * (bsm.NOALLOC_MAX_PATCHES + 1)
     rc = bsm.lib().bsm_softmax_noalloc(ctypes.c_void_p(256), ctypes.c_void_p(1 << 40), 1, rows,
                                        512, bsm.F32, 0, None)
     assert rc == bsm.ERR_TOO_LARGE
