@@ -165,13 +165,15 @@ def test_backward_mixed_short_and_long_rows():
     assert bsm.bsm_device_status() == 0
 
 
-def test_backward_many_long_rows_one_launch():
-    """Two waves of backward long rows: each row streams twice in one launch."""
+@pytest.mark.parametrize("chunks", [2, 3])
+def test_backward_many_long_rows_one_launch(chunks):
+    """Two waves of backward long rows: each row streams twice in one launch,
+    the second pass from its last chunk (still staged) backwards."""
     import torch
     n_sm = torch.cuda.get_device_properties(0).multi_processor_count
     half = bsm.bsm_max_row_bytes() // 2 // 4
-    R, C = 2 * n_sm + 8, half + 4
-    w = workload.uniform("bwd many long", workload.F32, 1, R, C, 3.0, 0xB77).materialize()
+    R, C = 2 * n_sm + 8, (chunks - 1) * half + 4
+    w = workload.uniform("bwd many long", workload.F32, 1, R, C, 3.0, 0xB77 + chunks).materialize()
     y, dy = _inputs(w)
     yd, dyd = to_device(y), to_device(dy)
     outs = []

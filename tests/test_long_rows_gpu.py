@@ -117,3 +117,27 @@ def test_few_long_rows_are_segmented_over_two_launches():
     p.close()
     y = _all(w, x)
     check_all_against_oracle(w, to_host(y))
+
+
+@pytest.mark.parametrize("dtype", [workload.F32, workload.BF16])
+@pytest.mark.parametrize("chunks,flags", [(3, workload.CAUSAL), (4, 0)])
+def test_many_long_rows_of_several_chunks(dtype, chunks, flags):
+    """Whole rows of three and four chunks in the one-launch path: the
+    second pass starts on the chunk still staged and runs backwards; under
+    the causal mask most of every row is masked (the row index is below the
+    column count), so the kept last chunk is a masked one."""
+    import torch
+    es = 4 if dtype == workload.F32 else 2
+    limit = bsm.bsm_max_row_bytes() // es
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    R, C = 2 * n_sm + 3, (chunks - 1) * limit + 16 // es * 7
+    w = workload.uniform("many long %d" % chunks, dtype, 1, R, C, 3.0, 0x10B0 + chunks + dtype,
+                         flags).materialize()
+    x = to_device(w.x)
+    p = bsm.bsm_plan_create(x, x, w.rows, w.cols, dtype, bsm.POLICY_DYNAMIC, flags=flags)
+    st = p.stats()
+    assert st["long_items"] == R and st["launches"] == 1
+    p.close()
+    y = _all(w, x)
+    check_all_against_oracle(w, to_host(y))
+    assert bsm.bsm_device_status() == 0
