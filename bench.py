@@ -61,17 +61,17 @@ def kernel_hash() -> str:
 
 
 def profiled_traffic(workload_k: int, dtype_name: str):
-    """DRAM bytes per launch of the softmax kernel from the committed ncu
-    summary for this workload, if it was taken on the current kernel source."""
-    path = os.path.join(PROFILE_DIR, "softmax_persistent_workload%d.md" % workload_k)
-    if not os.path.exists(path):
-        return None
-    text = open(path).read()
-    m_hash = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]{16})", text)
-    m_traf = re.search(r"dram_bytes_per_launch:\s*([0-9]+)", text)
-    if not m_hash or not m_traf or m_hash.group(1) != kernel_hash():
-        return None
-    return int(m_traf.group(1))
+    """DRAM bytes per launch of the softmax kernel on workload k (steady
+    state: consecutive launches, caches not flushed) from a committed ncu
+    summary taken on the current kernel source, else None."""
+    import glob
+    for path in sorted(glob.glob(os.path.join(PROFILE_DIR, "softmax_persistent*.md"))):
+        text = open(path).read()
+        m_hash = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]{16})", text)
+        m_traf = re.search(r"dram_bytes_per_launch_workload%d:\s*([0-9]+)" % workload_k, text)
+        if m_hash and m_traf and m_hash.group(1) == kernel_hash():
+            return int(m_traf.group(1))
+    return None
 
 
 class ClockSampler:
