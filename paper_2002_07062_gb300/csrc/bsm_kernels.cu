@@ -826,11 +826,13 @@ __device__ __forceinline__ int consume_stage_bwd(const unsigned char *sbuf, int 
 
 // ------------------------------------------------------------ long rows
 // A row longer than a stage is streamed through the stages twice, in
-// chunks; all consumer warps share every chunk (warp w takes the vectors
-// w*32 + lane, + 512, ...).  Pass 0 keeps a running (max m, sum s of
-// exp(v - m)) per lane -- when the max grows, s is rescaled by exp(m_old -
+// chunks of equal length; all consumer warps share every chunk (warp w takes
+// the vectors w*32 + lane, + 512, ...).  Pass 0 keeps a running (max m, sum s
+// of exp(v - m)) per lane -- when the max grows, s is rescaled by exp(m_old -
 // m_new) -- then the lanes, the warps (through shared memory) combine their
-// pairs in a fixed order; pass 1 writes exp(v - m) / s.
+// pairs in a fixed order; pass 1 writes exp(v - m) / s.  For a whole row in
+// one launch, pass 1 starts on the last chunk, still in its stage, and takes
+// the others in reverse order.
 
 // (m, s) of two partials; a -inf maximum contributes nothing.
 __device__ __forceinline__ void combine_ms(float &m, float &s, float mo, float so)
