@@ -174,3 +174,25 @@ def test_shape_errors_and_empty_batches():
     assert e.value.status == bsm.ERR_INVALID_ARG
     torch.cuda.synchronize()
     assert bsm.bsm_device_status() == 0
+
+
+@pytest.mark.parametrize("N", [64, 128, 256])
+@pytest.mark.parametrize("extra", [5, 76 + 7])
+@pytest.mark.parametrize("out", [W.F32, W.BF16])
+def test_ragged_tile_counts_are_exact(N, extra, out):
+    """Tile counts one or two waves plus a few over the SMs, every tile
+    width: integer operands make every result exact, equal to the oracle and,
+    bit for bit, between the dynamic and the round-robin schedules."""
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    B, M, K = n_sm // 2 + extra, 256, 192
+    w = W.BmmWorkload("ragged waves", B, M, N, K, out, seed=29 + N + extra, kind="int")
+    a, bt = w.operands()
+    ref = O.bmm_f64(a, bt, B, M, N, K)
+    dyn = _run(w, a, bt, bsm.POLICY_DYNAMIC)
+    rr = _run(w, a, bt, bsm.POLICY_RR)
+    assert torch.equal(dyn, rr)
+    c = dyn.cpu().numpy()
+    if out == W.F32:
+        assert np.array_equal(c.reshape(B, M, N), ref.astype(np.float32))
+    else:
+        assert np.array_equal(c.view(np.uint16).reshape(B, M, N), O.round_bf16(ref))
