@@ -270,7 +270,22 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     const int64_t row_cap =
         std::min<int64_t>((max_row + 127) & ~int64_t(127), (max_row_bytes_for(*c) / in_arrays) & ~int64_t(127));
     const int64_t min_stage = kMinStageBytes;
-    const int64_t stage = std::max<int64_t>(min_stage, in_arrays * row_cap);
+    int64_t stage = std::max<int64_t>(min_stage, in_arrays * row_cap);
+    // Rows longer than that cap but whose halves fit three stages (with the
+    // shorter rows of the batch): stages of half such a row, so that each of
+    // them (two chunks) stays staged for its second pass while the third
+    // stage takes the next row's first chunk -- one copy per row
+    if (max_row > max_row_bytes_for(*c) / in_arrays) {
+        int64_t max_short = 0;
+        for (const SliceView &v : slices)
+            if (v.R > 0 && int64_t(v.C) * es <= max_row_bytes_for(*c) / in_arrays)
+                max_short = std::max<int64_t>(max_short, int64_t(v.C) * es);
+        const int64_t half = std::max<int64_t>((max_short + 127) & ~int64_t(127),
+                                               ((max_row + 1) / 2 + 127) & ~int64_t(127));
+        const int64_t two_chunk = std::max<int64_t>(min_stage, in_arrays * half);
+        if (3 * two_chunk <= avail)
+            stage = two_chunk;
+    }
     const int n_stages = static_cast<int>(std::min<int64_t>(kMaxStages, avail / stage));
     if (n_stages < 2)
         return BSM_ERR_UNSUPPORTED;

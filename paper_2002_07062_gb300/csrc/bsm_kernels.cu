@@ -56,7 +56,8 @@ struct alignas(16) StageMeta {
     int32_t part;       // KIND_LONG: the segment's partial slot
     int32_t part_first; // KIND_LONG: the row's first partial slot
     int32_t part_count; // KIND_LONG: the row's number of segments
-    int32_t pad[2];
+    int32_t resident;   // KIND_LONG: the whole row stays staged for its second pass
+    int32_t pad;
 };
 static_assert(sizeof(StageMeta) == 64, "StageMeta layout");
 
@@ -1250,8 +1251,11 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                         // the segment in chunks of one stage: a whole row (one
                         // segment) streams twice in this launch; a segment of a
                         // longer row streams once, for this launch's phase
+                        // a whole row with fewer chunks than stages stays staged:
+                        // its second pass needs no copies
+                        const bool resident = sg.part_count == 1 && nch < S;
                         const int p_lo = sg.part_count == 1 ? 0 : a.phase;
-                        const int p_hi = sg.part_count == 1 ? 1 : a.phase;
+                        const int p_hi = sg.part_count == 1 && !resident ? 1 : a.phase;
                         bool first_stage = true;
                         for (int pass = p_lo; pass <= p_hi && !aborted; ++pass) {
                         // a whole row's second pass runs backwards from its
@@ -1279,6 +1283,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                             lm.part = sg.part;
                             lm.part_first = sg.part_first;
                             lm.part_count = sg.part_count;
+                            lm.resident = resident;
                             lm.kind = KIND_LONG;
                             const uint32_t cb = static_cast<uint32_t>(cn * E::kSize);
                             unsigned char *ldst = stages + (size_t)s * a.stage_bytes;
@@ -1375,6 +1380,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
     // offset and reciprocal; which partial buffer and barrier phase is next
     float m_l = -INFINITY, s_l = 0.0f, long_mL = 0.0f, long_inv = 0.0f;
     uint32_t long_rows = 0;
+    uint32_t long_first_it = 0;  // stage iteration of the current row's first chunk
     (void)m_l, (void)s_l, (void)long_mL, (void)long_inv, (void)long_rows;
     for (uint32_t it = 0;; ++it) {
         const int s = it % S;
@@ -1415,8 +1421,11 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                 long_chunk<Tag, Checked>(stages + (size_t)s * a.stage_bytes, mt, y, causal, warp, lane, bd, m_l,
                                          s_l, long_mL, long_inv);
             __syncwarp();
-            // a whole row keeps its last chunk staged for the second pass
-            const bool keep = mt.pass == 0 && mt.last && mt.part_count == 1;
+            if (mt.pass == 0 && mt.first)
+                long_first_it = it;
+            // a whole row keeps its last chunk (a resident row: every chunk)
+            // staged for the second pass
+            const bool keep = mt.resident || (mt.pass == 0 && mt.last && mt.part_count == 1);
             if (lane == 0 && !keep)
                 mbar_arrive(&h.empty[s]);
             if (mt.pass == 0 && mt.last) {
@@ -1462,17 +1471,36 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
                         long_mL = m * kLog2e;
                         long_inv = __frcp_rn(sum);
                     }
-                    StageMeta m1 = mt;
-                    m1.pass = 1;
-                    if constexpr (kBwd)
-                        long_chunk_bwd<Tag, Checked>(stages + (size_t)s * a.stage_bytes, a.stage_bytes / 2, m1, y,
-                                                     warp, lane, bd, s_l, long_mL);
-                    else
-                        long_chunk<Tag, Checked>(stages + (size_t)s * a.stage_bytes, m1, y, causal, warp, lane, bd,
-                                                 m_l, s_l, long_mL, long_inv);
-                    __syncwarp();
-                    if (lane == 0)
-                        mbar_arrive(&h.empty[s]);
+                    if (!mt.resident) {
+                        StageMeta m1 = mt;
+                        m1.pass = 1;
+                        if constexpr (kBwd)
+                            long_chunk_bwd<Tag, Checked>(stages + (size_t)s * a.stage_bytes, a.stage_bytes / 2, m1,
+                                                         y, warp, lane, bd, s_l, long_mL);
+                        else
+                            long_chunk<Tag, Checked>(stages + (size_t)s * a.stage_bytes, m1, y, causal, warp, lane,
+                                                     bd, m_l, s_l, long_mL, long_inv);
+                        __syncwarp();
+                        if (lane == 0)
+                            mbar_arrive(&h.empty[s]);
+                    } else {
+                        // a resident row: every chunk, from the first one's stage
+                        for (uint32_t j = long_first_it; j <= it; ++j) {
+                            const int sj = static_cast<int>(j % S);
+                            StageMeta m1 = h.meta[sj];
+                            m1.pass = 1;
+                            if constexpr (kBwd)
+                                long_chunk_bwd<Tag, Checked>(stages + (size_t)sj * a.stage_bytes,
+                                                             a.stage_bytes / 2, m1, y, warp, lane, bd, s_l, long_mL);
+                            else
+                                long_chunk<Tag, Checked>(stages + (size_t)sj * a.stage_bytes, m1, y, causal, warp,
+                                                         lane, bd, m_l, s_l, long_mL, long_inv);
+                        }
+                        __syncwarp();
+                        if (lane == 0)
+                            for (uint32_t j = long_first_it; j <= it; ++j)
+                                mbar_arrive(&h.empty[j % S]);
+                    }
                 } else if (warp == 0 && lane == 0) {
                     a.partials[2 * static_cast<int64_t>(mt.part)] = m;
                     a.partials[2 * static_cast<int64_t>(mt.part) + 1] = sum;

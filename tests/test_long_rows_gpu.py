@@ -87,8 +87,10 @@ def test_non_finite_long_rows():
 @pytest.mark.parametrize("dtype", [workload.F32, workload.BF16])
 def test_many_long_rows_stream_whole_rows_in_one_launch(dtype):
     """With at least two waves of long rows each row is one segment that one
-    CTA streams twice in a single launch (fewer rows are cut into segments
-    over two launches); both against the oracle, all policies bit-identical."""
+    CTA streams in a single launch (fewer rows are cut into segments over two
+    launches).  Rows just over the cap get three stages of half a row: a row
+    (two chunks) stays staged for its second pass.  Against the oracle, all
+    policies bit-identical."""
     import torch
     es = 4 if dtype == workload.F32 else 2
     limit = bsm.bsm_max_row_bytes() // es
@@ -99,6 +101,7 @@ def test_many_long_rows_stream_whole_rows_in_one_launch(dtype):
     p = bsm.bsm_plan_create(x, x, w.rows, w.cols, dtype, bsm.POLICY_DYNAMIC)
     st = p.stats()
     assert st["long_items"] == R and st["launches"] == 1 and st["n_items"] == R
+    assert st["n_stages"] == 3 and 2 * st["stage_bytes"] >= C * es
     p.close()
     y = _all(w, x)
     check_all_against_oracle(w, to_host(y))
