@@ -51,12 +51,14 @@ def test_checked_forward_every_routine(dtype, flags, col_steps):
         assert __import__("torch").equal(bits(a), bits(b))
 
 
-@pytest.mark.parametrize("R", [3, 400])
-def test_checked_long_rows(R):
-    """3 rows: segments over two launches; 400 rows: one launch per row."""
+@pytest.mark.parametrize("R,caps", [(3, 1), (400, 1), (400, 2)])
+def test_checked_long_rows(R, caps):
+    """3 rows: segments over two launches; 400 rows: one launch per row, of
+    two chunks (staged whole between the passes) or three (the last chunk
+    kept, the others copied again)."""
     import torch
     es = 4
-    C = bsm.bsm_max_row_bytes() // es + 64
+    C = caps * (bsm.bsm_max_row_bytes() // es) + 64
     w = workload.uniform("checked long", workload.F32, 1, R, C, 2.0, 0xC4E + R).materialize()
     x = to_device(w.x)
     a, b = _both(lambda: run(w, x, bsm.POLICY_DYNAMIC))
