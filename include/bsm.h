@@ -52,13 +52,15 @@
  *     (BSM_ERR_INVALID_ARG).
  *   - Row length: a row of up to bsm_max_row_bytes() (half of it for the
  *     backward pass, where y and dy share a stage) is read once from one
- *     shared-memory stage.  Longer rows stream through the stages in chunks
- *     twice -- a running maximum and rescaled sum (backward: the dot
- *     product), then the output -- so they cost one extra read.  When a
- *     batch has fewer such rows than two per SM, each is cut into segments
- *     spread over the SMs and the execute takes two launches (segment
- *     partials, then combine and write); otherwise each row stays on one SM
- *     within one launch.
+ *     shared-memory stage.  Longer rows go through the stages in chunks, in
+ *     two passes -- a running maximum and rescaled sum (backward: the dot
+ *     product), then the output.  A row of two chunks whose halves fit three
+ *     stages (with the batch's shorter rows) stays staged between the passes
+ *     and is read once; longer rows are read again, all but their last
+ *     chunk.  When a batch has fewer such rows than two per SM, each is cut
+ *     into segments spread over the SMs and the execute takes two launches
+ *     (segment partials, then combine and write); otherwise each row stays
+ *     on one SM within one launch.
  */
 #ifndef BSM_H
 #define BSM_H
@@ -302,7 +304,7 @@ typedef struct {
     int32_t steal;              /* 1 if CTAs steal from other dies' queues */
     int64_t map_chunk_bytes;    /* granularity of the address->die map used */
     double plan_ms;             /* host time spent in bsm_plan_create */
-    int64_t long_items;         /* rows longer than a stage (streamed in two passes) */
+    int64_t long_items;         /* rows longer than a stage (two passes over chunks) */
 } bsm_plan_stats;
 
 int bsm_plan_get_stats(const bsm_plan *plan, bsm_plan_stats *out);
@@ -431,7 +433,7 @@ void bsm_set_device_checks(int on);
 const char *bsm_last_cuda_error(void);
 
 /* Largest row (C * element size) processed from a single shared-memory stage
- * on this device, bytes; longer forward rows take two passes. */
+ * on this device, bytes; longer rows take two passes (see Row length). */
 int64_t bsm_max_row_bytes(int device);
 
 /* Static description of a status code. */
