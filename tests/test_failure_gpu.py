@@ -82,3 +82,63 @@ def test_corrupted_patch_is_skipped_with_bounds_status():
     torch.cuda.synchronize()
     assert bsm.bsm_device_status() == 0
     check_all_against_oracle(w, to_host(y2))
+
+
+def _w_long():
+    """Two waves of rows just over a stage: the one-launch long-row path
+    (rows staged whole between their passes)."""
+    import torch
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    C = bsm.bsm_max_row_bytes() // 4 + 64
+    return workload.uniform("fail long", workload.F32, 1, 2 * n_sm + 3, C, 2.0, 0xFA12).materialize()
+
+
+def test_withheld_stage_times_out_on_long_rows():
+    import time
+    import torch
+    w = _w_long()
+    x = to_device(w.x)
+    y = torch.zeros_like(x)
+    bsm.bsm_device_status_clear()
+    p = bsm.bsm_plan_create(x, y, w.rows, w.cols, w.dtype, bsm.POLICY_DYNAMIC)
+    assert p.stats()["long_items"] == int(w.rows[0]) and p.stats()["launches"] == 1
+    bsm.bsm_plan_debug(p, bsm.DEBUG_WITHHOLD_STAGE, 100_000_000)      # 0.1 s waits
+    t0 = time.time()
+    p.execute()
+    torch.cuda.synchronize()
+    assert time.time() - t0 < 5.0
+    assert bsm.bsm_device_status() & bsm.DEV_TIMEOUT
+    bsm.bsm_plan_debug(p, bsm.DEBUG_NONE)
+    bsm.bsm_device_status_clear()
+    y.fill_(float("nan"))
+    p.execute()
+    torch.cuda.synchronize()
+    assert bsm.bsm_device_status() == 0
+    check_all_against_oracle(w, to_host(y))
+    p.close()
+
+
+def test_corrupted_long_patch_is_skipped_with_bounds_status():
+    import torch
+    w = _w_long()
+    C = int(w.cols[0])
+    x = to_device(w.x)
+    sentinel = -7.0
+    y = torch.full_like(x, sentinel)
+    bsm.bsm_device_status_clear()
+    p = bsm.bsm_plan_create(x, y, w.rows, w.cols, w.dtype, bsm.POLICY_RR)
+    n = p.stats()["n_items"]
+    assert n == int(w.rows[0])                                 # one patch per long row
+    bsm.bsm_plan_debug(p, bsm.DEBUG_CORRUPT_PATCH, n // 2)
+    p.execute()
+    torch.cuda.synchronize()
+    assert bsm.bsm_device_status() & bsm.DEV_BOUNDS
+    yh = to_host(y).reshape(-1, C)
+    untouched = np.all(yh == sentinel, axis=1)
+    assert untouched.sum() == 1 and untouched[n // 2]
+    from oracle import softmax as O
+    y64, _ = O.softmax_batched(w.x, w.offsets, w.rows, w.cols)
+    ok = ~untouched
+    assert np.max(np.abs(yh[ok].astype(np.float64) - y64.reshape(-1, C)[ok])) <= 2e-6
+    p.close()
+    bsm.bsm_device_status_clear()
