@@ -357,7 +357,7 @@ def main():
     if args.bmm:
         return run_bmm(args, bsm, workload, ws, rank, dev)
     if args.long_rows:
-        return run_long_rows(args, bsm, rank, dev)
+        return run_long_rows(args, bsm, ws, rank, dev)
 
     w = workload.config(args.workload).materialize()
     pol = policy_code(args.policy)
@@ -452,7 +452,12 @@ def main():
         for _ in range(3):
             e2e_step()
         stream.synchronize()
+        if ws > 1:
+            dist.barrier()
         e_ms, _ = time_steps(e2e_step, args.e2e_steps, stream, per_launch=False)
+        if ws > 1:
+            dist.barrier()
+            e_ms = reduce_max_ms(e_ms, device="cuda")
         e_ms /= args.e2e_steps
         nb = x.numel() * x.element_size()
         out["e2e"] = {"value": round(ws * bytes_step / (e_ms * 1e-3) / 1e9, 2), "unit": "GB/s",
@@ -580,14 +585,21 @@ def run_bmm(args, bsm, workload, ws, rank, dev):
         step()
     stream.synchronize()
     launches = w.B if pol == bsm.POLICY_WHOLE_GPU else 1
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
     with ClockSampler(dev) as clk:
         total_ms, _ = time_steps(step, args.steps, stream)
     torch.cuda.synchronize()
+    if ws > 1:
+        dist.barrier()
+        total_ms = reduce_max_ms(total_ms, device="cuda")
     ms = total_ms / args.steps
-    gbs = w.algorithmic_bytes / (ms * 1e-3) / 1e9
+    gbs = w.algorithmic_bytes / (ms * 1e-3) / 1e9          # per GPU (the roofline)
     peak, peak_src = measured_peak()
-    out = {"metric": "batched matmul GB/s (operands read + product written)", "value": round(gbs, 2),
-           "unit": "GB/s", "n_gpus": 1, "steps": args.steps, "warmup": max(3, args.warmup),
+    out = {"metric": "batched matmul GB/s (operands read + product written)",
+           "value": round(job_gbs(ws, w.algorithmic_bytes, args.steps, total_ms), 2),
+           "unit": "GB/s", "n_gpus": ws, "steps": args.steps, "warmup": max(3, args.warmup),
            "ms_per_step": round(ms, 5), "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
            "config": {"workload": w.name, "policy": args.policy, "bytes_per_step": w.algorithmic_bytes,
@@ -607,7 +619,7 @@ def run_bmm(args, bsm, workload, ws, rank, dev):
     return 0
 
 
-def run_long_rows(args, bsm, rank, dev):
+def run_long_rows(args, bsm, ws, rank, dev):
     """One JSON line for fp32 rows longer than a shared-memory stage (256 MiB
     of input, dynamic policy): GB/s of algorithmic traffic (x read once, y
     written once) and of the bytes the two passes move (x read twice)."""
@@ -626,13 +638,19 @@ def run_long_rows(args, bsm, rank, dev):
     for _ in range(max(3, args.warmup)):
         step()
     stream.synchronize()
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
     with ClockSampler(dev) as clk:
         total_ms, _ = time_steps(step, args.steps, stream)
     torch.cuda.synchronize()
+    if ws > 1:
+        dist.barrier()
+        total_ms = reduce_max_ms(total_ms, device="cuda")
     ms = total_ms / args.steps
     alg = 2 * R * C * 4
     out = {"metric": "softmax of rows longer than a stage, GB/s (read+write)",
-           "value": round(alg / (ms * 1e-3) / 1e9, 2), "unit": "GB/s", "n_gpus": 1,
+           "value": round(job_gbs(ws, alg, args.steps, total_ms), 2), "unit": "GB/s", "n_gpus": ws,
            "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": round(ms, 5),
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
            "data": "synthetic", "config": {"workload": "fp32 %d rows x %d" % (R, C),
