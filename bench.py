@@ -134,6 +134,9 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
+COLL_DEVICE = "cuda"      # where the timing reduction's tensor lives (NCCL: the GPU)
+
+
 def dist_env():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -343,8 +346,14 @@ def main():
     ws, rank, local = dist_env()
     if ws > 1:
         import torch.distributed as dist
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl")
+        global COLL_DEVICE
+        # one rank per GPU (a rank past the GPU count shares one: only the
+        # gloo test of this path does that); the barrier and the max-reduce
+        # of the timings go over NCCL (gloo when BSM_BENCH_DIST_BACKEND says so)
+        torch.cuda.set_device(local % max(1, torch.cuda.device_count()))
+        backend = os.environ.get("BSM_BENCH_DIST_BACKEND", "nccl")
+        COLL_DEVICE = "cuda" if backend == "nccl" else "cpu"
+        dist.init_process_group(backend)
     else:
         torch.cuda.set_device(0)
     if rank == 0 or ws == 1:
@@ -397,7 +406,7 @@ def main():
     torch.cuda.synchronize()
     if ws > 1:
         dist.barrier()
-        total_ms = reduce_max_ms(total_ms, device="cuda")
+        total_ms = reduce_max_ms(total_ms, device=COLL_DEVICE)
     status = bsm.bsm_device_status()
     ms = total_ms / args.steps
     bytes_step = w.algorithmic_bytes
@@ -457,7 +466,7 @@ def main():
         e_ms, _ = time_steps(e2e_step, args.e2e_steps, stream, per_launch=False)
         if ws > 1:
             dist.barrier()
-            e_ms = reduce_max_ms(e_ms, device="cuda")
+            e_ms = reduce_max_ms(e_ms, device=COLL_DEVICE)
         e_ms /= args.e2e_steps
         nb = x.numel() * x.element_size()
         out["e2e"] = {"value": round(ws * bytes_step / (e_ms * 1e-3) / 1e9, 2), "unit": "GB/s",
@@ -593,7 +602,7 @@ def run_bmm(args, bsm, workload, ws, rank, dev):
     torch.cuda.synchronize()
     if ws > 1:
         dist.barrier()
-        total_ms = reduce_max_ms(total_ms, device="cuda")
+        total_ms = reduce_max_ms(total_ms, device=COLL_DEVICE)
     ms = total_ms / args.steps
     gbs = w.algorithmic_bytes / (ms * 1e-3) / 1e9          # per GPU (the roofline)
     peak, peak_src = measured_peak()
@@ -646,7 +655,7 @@ def run_long_rows(args, bsm, ws, rank, dev):
     torch.cuda.synchronize()
     if ws > 1:
         dist.barrier()
-        total_ms = reduce_max_ms(total_ms, device="cuda")
+        total_ms = reduce_max_ms(total_ms, device=COLL_DEVICE)
     ms = total_ms / args.steps
     alg = 2 * R * C * 4
     out = {"metric": "softmax of rows longer than a stage, GB/s (read+write)",
