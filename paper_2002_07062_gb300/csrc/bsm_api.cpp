@@ -138,6 +138,7 @@ struct bsm_plan {
     bsm::KernelArgs args1{};         // phase 1 of plans with rows longer than a stage
     int64_t n_phase1 = 0;
     std::vector<Launch> whole_gpu;   // WHOLE_GPU: one launch per slice
+    cudaGraphExec_t whole_graph = nullptr;   // ... captured once as a CUDA graph (or null)
     void *blob = nullptr;            // device tables (patches, slice index, sm_die, heads)
     bsm_plan_stats stats{};
     // identity of the plan for the cache
@@ -240,6 +241,64 @@ int validate(const bsm_plan_desc *d, std::vector<SliceView> &slices,
         }
     }
     return BSM_OK;
+}
+
+// WHOLE_GPU runs one kernel per slice, one after another (Sec. 3): a
+// launch-bound loop.  Plans of up to this many launches capture it once, at
+// creation, as a CUDA graph, so an execute is one graph launch (the kernels
+// still run in slice order, each on the whole device); larger plans launch
+// kernel by kernel.
+constexpr size_t kMaxGraphLaunches = 4096;
+
+cudaGraphExec_t capture_whole_gpu(const bsm_plan *p)
+{
+    cudaStream_t st = nullptr;
+    if (cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking) != cudaSuccess) {
+        cudaGetLastError();
+        return nullptr;
+    }
+    cudaGraph_t g = nullptr;
+    cudaGraphExec_t e = nullptr;
+    bool ok = cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal) == cudaSuccess;
+    if (ok) {
+        KernelArgs a = p->args, a1 = p->args1;
+        for (const auto &l : p->whole_gpu) {
+            KernelArgs &al = l.phase ? a1 : a;
+            al.item_begin = l.begin;
+            al.item_end = l.end;
+            if (launch_softmax(al, p->dtype, p->kernel_op, l.grid, st, false)) {
+                ok = false;
+                break;
+            }
+        }
+        const cudaError_t ec = cudaStreamEndCapture(st, &g);   // always ends the capture
+        ok = ok && ec == cudaSuccess && g != nullptr;
+    }
+    if (ok && cudaGraphInstantiate(&e, g, 0) != cudaSuccess)
+        e = nullptr;
+    if (g)
+        cudaGraphDestroy(g);
+    cudaStreamDestroy(st);
+    cudaGetLastError();   // a failed capture leaves plain launches, not an error
+    return e;
+}
+
+void free_plan(bsm_plan *p)
+{
+    if (!p)
+        return;
+    if (p->whole_graph) {
+        // the graph may still be running: let the plan's device finish first
+        int prev = -1;
+        cudaGetDevice(&prev);
+        cudaSetDevice(p->device);
+        cudaDeviceSynchronize();
+        cudaGraphExecDestroy(p->whole_graph);
+        if (prev >= 0)
+            cudaSetDevice(prev);
+    }
+    cudaFree(p->blob);
+    delete p;
 }
 
 int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
@@ -682,6 +741,14 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
         break;
     }
     p->args1.mode = a.mode;
+    if (d->policy == BSM_POLICY_WHOLE_GPU && !p->whole_gpu.empty() && p->whole_gpu.size() <= kMaxGraphLaunches) {
+        int prev_dev = -1;
+        cudaGetDevice(&prev_dev);
+        cudaSetDevice(device);
+        p->whole_graph = capture_whole_gpu(p);
+        if (prev_dev >= 0)
+            cudaSetDevice(prev_dev);
+    }
     st.grid = p->grid;
     st.steal = a.steal;
     st.plan_ms = std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t0).count();
@@ -701,7 +768,10 @@ int plan_execute_impl(const bsm_plan *p, bsm_stream_t stream)
         return BSM_ERR_NO_DEVICE;
     int err = 0;
     const bool checked = g_checked.load(std::memory_order_relaxed) != 0;
-    if (p->policy == BSM_POLICY_WHOLE_GPU) {
+    if (p->policy == BSM_POLICY_WHOLE_GPU && p->whole_graph && !checked && p->args.debug == 0 &&
+        p->args.wait_limit_ns == 0) {
+        err = static_cast<int>(cudaGraphLaunch(p->whole_graph, static_cast<cudaStream_t>(stream)));
+    } else if (p->policy == BSM_POLICY_WHOLE_GPU) {
         KernelArgs a = p->args, a1 = p->args1;
         for (const auto &l : p->whole_gpu) {
             KernelArgs &al = l.phase ? a1 : a;
@@ -806,8 +876,7 @@ int cached_run(const CacheKey &k, int64_t B, int64_t R, int64_t C, int64_t n, co
     while (g_cache.size() > kCacheMax) {
         bsm_plan *old = g_cache.back();
         g_cache.pop_back();
-        cudaFree(old->blob);
-        delete old;
+        free_plan(old);
     }
     return plan_execute_impl(p, stream);
 }
@@ -890,19 +959,14 @@ int bsm_plan_debug(bsm_plan *plan, int what, int64_t arg)
 
 void bsm_plan_destroy(bsm_plan *plan)
 {
-    if (!plan)
-        return;
-    cudaFree(plan->blob);
-    delete plan;
+    bsm::free_plan(plan);
 }
 
 void bsm_cache_clear(void)
 {
     std::lock_guard<std::mutex> lk(g_cache_mu);
-    for (bsm_plan *p : g_cache) {
-        cudaFree(p->blob);
-        delete p;
-    }
+    for (bsm_plan *p : g_cache)
+        bsm::free_plan(p);
     g_cache.clear();
 }
 

@@ -142,3 +142,33 @@ def test_corrupted_long_patch_is_skipped_with_bounds_status():
     assert np.max(np.abs(yh[ok].astype(np.float64) - y64.reshape(-1, C)[ok])) <= 2e-6
     p.close()
     bsm.bsm_device_status_clear()
+
+
+def test_whole_gpu_graph_and_debug_launches():
+    """WHOLE_GPU plans run their per-slice launches as one captured graph; a
+    plan under a debug setting launches kernel by kernel (the withheld stage
+    times out), and back on the graph afterwards gives correct results."""
+    import torch
+    w = _w()
+    x = to_device(w.x)
+    y = torch.full_like(x, float("nan"))
+    bsm.bsm_device_status_clear()
+    p = bsm.bsm_plan_create(x, y, w.rows, w.cols, w.dtype, bsm.POLICY_WHOLE_GPU)
+    assert p.stats()["launches"] == w.nslices
+    p.execute()
+    torch.cuda.synchronize()
+    assert bsm.bsm_device_status() == 0
+    check_all_against_oracle(w, to_host(y))
+    bsm.bsm_plan_debug(p, bsm.DEBUG_WITHHOLD_STAGE, 100_000_000)
+    p.execute()
+    torch.cuda.synchronize()
+    assert bsm.bsm_device_status() & bsm.DEV_TIMEOUT
+    bsm.bsm_plan_debug(p, bsm.DEBUG_NONE)
+    bsm.bsm_device_status_clear()
+    y.fill_(float("nan"))
+    for _ in range(3):
+        p.execute()
+    torch.cuda.synchronize()
+    assert bsm.bsm_device_status() == 0
+    check_all_against_oracle(w, to_host(y))
+    p.close()
