@@ -107,6 +107,7 @@ struct GemmPlan {
     CUtensorMap ta{}, tb{}, tc{};
     GemmArgs args{};
     std::vector<int32_t> whole_begin;   // WHOLE_GPU: first tile of each slice
+    cudaGraphExec_t whole_graph = nullptr;   // WHOLE_GPU: the per-slice launches as one graph
     void *blob = nullptr;
 };
 
@@ -115,9 +116,56 @@ std::list<GemmPlan *> g_gcache;
 void free_plan(GemmPlan *p)
 {
     if (p) {
+        if (p->whole_graph) {
+            // the graph may still be running: let the plan's device finish first
+            int prev = -1;
+            cudaGetDevice(&prev);
+            cudaSetDevice(p->device);
+            cudaDeviceSynchronize();
+            cudaGraphExecDestroy(p->whole_graph);
+            if (prev >= 0)
+                cudaSetDevice(prev);
+        }
         cudaFree(p->blob);
         delete p;
     }
+}
+
+// WHOLE_GPU: one launch per slice, one after another (Sec. 3), a
+// launch-bound loop; captured once as a CUDA graph when the batch has at
+// most this many slices (null if the capture fails: kernel-by-kernel launches)
+constexpr int64_t kMaxGraphLaunches = 4096;
+
+cudaGraphExec_t capture_whole_gpu(const GemmPlan *p)
+{
+    cudaStream_t st = nullptr;
+    if (cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking) != cudaSuccess) {
+        cudaGetLastError();
+        return nullptr;
+    }
+    cudaGraph_t g = nullptr;
+    cudaGraphExec_t e = nullptr;
+    bool ok = cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal) == cudaSuccess;
+    if (ok) {
+        GemmArgs a = p->args;
+        for (int64_t s = 0; s < p->B; ++s) {
+            a.item_begin = p->whole_begin[s];
+            a.item_end = p->whole_begin[s + 1];
+            if (launch_bmm(&p->ta, &p->tb, &p->tc, a, p->bn, p->out_bf16, p->grid, st)) {
+                ok = false;
+                break;
+            }
+        }
+        const cudaError_t ec = cudaStreamEndCapture(st, &g);
+        ok = ok && ec == cudaSuccess && g != nullptr;
+    }
+    if (ok && cudaGraphInstantiate(&e, g, 0) != cudaSuccess)
+        e = nullptr;
+    if (g)
+        cudaGraphDestroy(g);
+    cudaStreamDestroy(st);
+    cudaGetLastError();
+    return e;
 }
 
 int build_plan(GemmPlan *p, const GemmDev &dev)
@@ -313,7 +361,9 @@ int build_plan(GemmPlan *p, const GemmDev &dev)
 int run_plan(GemmPlan *p, bsm_stream_t stream)
 {
     int err = 0;
-    if (p->policy == BSM_POLICY_WHOLE_GPU) {
+    if (p->policy == BSM_POLICY_WHOLE_GPU && p->whole_graph) {
+        err = static_cast<int>(cudaGraphLaunch(p->whole_graph, static_cast<cudaStream_t>(stream)));
+    } else if (p->policy == BSM_POLICY_WHOLE_GPU) {
         GemmArgs a = p->args;
         for (int64_t s = 0; s < p->B; ++s) {
             a.item_begin = p->whole_begin[s];
@@ -387,6 +437,8 @@ int bmm_impl(const void *a, const void *bt, void *c, int64_t B, int64_t M, int64
         free_plan(p);
         return rc;
     }
+    if (p->policy == BSM_POLICY_WHOLE_GPU && p->B > 0 && p->B <= kMaxGraphLaunches)
+        p->whole_graph = capture_whole_gpu(p);
     g_gcache.push_front(p);
     while (g_gcache.size() > 16) {
         free_plan(g_gcache.back());
