@@ -275,6 +275,9 @@ int bsm_plan_desc_init(bsm_plan_desc *d);
 /* Build a plan: validate, cut slices into patches, and for CBMF / CBMF_LB
  * probe the topology (cached per device) and the die of every chunk of x and
  * y, then run the Sec. 4.1 / 4.2 steps on the host and upload the tables.
+ * A WHOLE_GPU plan of up to 4096 launches also captures them as one CUDA
+ * graph (executed without per-kernel launches; a debug setting or the
+ * self-checking kernels bring back kernel-by-kernel launches).
  * Synchronous; allocates device memory owned by the plan. */
 int bsm_plan_create(bsm_plan **plan, const bsm_plan_desc *d);
 
