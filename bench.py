@@ -408,6 +408,18 @@ def main():
         dist.barrier()
         total_ms = reduce_max_ms(total_ms, device=COLL_DEVICE)
     status = bsm.bsm_device_status()
+    # context on this very box: a plain device-to-device copy of the same
+    # bytes (x into y: one read and one write of every element), timed the
+    # same way; the roofline's peak stays the measured copy bandwidth
+    copy_reps = 50
+
+    def copy_step():
+        with torch.cuda.stream(stream):
+            y.copy_(x)
+    for _ in range(3):
+        copy_step()
+    stream.synchronize()
+    copy_ms, _ = time_steps(copy_step, copy_reps, stream, per_launch=False)
     ms = total_ms / args.steps
     bytes_step = w.algorithmic_bytes
     value = job_gbs(ws, bytes_step, args.steps, total_ms)
@@ -439,6 +451,9 @@ def main():
                      "peak_source": peak_src, "kernel": "softmax_persistent",
                      "launch_ms": round(launch_ms, 5)},
         "clocks": clk.summary(),
+        "copy_context": {"GBps": round(bytes_step / (copy_ms / copy_reps * 1e-3) / 1e9, 2),
+                         "what": "torch copy of x into y on the same stream (device to device), "
+                                 "same bytes, mean of %d back-to-back copies" % copy_reps},
         "plan": {k: st[k] for k in ("n_items", "n_die", "stage_bytes", "n_stages", "grid",
                                      "moved_items", "overlap_items", "tie_items", "L", "N",
                                      "map_chunk_bytes", "plan_ms", "steal")},
