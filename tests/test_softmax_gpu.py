@@ -253,3 +253,40 @@ def test_topology_and_plan_stats():
         assert sum(st["N"][:st["n_die"]]) >= n                         # sum N >= N
         assert sum(st["queue_items"][:st["n_die"]]) == n
         p.close()
+
+
+@pytest.mark.parametrize("dtype", [workload.F32, workload.BF16])
+def test_ragged_batch_with_empty_slices(dtype):
+    """Zero-row slices anywhere in a ragged batch (first, between same-shape
+    slices, before a long row, last) are skipped; the other slices match the
+    oracle and every policy gives the same bits; elements outside the slices
+    (a gap) keep their sentinel."""
+    import torch
+    es = 4 if dtype == workload.F32 else 2
+    long_c = bsm.bsm_max_row_bytes() // es + 16 // es
+    rows = np.array([0, 3, 0, 3, 5, 0, 2, 1, 0], np.int32)
+    cols = np.array([64, 128, 128, 128, 256, long_c, long_c, 512, 64], np.int32)
+    sizes = rows.astype(np.int64) * cols
+    off = np.zeros(len(rows), np.int64)
+    pos = 0
+    for i in range(len(rows)):
+        off[i] = pos
+        pos += int(sizes[i]) + (64 if i == 4 else 0)      # a gap after slice 4
+    w = workload.Workload("empty slices", dtype, rows, cols, off, 0, 0xE3B7, 2.0)
+    w.x = workload.fill_normal(pos, dtype, w.seed, w.sigma)
+    x = to_device(w.x)
+    outs = []
+    for pol in (bsm.POLICY_WHOLE_GPU, bsm.POLICY_RR, bsm.POLICY_DYNAMIC, bsm.POLICY_CBMF,
+                bsm.POLICY_CBMF_LB, bsm.POLICY_MINIMAX):
+        y = torch.full_like(x, -7.0)
+        bsm.bsm_softmax_ragged(x, y, w.offsets, w.rows, w.cols, dtype, pol)
+        outs.append(y)
+    torch.cuda.synchronize()
+    for y in outs[1:]:
+        assert torch.equal(bits(y), bits(outs[0]))
+    yh = to_host(outs[0])
+    gap = slice(int(off[4] + sizes[4]), int(off[4] + sizes[4]) + 64)
+    sentinel = to_host(torch.full((1,), -7.0, dtype=x.dtype, device="cuda"))[0]
+    assert np.all(yh[gap] == sentinel)
+    check_all_against_oracle(w, yh)
+    assert bsm.bsm_device_status() == 0
