@@ -605,9 +605,9 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
             st.moved_items = so.n_moved;
             st.n_die = nb;
             std::memcpy(sm_die_tab, topo.sm_die, sizeof sm_die_tab);
-            for (int s = 0; s < BSM_MAX_SM; ++s)
-                if (sm_die_tab[s] < 0)
-                    sm_die_tab[s] = 0;
+            for (int sm = 0; sm < BSM_MAX_SM; ++sm)
+                if (sm_die_tab[sm] < 0)
+                    sm_die_tab[sm] = 0;
             use_sm_die = true;
             p->args.steal = (lb || minimax) ? 1 : 0;
         }
@@ -718,13 +718,13 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     switch (d->policy) {
     case BSM_POLICY_WHOLE_GPU:
         a.mode = PULL_STATIC;
-        for (size_t s = 0; s < slices.size(); ++s) {
-            const int32_t n = slice_first[s + 1] - slice_first[s];
+        for (size_t k = 0; k < slices.size(); ++k) {
+            const int32_t n = slice_first[k + 1] - slice_first[k];
             if (n > 0)
-                p->whole_gpu.push_back({slice_first[s], slice_first[s + 1], std::min(n, c->n_sm), 0});
-            const int32_t n1s = slice_first1[s + 1] - slice_first1[s];
+                p->whole_gpu.push_back({slice_first[k], slice_first[k + 1], std::min(n, c->n_sm), 0});
+            const int32_t n1s = slice_first1[k + 1] - slice_first1[k];
             if (n1s > 0)
-                p->whole_gpu.push_back({slice_first1[s], slice_first1[s + 1], std::min(n1s, c->n_sm), 1});
+                p->whole_gpu.push_back({slice_first1[k], slice_first1[k + 1], std::min(n1s, c->n_sm), 1});
         }
         p->grid = c->n_sm;
         st.launches = static_cast<int32_t>(p->whole_gpu.size());

@@ -156,7 +156,7 @@ void analyse_topology(const std::vector<float> &lat, const std::vector<int32_t> 
         group[k] = c >= 0 ? 0 : 1;
         sep += std::fabs(c);
     }
-    sep = sms.size() > 1 ? sep / (sms.size() - 1) : 0.0;
+    sep = sms.size() > 1 ? sep / double(sms.size() - 1) : 0.0;
     int cnt[2] = {0, 0};
     for (int g : group)
         ++cnt[g];
