@@ -313,6 +313,45 @@ typedef struct {
 int bsm_plan_get_stats(const bsm_plan *plan, bsm_plan_stats *out);
 void bsm_plan_destroy(bsm_plan *plan);
 
+/* ---- the patch table alone, on the host (no GPU needed) ----
+ * Cuts the descriptor's slices into patches exactly as bsm_plan_create does,
+ * for a device with n_sm SMs and smem_optin bytes of opt-in shared memory per
+ * block (Sec. 4: a patch is a block of consecutive rows of one slice -- under
+ * the queue policies, of back-to-back slices of one shape -- that fills at
+ * most one stage; a row longer than a stage is one patch, or, when such rows
+ * are too few to fill the SMs twice, several segments of whole chunks that
+ * run in two launches).  d->x, d->y and d->x2 only take part in the
+ * alignment and overlap checks and are never dereferenced.  Phase-0 patches
+ * come in slice order (before any queue ordering), phase-1 segments in the
+ * order the second launch takes them.  At most cap0 / cap1 records are
+ * written to phase0 / phase1 (host memory owned by the caller; NULL with a
+ * capacity of 0); *out always receives the counts, so a first call with both
+ * capacities 0 sizes the arrays.  Returns BSM_ERR_INVALID_ARG for a null d or
+ * out, n_sm outside 1..BSM_MAX_SM, smem_optin outside (1024, 1 MiB] or a
+ * capacity without an array, and the errors of bsm_plan_create's validation
+ * (BSM_ERR_MISALIGNED, BSM_ERR_UNSUPPORTED when fewer than two stages fit). */
+typedef struct {
+    int64_t elem_offset;        /* first element of the patch in x and y */
+    int32_t cols;               /* elements of each of its rows (a segment: its length) */
+    int32_t nrows;              /* rows in the patch (1 for a long row) */
+    int32_t row0;               /* index of its first row within its slice */
+    int32_t slice_rows;         /* R of that slice */
+    int32_t col0;               /* long rows: the segment's first column; else 0 */
+    int32_t part_count;         /* long rows: segments of the row (1 = the whole row); else 0 */
+} bsm_patch;
+
+typedef struct {
+    int64_t stage_bytes;        /* bytes per shared-memory stage */
+    int32_t n_stages;           /* stages per CTA */
+    int32_t pad;
+    int64_t n_patches;          /* phase 0 (the first or only launch) */
+    int64_t n_patches_phase1;   /* segments of rows cut into several (the second launch) */
+    int64_t long_rows;          /* rows longer than a stage */
+} bsm_layout;
+
+int bsm_plan_layout_host(const bsm_plan_desc *d, int32_t n_sm, int64_t smem_optin, bsm_patch *phase0,
+                         int64_t cap0, bsm_patch *phase1, int64_t cap1, bsm_layout *out);
+
 /* Fault injection on one plan, for the library's failure-detection tests
  * (nothing here faults, traps or hangs the GPU):
  *   BSM_DEBUG_WITHHOLD_STAGE  later executes never fill the first shared-memory

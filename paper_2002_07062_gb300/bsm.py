@@ -56,6 +56,18 @@ class PlanDesc(ctypes.Structure):
                 ("device", ctypes.c_int32), ("op", ctypes.c_int32), ("x2", ctypes.c_void_p)]
 
 
+class Patch(ctypes.Structure):
+    _fields_ = [("elem_offset", ctypes.c_int64), ("cols", ctypes.c_int32), ("nrows", ctypes.c_int32),
+                ("row0", ctypes.c_int32), ("slice_rows", ctypes.c_int32), ("col0", ctypes.c_int32),
+                ("part_count", ctypes.c_int32)]
+
+
+class Layout(ctypes.Structure):
+    _fields_ = [("stage_bytes", ctypes.c_int64), ("n_stages", ctypes.c_int32), ("pad", ctypes.c_int32),
+                ("n_patches", ctypes.c_int64), ("n_patches_phase1", ctypes.c_int64),
+                ("long_rows", ctypes.c_int64)]
+
+
 class PlanStats(ctypes.Structure):
     _fields_ = [("policy", ctypes.c_int32), ("n_die", ctypes.c_int32), ("n_items", ctypes.c_int64),
                 ("N", ctypes.c_int64 * MAX_DIES), ("L", ctypes.c_int64 * MAX_DIES),
@@ -127,6 +139,8 @@ def lib():
         "bsm_plan_get_stats": ([vp, ctypes.POINTER(PlanStats)], ctypes.c_int),
         "bsm_plan_destroy": ([vp], None),
         "bsm_plan_debug": ([vp, ctypes.c_int, i64], ctypes.c_int),
+        "bsm_plan_layout_host": ([ctypes.POINTER(PlanDesc), i32, i64, ctypes.POINTER(Patch), i64,
+                                  ctypes.POINTER(Patch), i64, ctypes.POINTER(Layout)], ctypes.c_int),
         "bsm_cache_clear": ([], None),
         "bsm_topology_probe": ([ctypes.c_int, ctypes.c_int, ctypes.POINTER(Topology)], ctypes.c_int),
         "bsm_addr_die_map": ([ctypes.c_int, vp, i64, i64, ctypes.POINTER(ctypes.c_int8)], ctypes.c_int),
@@ -378,6 +392,41 @@ def bsm_probe_latency(line_off, reps: int = 8, device: int = -1):
                                    lat.ctypes.data_as(ctypes.POINTER(ctypes.c_float)),
                                    seen.ctypes.data_as(c_i32p)), "bsm_probe_latency")
     return lat, seen
+
+
+def bsm_plan_layout_host(rows, cols, dtype: int, policy: int, n_sm: int, smem_optin: int,
+                         offsets=None, rows_per_item: int = 0, op: int = 0, x: int = 1 << 40,
+                         y: int = 1 << 41, x2: int = 1 << 42) -> dict:
+    """The patch table bsm_plan_create would build on a device with n_sm SMs
+    and smem_optin bytes of opt-in shared memory (host only).  x, y, x2 are
+    addresses for the alignment and overlap checks, never dereferenced.
+    Returns the stage figures and two structured arrays of patches (fields of
+    bsm_patch): phase 0 in slice order, phase 1 in launch order."""
+    d = PlanDesc()
+    _check(lib().bsm_plan_desc_init(ctypes.byref(d)), "bsm_plan_desc_init")
+    r = _np(rows, np.int32)
+    c = _np(cols, np.int32)
+    off = None if offsets is None else _np(offsets, np.int64)
+    d.x, d.y, d.x2 = x, y, x2
+    d.num_slices = len(r)
+    d.rows = r.ctypes.data_as(c_i32p)
+    d.cols = c.ctypes.data_as(c_i32p)
+    if off is not None:
+        d.offsets = off.ctypes.data_as(c_i64p)
+    d.dtype, d.policy, d.rows_per_item, d.op = dtype, policy, rows_per_item, op
+    out = Layout()
+    _check(lib().bsm_plan_layout_host(ctypes.byref(d), n_sm, smem_optin, None, 0, None, 0,
+                                      ctypes.byref(out)), "bsm_plan_layout_host")
+    n0, n1 = out.n_patches, out.n_patches_phase1
+    p0 = (Patch * max(n0, 1))()
+    p1 = (Patch * max(n1, 1))()
+    _check(lib().bsm_plan_layout_host(ctypes.byref(d), n_sm, smem_optin, p0, n0, p1, n1,
+                                      ctypes.byref(out)), "bsm_plan_layout_host")
+    dt = np.dtype([(name, np.int64 if ct is ctypes.c_int64 else np.int32) for name, ct in Patch._fields_])
+    a0 = np.frombuffer(bytes(p0), dtype=dt, count=n0) if n0 else np.zeros(0, dt)
+    a1 = np.frombuffer(bytes(p1), dtype=dt, count=n1) if n1 else np.zeros(0, dt)
+    return {"stage_bytes": out.stage_bytes, "n_stages": out.n_stages, "long_rows": out.long_rows,
+            "phase0": a0, "phase1": a1}
 
 
 def bsm_schedule_host(patches: Sequence, maps: Sequence, n_banks: int, tie_seed: int,

@@ -114,10 +114,12 @@ int device_status_word(int device, uint32_t **out)
 
 namespace {
 
-int64_t max_row_bytes_for(const DeviceCtx &c)
+int64_t max_row_bytes_for(int64_t smem_optin)
 {
-    return ((static_cast<int64_t>(c.smem_optin) - kSmemHeader) / 2) & ~int64_t(127);
+    return ((smem_optin - kSmemHeader) / 2) & ~int64_t(127);
 }
+
+int64_t max_row_bytes_for(const DeviceCtx &c) { return max_row_bytes_for(static_cast<int64_t>(c.smem_optin)); }
 
 int esize(int dtype) { return dtype == BSM_F32 ? 4 : 2; }
 
@@ -243,6 +245,164 @@ int validate(const bsm_plan_desc *d, std::vector<SliceView> &slices,
     return BSM_OK;
 }
 
+// The patch table of a plan: a host computation from the descriptor and two
+// figures of the device (its SM count and the opt-in shared memory of a
+// block), with no CUDA call.
+struct PatchLayout {
+    int64_t stage = 0;                  // bytes per shared-memory stage
+    int n_stages = 0;
+    std::vector<Item> items;            // phase 0, in slice order
+    std::vector<LongSeg> segs;          // parallel to items when there are long rows
+    std::vector<Item> items1;           // phase 1: the segments of rows cut into several
+    std::vector<LongSeg> segs1;
+    std::vector<int32_t> slice_first, slice_first1;
+    int64_t n_parts = 0;                // segments of rows cut into several
+    int64_t long_rows = 0;              // rows longer than a stage
+};
+
+int cut_patches(const bsm_plan_desc *d, const std::vector<SliceView> &slices, int64_t max_row, int n_sm,
+                int64_t smem_optin, PatchLayout &L)
+{
+    const int es = esize(d->dtype);
+    // ---- stages: one CTA per SM, as many stages as fit the shared memory
+    const int64_t avail = smem_optin - kSmemHeader;
+    const int in_arrays = d->op == BSM_OP_BACKWARD ? 2 : 1;   // inputs sharing a stage
+    // a stage holds the longest row (for the backward pass: the row of y and
+    // the row of dy), up to half the shared memory; longer rows go through
+    // the stages in chunks, twice
+    const int64_t row_cap = std::min<int64_t>((max_row + 127) & ~int64_t(127),
+                                              (max_row_bytes_for(smem_optin) / in_arrays) & ~int64_t(127));
+    const int64_t min_stage = kMinStageBytes;
+    int64_t stage = std::max<int64_t>(min_stage, in_arrays * row_cap);
+    // Rows longer than that cap but whose halves fit three stages (with the
+    // shorter rows of the batch): stages of half such a row, so that each of
+    // them (two chunks) stays staged for its second pass while the third
+    // stage takes the next row's first chunk -- one copy per row
+    if (max_row > max_row_bytes_for(smem_optin) / in_arrays) {
+        int64_t max_short = 0;
+        for (const SliceView &v : slices)
+            if (v.R > 0 && int64_t(v.C) * es <= max_row_bytes_for(smem_optin) / in_arrays)
+                max_short = std::max<int64_t>(max_short, int64_t(v.C) * es);
+        const int64_t half = std::max<int64_t>((max_short + 127) & ~int64_t(127),
+                                               ((max_row + 1) / 2 + 127) & ~int64_t(127));
+        const int64_t two_chunk = std::max<int64_t>(min_stage, in_arrays * half);
+        if (3 * two_chunk <= avail)
+            stage = two_chunk;
+    }
+    const int n_stages = static_cast<int>(std::min<int64_t>(kMaxStages, avail / stage));
+    if (n_stages < 2)
+        return BSM_ERR_UNSUPPORTED;
+    L.stage = stage;
+    L.n_stages = n_stages;
+
+    // ---- patches: consecutive rows filling (at most) one stage.  Under the
+    // queue policies a patch may run on into the next slices when they have
+    // the same shape and follow back to back (a "segment"); under RR and
+    // WHOLE_GPU a patch stays inside its slice, the unit those policies place.
+    const bool spanning = d->policy == BSM_POLICY_DYNAMIC || d->policy == BSM_POLICY_CBMF ||
+                          d->policy == BSM_POLICY_CBMF_LB || d->policy == BSM_POLICY_MINIMAX;
+    std::vector<Item> &items = L.items;
+    std::vector<int32_t> &slice_first = L.slice_first;
+    slice_first.assign(slices.size() + 1, 0);
+    // rows longer than a stage: when they are too few to fill two waves of
+    // the SMs, cut into segments of whole chunks, about eight per SM over the
+    // batch, so that a few long rows still spread over the device (two
+    // launches, see LongSeg; eight rather than four evens out the last wave
+    // of each launch: +1 to +6.5 % measured, sixteen is no better); otherwise
+    // each row is one segment that one CTA streams twice within the launch
+    // (its second read mostly hits L2)
+    int64_t n_long_rows = 0;
+    for (const SliceView &v : slices)
+        if (v.R > 0 && int64_t(v.C) * es > stage / in_arrays)
+            n_long_rows += v.R;
+    const int64_t chunk_elems = stage / in_arrays / es;
+    const int64_t want_segs = n_long_rows > 0 && n_long_rows < 2 * n_sm
+                                  ? std::max<int64_t>(1, (8 * n_sm + n_long_rows - 1) / n_long_rows)
+                                  : 1;
+    std::vector<LongSeg> &segs = L.segs;
+    std::vector<Item> &items1 = L.items1;
+    std::vector<LongSeg> &segs1 = L.segs1;
+    std::vector<int32_t> &slice_first1 = L.slice_first1;
+    slice_first1.assign(slices.size() + 1, 0);
+    int64_t &n_parts = L.n_parts;
+    int64_t &long_rows = L.long_rows;
+    size_t s = 0;
+    while (s < slices.size()) {
+        slice_first[s] = static_cast<int32_t>(items.size());
+        slice_first1[s] = static_cast<int32_t>(items1.size());
+        const SliceView &v = slices[s];
+        size_t e = s + 1;
+        if (spanning && v.R > 0) {
+            while (e < slices.size() && slices[e].R == v.R && slices[e].C == v.C &&
+                   slices[e].off == slices[e - 1].off + int64_t(v.R) * v.C) {
+                slice_first[e] = static_cast<int32_t>(items.size());
+                slice_first1[e] = static_cast<int32_t>(items1.size());
+                ++e;
+            }
+        }
+        if (v.R > 0 && int64_t(v.C) * es > stage / in_arrays) {
+            const int64_t seg_rows = int64_t(v.R) * static_cast<int64_t>(e - s);
+            long_rows += seg_rows;
+            const int64_t nch = (v.C + chunk_elems - 1) / chunk_elems;
+            const int64_t per_row = std::min<int64_t>(nch, want_segs);
+            const int64_t seg_elems = (nch + per_row - 1) / per_row * chunk_elems;
+            const int64_t n_seg = (v.C + seg_elems - 1) / seg_elems;
+            if (segs.size() < items.size())
+                segs.resize(items.size(), LongSeg{0, 0, 0, 0});
+            for (int64_t g = 0; g < seg_rows; ++g) {
+                if (items.size() + n_seg >= static_cast<size_t>(INT32_MAX) || n_parts + n_seg >= INT32_MAX)
+                    return BSM_ERR_UNSUPPORTED;
+                for (int64_t k = 0; k < n_seg; ++k) {
+                    const int64_t c0 = k * seg_elems;
+                    const Item it{v.off + g * v.C + c0, static_cast<int32_t>(std::min<int64_t>(seg_elems, v.C - c0)),
+                                  1, static_cast<int32_t>(g % v.R), v.R};
+                    if (n_seg == 1) {       // the whole row, both passes in one launch
+                        items.push_back(it);
+                        segs.push_back(LongSeg{0, 0, 0, 1});
+                        continue;
+                    }
+                    const LongSeg sg{static_cast<int32_t>(c0), static_cast<int32_t>(n_parts + k),
+                                     static_cast<int32_t>(n_parts), static_cast<int32_t>(n_seg)};
+                    items.push_back(it);
+                    segs.push_back(sg);
+                    items1.push_back(it);
+                    segs1.push_back(sg);
+                }
+                if (n_seg > 1)
+                    n_parts += n_seg;
+            }
+        } else if (v.R > 0) {
+            const int64_t seg_rows = int64_t(v.R) * static_cast<int64_t>(e - s);
+            const int64_t row_bytes = int64_t(v.C) * es;
+            int64_t rpi = std::max<int64_t>(1, stage / in_arrays / row_bytes);
+            if (d->rows_per_item > 0)
+                rpi = std::min<int64_t>(rpi, d->rows_per_item);
+            if (d->policy == BSM_POLICY_WHOLE_GPU)
+                rpi = std::min<int64_t>(rpi, (v.R + n_sm - 1) / n_sm);
+            rpi = std::max<int64_t>(1, std::min<int64_t>(rpi, seg_rows));
+            for (int64_t g0 = 0; g0 < seg_rows; g0 += rpi) {
+                if (items.size() >= static_cast<size_t>(INT32_MAX))
+                    return BSM_ERR_UNSUPPORTED;
+                const int64_t nr = std::min<int64_t>(rpi, seg_rows - g0);
+                items.push_back({v.off + g0 * v.C, v.C, static_cast<int32_t>(nr),
+                                 static_cast<int32_t>(g0 % v.R), v.R});
+            }
+        }
+        s = e;
+    }
+    slice_first[slices.size()] = static_cast<int32_t>(items.size());
+    slice_first1[slices.size()] = static_cast<int32_t>(items1.size());
+    if (!segs.empty())
+        segs.resize(items.size(), LongSeg{0, 0, 0, 0});
+    if (spanning && !items1.empty()) {
+        // phase 1 takes the segments in reverse: it starts with those phase 0
+        // read last, which are most likely still in L2
+        std::reverse(items1.begin(), items1.end());
+        std::reverse(segs1.begin(), segs1.end());
+    }
+    return BSM_OK;
+}
+
 // WHOLE_GPU runs one kernel per slice, one after another (Sec. 3): a
 // launch-bound loop.  Plans of up to this many launches capture it once, at
 // creation, as a CUDA graph, so an execute is one graph launch (the kernels
@@ -319,139 +479,19 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     if ((rc = validate(d, slices, total, max_row)))
         return rc;
     const int es = esize(d->dtype);
-
-    // ---- stages: one CTA per SM, as many stages as fit the shared memory
-    const int64_t avail = c->smem_optin - kSmemHeader;
-    const int in_arrays = d->op == BSM_OP_BACKWARD ? 2 : 1;   // inputs sharing a stage
-    // a stage holds the longest row (for the backward pass: the row of y and
-    // the row of dy), up to half the shared memory; longer rows go through
-    // the stages in chunks, twice
-    const int64_t row_cap =
-        std::min<int64_t>((max_row + 127) & ~int64_t(127), (max_row_bytes_for(*c) / in_arrays) & ~int64_t(127));
-    const int64_t min_stage = kMinStageBytes;
-    int64_t stage = std::max<int64_t>(min_stage, in_arrays * row_cap);
-    // Rows longer than that cap but whose halves fit three stages (with the
-    // shorter rows of the batch): stages of half such a row, so that each of
-    // them (two chunks) stays staged for its second pass while the third
-    // stage takes the next row's first chunk -- one copy per row
-    if (max_row > max_row_bytes_for(*c) / in_arrays) {
-        int64_t max_short = 0;
-        for (const SliceView &v : slices)
-            if (v.R > 0 && int64_t(v.C) * es <= max_row_bytes_for(*c) / in_arrays)
-                max_short = std::max<int64_t>(max_short, int64_t(v.C) * es);
-        const int64_t half = std::max<int64_t>((max_short + 127) & ~int64_t(127),
-                                               ((max_row + 1) / 2 + 127) & ~int64_t(127));
-        const int64_t two_chunk = std::max<int64_t>(min_stage, in_arrays * half);
-        if (3 * two_chunk <= avail)
-            stage = two_chunk;
-    }
-    const int n_stages = static_cast<int>(std::min<int64_t>(kMaxStages, avail / stage));
-    if (n_stages < 2)
-        return BSM_ERR_UNSUPPORTED;
-
-    // ---- patches: consecutive rows filling (at most) one stage.  Under the
-    // queue policies a patch may run on into the next slices when they have
-    // the same shape and follow back to back (a "segment"); under RR and
-    // WHOLE_GPU a patch stays inside its slice, the unit those policies place.
-    const bool spanning = d->policy == BSM_POLICY_DYNAMIC || d->policy == BSM_POLICY_CBMF ||
-                          d->policy == BSM_POLICY_CBMF_LB || d->policy == BSM_POLICY_MINIMAX;
-    std::vector<Item> items;
-    std::vector<int32_t> slice_first(slices.size() + 1, 0);
-    // rows longer than a stage: when they are too few to fill two waves of
-    // the SMs, cut into segments of whole chunks, about eight per SM over the
-    // batch, so that a few long rows still spread over the device (two
-    // launches, see LongSeg; eight rather than four evens out the last wave
-    // of each launch: +1 to +6.5 % measured, sixteen is no better); otherwise
-    // each row is one segment that one CTA streams twice within the launch
-    // (its second read mostly hits L2)
-    int64_t n_long_rows = 0;
-    for (const SliceView &v : slices)
-        if (v.R > 0 && int64_t(v.C) * es > stage / in_arrays)
-            n_long_rows += v.R;
-    const int64_t chunk_elems = stage / in_arrays / es;
-    const int64_t want_segs = n_long_rows > 0 && n_long_rows < 2 * c->n_sm
-                                  ? std::max<int64_t>(1, (8 * c->n_sm + n_long_rows - 1) / n_long_rows)
-                                  : 1;
-    std::vector<LongSeg> segs;              // parallel to items when there are long rows
-    std::vector<Item> items1;               // phase 1: the long-row segments
-    std::vector<LongSeg> segs1;
-    std::vector<int32_t> slice_first1(slices.size() + 1, 0);
-    int64_t n_parts = 0;
-    int64_t long_rows = 0;
-    size_t s = 0;
-    while (s < slices.size()) {
-        slice_first[s] = static_cast<int32_t>(items.size());
-        slice_first1[s] = static_cast<int32_t>(items1.size());
-        const SliceView &v = slices[s];
-        size_t e = s + 1;
-        if (spanning && v.R > 0) {
-            while (e < slices.size() && slices[e].R == v.R && slices[e].C == v.C &&
-                   slices[e].off == slices[e - 1].off + int64_t(v.R) * v.C) {
-                slice_first[e] = static_cast<int32_t>(items.size());
-                slice_first1[e] = static_cast<int32_t>(items1.size());
-                ++e;
-            }
-        }
-        if (v.R > 0 && int64_t(v.C) * es > stage / in_arrays) {
-            const int64_t seg_rows = int64_t(v.R) * static_cast<int64_t>(e - s);
-            long_rows += seg_rows;
-            const int64_t nch = (v.C + chunk_elems - 1) / chunk_elems;
-            const int64_t per_row = std::min<int64_t>(nch, want_segs);
-            const int64_t seg_elems = (nch + per_row - 1) / per_row * chunk_elems;
-            const int64_t n_seg = (v.C + seg_elems - 1) / seg_elems;
-            if (segs.size() < items.size())
-                segs.resize(items.size(), LongSeg{0, 0, 0, 0});
-            for (int64_t g = 0; g < seg_rows; ++g) {
-                if (items.size() + n_seg >= static_cast<size_t>(INT32_MAX) || n_parts + n_seg >= INT32_MAX)
-                    return BSM_ERR_UNSUPPORTED;
-                for (int64_t k = 0; k < n_seg; ++k) {
-                    const int64_t c0 = k * seg_elems;
-                    const Item it{v.off + g * v.C + c0, static_cast<int32_t>(std::min<int64_t>(seg_elems, v.C - c0)),
-                                  1, static_cast<int32_t>(g % v.R), v.R};
-                    if (n_seg == 1) {       // the whole row, both passes in one launch
-                        items.push_back(it);
-                        segs.push_back(LongSeg{0, 0, 0, 1});
-                        continue;
-                    }
-                    const LongSeg sg{static_cast<int32_t>(c0), static_cast<int32_t>(n_parts + k),
-                                     static_cast<int32_t>(n_parts), static_cast<int32_t>(n_seg)};
-                    items.push_back(it);
-                    segs.push_back(sg);
-                    items1.push_back(it);
-                    segs1.push_back(sg);
-                }
-                if (n_seg > 1)
-                    n_parts += n_seg;
-            }
-        } else if (v.R > 0) {
-            const int64_t seg_rows = int64_t(v.R) * static_cast<int64_t>(e - s);
-            const int64_t row_bytes = int64_t(v.C) * es;
-            int64_t rpi = std::max<int64_t>(1, stage / in_arrays / row_bytes);
-            if (d->rows_per_item > 0)
-                rpi = std::min<int64_t>(rpi, d->rows_per_item);
-            if (d->policy == BSM_POLICY_WHOLE_GPU)
-                rpi = std::min<int64_t>(rpi, (v.R + c->n_sm - 1) / c->n_sm);
-            rpi = std::max<int64_t>(1, std::min<int64_t>(rpi, seg_rows));
-            for (int64_t g0 = 0; g0 < seg_rows; g0 += rpi) {
-                if (items.size() >= static_cast<size_t>(INT32_MAX))
-                    return BSM_ERR_UNSUPPORTED;
-                const int64_t nr = std::min<int64_t>(rpi, seg_rows - g0);
-                items.push_back({v.off + g0 * v.C, v.C, static_cast<int32_t>(nr),
-                                 static_cast<int32_t>(g0 % v.R), v.R});
-            }
-        }
-        s = e;
-    }
-    slice_first[slices.size()] = static_cast<int32_t>(items.size());
-    slice_first1[slices.size()] = static_cast<int32_t>(items1.size());
-    if (!segs.empty())
-        segs.resize(items.size(), LongSeg{0, 0, 0, 0});
-    if (spanning && !items1.empty()) {
-        // phase 1 takes the segments in reverse: it starts with those phase 0
-        // read last, which are most likely still in L2
-        std::reverse(items1.begin(), items1.end());
-        std::reverse(segs1.begin(), segs1.end());
-    }
+    PatchLayout lay;
+    if ((rc = cut_patches(d, slices, max_row, c->n_sm, c->smem_optin, lay)))
+        return rc;
+    const int64_t stage = lay.stage;
+    const int n_stages = lay.n_stages;
+    std::vector<Item> &items = lay.items;
+    std::vector<LongSeg> &segs = lay.segs;
+    const std::vector<Item> &items1 = lay.items1;
+    const std::vector<LongSeg> &segs1 = lay.segs1;
+    const std::vector<int32_t> &slice_first = lay.slice_first;
+    const std::vector<int32_t> &slice_first1 = lay.slice_first1;
+    const int64_t n_parts = lay.n_parts;
+    const int64_t long_rows = lay.long_rows;
     const int64_t n_items = static_cast<int64_t>(items.size());
 
     bsm_plan *p = new bsm_plan();
@@ -756,6 +796,43 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     return BSM_OK;
 }
 
+int plan_layout_host_impl(const bsm_plan_desc *d, int32_t n_sm, int64_t smem_optin, bsm_patch *phase0,
+                          int64_t cap0, bsm_patch *phase1, int64_t cap1, bsm_layout *out)
+{
+    if (!d || !out || n_sm < 1 || n_sm > BSM_MAX_SM || smem_optin <= kSmemHeader ||
+        smem_optin > (int64_t(1) << 20) || cap0 < 0 || cap1 < 0 || (cap0 > 0 && !phase0) ||
+        (cap1 > 0 && !phase1))
+        return BSM_ERR_INVALID_ARG;
+    std::memset(out, 0, sizeof *out);
+    std::vector<SliceView> slices;
+    int64_t total = 0, max_row = 0;
+    int rc = validate(d, slices, total, max_row);
+    if (rc)
+        return rc;
+    PatchLayout lay;
+    if ((rc = cut_patches(d, slices, max_row, n_sm, smem_optin, lay)))
+        return rc;
+    out->stage_bytes = lay.stage;
+    out->n_stages = lay.n_stages;
+    out->n_patches = static_cast<int64_t>(lay.items.size());
+    out->n_patches_phase1 = static_cast<int64_t>(lay.items1.size());
+    out->long_rows = lay.long_rows;
+    auto put = [](const Item &it, const LongSeg *sg, bsm_patch &o) {
+        o.elem_offset = it.off;
+        o.cols = it.C;
+        o.nrows = it.nrows;
+        o.row0 = it.row0;
+        o.slice_rows = it.R;
+        o.col0 = sg ? sg->col0 : 0;
+        o.part_count = sg ? sg->part_count : 0;
+    };
+    for (size_t i = 0; i < lay.items.size() && static_cast<int64_t>(i) < cap0; ++i)
+        put(lay.items[i], lay.segs.empty() ? nullptr : &lay.segs[i], phase0[i]);
+    for (size_t i = 0; i < lay.items1.size() && static_cast<int64_t>(i) < cap1; ++i)
+        put(lay.items1[i], &lay.segs1[i], phase1[i]);
+    return BSM_OK;
+}
+
 int plan_execute_impl(const bsm_plan *p, bsm_stream_t stream)
 {
     if (!p)
@@ -960,6 +1037,12 @@ int bsm_plan_debug(bsm_plan *plan, int what, int64_t arg)
 void bsm_plan_destroy(bsm_plan *plan)
 {
     bsm::free_plan(plan);
+}
+
+int bsm_plan_layout_host(const bsm_plan_desc *d, int32_t n_sm, int64_t smem_optin, bsm_patch *phase0,
+                         int64_t cap0, bsm_patch *phase1, int64_t cap1, bsm_layout *out)
+{
+    BSM_GUARD(plan_layout_host_impl(d, n_sm, smem_optin, phase0, cap0, phase1, cap1, out))
 }
 
 void bsm_cache_clear(void)
