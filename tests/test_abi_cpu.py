@@ -105,7 +105,9 @@ def test_bmm_empty_batch_is_a_no_op():
 
 def test_header_is_plain_c_and_links_from_c(tmp_path):
     """include/bsm.h compiles as C11 under -pedantic, and a C program links
-    against libbsm.so and gets argument errors back without a GPU."""
+    against libbsm.so, gets argument errors back without a GPU, and reads the
+    host-only patch table of workload 2 (6144 patches of 32 rows, three
+    64 KiB stages) through the C structs."""
     import os
     import shutil
     gcc = shutil.which("gcc")
@@ -119,8 +121,22 @@ def test_header_is_plain_c_and_links_from_c(tmp_path):
         "int main(void) {\n"
         "  int rc = bsm_softmax(NULL, NULL, -1, 4, 4, BSM_F32, BSM_POLICY_DYNAMIC, NULL);\n"
         "  int rb = bsm_bmm(NULL, NULL, NULL, 1, 64, 64, 64, BSM_F32, BSM_POLICY_DYNAMIC, NULL);\n"
-        "  printf(\"%d %d %d\\n\", bsm_version(), rc, rb);\n"
-        "  return rc == BSM_ERR_INVALID_ARG && rb == BSM_ERR_UNSUPPORTED ? 0 : 1;\n}\n")
+        "  static int32_t R[384], C[384];\n"
+        "  for (int s = 0; s < 384; ++s) { R[s] = 512; C[s] = 512; }\n"
+        "  bsm_plan_desc d;\n"
+        "  bsm_plan_desc_init(&d);\n"
+        "  d.x = (const void *)(uintptr_t)(1ull << 40); d.y = (void *)(uintptr_t)(1ull << 41);\n"
+        "  d.num_slices = 384; d.rows = R; d.cols = C; d.dtype = BSM_F32;\n"
+        "  d.policy = BSM_POLICY_DYNAMIC;\n"
+        "  bsm_layout lay;\n"
+        "  int rl = bsm_plan_layout_host(&d, 152, 232448, NULL, 0, NULL, 0, &lay);\n"
+        "  static bsm_patch p[6144];\n"
+        "  int rl2 = bsm_plan_layout_host(&d, 152, 232448, p, 6144, NULL, 0, &lay);\n"
+        "  int ok = rl == BSM_OK && rl2 == BSM_OK && lay.n_patches == 6144 && lay.n_stages == 3 &&\n"
+        "           lay.stage_bytes == 65536 && lay.n_patches_phase1 == 0 && p[1].elem_offset == 32 * 512 &&\n"
+        "           p[1].nrows == 32 && p[1].row0 == 32 && p[6143].row0 == 480 && p[6143].slice_rows == 512;\n"
+        "  printf(\"%d %d %d %d\\n\", bsm_version(), rc, rb, ok);\n"
+        "  return rc == BSM_ERR_INVALID_ARG && rb == BSM_ERR_UNSUPPORTED && ok ? 0 : 1;\n}\n")
     exe = tmp_path / "capi"
     subprocess.run([gcc, "-std=c11", "-Wall", "-Wextra", "-pedantic", "-Werror", "-I", inc, str(src),
                     "-L", lib_dir, "-lbsm", "-Wl,-rpath," + lib_dir, "-o", str(exe)], check=True)
