@@ -202,3 +202,22 @@ def test_random_batches(trial):
     except bsm.BsmError as e:
         # only a device too small for two stages may refuse a valid batch
         assert e.status == bsm.ERR_UNSUPPORTED and smem - HEADER < 2 * MIN_STAGE * (2 if op else 1), e
+
+
+def test_edge_cases():
+    # only empty slices: no patches, the default stages
+    L = bsm.bsm_plan_layout_host([0, 0], [64, 64], bsm.F32, bsm.POLICY_RR, 152, SMEM)
+    assert len(L["phase0"]) == 0 and L["n_stages"] == 3
+    # in place (x == y) is allowed, a partial overlap is not
+    check_layout([4], [64], bsm.F32, bsm.POLICY_DYNAMIC)
+    assert len(bsm.bsm_plan_layout_host([4], [64], bsm.F32, bsm.POLICY_DYNAMIC, 152, SMEM,
+                                        x=1 << 40, y=1 << 40)["phase0"]) == 1
+    with pytest.raises(bsm.BsmError) as e:
+        bsm.bsm_plan_layout_host([4], [64], bsm.F32, bsm.POLICY_DYNAMIC, 152, SMEM,
+                                 x=1 << 40, y=(1 << 40) + 64)
+    assert e.value.status == bsm.ERR_INVALID_ARG
+    # three 8 MiB bf16 rows, backward: segments of one chunk (28928 elements,
+    # half of the 113 KiB stage per array), 145 per row
+    L = check_layout([3], [1 << 22], bsm.BF16, bsm.POLICY_DYNAMIC, op=bsm.OP_BACKWARD)
+    assert len(L["phase0"]) == len(L["phase1"]) == 3 * 145
+    assert set(L["phase1"]["part_count"]) == {145}
