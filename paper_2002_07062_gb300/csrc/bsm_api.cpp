@@ -311,10 +311,21 @@ int cut_patches(const bsm_plan_desc *d, const std::vector<SliceView> &slices, in
     // of each launch: +1 to +6.5 % measured, sixteen is no better); otherwise
     // each row is one segment that one CTA streams twice within the launch
     // (its second read mostly hits L2)
-    int64_t n_long_rows = 0;
-    for (const SliceView &v : slices)
+    int64_t n_long_rows = 0, n_short_rows = 0;
+    for (const SliceView &v : slices) {
         if (v.R > 0 && int64_t(v.C) * es > stage / in_arrays)
             n_long_rows += v.R;
+        else
+            n_short_rows += v.R;
+    }
+    // Under the queue policies a CTA's first claim takes kFetch patches.  A
+    // batch of fewer than kFetch stage-filling patches per SM (up to a few
+    // tens of MB) is therefore cut into patches of at most
+    // ceil(rows / (kFetch * SMs)) rows, so that the first claims reach every
+    // SM instead of a few (8 x 64 x 64 fp32 ran on 2 SMs).  RR and WHOLE_GPU
+    // keep their own units.
+    const int64_t spread_rows =
+        std::max<int64_t>(1, (n_short_rows + int64_t(kFetch) * n_sm - 1) / (int64_t(kFetch) * n_sm));
     const int64_t chunk_elems = stage / in_arrays / es;
     const int64_t want_segs = n_long_rows > 0 && n_long_rows < 2 * n_sm
                                   ? std::max<int64_t>(1, (8 * n_sm + n_long_rows - 1) / n_long_rows)
@@ -379,6 +390,8 @@ int cut_patches(const bsm_plan_desc *d, const std::vector<SliceView> &slices, in
                 rpi = std::min<int64_t>(rpi, d->rows_per_item);
             if (d->policy == BSM_POLICY_WHOLE_GPU)
                 rpi = std::min<int64_t>(rpi, (v.R + n_sm - 1) / n_sm);
+            if (spanning)
+                rpi = std::min<int64_t>(rpi, spread_rows);
             rpi = std::max<int64_t>(1, std::min<int64_t>(rpi, seg_rows));
             for (int64_t g0 = 0; g0 < seg_rows; g0 += rpi) {
                 if (items.size() >= static_cast<size_t>(INT32_MAX))

@@ -59,6 +59,7 @@ def check_layout(rows, cols, dtype, policy, n_sm=152, smem=SMEM, offsets=None, r
     whole_cap = (((avail // 2) & ~127) // ins) & ~127
     assert all(C * es > whole_cap for (_, R, C) in sl if R > 0 and C * es * ins > stage)
     assert L["long_rows"] == len(long_rows)
+    n_short = len(row_owner) - len(long_rows)
 
     seen = Counter()
     segs = {}                                      # long row -> [(col0, cols, part_count)]
@@ -80,6 +81,8 @@ def check_layout(rows, cols, dtype, policy, n_sm=152, smem=SMEM, offsets=None, r
             assert n <= rows_per_item
         if policy == bsm.POLICY_WHOLE_GPU:
             assert n <= -(-R // n_sm)
+        if policy in QUEUE_POLICIES:
+            assert n <= max(1, -(-n_short // (4 * n_sm)))
         if policy not in QUEUE_POLICIES:
             assert r0 + n <= R                     # RR / WHOLE_GPU: inside its slice
         for k in range(n):
@@ -138,10 +141,27 @@ def test_rows_of_two_chunks_stay_staged():
 
 @pytest.mark.parametrize("policy", [bsm.POLICY_WHOLE_GPU, bsm.POLICY_RR] + list(QUEUE_POLICIES))
 def test_patches_never_cross_slices_under_rr_and_whole_gpu(policy):
-    rows, cols = [40, 40, 40, 7], [256, 256, 256, 256]
+    # 9010 rows: the queue policies' patches are 15 rows (ceil(9010 / 608)),
+    # which do not divide 3001
+    rows, cols = [3001, 3001, 3001, 7], [256, 256, 256, 256]
     L = check_layout(rows, cols, bsm.F32, policy, rows_per_item=16)
     spans = any(int(p["row0"]) + int(p["nrows"]) > int(p["slice_rows"]) for p in L["phase0"])
     assert spans == (policy in QUEUE_POLICIES)
+
+
+def test_small_batches_spread_over_every_sm():
+    """A CTA's first claim takes four patches: a batch of fewer than four
+    stage-filling patches per SM is cut into patches of ceil(rows / (4 x SMs))
+    rows under the queue policies, so that the first claims reach every SM."""
+    L = check_layout([64] * 8, [64] * 8, bsm.F32, bsm.POLICY_DYNAMIC)     # 8 x 64 x 64
+    assert len(L["phase0"]) == 512 and set(L["phase0"]["nrows"]) == {1}
+    L = check_layout([64] * 8, [64] * 8, bsm.F32, bsm.POLICY_RR)          # one patch per slice
+    assert len(L["phase0"]) == 8
+    L = check_layout([512] * 30, [512] * 30, bsm.F32, bsm.POLICY_CBMF_LB)  # 15360 rows
+    assert len(L["phase0"]) == 591 and max(L["phase0"]["nrows"]) == 26
+    # past four stage-filling patches per SM nothing changes
+    L = check_layout([512] * 40, [512] * 40, bsm.F32, bsm.POLICY_DYNAMIC)
+    assert set(L["phase0"]["nrows"]) == {32}
 
 
 def test_backward_stage_holds_two_rows():
@@ -211,7 +231,7 @@ def test_edge_cases():
     # in place (x == y) is allowed, a partial overlap is not
     check_layout([4], [64], bsm.F32, bsm.POLICY_DYNAMIC)
     assert len(bsm.bsm_plan_layout_host([4], [64], bsm.F32, bsm.POLICY_DYNAMIC, 152, SMEM,
-                                        x=1 << 40, y=1 << 40)["phase0"]) == 1
+                                        x=1 << 40, y=1 << 40)["phase0"]) == 4   # a row each
     with pytest.raises(bsm.BsmError) as e:
         bsm.bsm_plan_layout_host([4], [64], bsm.F32, bsm.POLICY_DYNAMIC, 152, SMEM,
                                  x=1 << 40, y=(1 << 40) + 64)
