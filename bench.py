@@ -10,7 +10,9 @@ built once up front, as the paper's scheduler builds its table once).
 Default workload: fp32 softmax over the last dim of 384 slices of 512 x 512
 (a 196608 x 512 tensor), values 3*N(0,1) from a fixed seed -- the shape of
 the paper's SOFTMAX experiment (Sec. 6).  Inputs (805 MB with the output)
-are larger than the 129 MB L2, so no flush is needed between steps.
+are larger than the 129 MB L2, so no flush is needed between steps.  A
+working set under twice the L2 (--workload 1, 256 KB) is timed step by step
+instead, with a buffer of twice the L2 written before every step.
 
 Metric: GB/s of algorithmic traffic (every input element read once, every
 output element written once) per step; also % of the measured HBM copy
