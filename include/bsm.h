@@ -113,7 +113,10 @@ typedef enum {
  * Softmax over B slices of R x C stored back to back, i.e. a (B*R) x C
  * row-major tensor (the layout of Sec. 2).  Equivalent to bsm_softmax_ex with
  * flags = 0.  The plan (patch table, die queues) is built on first use for a
- * given (device, x, y, shape, dtype, policy, flags) and cached.
+ * given (device, x, y, shape, dtype, policy, flags) and cached.  Calls that
+ * share a cached plan share its queue counters, which the last CTA of an
+ * execution resets.  Such calls must therefore not run at the same time on
+ * different streams; they write the same y anyway, so order them.
  *   x, y    device pointers, B*R*C elements of `dtype` each.
  *   B, R, C B >= 0, R >= 0, C >= 1; B*R*C < 2^62.
  *   dtype   bsm_dtype; policy bsm_policy.
