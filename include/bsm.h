@@ -226,7 +226,9 @@ int bsm_softmax_backward_ragged(const void *y, const void *dy, void *dx, int64_t
  *       rounded to nearest even for bf16)
  *   M a multiple of 128, N of 64, K of 64 (else BSM_ERR_UNSUPPORTED);
  *   pointers 16-byte aligned; c must not overlap a or bt.
- * Plans are cached like bsm_softmax's.  Errors as bsm_softmax.
+ * Plans are cached like bsm_softmax's, with the same rule: calls that share
+ * one (same pointers, shapes, dtype, policy) must not run at the same time on
+ * different streams.  Errors as bsm_softmax.
  */
 int bsm_bmm(const void *a, const void *bt, void *c, int64_t B, int64_t M, int64_t N, int64_t K,
             int out_dtype, int policy, bsm_stream_t stream);
