@@ -19,6 +19,7 @@
 #include <vector>
 
 #include "bsm_internal.h"
+#include "bsm_trace.h"
 
 namespace bsm {
 
@@ -476,6 +477,7 @@ void free_plan(bsm_plan *p)
 
 int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
 {
+    TraceRange trace("bsm_plan_create");
     const auto t0 = std::chrono::steady_clock::now();
     if (!out || !d)
         return BSM_ERR_INVALID_ARG;
@@ -848,6 +850,7 @@ int plan_layout_host_impl(const bsm_plan_desc *d, int32_t n_sm, int64_t smem_opt
 
 int plan_execute_impl(const bsm_plan *p, bsm_stream_t stream)
 {
+    TraceRange trace("bsm_plan_execute");
     if (!p)
         return BSM_ERR_INVALID_ARG;
     if (p->args.n_items == 0)

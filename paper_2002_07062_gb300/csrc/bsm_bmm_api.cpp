@@ -15,6 +15,7 @@
 #include <vector>
 
 #include "bsm_internal.h"
+#include "bsm_trace.h"
 
 namespace bsm {
 
@@ -170,6 +171,7 @@ cudaGraphExec_t capture_whole_gpu(const GemmPlan *p)
 
 int build_plan(GemmPlan *p, const GemmDev &dev)
 {
+    TraceRange trace("bsm_bmm_plan_create");
     const int bn = p->bn;
     const int64_t mt = p->M / 128, nt = p->N / bn;
     const int64_t n_items = p->B * mt * nt;
@@ -360,6 +362,7 @@ int build_plan(GemmPlan *p, const GemmDev &dev)
 
 int run_plan(GemmPlan *p, bsm_stream_t stream)
 {
+    TraceRange trace("bsm_bmm_execute");
     int err = 0;
     if (p->policy == BSM_POLICY_WHOLE_GPU && p->whole_graph) {
         err = static_cast<int>(cudaGraphLaunch(p->whole_graph, static_cast<cudaStream_t>(stream)));

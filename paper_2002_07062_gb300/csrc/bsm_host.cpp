@@ -21,6 +21,7 @@
 #include <mutex>
 
 #include "bsm_internal.h"
+#include "bsm_trace.h"
 
 namespace bsm {
 namespace {
@@ -87,6 +88,7 @@ int pipe_reserve(HostPipe &p, int64_t bytes)
 int softmax_host(const void *x_host, void *y_host, int64_t B, int64_t R, int64_t C, int dtype, int policy,
                  uint32_t flags, bsm_stream_t stream)
 {
+    TraceRange trace("bsm_softmax_host");
     if (B < 0 || R < 0 || C < 1 || (dtype != BSM_F32 && dtype != BSM_BF16) || (flags & ~BSM_FLAG_CAUSAL) ||
         policy < BSM_POLICY_WHOLE_GPU || policy > BSM_POLICY_MINIMAX)
         return BSM_ERR_INVALID_ARG;

@@ -142,3 +142,26 @@ def test_header_is_plain_c_and_links_from_c(tmp_path):
                     "-L", lib_dir, "-lbsm", "-Wl,-rpath," + lib_dir, "-o", str(exe)], check=True)
     out = subprocess.run([str(exe)], capture_output=True, text=True)
     assert out.returncode == 0, out.stdout + out.stderr
+
+
+def test_plan_create_without_gpu_reports_no_device():
+    """A well-formed descriptor reaches the device query (inside the plan's
+    trace range, a no-op without a profiler) and comes back as
+    BSM_ERR_NO_DEVICE; execute and stats reject a null plan."""
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    d = bsm.PlanDesc()
+    assert bsm.lib().bsm_plan_desc_init(ctypes.byref(d)) == bsm.OK
+    r = (ctypes.c_int32 * 1)(4)
+    c = (ctypes.c_int32 * 1)(64)
+    d.x, d.y, d.num_slices = 1 << 40, 1 << 41, 1
+    d.rows = ctypes.cast(r, bsm.c_i32p)
+    d.cols = ctypes.cast(c, bsm.c_i32p)
+    h = ctypes.c_void_p()
+    for _ in range(2):
+        assert bsm.lib().bsm_plan_create(ctypes.byref(h), ctypes.byref(d)) == bsm.ERR_NO_DEVICE
+        assert not h.value
+    assert bsm.lib().bsm_plan_execute(None, None) == bsm.ERR_INVALID_ARG
+    s = bsm.PlanStats()
+    assert bsm.lib().bsm_plan_get_stats(None, ctypes.byref(s)) == bsm.ERR_INVALID_ARG
