@@ -181,13 +181,43 @@ def _check(rc: int, where: str):
         raise BsmError(rc, where)
 
 
-def _dptr(t) -> Optional[int]:
-    """Device address of a torch tensor, or an int passed through."""
+def _dptr(t, nbytes: Optional[int] = None, what: str = "buffer") -> Optional[int]:
+    """Device address of a torch tensor, or an int passed through unchecked.
+    A tensor must live on a CUDA device, be contiguous and (when nbytes is
+    given) hold at least nbytes: the C ABI sees only the address, so these are
+    checked here, before any launch."""
     if t is None:
         return None
     if isinstance(t, int):
         return t
+    if not getattr(t, "is_cuda", True):
+        raise ValueError("%s must be a CUDA tensor (got one on %s)" % (what, t.device))
+    if hasattr(t, "is_contiguous") and not t.is_contiguous():
+        raise ValueError("%s must be contiguous" % what)
+    if nbytes is not None and hasattr(t, "numel") and t.numel() * t.element_size() < nbytes:
+        raise ValueError("%s holds %d bytes, the call needs %d"
+                         % (what, t.numel() * t.element_size(), nbytes))
     return int(t.data_ptr())
+
+
+def _esize(dtype: int) -> int:
+    return 4 if dtype == F32 else 2
+
+
+def _bmm_bytes(B: int, M: int, N: int, K: int, out_dtype: int):
+    """Bytes of a, bt and c for a batched product (bf16 operands)."""
+    if min(B, M, N, K) <= 0:
+        return 0, 0, 0
+    return B * M * K * 2, B * N * K * 2, B * M * N * _esize(out_dtype)
+
+
+def _extent(offsets, rows, cols) -> int:
+    """Elements a ragged batch spans (the end of its furthest non-empty slice)."""
+    end = 0
+    for o, r, c in zip(offsets, rows, cols):
+        if r > 0:
+            end = max(end, int(o) + int(r) * int(c))
+    return end
 
 
 def _stream(s) -> Optional[int]:
@@ -203,13 +233,15 @@ def _np(a, dt):
 
 
 def bsm_softmax(x, y, B: int, R: int, C: int, dtype: int, policy: int, stream=None):
-    _check(lib().bsm_softmax(_dptr(x), _dptr(y), B, R, C, dtype, policy, _stream(stream)),
-           "bsm_softmax")
+    n = max(B * R * C, 0) * _esize(dtype)
+    _check(lib().bsm_softmax(_dptr(x, n, "x"), _dptr(y, n, "y"), B, R, C, dtype, policy,
+                             _stream(stream)), "bsm_softmax")
 
 
 def bsm_softmax_ex(x, y, B: int, R: int, C: int, dtype: int, policy: int, flags: int = 0,
                    stream=None):
-    _check(lib().bsm_softmax_ex(_dptr(x), _dptr(y), B, R, C, dtype, policy, flags,
+    n = max(B * R * C, 0) * _esize(dtype)
+    _check(lib().bsm_softmax_ex(_dptr(x, n, "x"), _dptr(y, n, "y"), B, R, C, dtype, policy, flags,
                                 _stream(stream)), "bsm_softmax_ex")
 
 
@@ -229,27 +261,33 @@ def bsm_softmax_host(x_host, y_host, B: int, R: int, C: int, dtype: int, policy:
 
 def bsm_softmax_noalloc(x, y, B: int, R: int, C: int, dtype: int, flags: int = 0, stream=None):
     """The allocation-free entry point (fixed scratch inside the library)."""
-    _check(lib().bsm_softmax_noalloc(_dptr(x), _dptr(y), B, R, C, dtype, flags, _stream(stream)),
-           "bsm_softmax_noalloc")
+    n = max(B * R * C, 0) * _esize(dtype)
+    _check(lib().bsm_softmax_noalloc(_dptr(x, n, "x"), _dptr(y, n, "y"), B, R, C, dtype, flags,
+                                     _stream(stream)), "bsm_softmax_noalloc")
 
 
 def bsm_bmm(a, bt, c, B: int, M: int, N: int, K: int, out_dtype: int, policy: int, stream=None):
     """C_s = A_s Bt_s^T for every slice (bf16 inputs, fp32 or bf16 output)."""
-    _check(lib().bsm_bmm(_dptr(a), _dptr(bt), _dptr(c), B, M, N, K, out_dtype, policy,
-                         _stream(stream)), "bsm_bmm")
+    na, nb, nc = _bmm_bytes(B, M, N, K, out_dtype)
+    _check(lib().bsm_bmm(_dptr(a, na, "a"), _dptr(bt, nb, "bt"), _dptr(c, nc, "c"), B, M, N, K,
+                         out_dtype, policy, _stream(stream)), "bsm_bmm")
 
 
 def bsm_bmm_ex(a, bt, c, B: int, M: int, N: int, K: int, out_dtype: int, policy: int,
                n_stages: int = 0, epi_bufs: int = 0, k_blocks_per_stage: int = 0, stream=None):
     """bsm_bmm with the shared-memory split (stages, store buffers, K blocks
     per stage) chosen."""
-    _check(lib().bsm_bmm_ex(_dptr(a), _dptr(bt), _dptr(c), B, M, N, K, out_dtype, policy,
-                            n_stages, epi_bufs, k_blocks_per_stage, _stream(stream)), "bsm_bmm_ex")
+    na, nb, nc = _bmm_bytes(B, M, N, K, out_dtype)
+    _check(lib().bsm_bmm_ex(_dptr(a, na, "a"), _dptr(bt, nb, "bt"), _dptr(c, nc, "c"), B, M, N, K,
+                            out_dtype, policy, n_stages, epi_bufs, k_blocks_per_stage,
+                            _stream(stream)), "bsm_bmm_ex")
 
 
 def bsm_softmax_backward(y, dy, dx, B: int, R: int, C: int, dtype: int, policy: int, stream=None):
-    _check(lib().bsm_softmax_backward(_dptr(y), _dptr(dy), _dptr(dx), B, R, C, dtype, policy,
-                                      _stream(stream)), "bsm_softmax_backward")
+    n = max(B * R * C, 0) * _esize(dtype)
+    _check(lib().bsm_softmax_backward(_dptr(y, n, "y"), _dptr(dy, n, "dy"), _dptr(dx, n, "dx"),
+                                      B, R, C, dtype, policy, _stream(stream)),
+           "bsm_softmax_backward")
 
 
 def bsm_softmax_backward_ragged(y, dy, dx, offsets, rows, cols, dtype: int, policy: int,
@@ -259,7 +297,9 @@ def bsm_softmax_backward_ragged(y, dy, dx, offsets, rows, cols, dtype: int, poli
     c = _np(cols, np.int32)
     if not (len(off) == len(r) == len(c)):
         raise ValueError("offsets, rows and cols must have the same length")
-    _check(lib().bsm_softmax_backward_ragged(_dptr(y), _dptr(dy), _dptr(dx), len(off),
+    n = _extent(off, r, c) * _esize(dtype)
+    _check(lib().bsm_softmax_backward_ragged(_dptr(y, n, "y"), _dptr(dy, n, "dy"), _dptr(dx, n, "dx"),
+                                             len(off),
                                              off.ctypes.data_as(c_i64p), r.ctypes.data_as(c_i32p),
                                              c.ctypes.data_as(c_i32p), dtype, policy,
                                              _stream(stream)), "bsm_softmax_backward_ragged")
@@ -272,7 +312,8 @@ def bsm_softmax_ragged(x, y, offsets, rows, cols, dtype: int, policy: int, flags
     c = _np(cols, np.int32)
     if not (len(off) == len(r) == len(c)):
         raise ValueError("offsets, rows and cols must have the same length")
-    _check(lib().bsm_softmax_ragged(_dptr(x), _dptr(y), len(off),
+    n = _extent(off, r, c) * _esize(dtype)
+    _check(lib().bsm_softmax_ragged(_dptr(x, n, "x"), _dptr(y, n, "y"), len(off),
                                     off.ctypes.data_as(c_i64p), r.ctypes.data_as(c_i32p),
                                     c.ctypes.data_as(c_i32p), dtype, policy, flags,
                                     _stream(stream)), "bsm_softmax_ragged")
@@ -312,8 +353,12 @@ def bsm_plan_create(x, y, rows, cols, dtype: int, policy: int, offsets=None, fla
     r = _np(rows, np.int32)
     c = _np(cols, np.int32)
     off = None if offsets is None else _np(offsets, np.int64)
-    d.x = _dptr(x)
-    d.y = _dptr(y)
+    if off is None:
+        n = int(np.sum(r.astype(np.int64) * c.astype(np.int64))) * _esize(dtype)
+    else:
+        n = _extent(off, r, c) * _esize(dtype)
+    d.x = _dptr(x, n, "x")
+    d.y = _dptr(y, n, "y")
     d.num_slices = len(r)
     d.rows = r.ctypes.data_as(c_i32p)
     d.cols = c.ctypes.data_as(c_i32p)
@@ -329,7 +374,7 @@ def bsm_plan_create(x, y, rows, cols, dtype: int, policy: int, offsets=None, fla
     d.count_output_bytes = 1 if count_output_bytes else 0
     d.device = device
     d.op = op
-    d.x2 = _dptr(x2)
+    d.x2 = _dptr(x2, n, "x2")
     h = ctypes.c_void_p()
     _check(lib().bsm_plan_create(ctypes.byref(h), ctypes.byref(d)), "bsm_plan_create")
     return Plan(h.value, (x, y, x2))

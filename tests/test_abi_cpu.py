@@ -165,3 +165,62 @@ def test_plan_create_without_gpu_reports_no_device():
     assert bsm.lib().bsm_plan_execute(None, None) == bsm.ERR_INVALID_ARG
     s = bsm.PlanStats()
     assert bsm.lib().bsm_plan_get_stats(None, ctypes.byref(s)) == bsm.ERR_INVALID_ARG
+
+
+class _FakeDevTensor:
+    """Stands in for a CUDA tensor: the binding only asks where it lives,
+    whether it is contiguous, its size and its address."""
+    is_cuda = True
+    device = "cuda:0"
+
+    def __init__(self, n, es=4, contiguous=True):
+        self._n, self._es, self._c = n, es, contiguous
+
+    def is_contiguous(self):
+        return self._c
+
+    def numel(self):
+        return self._n
+
+    def element_size(self):
+        return self._es
+
+    def data_ptr(self):
+        return 1 << 40
+
+
+def test_binding_rejects_host_strided_and_short_tensors():
+    """The C ABI sees only addresses, so the binding checks device, layout and
+    size before the call; a well-formed call reaches the library (which, on a
+    machine without a GPU, answers BSM_ERR_NO_DEVICE)."""
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    F = _FakeDevTensor
+    with pytest.raises(ValueError, match="CUDA tensor"):
+        bsm.bsm_softmax(torch.zeros(256), F(256), 4, 1, 64, bsm.F32, bsm.POLICY_RR)
+    with pytest.raises(ValueError, match="contiguous"):
+        bsm.bsm_softmax(F(256), F(256, contiguous=False), 4, 1, 64, bsm.F32, bsm.POLICY_RR)
+    with pytest.raises(ValueError, match="needs 1024"):
+        bsm.bsm_softmax_ex(F(255), F(256), 4, 1, 64, bsm.F32, bsm.POLICY_RR, 0)
+    with pytest.raises(ValueError, match="needs 512"):              # bf16: 2 bytes each
+        bsm.bsm_softmax(F(256, es=2), F(255, es=2), 4, 1, 64, bsm.BF16, bsm.POLICY_RR)
+    with pytest.raises(ValueError, match="needs"):                  # ragged: the furthest slice
+        bsm.bsm_softmax_ragged(F(1000), F(1000), [0, 960], [1, 1], [64, 64], bsm.F32, bsm.POLICY_RR)
+    with pytest.raises(ValueError, match="needs"):
+        bsm.bsm_softmax_backward(F(256), F(128), F(256), 4, 1, 64, bsm.F32, bsm.POLICY_RR)
+    with pytest.raises(ValueError, match="needs"):                  # c: 128 x 64 fp32
+        bsm.bsm_bmm(F(128 * 64, es=2), F(64 * 64, es=2), F(128 * 64 - 1), 1, 128, 64, 64,
+                    bsm.F32, bsm.POLICY_DYNAMIC)
+    with pytest.raises(ValueError, match="needs"):
+        bsm.bsm_plan_create(F(100), F(256), [4], [64], bsm.F32, bsm.POLICY_DYNAMIC)
+    # well-formed: the call reaches the library
+    with pytest.raises(bsm.BsmError) as e:
+        bsm.bsm_softmax(F(256), F(256), 4, 1, 64, bsm.F32, bsm.POLICY_RR)
+    assert e.value.status == bsm.ERR_NO_DEVICE
+    with pytest.raises(bsm.BsmError) as e:
+        bsm.bsm_softmax_ragged(F(1024), F(1024), [0, 960], [1, 1], [64, 64], bsm.F32,
+                               bsm.POLICY_RR)
+    assert e.value.status == bsm.ERR_NO_DEVICE
+    # empty batches need no buffer at all
+    bsm.bsm_softmax(None, None, 0, 4, 64, bsm.F32, bsm.POLICY_RR)
