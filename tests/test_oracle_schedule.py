@@ -166,6 +166,26 @@ def test_minimax_lpt_against_brute_force(trial):
         assert 6 * got[0] * opt[1] <= 7 * opt[0] * got[1]
 
 
+@pytest.mark.parametrize("trial", range(20))
+def test_minimax_lpt_three_banks_against_brute_force(trial):
+    """Three banks: every patch assigned once, never better than the exact
+    optimum, and with identical units and equal weights within Graham's LPT
+    bound for m = 3 machines, (4/3 - 1/9) OPT = 11/9 OPT."""
+    rng = random.Random(7000 + trial)
+    n = rng.randrange(1, 8)
+    t = _rand_table(rng, n, 3)
+    identical = trial % 2 == 0
+    units = [1, 1, 1] if identical else [rng.randrange(1, 4) for _ in range(3)]
+    ln, lf = (1, 1) if identical else (2, 5)
+    queues, W = S.minimax_lpt(t, units, ln, lf)
+    assert sorted(queues[0] + queues[1] + queues[2]) == list(range(n))
+    got = S.makespan_num_den(W, units)
+    opt = S.brute_force_minimax_table(t, units, ln, lf)
+    assert got[0] * opt[1] >= opt[0] * got[1]
+    if identical:
+        assert 9 * got[0] * opt[1] <= 11 * opt[0] * got[1]
+
+
 def test_minimax_queues_are_longest_first():
     m = S.BankMap(256, [0, 1] * 40)
     patches = [(0, 256), (256, 1280), (1280, 1536), (1536, 3584), (3584, 3840)]
