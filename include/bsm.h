@@ -170,25 +170,35 @@ int bsm_softmax_ragged(const void *x, void *y, int64_t num_slices, const int64_t
  * pick up the device-wide synchronisation of cudaMalloc/cudaFree.  The paper
  * has no counterpart; this is a deployment variant of the dynamic schedule.
  *
- * Same computation and the same kernel as bsm_softmax_ex with
- * BSM_POLICY_DYNAMIC (results are identical), for B slices of R x C packed
- * back to back.  Instead of a plan, the patch table and queue counters live
- * in one fixed device array inside the library: every GPU that loads the
- * library holds it (about 1.5 MiB) until the process exits.  The first call
- * on a device, with that device current, looks the array's address up
- * (cudaGetSymbolAddress): make that first call before any stream capture.
- * Every call shares the array and it keeps the last call's contents; each
- * call rewrites the patch table and zeroes the counters on `stream` first,
- * so calls that overlap on the GPU (other streams, unordered threads) race.
- * Device-side error bits of this entry point stay in the array and are not
- * reported.  Nothing is allocated and nothing synchronises.
+ * The same kernel, row routine and patches as bsm_softmax_ex with
+ * BSM_POLICY_DYNAMIC, for B slices of R x C packed back to back, so the
+ * results are bit for bit the same -- for rows that fit one shared-memory
+ * stage: at most BSM_NOALLOC_MAX_ROW_BYTES (C * element size), and at most
+ * the device's own stage limit (half its opt-in shared memory per block less
+ * 1 KiB, rounded down to 128 bytes: the same 113 KiB on GB300).  Longer rows
+ * get BSM_ERR_UNSUPPORTED here (bsm_softmax_ex streams them in two passes,
+ * which needs buffers this entry point does not have).
+ *
+ * Instead of a plan, the patch table and queue counters live in one fixed
+ * device array inside the library: every GPU that loads the library holds it
+ * (about 1.5 MiB) until the process exits.  The first call on a device, with
+ * that device current, looks the array's address up (cudaGetSymbolAddress):
+ * make that first call before any stream capture.  Every call shares the
+ * array and it keeps the last call's contents; each call rewrites the patch
+ * table and zeroes the counters on `stream` first, so calls that overlap on
+ * the GPU (other streams, unordered threads) race.  Device-side error bits
+ * of this entry point are sticky in the array: bsm_device_status reports
+ * them (OR-ed with the library's own word) and bsm_device_status_clear
+ * zeroes them.  Nothing is allocated and nothing synchronises.
  *   x, y, B, R, C, dtype, flags, stream: as bsm_softmax_ex.
- * Errors: as bsm_softmax_ex, plus BSM_ERR_TOO_LARGE when the batch needs more
- * than BSM_NOALLOC_MAX_PATCHES patches (a patch is the rows that fill one
- * 64 KiB shared-memory stage: for 2 KiB rows, 32 rows; 65536 patches cover
- * 4 GiB of input).
+ * Errors: as bsm_softmax_ex; BSM_ERR_UNSUPPORTED for a row past the limit
+ * above; BSM_ERR_TOO_LARGE when the batch needs more than
+ * BSM_NOALLOC_MAX_PATCHES patches (a patch is the rows that fill one 64 KiB
+ * shared-memory stage: for 2 KiB rows, 32 rows; 65536 patches cover 4 GiB of
+ * input).  The row and patch limits are checked before the device is touched.
  */
 #define BSM_NOALLOC_MAX_PATCHES 65536
+#define BSM_NOALLOC_MAX_ROW_BYTES 115712   /* 113 KiB */
 int bsm_softmax_noalloc(const void *x, void *y, int64_t B, int64_t R, int64_t C, int dtype,
                         uint32_t flags, bsm_stream_t stream);
 
@@ -360,7 +370,10 @@ int bsm_plan_layout_host(const bsm_plan_desc *d, int32_t n_sm, int64_t smem_opti
                          int64_t cap0, bsm_patch *phase1, int64_t cap1, bsm_layout *out);
 
 /* Fault injection on one plan, for the library's failure-detection tests
- * (nothing here faults, traps or hangs the GPU):
+ * (nothing here faults, traps or hangs the GPU).  plan = NULL applies
+ * BSM_DEBUG_WITHHOLD_STAGE / BSM_DEBUG_NONE to the bsm_softmax_noalloc
+ * launches that follow, in every thread (its timeout then shows in
+ * bsm_device_status); BSM_DEBUG_CORRUPT_PATCH needs a plan.
  *   BSM_DEBUG_WITHHOLD_STAGE  later executes never fill the first shared-memory
  *                             stage of each CTA, so the consumers' bounded waits
  *                             run out; arg = the wait limit in ns (> 0).  The
@@ -458,8 +471,12 @@ int bsm_schedule_host(const bsm_schedule_desc *d, bsm_schedule_out *out);
 
 /* ---- status ---- */
 
-/* Sticky device-side status word of `device` (-1 = current), BSM_DEV_* bits.
- * Synchronises the device.  bsm_device_status_clear zeroes it. */
+/* Sticky device-side status word of `device` (-1 = current), BSM_DEV_* bits:
+ * the library's own word OR-ed with the words of bsm_softmax_noalloc's fixed
+ * array (so a timeout or bounds error there is not lost).  Synchronises the
+ * device; allocates nothing.  bsm_device_status_clear zeroes both.  (The
+ * contract's `int bsm_device_status(void)` gained the device and an output
+ * argument, so that the status code and the bits travel separately.) */
 int bsm_device_status(int device, uint32_t *status_out);
 int bsm_device_status_clear(int device);
 

@@ -33,6 +33,7 @@ DEV_BOUNDS, DEV_TIMEOUT, DEV_CHECK = 1, 2, 4
 (OK, ERR_INVALID_ARG, ERR_MISALIGNED, ERR_UNSUPPORTED, ERR_CUDA, ERR_DEVICE_BOUNDS,
  ERR_TIMEOUT, ERR_NO_DEVICE, ERR_NOMEM, ERR_TOO_LARGE) = range(10)
 NOALLOC_MAX_PATCHES = 65536
+NOALLOC_MAX_ROW_BYTES = 115712      # 113 KiB: rows of bsm_softmax_noalloc fit one stage
 
 c_i64p = ctypes.POINTER(ctypes.c_int64)
 c_i32p = ctypes.POINTER(ctypes.c_int32)
@@ -397,9 +398,11 @@ def bsm_plan_get_stats(plan: Plan) -> dict:
 DEBUG_NONE, DEBUG_WITHHOLD_STAGE, DEBUG_CORRUPT_PATCH = 0, 1, 2
 
 
-def bsm_plan_debug(plan: Plan, what: int, arg: int = 0):
-    """Test-only fault injection (see include/bsm.h)."""
-    _check(lib().bsm_plan_debug(plan.handle, what, arg), "bsm_plan_debug")
+def bsm_plan_debug(plan, what: int, arg: int = 0):
+    """Test-only fault injection (see include/bsm.h); plan None targets the
+    launches of bsm_softmax_noalloc."""
+    _check(lib().bsm_plan_debug(None if plan is None else plan.handle, what, arg),
+           "bsm_plan_debug")
 
 
 def bsm_plan_destroy(plan: Plan):

@@ -1017,7 +1017,7 @@ int bsm_plan_get_stats(const bsm_plan *plan, bsm_plan_stats *out)
 int bsm_plan_debug(bsm_plan *plan, int what, int64_t arg)
 {
     if (!plan)
-        return BSM_ERR_INVALID_ARG;
+        return noalloc_debug(what, arg);
     switch (what) {
     case BSM_DEBUG_NONE:
         plan->args.debug = 0;
@@ -1194,14 +1194,31 @@ int bsm_device_status(int device, uint32_t *status_out)
 {
     if (!status_out)
         return BSM_ERR_INVALID_ARG;
-    DeviceCtx *c = nullptr;
-    int rc = device_ctx(device, &c);
-    if (rc)
-        return rc;
+    if (device < 0 && cudaGetDevice(&device) != cudaSuccess)
+        return BSM_ERR_NO_DEVICE;
+    int count = 0;
+    if (cudaGetDeviceCount(&count) != cudaSuccess || device >= count || device >= kMaxDevices)
+        return BSM_ERR_NO_DEVICE;
     if (cudaError_t e = cudaDeviceSynchronize())
         return cuda_error(e, "cudaDeviceSynchronize");
-    if (cudaError_t e = cudaMemcpy(status_out, c->status, sizeof(uint32_t), cudaMemcpyDeviceToHost))
-        return cuda_error(e, "cudaMemcpy(status)");
+    // the library's word exists once a plan or probe initialised the device;
+    // reading it allocates nothing (a caller of bsm_softmax_noalloc alone
+    // has only the fixed array's words)
+    uint32_t *word = nullptr;
+    {
+        std::lock_guard<std::mutex> lk(g_mu);
+        if (g_dev[device].ready)
+            word = g_dev[device].status;
+    }
+    uint32_t bits = 0;
+    if (word) {
+        if (cudaError_t e = cudaMemcpy(&bits, word, sizeof(uint32_t), cudaMemcpyDeviceToHost))
+            return cuda_error(e, "cudaMemcpy(status)");
+    }
+    uint32_t na = 0;
+    if (int rc = noalloc_status(device, &na, 0))
+        return rc;
+    *status_out = bits | na;
     return BSM_OK;
 }
 
@@ -1211,8 +1228,15 @@ int bsm_device_status_clear(int device)
     int rc = device_ctx(device, &c);
     if (rc)
         return rc;
+    if (device < 0)
+        cudaGetDevice(&device);
+    if (cudaError_t e = cudaDeviceSynchronize())
+        return cuda_error(e, "cudaDeviceSynchronize");
     if (cudaError_t e = cudaMemset(c->status, 0, 8 * sizeof(uint32_t)))
         return cuda_error(e, "cudaMemset(status)");
+    uint32_t na = 0;
+    if ((rc = noalloc_status(device, &na, 1)))
+        return rc;
     if (cudaError_t e = cudaDeviceSynchronize())
         return cuda_error(e, "cudaDeviceSynchronize");
     return BSM_OK;

@@ -156,6 +156,13 @@ int probe_map_run(const void *buf, int64_t bytes, int64_t chunk, int reps, const
 // returns BSM_ERR_CUDA.
 int record_cuda_error(int cuda_error, const char *where);
 
+// Sticky status bits left by bsm_softmax_noalloc on `device` (bsm_noalloc.cu;
+// 0 if it never ran there); clear != 0 zeroes them afterwards.
+int noalloc_status(int device, uint32_t *bits, int clear);
+// Fault injection for bsm_softmax_noalloc's launches (bsm_plan_debug with a
+// null plan): BSM_DEBUG_NONE or BSM_DEBUG_WITHHOLD_STAGE.
+int noalloc_debug(int what, int64_t arg);
+
 // Host planner (bsm_planner.cpp).
 int schedule_host(const bsm_schedule_desc *d, bsm_schedule_out *out);
 

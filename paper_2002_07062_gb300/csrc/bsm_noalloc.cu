@@ -11,7 +11,9 @@
 // persistent kernel under the one-queue dynamic schedule, with its scratch
 // (patch table, queue counters, status words) in one file-scope __device__
 // array of fixed size instead of allocated memory.  The caller still passes
-// x and y.
+// x and y.  Rows must fit one shared-memory stage (BSM_NOALLOC_MAX_ROW_BYTES,
+// and the device's own stage limit): the two-pass path of longer rows needs
+// per-plan buffers this entry point does not have.
 //
 // The array is part of the library's device image: every GPU that loads the
 // library holds it (about 1.5 MiB) until the process exits.  Host code cannot
@@ -21,10 +23,13 @@
 // capture).  All calls share the array and it keeps the last call's contents:
 // every call first rewrites the patch table and zeroes the queue counters on
 // its stream, and two calls that overlap on the GPU (different streams, or
-// different host threads without ordering) race on it.
+// different host threads without ordering) race on it.  The status words in
+// the array are sticky, like the library's own status word: they are read
+// (OR-ed into it) by bsm_device_status and zeroed by bsm_device_status_clear.
 
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cstdint>
 #include <mutex>
 
@@ -52,16 +57,19 @@ struct NoAllocDevice {
 std::mutex g_na_mu;
 NoAllocDevice g_na_dev[64];
 
+// Test-only fault injection for this entry point's launches (set through
+// bsm_plan_debug with a null plan): KDEBUG_* bits and the wait bound.
+std::atomic<uint32_t> g_na_debug{0};
+std::atomic<uint64_t> g_na_wait_ns{0};
+
 // Patch i covers rows [i*rpi, min((i+1)*rpi, B*R)) of the (B*R) x C matrix;
-// also zero the queue counters and the status words.
-__global__ void noalloc_fill(Item *items, uint32_t *heads, uint32_t *status, int64_t total_rows,
-                             int32_t R, int32_t C, int32_t rpi, int32_t n_items)
+// also zero the queue counters (the status words stay: they are sticky).
+__global__ void noalloc_fill(Item *items, uint32_t *heads, int64_t total_rows, int32_t R, int32_t C,
+                             int32_t rpi, int32_t n_items)
 {
     const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (i < 8) {
+    if (i < 8)
         heads[i] = 0u;
-        status[i] = 0u;
-    }
     if (i >= n_items)
         return;
     const int64_t g0 = i * rpi;
@@ -102,24 +110,27 @@ int softmax_noalloc(const void *x, void *y, int64_t B, int64_t R, int64_t C, int
     const int64_t rows = B * R;
     if (rows == 0)
         return BSM_OK;
-    if (C > (int64_t(1) << 61) / rows)
-        return BSM_ERR_INVALID_ARG;
     const int es = dtype == BSM_F32 ? 4 : 2;
+    const int64_t row_bytes = C * es;   // C < 2^31: no overflow
+    // no two-pass path here: a row must fit one stage (checked again against
+    // the device's shared memory below)
+    if (row_bytes > BSM_NOALLOC_MAX_ROW_BYTES)
+        return BSM_ERR_UNSUPPORTED;
+    // patches of the rows that fill one stage, as the planned path cuts them
+    // for large batches (device independent); the count bounds rows * C
+    // before any product of them is formed
+    const int64_t stage = row_bytes > kMinStageBytes ? (row_bytes + 127) & ~int64_t(127) : kMinStageBytes;
+    const int64_t rpi_stage = stage / row_bytes;
+    if ((rows + rpi_stage - 1) / rpi_stage > kNoAllocMaxPatches)
+        return BSM_ERR_TOO_LARGE;
     if (!x || !y)
         return BSM_ERR_INVALID_ARG;
     const uintptr_t xa = reinterpret_cast<uintptr_t>(x), ya = reinterpret_cast<uintptr_t>(y);
-    const uintptr_t len = static_cast<uintptr_t>(rows * C * es);
+    const uintptr_t len = static_cast<uintptr_t>(rows * row_bytes);   // < 2^16 stages of < 2^17 bytes
     if (xa != ya && xa < ya + len && ya < xa + len)
         return BSM_ERR_INVALID_ARG;
-    if ((xa & 15) || (ya & 15) || (C * es) % 16 != 0)
+    if ((xa & 15) || (ya & 15) || row_bytes % 16 != 0)
         return BSM_ERR_MISALIGNED;
-    // patches (device independent): the rows that fill one stage
-    const int64_t row_bytes = C * es;
-    const int64_t stage = row_bytes > kMinStageBytes ? (row_bytes + 127) & ~int64_t(127) : kMinStageBytes;
-    const int64_t rpi = stage / row_bytes;
-    const int64_t n_items = (rows + rpi - 1) / rpi;
-    if (n_items > kNoAllocMaxPatches)
-        return BSM_ERR_TOO_LARGE;
     int device = 0;
     if (cudaGetDevice(&device) != cudaSuccess)
         return BSM_ERR_NO_DEVICE;
@@ -130,6 +141,14 @@ int softmax_noalloc(const void *x, void *y, int64_t B, int64_t R, int64_t C, int
     if (row_bytes > ((avail / 2) & ~int64_t(127)))
         return BSM_ERR_UNSUPPORTED;
     const int n_stages = static_cast<int>(avail / stage < kMaxStages ? avail / stage : kMaxStages);
+    // a small batch (fewer than kFetch stage-filling patches per SM) is cut
+    // into patches of at most ceil(rows / (kFetch * SMs)) rows, as the planned
+    // dynamic schedule cuts it, so that the CTAs' first claims reach every SM
+    const int64_t spread = (rows + int64_t(kFetch) * nd->n_sm - 1) / (int64_t(kFetch) * nd->n_sm);
+    const int64_t rpi = spread < rpi_stage ? (spread > 0 ? spread : 1) : rpi_stage;
+    const int64_t n_items = (rows + rpi - 1) / rpi;
+    if (n_items > kNoAllocMaxPatches)
+        return BSM_ERR_TOO_LARGE;
 
     Item *items = reinterpret_cast<Item *>(nd->scratch);
     uint32_t *heads = reinterpret_cast<uint32_t *>(nd->scratch + kHeadsOffset);
@@ -137,7 +156,7 @@ int softmax_noalloc(const void *x, void *y, int64_t B, int64_t R, int64_t C, int
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     const int threads = 256;
     const int blocks = static_cast<int>((n_items + threads - 1) / threads);
-    noalloc_fill<<<blocks, threads, 0, st>>>(items, heads, status, rows, static_cast<int32_t>(R),
+    noalloc_fill<<<blocks, threads, 0, st>>>(items, heads, rows, static_cast<int32_t>(R),
                                              static_cast<int32_t>(C), static_cast<int32_t>(rpi),
                                              static_cast<int32_t>(n_items));
     if (cudaError_t e = cudaGetLastError())
@@ -160,12 +179,62 @@ int softmax_noalloc(const void *x, void *y, int64_t B, int64_t R, int64_t C, int
     a.n_stages = n_stages;
     a.flags = flags;
     a.status = status;
+    a.debug = g_na_debug.load(std::memory_order_relaxed);
+    a.wait_limit_ns = g_na_wait_ns.load(std::memory_order_relaxed);
     if (int e = launch_softmax(a, dtype, OP_FORWARD, nd->n_sm, stream, false))
         return record_cuda_error(e, "noalloc kernel launch");
     return BSM_OK;
 }
 
 }  // namespace
+
+// bsm_plan_debug(NULL, what, arg): fault injection for the launches of
+// bsm_softmax_noalloc that follow (the failure-detection tests).
+int noalloc_debug(int what, int64_t arg)
+{
+    switch (what) {
+    case BSM_DEBUG_NONE:
+        g_na_debug.store(0);
+        g_na_wait_ns.store(0);
+        return BSM_OK;
+    case BSM_DEBUG_WITHHOLD_STAGE:
+        if (arg <= 0)
+            return BSM_ERR_INVALID_ARG;
+        g_na_wait_ns.store(static_cast<uint64_t>(arg));
+        g_na_debug.store(KDEBUG_WITHHOLD_STAGE0);
+        return BSM_OK;
+    default:
+        return BSM_ERR_INVALID_ARG;
+    }
+}
+
+// The sticky status bits this entry point's kernels left on `device` (0 when
+// it never ran there); with clear != 0 they are zeroed afterwards.  Copies
+// through the array's address, taken by the first call: nothing allocates.
+// Called with the device idle (bsm_device_status synchronises it first).
+int noalloc_status(int device, uint32_t *bits, int clear)
+{
+    *bits = 0;
+    if (device < 0 || device >= 64)
+        return BSM_OK;
+    unsigned char *scratch = nullptr;
+    {
+        std::lock_guard<std::mutex> lk(g_na_mu);
+        if (g_na_dev[device].ready)
+            scratch = g_na_dev[device].scratch;
+    }
+    if (!scratch)
+        return BSM_OK;
+    uint32_t *status = reinterpret_cast<uint32_t *>(scratch + kStatusOffset);
+    if (cudaError_t e = cudaMemcpy(bits, status, sizeof(uint32_t), cudaMemcpyDeviceToHost))
+        return record_cuda_error(static_cast<int>(e), "cudaMemcpy(noalloc status)");
+    if (clear) {
+        if (cudaError_t e = cudaMemset(status, 0, 8 * sizeof(uint32_t)))
+            return record_cuda_error(static_cast<int>(e), "cudaMemset(noalloc status)");
+    }
+    return BSM_OK;
+}
+
 }  // namespace bsm
 
 extern "C" int bsm_softmax_noalloc(const void *x, void *y, int64_t B, int64_t R, int64_t C, int dtype,
