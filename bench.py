@@ -62,7 +62,7 @@ def kernel_hash() -> str:
     return hashlib.sha256(open(KERNEL_SRC, "rb").read()).hexdigest()[:16]
 
 
-def profiled_traffic(workload_k: int, dtype_name: str):
+def profiled_traffic(workload_k: int):
     """DRAM bytes per launch of the softmax kernel on workload k (steady
     state: consecutive launches, caches not flushed) from a committed ncu
     summary taken on the current kernel source, else None."""
@@ -352,7 +352,13 @@ def main():
                     help="time the Sec. 6 batched product 1 or 2 instead of the softmax")
     ap.add_argument("--long-rows", type=int, default=0,
                     help="time fp32 rows of this many elements (longer than a stage), 256 MiB in all")
+    ap.add_argument("--die-check", action="store_true",
+                    help="check the probed address -> die map: each die's SMs read only the "
+                         "chunks it maps there (then the inverse, then a random map); one JSON line")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-workloads", action="store_true",
+                    help="skip the other workloads, the policy ratios and the Sec. 6 products "
+                         "(nested under 'workloads' in the JSON line)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=20)
     args = ap.parse_args()
@@ -387,6 +393,8 @@ def main():
         g.build()
     dev = torch.cuda.current_device()
 
+    if args.die_check:
+        return run_die_check(bsm, dev)
     if args.bmm:
         return run_bmm(args, bsm, workload, ws, rank, dev)
     if args.long_rows:
@@ -463,7 +471,7 @@ def main():
     # step is nothing but its launches)
     launch_ms = total_ms / (args.steps * launches_per_step)
     achieved = bytes_step / launches_per_step / (launch_ms * 1e-3) / 1e9
-    traffic = profiled_traffic(args.workload, "f32")
+    traffic = profiled_traffic(args.workload)
 
     out = {
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": ws,
@@ -529,6 +537,15 @@ def main():
     if not args.no_cpu_baseline and rank == 0 and ws == 1:
         out["cpu_baseline"] = cpu_baseline(w)
 
+    if not args.no_workloads and ws == 1 and args.workload == 2 and args.policy == "dynamic":
+        # the paper's policies against its round-robin baseline on this very
+        # workload (Sec. 6 SOFTMAX table gives 1.08x for CBMF over RR, on
+        # Intel NNP-T), then the other workloads and the Sec. 6 products
+        out["policies"] = policy_ratios(bsm, w, x, y, stream)
+        del x, y
+        torch.cuda.empty_cache()
+        out["workloads"] = other_workloads(bsm, workload, stream, dev)
+
     if rank == 0:
         print(json.dumps(out), flush=True)
 
@@ -537,6 +554,186 @@ def main():
     if ws > 1:
         dist.destroy_process_group()
     return 0
+
+
+def _softmax_tensors(w):
+    import numpy as np
+    import torch
+    from paper_2002_07062_gb300 import workload
+    xh = w.x.view(np.int16) if w.dtype == workload.BF16 else w.x
+    x = torch.from_numpy(xh).cuda()
+    if w.dtype == workload.BF16:
+        x = x.view(torch.bfloat16)
+    return x, torch.empty_like(x)
+
+
+def _steps_for(fn, stream, target_s, lo=20, hi=20000, small=False, flush_buf=None):
+    """Steps that fill about target_s seconds, from three calibration steps."""
+    if small:
+        t, _ = time_steps_flushed(fn, 3, stream, flush_buf)
+    else:
+        t, _ = time_steps(fn, 3, stream)
+    per = max(t / 3, 1e-3)
+    return int(min(hi, max(lo, target_s * 1e3 / per)))
+
+
+def time_softmax(bsm, w, x, y, pol, stream, dev, target_s=1.0, clocks=True):
+    """One softmax workload under one policy, timed like the main line:
+    back-to-back steps under one event pair (working sets over twice the L2),
+    or step by step after an L2 flush (smaller ones).  Returns a dict."""
+    import torch
+    from paper_2002_07062_gb300 import workload
+    uniform = w.uniform
+    B, R, C = w.nslices, int(w.rows[0]), int(w.cols[0])
+
+    def step():
+        if uniform:
+            bsm.bsm_softmax_ex(x, y, B, R, C, w.dtype, pol, w.flags, stream)
+        else:
+            bsm.bsm_softmax_ragged(x, y, w.offsets, w.rows, w.cols, w.dtype, pol, w.flags, stream)
+    with torch.cuda.stream(stream):
+        step()
+    stream.synchronize()
+    plan = bsm.bsm_plan_create(x, y, w.rows, w.cols, w.dtype, pol, offsets=w.offsets, flags=w.flags)
+    st = plan.stats()
+    plan.close()
+    launches = int(st["launches"])
+    small = w.algorithmic_bytes < 2 * L2_BYTES
+    flush_buf = torch.zeros(2 * L2_BYTES // 4, dtype=torch.int32, device="cuda") if small else None
+    for _ in range(5):
+        step()
+    stream.synchronize()
+    steps = _steps_for(step, stream, target_s, small=small, flush_buf=flush_buf)
+    torch.cuda.synchronize()
+    if clocks:
+        with ClockSampler(dev) as clk:
+            total_ms, _ = (time_steps_flushed(step, steps, stream, flush_buf) if small
+                           else time_steps(step, steps, stream))
+    else:
+        clk = None
+        total_ms, _ = (time_steps_flushed(step, steps, stream, flush_buf) if small
+                       else time_steps(step, steps, stream))
+    ms = total_ms / steps
+    gbs = w.algorithmic_bytes / (ms * 1e-3) / 1e9
+    peak, peak_src = measured_peak()
+    launch_ms = ms / max(1, launches)
+    achieved = w.algorithmic_bytes / max(1, launches) / (launch_ms * 1e-3) / 1e9
+    out = {"value": round(gbs, 2), "unit": "GB/s", "ms_per_step": round(ms, 5), "steps": steps,
+           "dtype": "f32" if w.dtype == workload.F32 else "bf16",
+           "slices_per_s": round(B / (ms * 1e-3), 1),
+           "config": {"workload": w.name, "policy": bsm.POLICY_NAMES[pol],
+                      "bytes_per_step": w.algorithmic_bytes,
+                      "l2": ("working set %d KB under twice the L2: a %d MB buffer written before "
+                             "every step, each step timed alone"
+                             % (w.algorithmic_bytes >> 10, 2 * L2_BYTES // 10**6) if small else
+                             "inputs larger than L2 (%d MB vs 129 MB), no flush"
+                             % (w.algorithmic_bytes >> 20))},
+           "gpu_launches": launches * steps,
+           "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak,
+                        "unit": "GB/s", "frac": round(achieved / peak, 4),
+                        "traffic": None, "peak_source": peak_src,
+                        "kernel": "softmax_persistent", "launch_ms": round(launch_ms, 5)},
+           "device_status": bsm.bsm_device_status()}
+    if clk is not None:
+        out["clocks"] = clk.summary()
+    return out
+
+
+def policy_ratios(bsm, w, x, y, stream, target_s=0.5):
+    """Every policy on the main workload (GB/s), and the ratios of the paper's
+    policies to its round-robin baseline, beside the paper's own figure."""
+    res = {}
+    for name in ("whole_gpu", "rr", "dynamic", "cbmf", "cbmf_lb", "minimax"):
+        r = time_softmax(bsm, w, x, y, bsm.POLICIES[name], stream, None, target_s=target_s,
+                         clocks=False)
+        res[name] = r["value"]
+    rr = res["rr"]
+    return {"GBps": res,
+            "cbmf_over_rr": round(res["cbmf"] / rr, 4),
+            "cbmf_lb_over_rr": round(res["cbmf_lb"] / rr, 4),
+            "minimax_over_rr": round(res["minimax"] / rr, 4),
+            "best_over_rr": round(max(res.values()) / rr, 4),
+            "best": max(res, key=res.get),
+            "paper_context": {"cbmf_over_rr": 1.08, "what": "HW utilization, CBMF over RR, "
+                              "SOFTMAX on 384 slices of 512 x 512", "hardware": "Intel NNP-T",
+                              "source": "Sec. 6, SOFTMAX table"}}
+
+
+def time_bmm(bsm, workload, k, pol, stream, dev, target_s=1.0, clocks=True):
+    """A Sec. 6 batched product on the tensor cores: operands resident,
+    back-to-back launches, one event pair.  Returns a dict."""
+    import numpy as np
+    import torch
+    w = workload.bmm_config(k)
+    a_bits, bt_bits = w.operands()
+    a = torch.from_numpy(a_bits.view(np.int16)).cuda()
+    bt = torch.from_numpy(bt_bits.view(np.int16)).cuda()
+    c = torch.empty(w.B * w.M * w.N, dtype=torch.int16, device="cuda")
+
+    def step():
+        bsm.bsm_bmm(a, bt, c, w.B, w.M, w.N, w.K, w.out_dtype, pol, stream)
+    for _ in range(5):
+        step()
+    stream.synchronize()
+    steps = _steps_for(step, stream, target_s)
+    launches = w.B if pol == bsm.POLICY_WHOLE_GPU else 1
+    torch.cuda.synchronize()
+    clk = None
+    if clocks:
+        with ClockSampler(dev) as clk:
+            total_ms, _ = time_steps(step, steps, stream)
+    else:
+        total_ms, _ = time_steps(step, steps, stream)
+    ms = total_ms / steps
+    gbs = w.algorithmic_bytes / (ms * 1e-3) / 1e9
+    peak, peak_src = measured_peak()
+    # cuBLAS on the same operands and stream, as context
+    A3 = a.view(torch.bfloat16).view(w.B, w.M, w.K)
+    B3 = bt.view(torch.bfloat16).view(w.B, w.N, w.K)
+    with torch.cuda.stream(stream):
+        def lib_step():
+            torch.bmm(A3, B3.transpose(1, 2))
+        for _ in range(3):
+            lib_step()
+        stream.synchronize()
+        lib_ms = _median_ms(lib_step, 50, stream)
+    out = {"value": round(gbs, 2), "unit": "GB/s", "ms_per_step": round(ms, 5), "steps": steps,
+           "dtype": "bf16", "tflops": round(w.flops / (ms * 1e-3) / 1e12, 2),
+           "config": {"workload": w.name, "policy": bsm.POLICY_NAMES[pol],
+                      "bytes_per_step": w.algorithmic_bytes, "flops_per_step": w.flops,
+                      "l2": "operands + product %d MB vs 129 MB L2, no flush"
+                            % (w.algorithmic_bytes >> 20)},
+           "gpu_launches": launches * steps,
+           "roofline": {"bound": "hbm", "achieved": round(gbs, 2), "peak": peak, "unit": "GB/s",
+                        "frac": round(gbs / peak, 4), "traffic": profiled_bmm_traffic(k),
+                        "peak_source": peak_src, "kernel": "bmm_persistent",
+                        "launch_ms": round(ms / launches, 5)},
+           "torch_bmm_context_ms": round(lib_ms, 5),
+           "vs_torch_bmm_time": round(ms / lib_ms, 4),
+           "device_status": bsm.bsm_device_status()}
+    if clk is not None:
+        out["clocks"] = clk.summary()
+    del a, bt, c
+    return out
+
+
+def other_workloads(bsm, workload, stream, dev):
+    """The other softmax workloads (1, 3, 4, 5) under the default policy and
+    both Sec. 6 batched products, each timed like the main line."""
+    import torch
+    res = {}
+    for k in (1, 3, 4, 5):
+        w = workload.config(k).materialize()
+        x, y = _softmax_tensors(w)
+        r = time_softmax(bsm, w, x, y, bsm.POLICY_DYNAMIC, stream, dev)
+        r["roofline"]["traffic"] = profiled_traffic(k)
+        res["workload%d" % k] = r
+        del x, y, w
+        torch.cuda.empty_cache()
+    for k in (1, 2):
+        res["bmm_E%d" % k] = time_bmm(bsm, workload, k, bsm.POLICY_DYNAMIC, stream, dev)
+        torch.cuda.empty_cache()
+    return res
 
 
 def sweep(args, bsm, workload, stream):
@@ -725,6 +922,58 @@ def run_long_rows(args, bsm, ws, rank, dev):
     plan.close()
     if rank == 0:
         print(json.dumps(out), flush=True)
+    return 0
+
+
+def run_die_check(bsm, dev):
+    """The Sec. 4.1 bank map on GB300 (address -> die, probed by latency),
+    checked by its consequence: reading only the chunks mapped to the reader's
+    own die.  Launches of die_check_kernel, in order: the map at 128 B (the L2
+    line), its inverse, a random map of the same buffer (the control), then
+    the map and its inverse at the plans' chunk size.  A profiler's
+    lts__t_sectors_srcunit_ltcfabric / lts__t_sectors_srcunit_tex on these
+    launches is the share of the traffic that crossed dies.  Also: how often
+    the majority rule puts a 64 KiB patch on die 0, against what the map's
+    die-0 share would give if every line were an independent draw."""
+    import math
+    import numpy as np
+    import torch
+    topo = bsm.bsm_topology_probe()
+    if not topo["separable"]:
+        print(json.dumps({"die_check": "topology not separable"}))
+        return 0
+    nbytes = 256 << 20                     # larger than the L2: every read streams from DRAM
+    g = torch.Generator(device="cuda").manual_seed(0xD1E)
+    buf = torch.randint(-2**31, 2**31 - 1, (nbytes // 4,), device="cuda", dtype=torch.int32,
+                        generator=g)
+    want = int(np.bitwise_xor.reduce(buf.cpu().numpy().view(np.uint32)))
+    plan_chunk = max(128, (int(topo["granularity"]) + 127) // 128 * 128)
+    out = {"die_check": True, "buffer_bytes": nbytes, "sm_per_die": topo["sm_per_die"][:2],
+           "granularity": topo["granularity"], "plan_chunk": plan_chunk, "launches": []}
+    m128 = bsm.bsm_addr_die_map(buf, nbytes, 128)
+    m128b = bsm.bsm_addr_die_map(buf, nbytes, 128)
+    rnd = np.random.default_rng(7).integers(0, 2, m128.size).astype(np.int8)
+    mplan = bsm.bsm_addr_die_map(buf, nbytes, plan_chunk)
+    out["share_die0_128"] = round(float(np.mean(m128 == 0)), 5)
+    out["share_die0_plan_chunk"] = round(float(np.mean(mplan == 0)), 5)
+    out["probe_agreement_128"] = round(float(np.mean(m128 == m128b)), 5)
+    # majority of 64 KiB patches (input bytes only) against a binomial model
+    lines = (64 << 10) // 128
+    per = m128.reshape(-1, lines)
+    maj0 = float(np.mean((per == 0).sum(axis=1) > lines // 2))
+    p = float(np.mean(m128 == 0))
+    z = (0.5 - p) * math.sqrt(lines) / math.sqrt(max(p * (1 - p), 1e-12))
+    out["patches_64k_majority_die0"] = round(maj0, 4)
+    out["binomial_prediction"] = round(0.5 * math.erfc(z / math.sqrt(2)), 4)
+    for name, m, ch, inv in (("map 128 B", m128, 128, False), ("inverse 128 B", m128, 128, True),
+                             ("random 128 B", rnd, 128, False),
+                             ("map plan chunk", mplan, plan_chunk, False),
+                             ("inverse plan chunk", mplan, plan_chunk, True)):
+        got, ms = bsm.bsm_die_check_read(buf, nbytes, ch, m, invert=inv)
+        out["launches"].append({"what": name, "ms": round(ms, 4), "covers_once": got == want,
+                                "GBps": round(nbytes / (ms * 1e-3) / 1e9, 1)})
+    out["device_status"] = bsm.bsm_device_status()
+    print(json.dumps(out), flush=True)
     return 0
 
 

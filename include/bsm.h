@@ -154,7 +154,11 @@ int bsm_softmax_host(const void *x_host, void *y_host, int64_t B, int64_t R, int
 
 /*
  * Ragged batch: slice s has rows[s] x cols[s] elements at element offset
- * offsets[s] of x (and of y).  offsets/rows/cols are HOST arrays of
+ * offsets[s] of x (and of y).  The paper's slices are uniform (Sec. 2); its
+ * load balance (Sec. 4.2) exists because patches differ in size, and a batch
+ * of slices of different shapes is where they do.  The paper has no call of
+ * this shape; it is the ragged form the scheduling contract asks for, with
+ * the same per-row computation as bsm_softmax.  offsets/rows/cols are HOST arrays of
  * num_slices entries, copied.  Slices must not overlap each other; they need
  * not be contiguous or ordered.  Same errors as bsm_softmax.
  */
@@ -298,8 +302,11 @@ int bsm_plan_desc_init(bsm_plan_desc *d);
  * Synchronous; allocates device memory owned by the plan. */
 int bsm_plan_create(bsm_plan **plan, const bsm_plan_desc *d);
 
-/* Launch the plan on `stream` (async).  Allocates nothing and does not
- * synchronise.  Executions of one plan must not overlap in time (they share
+/* Launch the plan on `stream` (async): the persistent kernel walks the
+ * table built up front (Sec. 5: the scheduler fills its mapping table once,
+ * then feeds patch coordinates to one templated kernel; Sec. 4.1: each
+ * compute unit takes its bank's patches in order).  Allocates nothing and
+ * does not synchronise.  Executions of one plan must not overlap in time (they share
  * the plan's queue counters and its long-row partials): keep them on one
  * stream, or order them. */
 int bsm_plan_execute(const bsm_plan *plan, bsm_stream_t stream);
@@ -329,6 +336,45 @@ typedef struct {
 
 int bsm_plan_get_stats(const bsm_plan *plan, bsm_plan_stats *out);
 void bsm_plan_destroy(bsm_plan *plan);
+
+/* ---- the schedule a plan was built with (for checking it against an
+ * independent restatement of Sec. 4.1 / 4.2, and for diagnosis) ----
+ * bsm_plan_get_schedule fills the scalar fields always; each array pointer
+ * the caller sets (non-NULL) receives its data -- a first call with all
+ * arrays NULL gives the sizes.  Host only; no device access.
+ *   queue    n_items entries: for every queue slot, the index of its patch in
+ *            slice order (the order of bsm_plan_layout_host's phase 0); the
+ *            slots of die d's queue are [queue_begin[d], + queue_len[d]).
+ *            Written only for the queue policies (n_queues > 0).
+ *   x_map    n_map_chunks entries: die of every map_chunk_bytes chunk of x,
+ *            as probed at plan creation (CBMF, CBMF_LB, MINIMAX on a
+ *            separable device; otherwise n_map_chunks = 0).
+ *   y_map    the same for y, when the table counted output bytes and y != x.
+ *   moved    n_moved entries: the patches the Sec. 4.2 balance moved, in
+ *            order (CBMF_LB).
+ * units, l_near, l_far and tie_seed are the planner's other inputs (SMs per
+ * die, integer latency weights, the tie coin's seed).  Returns
+ * BSM_ERR_INVALID_ARG for a null plan or out. */
+typedef struct {
+    int32_t n_queues;           /* 0: the policy takes patches statically (RR, WHOLE_GPU) */
+    int32_t count_output_bytes;
+    int32_t queue_begin[BSM_MAX_DIES];
+    int32_t queue_len[BSM_MAX_DIES];
+    int32_t units[BSM_MAX_DIES];
+    int64_t l_near, l_far;
+    uint64_t tie_seed;
+    int64_t n_items;
+    int64_t map_chunk_bytes;
+    int64_t n_map_chunks;
+    int64_t n_moved;
+    int32_t *queue;
+    int8_t *x_map;
+    int8_t *y_map;
+    int32_t *moved;
+} bsm_plan_schedule;
+
+int bsm_plan_get_schedule(const bsm_plan *plan, bsm_plan_schedule *out);
+
 
 /* ---- the patch table alone, on the host (no GPU needed) ----
  * Cuts the descriptor's slices into patches exactly as bsm_plan_create does,
@@ -368,6 +414,15 @@ typedef struct {
 
 int bsm_plan_layout_host(const bsm_plan_desc *d, int32_t n_sm, int64_t smem_optin, bsm_patch *phase0,
                          int64_t cap0, bsm_patch *phase1, int64_t cap1, bsm_layout *out);
+
+/* The patch records as the kernel reads them from the plan's device table
+ * (queue policies: in queue order, so that slot k holds patch queue[k]),
+ * phase 0 or 1 (the second launch of rows cut into segments).  At most cap
+ * records go to out (host, caller-owned); *n_out receives the count.
+ * Synchronous (a device-to-host copy).  BSM_ERR_INVALID_ARG for a null plan
+ * or n_out, a phase other than 0/1, or a capacity without an array. */
+int bsm_plan_device_table(const bsm_plan *plan, int phase, bsm_patch *out, int64_t cap,
+                          int64_t *n_out);
 
 /* Fault injection on one plan, for the library's failure-detection tests
  * (nothing here faults, traps or hangs the GPU).  plan = NULL applies
@@ -424,6 +479,20 @@ int bsm_topology_probe(int device, int force, bsm_topology *out);
  * Synchronous. */
 int bsm_addr_die_map(int device, const void *ptr, int64_t bytes, int64_t chunk, int8_t *die_out);
 
+/* Check of such a map (Sec. 4.1: a patch is "created" in the bank that holds
+ * it): the SMs of each die read, once, only the chunk-byte chunks of
+ * [ptr, ptr + bytes) that die_of_chunk (host, bytes / chunk entries of 0 or
+ * 1) places on their die -- with invert != 0, only the others.  Run under a
+ * profiler, the L2's die-to-die (fabric) sector counters then say how much
+ * of the traffic the map failed to keep on its die: none for a right map,
+ * all of it inverted.  *xor_out gets the XOR of every 32-bit word read (each
+ * chunk is read once, so it equals the XOR of the whole buffer); *ms_out
+ * (may be NULL) the kernel's time.  bytes a multiple of chunk, chunk of 16;
+ * ptr 16-byte aligned.  Needs a separable topology (else
+ * BSM_ERR_UNSUPPORTED).  Synchronous; allocates and frees small tables. */
+int bsm_die_check_read(int device, const void *ptr, int64_t bytes, int64_t chunk,
+                       const int8_t *die_of_chunk, int invert, uint32_t *xor_out, float *ms_out);
+
 /* Raw probe matrix, for diagnostics: lat_out (host, BSM_MAX_SM x n_lines,
  * row = %smid) gets the mean cycles of a dependent L2-hit load from that SM to
  * byte offset line_off[i] of a 32 MiB scratch buffer (line_off multiples of
@@ -471,7 +540,9 @@ int bsm_schedule_host(const bsm_schedule_desc *d, bsm_schedule_out *out);
 
 /* ---- status ---- */
 
-/* Sticky device-side status word of `device` (-1 = current), BSM_DEV_* bits:
+/* Sticky device-side status word of `device` (-1 = current), BSM_DEV_* bits
+ * (the paper has no error reporting; the word is the contract's "device
+ * faults are sticky" rule):
  * the library's own word OR-ed with the words of bsm_softmax_noalloc's fixed
  * array (so a timeout or bounds error there is not lost).  Synchronises the
  * device; allocates nothing.  bsm_device_status_clear zeroes both.  (The

@@ -83,6 +83,17 @@ class PlanStats(ctypes.Structure):
                 ("long_items", ctypes.c_int64)]
 
 
+class PlanSchedule(ctypes.Structure):
+    _fields_ = [("n_queues", ctypes.c_int32), ("count_output_bytes", ctypes.c_int32),
+                ("queue_begin", ctypes.c_int32 * MAX_DIES), ("queue_len", ctypes.c_int32 * MAX_DIES),
+                ("units", ctypes.c_int32 * MAX_DIES), ("l_near", ctypes.c_int64),
+                ("l_far", ctypes.c_int64), ("tie_seed", ctypes.c_uint64), ("n_items", ctypes.c_int64),
+                ("map_chunk_bytes", ctypes.c_int64), ("n_map_chunks", ctypes.c_int64),
+                ("n_moved", ctypes.c_int64), ("queue", c_i32p),
+                ("x_map", ctypes.POINTER(ctypes.c_int8)), ("y_map", ctypes.POINTER(ctypes.c_int8)),
+                ("moved", c_i32p)]
+
+
 class Topology(ctypes.Structure):
     _fields_ = [("device", ctypes.c_int32), ("n_sm", ctypes.c_int32), ("n_die", ctypes.c_int32),
                 ("separable", ctypes.c_int32), ("sm_die", ctypes.c_int8 * MAX_SM),
@@ -140,6 +151,11 @@ def lib():
         "bsm_plan_get_stats": ([vp, ctypes.POINTER(PlanStats)], ctypes.c_int),
         "bsm_plan_destroy": ([vp], None),
         "bsm_plan_debug": ([vp, ctypes.c_int, i64], ctypes.c_int),
+        "bsm_plan_get_schedule": ([vp, ctypes.POINTER(PlanSchedule)], ctypes.c_int),
+        "bsm_plan_device_table": ([vp, ctypes.c_int, ctypes.POINTER(Patch), i64, ctypes.POINTER(i64)],
+                                  ctypes.c_int),
+        "bsm_die_check_read": ([ctypes.c_int, vp, i64, i64, ctypes.POINTER(ctypes.c_int8), ctypes.c_int,
+                                ctypes.POINTER(u32), ctypes.POINTER(ctypes.c_float)], ctypes.c_int),
         "bsm_plan_layout_host": ([ctypes.POINTER(PlanDesc), i32, i64, ctypes.POINTER(Patch), i64,
                                   ctypes.POINTER(Patch), i64, ctypes.POINTER(Layout)], ctypes.c_int),
         "bsm_cache_clear": ([], None),
@@ -393,6 +409,63 @@ def bsm_plan_get_stats(plan: Plan) -> dict:
         v = getattr(s, name)
         out[name] = list(v) if not isinstance(v, (int, float)) else v
     return out
+
+
+def _patch_array(buf, n):
+    dt = np.dtype([(name, np.int64 if ct is ctypes.c_int64 else np.int32) for name, ct in Patch._fields_])
+    return np.frombuffer(bytes(buf), dtype=dt, count=n) if n else np.zeros(0, dt)
+
+
+def bsm_plan_get_schedule(plan: Plan) -> dict:
+    """The schedule a plan was built with: queue slots (phase-0 patch index
+    in slice order), the probed address -> die maps, moved patches and the
+    planner's inputs (see include/bsm.h)."""
+    sc = PlanSchedule()
+    _check(lib().bsm_plan_get_schedule(plan.handle, ctypes.byref(sc)), "bsm_plan_get_schedule")
+    q = np.zeros(max(sc.n_items, 1), np.int32)
+    xm = np.zeros(max(sc.n_map_chunks, 1), np.int8)
+    ym = np.full(max(sc.n_map_chunks, 1), -1, np.int8)
+    mv = np.zeros(max(sc.n_moved, 1), np.int32)
+    sc.queue = q.ctypes.data_as(c_i32p)
+    sc.x_map = xm.ctypes.data_as(ctypes.POINTER(ctypes.c_int8))
+    sc.y_map = ym.ctypes.data_as(ctypes.POINTER(ctypes.c_int8))
+    sc.moved = mv.ctypes.data_as(c_i32p)
+    _check(lib().bsm_plan_get_schedule(plan.handle, ctypes.byref(sc)), "bsm_plan_get_schedule")
+    n, nm = sc.n_items, sc.n_map_chunks
+    return {"n_queues": sc.n_queues, "count_output_bytes": sc.count_output_bytes,
+            "queue_begin": list(sc.queue_begin), "queue_len": list(sc.queue_len),
+            "units": list(sc.units), "l_near": sc.l_near, "l_far": sc.l_far,
+            "tie_seed": sc.tie_seed, "n_items": n, "map_chunk_bytes": sc.map_chunk_bytes,
+            "queue": q[:n] if sc.n_queues else None,
+            "x_map": xm[:nm], "y_map": ym[:nm] if nm and ym[0] >= 0 else None,
+            "moved": mv[:sc.n_moved]}
+
+
+def bsm_plan_device_table(plan: Plan, phase: int = 0) -> np.ndarray:
+    """The plan's device patch table as the kernel reads it (structured
+    array with the fields of bsm_patch)."""
+    n = ctypes.c_int64()
+    _check(lib().bsm_plan_device_table(plan.handle, phase, None, 0, ctypes.byref(n)),
+           "bsm_plan_device_table")
+    buf = (Patch * max(n.value, 1))()
+    _check(lib().bsm_plan_device_table(plan.handle, phase, buf, n.value, ctypes.byref(n)),
+           "bsm_plan_device_table")
+    return _patch_array(buf, n.value)
+
+
+def bsm_die_check_read(ptr, nbytes: int, chunk: int, die_of_chunk, invert: bool = False,
+                       device: int = -1):
+    """SMs of each die read only the chunks the map places on their die (or,
+    inverted, the others); returns (XOR of the words read, kernel ms)."""
+    m = _np(die_of_chunk, np.int8)
+    assert len(m) * chunk == nbytes
+    xo = ctypes.c_uint32()
+    ms = ctypes.c_float()
+    _check(lib().bsm_die_check_read(device, _dptr(ptr, nbytes, "buffer"), nbytes, chunk,
+                                    m.ctypes.data_as(ctypes.POINTER(ctypes.c_int8)),
+                                    1 if invert else 0, ctypes.byref(xo), ctypes.byref(ms)),
+           "bsm_die_check_read")
+    return xo.value, ms.value
 
 
 DEBUG_NONE, DEBUG_WITHHOLD_STAGE, DEBUG_CORRUPT_PATCH = 0, 1, 2

@@ -36,6 +36,8 @@ int record_cuda_error(int cuda_error, const char *where)
 
 int topology_get(int device, int force, bsm_topology *out);
 int addr_die_map_host(int device, const void *ptr, int64_t bytes, int64_t chunk, int8_t *die_out);
+int die_check_host(int device, const void *ptr, int64_t bytes, int64_t chunk, const int8_t *die_of_chunk,
+                   int invert, uint32_t *xor_out, float *ms_out);
 int probe_latency_host(int device, const std::vector<int64_t> &lines, int reps, std::vector<float> &lat,
                        std::vector<int32_t> &seen);
 
@@ -144,6 +146,17 @@ struct bsm_plan {
     cudaGraphExec_t whole_graph = nullptr;   // ... captured once as a CUDA graph (or null)
     void *blob = nullptr;            // device tables (patches, slice index, sm_die, heads)
     bsm_plan_stats stats{};
+    // the schedule as built (bsm_plan_get_schedule): the phase-0 patch index
+    // (slice order) of every queue slot, the address -> die maps and the
+    // planner's inputs
+    std::vector<int32_t> queue;
+    std::vector<int8_t> xmap, ymap;
+    std::vector<int32_t> moved;
+    int64_t map_chunk = 0;
+    int32_t units[BSM_MAX_DIES] = {0, 0, 0, 0};
+    int64_t w_near = 0, w_far = 0;
+    int count_y = 0;
+    uint64_t tie_seed = 0;
     // identity of the plan for the cache
     const void *x = nullptr;
     void *y = nullptr;
@@ -631,6 +644,16 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
                 return rc;
             }
             queue = qi;
+            p->xmap = xmap;
+            p->ymap = count_y && d->y != d->x ? ymap : std::vector<int8_t>();
+            p->map_chunk = chunk;
+            p->moved.assign(moved.begin(), moved.begin() + so.n_moved);
+            for (int b = 0; b < nb; ++b)
+                p->units[b] = units[b];
+            p->w_near = sd.l_near;
+            p->w_far = sd.l_far;
+            p->count_y = count_y ? 1 : 0;
+            p->tie_seed = d->tie_seed;
             n_queues = nb;
             int32_t pos = 0;
             for (int b = 0; b < nb; ++b) {
@@ -668,6 +691,7 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
         }
     }
 
+    p->queue = queue;
     // ---- queue policies store the patches in queue order (die 0's queue,
     // then die 1's, ...), so a claimed queue slot is the patch record itself
     if (!queue.empty()) {
@@ -1012,6 +1036,81 @@ int bsm_plan_get_stats(const bsm_plan *plan, bsm_plan_stats *out)
         return BSM_ERR_INVALID_ARG;
     *out = plan->stats;
     return BSM_OK;
+}
+
+int bsm_plan_get_schedule(const bsm_plan *plan, bsm_plan_schedule *out)
+{
+    if (!plan || !out)
+        return BSM_ERR_INVALID_ARG;
+    const bsm_plan &p = *plan;
+    const bool queued = p.args.mode == PULL_QUEUE;
+    out->n_queues = queued ? p.args.n_queues : 0;
+    out->count_output_bytes = p.count_y;
+    for (int b = 0; b < BSM_MAX_DIES; ++b) {
+        out->queue_begin[b] = queued ? p.args.queue_begin[b] : 0;
+        out->queue_len[b] = queued ? p.args.queue_len[b] : 0;
+        out->units[b] = p.units[b];
+    }
+    out->l_near = p.w_near;
+    out->l_far = p.w_far;
+    out->tie_seed = p.tie_seed;
+    out->n_items = p.stats.n_items;
+    out->map_chunk_bytes = p.map_chunk;
+    out->n_map_chunks = static_cast<int64_t>(p.xmap.size());
+    out->n_moved = static_cast<int64_t>(p.moved.size());
+    if (out->queue && queued)
+        std::memcpy(out->queue, p.queue.data(), sizeof(int32_t) * p.queue.size());
+    if (out->x_map && !p.xmap.empty())
+        std::memcpy(out->x_map, p.xmap.data(), p.xmap.size());
+    if (out->y_map && !p.ymap.empty())
+        std::memcpy(out->y_map, p.ymap.data(), p.ymap.size());
+    if (out->moved && !p.moved.empty())
+        std::memcpy(out->moved, p.moved.data(), sizeof(int32_t) * p.moved.size());
+    return BSM_OK;
+}
+
+int bsm_plan_device_table(const bsm_plan *plan, int phase, bsm_patch *out, int64_t cap, int64_t *n_out)
+{
+    if (!plan || !n_out || (phase != 0 && phase != 1) || cap < 0 || (cap > 0 && !out))
+        return BSM_ERR_INVALID_ARG;
+    const KernelArgs &a = phase ? plan->args1 : plan->args;
+    const int64_t n = phase && !plan->n_phase1 ? 0 : a.n_items;
+    *n_out = n;
+    const int64_t m = std::min(n, cap);
+    if (m <= 0)
+        return BSM_OK;
+    std::vector<Item> items(static_cast<size_t>(m));
+    std::vector<LongSeg> segs;
+    int prev = -1;
+    cudaGetDevice(&prev);
+    cudaSetDevice(plan->device);
+    cudaError_t e = cudaMemcpy(items.data(), a.items, sizeof(Item) * items.size(), cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess && a.segs) {
+        segs.resize(static_cast<size_t>(m));
+        e = cudaMemcpy(segs.data(), a.segs, sizeof(LongSeg) * segs.size(), cudaMemcpyDeviceToHost);
+    }
+    if (prev >= 0)
+        cudaSetDevice(prev);
+    if (e != cudaSuccess)
+        return cuda_error(e, "cudaMemcpy(plan table)");
+    for (int64_t i = 0; i < m; ++i) {
+        out[i].elem_offset = items[i].off;
+        out[i].cols = items[i].C;
+        out[i].nrows = items[i].nrows;
+        out[i].row0 = items[i].row0;
+        out[i].slice_rows = items[i].R;
+        out[i].col0 = segs.empty() ? 0 : segs[i].col0;
+        out[i].part_count = segs.empty() ? 0 : segs[i].part_count;
+    }
+    return BSM_OK;
+}
+
+int bsm_die_check_read(int device, const void *ptr, int64_t bytes, int64_t chunk, const int8_t *die_of_chunk,
+                       int invert, uint32_t *xor_out, float *ms_out)
+{
+    if (device < 0 && cudaGetDevice(&device) != cudaSuccess)
+        return BSM_ERR_NO_DEVICE;
+    BSM_GUARD(die_check_host(device, ptr, bytes, chunk, die_of_chunk, invert, xor_out, ms_out))
 }
 
 int bsm_plan_debug(bsm_plan *plan, int what, int64_t arg)

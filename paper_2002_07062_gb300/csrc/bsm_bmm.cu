@@ -144,11 +144,6 @@ __device__ __forceinline__ void tma_load_3d(void *dst, const CUtensorMap *map, i
         : "memory");
 }
 
-// Shared-memory matrix descriptor of a K-major operand tile whose rows are
-// 128 bytes (64 bf16) laid out with the 128-byte swizzle by TMA: start
-// address (16-byte units), leading-dimension offset (unused for this
-// layout: 1), stride between 8-row groups = 1024 bytes, descriptor version 1,
-// base offset 0 (tiles are 1024-byte aligned), swizzle mode 2 = 128 bytes.
 // Tile record of queue entry idx: read from the plan, or computed when the
 // plan keeps tiles in their natural order (slice, row block, column block).
 template <int BN> __device__ __forceinline__ GemmItem tile_at(const GemmArgs &a, int32_t idx)
@@ -162,6 +157,11 @@ template <int BN> __device__ __forceinline__ GemmItem tile_at(const GemmArgs &a,
     return GemmItem{s, (r / a.tiles_n) * 128, (r % a.tiles_n) * BN, 0};
 }
 
+// Shared-memory matrix descriptor of a K-major operand tile whose rows are
+// 128 bytes (64 bf16) laid out with the 128-byte swizzle by TMA: start
+// address (16-byte units), leading-dimension offset (unused for this
+// layout: 1), stride between 8-row groups = 1024 bytes, descriptor version 1,
+// base offset 0 (tiles are 1024-byte aligned), swizzle mode 2 = 128 bytes.
 __device__ __forceinline__ uint64_t smem_desc(const void *tile)
 {
     const uint64_t a = (saddr(tile) & 0x3FFFFu) >> 4;

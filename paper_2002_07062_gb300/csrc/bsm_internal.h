@@ -151,6 +151,10 @@ int probe_latency_run(const void *buf, const int64_t *line_off_dev, int n_lines,
                       int grid, float *lat_dev, uint32_t *claim_dev);
 int probe_map_run(const void *buf, int64_t bytes, int64_t chunk, int reps, const int8_t *sm_die_dev, int want_die,
                   int n_sm, uint32_t *counter_dev, float *lat_dev);
+// Die-map check (bsm_probe.cu): SMs of die d read the chunks listed for d.
+int die_check_run(const void *buf, int64_t n_chunks, int64_t chunk, const int32_t *list0, int64_t len0,
+                  const int32_t *list1, int64_t len1, uint32_t *ctr, const int8_t *sm_die_dev, int n_sm,
+                  uint32_t *sink, float *ms);
 
 // Remember a failing CUDA call for bsm_last_cuda_error (bsm_api.cpp);
 // returns BSM_ERR_CUDA.

@@ -101,6 +101,56 @@ __global__ void probe_map_kernel(const unsigned char *buf, int64_t buf_bytes, in
     }
 }
 
+
+// Die-map check: every CTA reads, from the chunks of `buf`, only those in
+// the list of its own SM's die (claimed 32 at a time from that die's
+// counter), each chunk once, with 16-byte L2-only loads.  With the lists
+// built from an address -> die map (chunks of die d for SMs of die d), the
+// L2's fabric counters then show how much of that traffic still crossed to
+// the other die: none if the map is right.  The XOR of every word read goes
+// to `sink` (the host checks it covers the buffer).  List entries are
+// chunk indices checked on the host (< n_chunks); an index outside is
+// skipped here too.
+__global__ void die_check_kernel(const uint4 *buf, int64_t n_chunks, int32_t chunk_vecs,
+                                 const int32_t *list0, int64_t len0, const int32_t *list1, int64_t len1,
+                                 uint32_t *ctr, const int8_t *sm_die, uint32_t *sink)
+{
+    const int lane = threadIdx.x & 31;
+    const int my = sm_die[probe_smid() & (BSM_MAX_SM - 1)];
+    if (my != 0 && my != 1)
+        return;
+    const int32_t *list = my == 0 ? list0 : list1;
+    const int64_t len = my == 0 ? len0 : len1;
+    uint4 acc = make_uint4(0u, 0u, 0u, 0u);
+    for (int64_t guard = 0; guard <= len / 32 + 1; ++guard) {
+        uint32_t base = 0;
+        if (lane == 0)
+            base = atomicAdd(&ctr[my], 32u);
+        base = __shfl_sync(0xFFFFFFFFu, base, 0);
+        if (base >= len)
+            break;
+        for (int j = 0; j < 32 && base + j < len; ++j) {
+            const int64_t c = list[base + j];
+            if (c < 0 || c >= n_chunks)
+                continue;
+            const uint4 *p = buf + c * chunk_vecs;
+            for (int v = lane; v < chunk_vecs; v += 32) {
+                uint4 w;
+                asm volatile("ld.global.cg.v4.u32 {%0, %1, %2, %3}, [%4];"
+                             : "=r"(w.x), "=r"(w.y), "=r"(w.z), "=r"(w.w)
+                             : "l"(p + v));
+                acc.x ^= w.x;
+                acc.y ^= w.y;
+                acc.z ^= w.z;
+                acc.w ^= w.w;
+            }
+        }
+    }
+    const uint32_t a = acc.x ^ acc.y ^ acc.z ^ acc.w;
+    if (a)
+        atomicXor(sink, a);
+}
+
 }  // namespace
 
 int probe_latency_run(const void *buf, const int64_t *line_off_dev, int n_lines, int reps, int grid,
@@ -124,6 +174,31 @@ int probe_map_run(const void *buf, int64_t bytes, int64_t chunk, int reps, const
     cudaError_t e = cudaGetLastError();
     if (e == cudaSuccess)
         e = cudaDeviceSynchronize();
+    return static_cast<int>(e);
+}
+
+}  // namespace bsm
+
+namespace bsm {
+
+int die_check_run(const void *buf, int64_t n_chunks, int64_t chunk, const int32_t *list0, int64_t len0,
+                  const int32_t *list1, int64_t len1, uint32_t *ctr, const int8_t *sm_die_dev, int n_sm,
+                  uint32_t *sink, float *ms)
+{
+    cudaEvent_t e0 = nullptr, e1 = nullptr;
+    cudaEventCreate(&e0);
+    cudaEventCreate(&e1);
+    cudaEventRecord(e0);
+    die_check_kernel<<<n_sm, 256>>>(static_cast<const uint4 *>(buf), n_chunks, static_cast<int32_t>(chunk / 16),
+                                    list0, len0, list1, len1, ctr, sm_die_dev, sink);
+    cudaError_t e = cudaGetLastError();
+    cudaEventRecord(e1);
+    if (e == cudaSuccess)
+        e = cudaDeviceSynchronize();
+    if (e == cudaSuccess && ms)
+        cudaEventElapsedTime(ms, e0, e1);
+    cudaEventDestroy(e0);
+    cudaEventDestroy(e1);
     return static_cast<int>(e);
 }
 

@@ -303,4 +303,71 @@ int addr_die_map_host(int device, const void *ptr, int64_t bytes, int64_t chunk,
     return rc;
 }
 
+// Die-map check: the SMs of each die read only the chunks listed for that
+// die (the chunks `die_of_chunk` places there, or with invert the others),
+// so that a profiler's L2 fabric counters can say how much of the traffic
+// still crossed dies.  *xor_out = XOR of every 32-bit word read (each chunk
+// is read once: it equals the XOR of the whole buffer).
+int die_check_host(int device, const void *ptr, int64_t bytes, int64_t chunk, const int8_t *die_of_chunk,
+                   int invert, uint32_t *xor_out, float *ms_out)
+{
+    if (!ptr || !die_of_chunk || !xor_out || bytes <= 0 || chunk <= 0 || (chunk & 15) || bytes % chunk ||
+        (reinterpret_cast<uintptr_t>(ptr) & 15))
+        return BSM_ERR_INVALID_ARG;
+    const int64_t n_chunks = bytes / chunk;
+    if (n_chunks >= INT32_MAX || chunk / 16 > INT32_MAX)
+        return BSM_ERR_UNSUPPORTED;
+    std::vector<int32_t> list[2];
+    for (int64_t c = 0; c < n_chunks; ++c) {
+        const int d = die_of_chunk[c];
+        if (d != 0 && d != 1)
+            return BSM_ERR_INVALID_ARG;
+        list[invert ? 1 - d : d].push_back(static_cast<int32_t>(c));
+    }
+    bsm_topology t;
+    int rc = topology_get(device, 0, &t);
+    if (rc)
+        return rc;
+    if (!t.separable)
+        return BSM_ERR_UNSUPPORTED;
+    if (cudaSetDevice(device) != cudaSuccess)
+        return BSM_ERR_NO_DEVICE;
+    int32_t *d_list = nullptr;
+    int8_t *d_sm = nullptr;
+    uint32_t *d_words = nullptr;   // two counters, then the XOR sink
+    float ms = 0.0f;
+    do {
+        if ((rc = cuda_fail(cudaMalloc(&d_list, sizeof(int32_t) * static_cast<size_t>(n_chunks)))))
+            break;
+        if (!list[0].empty() &&
+            (rc = cuda_fail(cudaMemcpy(d_list, list[0].data(), sizeof(int32_t) * list[0].size(),
+                                       cudaMemcpyHostToDevice))))
+            break;
+        if (!list[1].empty() &&
+            (rc = cuda_fail(cudaMemcpy(d_list + list[0].size(), list[1].data(), sizeof(int32_t) * list[1].size(),
+                                       cudaMemcpyHostToDevice))))
+            break;
+        if ((rc = cuda_fail(cudaMalloc(&d_sm, BSM_MAX_SM))))
+            break;
+        if ((rc = cuda_fail(cudaMemcpy(d_sm, t.sm_die, BSM_MAX_SM, cudaMemcpyHostToDevice))))
+            break;
+        if ((rc = cuda_fail(cudaMalloc(&d_words, 4 * sizeof(uint32_t)))))
+            break;
+        if ((rc = cuda_fail(cudaMemset(d_words, 0, 4 * sizeof(uint32_t)))))
+            break;
+        if ((rc = cuda_fail(static_cast<cudaError_t>(
+                 die_check_run(ptr, n_chunks, chunk, d_list, static_cast<int64_t>(list[0].size()),
+                               d_list + list[0].size(), static_cast<int64_t>(list[1].size()), d_words, d_sm,
+                               t.n_sm, d_words + 2, &ms)))))
+            break;
+        rc = cuda_fail(cudaMemcpy(xor_out, d_words + 2, sizeof(uint32_t), cudaMemcpyDeviceToHost));
+    } while (false);
+    cudaFree(d_list);
+    cudaFree(d_sm);
+    cudaFree(d_words);
+    if (!rc && ms_out)
+        *ms_out = ms;
+    return rc;
+}
+
 }  // namespace bsm

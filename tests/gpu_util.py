@@ -104,20 +104,68 @@ def check_rows_against_oracle(w: workload.Workload, y_host: np.ndarray, pairs):
 
 def check_all_against_oracle(w: workload.Workload, y_host: np.ndarray):
     y64, yr = O.softmax_batched(w.x, w.offsets, w.rows, w.cols, w.flags)
-    covered = np.zeros(w.x.size, bool)
-    for s in range(w.nslices):
-        n = int(w.rows[s]) * int(w.cols[s])
-        covered[int(w.offsets[s]):int(w.offsets[s]) + n] = True
+    if is_packed(w) and w.numel == w.x.size:
+        covered = slice(None)                  # the slices cover the whole array
+    else:
+        covered = np.zeros(w.x.size, bool)
+        for s in range(w.nslices):
+            n = int(w.rows[s]) * int(w.cols[s])
+            covered[int(w.offsets[s]):int(w.offsets[s]) + n] = True
     if w.dtype == workload.F32:
         g = y_host[covered].astype(np.float64)
         o = y64[covered]
-        assert np.array_equal(np.isnan(g), np.isnan(o))
-        m = ~np.isnan(o)
-        err = float(np.max(np.abs(g[m] - o[m]))) if m.any() else 0.0
+        nan_o = np.isnan(o)
+        if nan_o.any():
+            assert np.array_equal(np.isnan(g), nan_o)
+            m = ~nan_o
+            err = float(np.max(np.abs(g[m] - o[m]))) if m.any() else 0.0
+        else:
+            # no NaN expected: a NaN in g makes the maximum NaN, which fails
+            np.subtract(g, o, out=g)
+            np.abs(g, out=g)
+            err = float(np.max(g)) if g.size else 0.0
         assert err <= FP32_TOL, err
         return err
     gi = y_host[covered].astype(np.int32)
     wi = yr[covered].astype(np.int32)
-    err = float(np.max(np.abs(gi - wi))) if gi.size else 0.0
+    np.subtract(gi, wi, out=gi)
+    np.abs(gi, out=gi)
+    err = float(np.max(gi)) if gi.size else 0.0
     assert err <= BF16_ULPS, err
     return err
+
+
+def check_every_element_against_oracle(w: workload.Workload, y_host: np.ndarray,
+                                       max_elems: int = 1 << 26):
+    """check_all_against_oracle over every slice of w, in groups of slices of
+    at most about max_elems elements (the oracle's double-precision output of
+    a whole 4.6 GB workload would need tens of GB of host memory at once).
+    Returns the worst error (fp32: absolute; bf16: ulps)."""
+    worst = 0.0
+    packed = is_packed(w)
+
+    def n_last(s):
+        return int(w.rows[s]) * int(w.cols[s])
+    s0 = 0
+    while s0 < w.nslices:
+        s1, n = s0, 0
+        while s1 < w.nslices and (s1 == s0 or n + int(w.rows[s1]) * int(w.cols[s1]) <= max_elems):
+            n += int(w.rows[s1]) * int(w.cols[s1])
+            s1 += 1
+        if packed:
+            # consecutive slices are one contiguous range of x and y
+            a, b = int(w.offsets[s0]), int(w.offsets[s1 - 1]) + n_last(s1 - 1)
+            sub = workload.Workload(w.name, w.dtype, w.rows[s0:s1], w.cols[s0:s1],
+                                    w.offsets[s0:s1] - a, w.flags, w.seed, w.sigma, w.x[a:b])
+            ys = y_host[a:b]
+        else:
+            idx = np.arange(s0, s1)
+            sub = workload.slice_sample(w, idx)
+            ys = np.empty_like(sub.x)
+            for j, s in enumerate(idx):
+                m = n_last(s)
+                ys[int(sub.offsets[j]):int(sub.offsets[j]) + m] = \
+                    y_host[int(w.offsets[s]):int(w.offsets[s]) + m]
+        worst = max(worst, check_all_against_oracle(sub, ys))
+        s0 = s1
+    return worst
