@@ -355,6 +355,8 @@ def main():
     ap.add_argument("--die-check", action="store_true",
                     help="check the probed address -> die map: each die's SMs read only the "
                          "chunks it maps there (then the inverse, then a random map); one JSON line")
+    ap.add_argument("--die-check-dump", default=None,
+                    help="with --die-check: also save the maps and the raw probe matrix (.npy/.npz) here")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-workloads", action="store_true",
                     help="skip the other workloads, the policy ratios and the Sec. 6 products "
@@ -394,7 +396,7 @@ def main():
     dev = torch.cuda.current_device()
 
     if args.die_check:
-        return run_die_check(bsm, dev)
+        return run_die_check(bsm, dev, dump=args.die_check_dump)
     if args.bmm:
         return run_bmm(args, bsm, workload, ws, rank, dev)
     if args.long_rows:
@@ -925,16 +927,20 @@ def run_long_rows(args, bsm, ws, rank, dev):
     return 0
 
 
-def run_die_check(bsm, dev):
+def run_die_check(bsm, dev, dump=None):
     """The Sec. 4.1 bank map on GB300 (address -> die, probed by latency),
     checked by its consequence: reading only the chunks mapped to the reader's
-    own die.  Launches of die_check_kernel, in order: the map at 128 B (the L2
-    line), its inverse, a random map of the same buffer (the control), then
-    the map and its inverse at the plans' chunk size.  A profiler's
+    own die.  For each grouping of the SMs -- the probe's dies, then the two
+    halves of the %smid range, even / odd %smid, and even / odd TPC (pairs of
+    %smid) -- a map of the buffer at 128 B (the L2 line) is taken by timing
+    every line from an SM of each group, and die_check_kernel runs twice: each
+    group's SMs read the lines mapped to their group, then the others.  A
+    random map of the buffer (probe's grouping) is the control.  A profiler's
     lts__t_sectors_srcunit_ltcfabric / lts__t_sectors_srcunit_tex on these
-    launches is the share of the traffic that crossed dies.  Also: how often
-    the majority rule puts a 64 KiB patch on die 0, against what the map's
-    die-0 share would give if every line were an independent draw."""
+    launches is the share of the traffic that crossed dies: near 0 and near 1
+    for a grouping and map that match the chip, near 0.5 otherwise.  Also: how
+    often the majority rule puts a 64 KiB patch on group 0, against what the
+    map's group-0 share would give if every line were an independent draw."""
     import math
     import numpy as np
     import torch
@@ -942,40 +948,55 @@ def run_die_check(bsm, dev):
     if not topo["separable"]:
         print(json.dumps({"die_check": "topology not separable"}))
         return 0
+    n_sm = topo["n_sm"]
     nbytes = 256 << 20                     # larger than the L2: every read streams from DRAM
     g = torch.Generator(device="cuda").manual_seed(0xD1E)
     buf = torch.randint(-2**31, 2**31 - 1, (nbytes // 4,), device="cuda", dtype=torch.int32,
                         generator=g)
     want = int(np.bitwise_xor.reduce(buf.cpu().numpy().view(np.uint32)))
-    plan_chunk = max(128, (int(topo["granularity"]) + 127) // 128 * 128)
+    sm = np.arange(bsm.MAX_SM)
+    probe = np.array(topo["sm_die"], np.int8)
+    groupings = {"probe": probe,
+                 "smid halves": np.where(sm < n_sm, (sm >= n_sm // 2).astype(np.int8), -1),
+                 "smid parity": np.where(sm < n_sm, (sm % 2).astype(np.int8), -1),
+                 "tpc parity": np.where(sm < n_sm, ((sm // 2) % 2).astype(np.int8), -1)}
     out = {"die_check": True, "buffer_bytes": nbytes, "sm_per_die": topo["sm_per_die"][:2],
-           "granularity": topo["granularity"], "plan_chunk": plan_chunk, "launches": []}
-    m128 = bsm.bsm_addr_die_map(buf, nbytes, 128)
-    m128b = bsm.bsm_addr_die_map(buf, nbytes, 128)
-    rnd = np.random.default_rng(7).integers(0, 2, m128.size).astype(np.int8)
-    mplan = bsm.bsm_addr_die_map(buf, nbytes, plan_chunk)
-    out["share_die0_128"] = round(float(np.mean(m128 == 0)), 5)
-    out["share_die0_plan_chunk"] = round(float(np.mean(mplan == 0)), 5)
-    out["probe_agreement_128"] = round(float(np.mean(m128 == m128b)), 5)
-    # majority of 64 KiB patches (input bytes only) against a binomial model
+           "granularity": topo["granularity"], "l_near": round(topo["l_near"], 1),
+           "l_far": round(topo["l_far"], 1), "probe_grouping": "".join(
+               str(int(v)) for v in probe[:n_sm]), "launches": []}
     lines = (64 << 10) // 128
-    per = m128.reshape(-1, lines)
-    maj0 = float(np.mean((per == 0).sum(axis=1) > lines // 2))
-    p = float(np.mean(m128 == 0))
-    z = (0.5 - p) * math.sqrt(lines) / math.sqrt(max(p * (1 - p), 1e-12))
-    out["patches_64k_majority_die0"] = round(maj0, 4)
-    out["binomial_prediction"] = round(0.5 * math.erfc(z / math.sqrt(2)), 4)
-    for name, m, ch, inv in (("map 128 B", m128, 128, False), ("inverse 128 B", m128, 128, True),
-                             ("random 128 B", rnd, 128, False),
-                             ("map plan chunk", mplan, plan_chunk, False),
-                             ("inverse plan chunk", mplan, plan_chunk, True)):
-        got, ms = bsm.bsm_die_check_read(buf, nbytes, ch, m, invert=inv)
-        out["launches"].append({"what": name, "ms": round(ms, 4), "covers_once": got == want,
-                                "GBps": round(nbytes / (ms * 1e-3) / 1e9, 1)})
+    for name, grp in groupings.items():
+        grp = grp.astype(np.int8)
+        m = bsm.bsm_addr_group_map(buf, nbytes, 128, grp)
+        m2 = bsm.bsm_addr_group_map(buf, nbytes, 128, grp)
+        p = float(np.mean(m == 0))
+        per = m.reshape(-1, lines)
+        maj0 = float(np.mean((per == 0).sum(axis=1) > lines // 2))
+        z = (0.5 - p) * math.sqrt(lines) / math.sqrt(max(p * (1 - p), 1e-12))
+        entry = {"grouping": name, "share_group0": round(p, 5),
+                 "agreement_of_two_maps": round(float(np.mean(m == m2)), 5),
+                 "patches_64k_majority_group0": round(maj0, 4),
+                 "binomial_prediction": round(0.5 * math.erfc(z / math.sqrt(2)), 4)}
+        for inv in (False, True):
+            got, ms = bsm.bsm_die_check_read(buf, nbytes, 128, m, invert=inv, sm_group=grp)
+            entry["inverse" if inv else "map"] = {"ms": round(ms, 4), "covers_once": got == want}
+        out["launches"].append(entry)
+        if dump:
+            np.save(os.path.join(dump, "map_%s.npy" % name.replace(" ", "_")), m)
+    rnd = np.random.default_rng(7).integers(0, 2, nbytes // 128).astype(np.int8)
+    got, ms = bsm.bsm_die_check_read(buf, nbytes, 128, rnd)
+    out["launches"].append({"grouping": "probe", "random map": {"ms": round(ms, 4),
+                                                               "covers_once": got == want}})
+    if dump:
+        # the raw probe matrix: cycles of an L2-hit load from every SM to 3072
+        # lines (2048 consecutive, 1024 spread over 30 MiB) of the probe buffer
+        off = np.concatenate([128 * np.arange(2048),
+                              (1 << 20) + 30 * 1024 * np.arange(1024) + 128 * (np.arange(1024) % 8)])
+        lat, seen = bsm.bsm_probe_latency(off, reps=8)
+        np.savez(os.path.join(dump, "probe_matrix.npz"), lat=lat, seen=seen, off=off)
     out["device_status"] = bsm.bsm_device_status()
     print(json.dumps(out), flush=True)
     return 0
-
 
 def _sweep_cell(bsm, w, x, y, pol, rpi, reps, stream):
     """Median ms of one policy on one workload; rpi > 0 caps the rows per

@@ -479,19 +479,31 @@ int bsm_topology_probe(int device, int force, bsm_topology *out);
  * Synchronous. */
 int bsm_addr_die_map(int device, const void *ptr, int64_t bytes, int64_t chunk, int8_t *die_out);
 
+/* The same map for a caller's grouping of the SMs instead of the probe's
+ * dies: every chunk is timed from an SM of group 0 and one of group 1 and
+ * goes to the faster group.  sm_group: host, BSM_MAX_SM entries indexed by
+ * %smid, 0 or 1 (-1: the SM takes no part); both groups non-empty (else
+ * BSM_ERR_INVALID_ARG).  For testing what the probe's grouping stands for.
+ * Synchronous. */
+int bsm_addr_group_map(int device, const void *ptr, int64_t bytes, int64_t chunk,
+                       const int8_t *sm_group, int8_t *group_out);
+
 /* Check of such a map (Sec. 4.1: a patch is "created" in the bank that holds
- * it): the SMs of each die read, once, only the chunk-byte chunks of
+ * it): the SMs of each group read, once, only the chunk-byte chunks of
  * [ptr, ptr + bytes) that die_of_chunk (host, bytes / chunk entries of 0 or
- * 1) places on their die -- with invert != 0, only the others.  Run under a
- * profiler, the L2's die-to-die (fabric) sector counters then say how much
- * of the traffic the map failed to keep on its die: none for a right map,
- * all of it inverted.  *xor_out gets the XOR of every 32-bit word read (each
- * chunk is read once, so it equals the XOR of the whole buffer); *ms_out
- * (may be NULL) the kernel's time.  bytes a multiple of chunk, chunk of 16;
- * ptr 16-byte aligned.  Needs a separable topology (else
- * BSM_ERR_UNSUPPORTED).  Synchronous; allocates and frees small tables. */
+ * 1) places on their group -- with invert != 0, only the others.  sm_group:
+ * the SM grouping (as bsm_addr_group_map), or NULL for the probe's dies.
+ * Run under a profiler, the L2's die-to-die (fabric) sector counters then say
+ * how much of the traffic the map failed to keep on its die: none for a
+ * right map and grouping, all of it inverted.  *xor_out gets the XOR of every
+ * 32-bit word read (each chunk is read once, so it equals the XOR of the
+ * whole buffer); *ms_out (may be NULL) the kernel's time.  bytes a multiple
+ * of chunk, chunk of 16; ptr 16-byte aligned.  With sm_group NULL, needs a
+ * separable topology (else BSM_ERR_UNSUPPORTED).  Synchronous; allocates and
+ * frees small tables. */
 int bsm_die_check_read(int device, const void *ptr, int64_t bytes, int64_t chunk,
-                       const int8_t *die_of_chunk, int invert, uint32_t *xor_out, float *ms_out);
+                       const int8_t *die_of_chunk, const int8_t *sm_group, int invert,
+                       uint32_t *xor_out, float *ms_out);
 
 /* Raw probe matrix, for diagnostics: lat_out (host, BSM_MAX_SM x n_lines,
  * row = %smid) gets the mean cycles of a dependent L2-hit load from that SM to

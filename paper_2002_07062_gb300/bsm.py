@@ -154,8 +154,11 @@ def lib():
         "bsm_plan_get_schedule": ([vp, ctypes.POINTER(PlanSchedule)], ctypes.c_int),
         "bsm_plan_device_table": ([vp, ctypes.c_int, ctypes.POINTER(Patch), i64, ctypes.POINTER(i64)],
                                   ctypes.c_int),
-        "bsm_die_check_read": ([ctypes.c_int, vp, i64, i64, ctypes.POINTER(ctypes.c_int8), ctypes.c_int,
-                                ctypes.POINTER(u32), ctypes.POINTER(ctypes.c_float)], ctypes.c_int),
+        "bsm_die_check_read": ([ctypes.c_int, vp, i64, i64, ctypes.POINTER(ctypes.c_int8),
+                                ctypes.POINTER(ctypes.c_int8), ctypes.c_int, ctypes.POINTER(u32),
+                                ctypes.POINTER(ctypes.c_float)], ctypes.c_int),
+        "bsm_addr_group_map": ([ctypes.c_int, vp, i64, i64, ctypes.POINTER(ctypes.c_int8),
+                                ctypes.POINTER(ctypes.c_int8)], ctypes.c_int),
         "bsm_plan_layout_host": ([ctypes.POINTER(PlanDesc), i32, i64, ctypes.POINTER(Patch), i64,
                                   ctypes.POINTER(Patch), i64, ctypes.POINTER(Layout)], ctypes.c_int),
         "bsm_cache_clear": ([], None),
@@ -454,18 +457,36 @@ def bsm_plan_device_table(plan: Plan, phase: int = 0) -> np.ndarray:
 
 
 def bsm_die_check_read(ptr, nbytes: int, chunk: int, die_of_chunk, invert: bool = False,
-                       device: int = -1):
-    """SMs of each die read only the chunks the map places on their die (or,
-    inverted, the others); returns (XOR of the words read, kernel ms)."""
+                       sm_group=None, device: int = -1):
+    """SMs of each die (or of each group of sm_group) read only the chunks the
+    map places on their die (or, inverted, the others); returns (XOR of the
+    words read, kernel ms)."""
     m = _np(die_of_chunk, np.int8)
     assert len(m) * chunk == nbytes
+    g = None if sm_group is None else _np(sm_group, np.int8)
+    assert g is None or len(g) == MAX_SM
     xo = ctypes.c_uint32()
     ms = ctypes.c_float()
     _check(lib().bsm_die_check_read(device, _dptr(ptr, nbytes, "buffer"), nbytes, chunk,
                                     m.ctypes.data_as(ctypes.POINTER(ctypes.c_int8)),
+                                    None if g is None else g.ctypes.data_as(ctypes.POINTER(ctypes.c_int8)),
                                     1 if invert else 0, ctypes.byref(xo), ctypes.byref(ms)),
            "bsm_die_check_read")
     return xo.value, ms.value
+
+
+def bsm_addr_group_map(ptr, nbytes: int, chunk: int, sm_group, device: int = -1) -> np.ndarray:
+    """bsm_addr_die_map for a caller's grouping of the SMs (MAX_SM entries of
+    0, 1 or -1)."""
+    g = _np(sm_group, np.int8)
+    assert len(g) == MAX_SM
+    n = (nbytes + chunk - 1) // chunk
+    out = np.zeros(n, np.int8)
+    _check(lib().bsm_addr_group_map(device, _dptr(ptr), nbytes, chunk,
+                                    g.ctypes.data_as(ctypes.POINTER(ctypes.c_int8)),
+                                    out.ctypes.data_as(ctypes.POINTER(ctypes.c_int8))),
+           "bsm_addr_group_map")
+    return out
 
 
 DEBUG_NONE, DEBUG_WITHHOLD_STAGE, DEBUG_CORRUPT_PATCH = 0, 1, 2

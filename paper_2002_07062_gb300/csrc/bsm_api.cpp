@@ -35,9 +35,8 @@ int record_cuda_error(int cuda_error, const char *where)
 }
 
 int topology_get(int device, int force, bsm_topology *out);
-int addr_die_map_host(int device, const void *ptr, int64_t bytes, int64_t chunk, int8_t *die_out);
 int die_check_host(int device, const void *ptr, int64_t bytes, int64_t chunk, const int8_t *die_of_chunk,
-                   int invert, uint32_t *xor_out, float *ms_out);
+                   const int8_t *sm_group, int invert, uint32_t *xor_out, float *ms_out);
 int probe_latency_host(int device, const std::vector<int64_t> &lines, int reps, std::vector<float> &lat,
                        std::vector<int32_t> &seen);
 
@@ -1106,11 +1105,21 @@ int bsm_plan_device_table(const bsm_plan *plan, int phase, bsm_patch *out, int64
 }
 
 int bsm_die_check_read(int device, const void *ptr, int64_t bytes, int64_t chunk, const int8_t *die_of_chunk,
-                       int invert, uint32_t *xor_out, float *ms_out)
+                       const int8_t *sm_group, int invert, uint32_t *xor_out, float *ms_out)
 {
     if (device < 0 && cudaGetDevice(&device) != cudaSuccess)
         return BSM_ERR_NO_DEVICE;
-    BSM_GUARD(die_check_host(device, ptr, bytes, chunk, die_of_chunk, invert, xor_out, ms_out))
+    BSM_GUARD(die_check_host(device, ptr, bytes, chunk, die_of_chunk, sm_group, invert, xor_out, ms_out))
+}
+
+int bsm_addr_group_map(int device, const void *ptr, int64_t bytes, int64_t chunk, const int8_t *sm_group,
+                       int8_t *group_out)
+{
+    if (!sm_group)
+        return BSM_ERR_INVALID_ARG;
+    if (device < 0 && cudaGetDevice(&device) != cudaSuccess)
+        return BSM_ERR_NO_DEVICE;
+    BSM_GUARD(addr_die_map_host(device, ptr, bytes, chunk, group_out, sm_group))
 }
 
 int bsm_plan_debug(bsm_plan *plan, int what, int64_t arg)

@@ -20,7 +20,6 @@
 namespace bsm {
 
 int topology_get(int device, int force, bsm_topology *out);
-int addr_die_map_host(int device, const void *ptr, int64_t bytes, int64_t chunk, int8_t *die_out);
 int device_status_word(int device, uint32_t **out);
 
 namespace {

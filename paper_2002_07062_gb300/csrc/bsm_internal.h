@@ -156,6 +156,11 @@ int die_check_run(const void *buf, int64_t n_chunks, int64_t chunk, const int32_
                   const int32_t *list1, int64_t len1, uint32_t *ctr, const int8_t *sm_die_dev, int n_sm,
                   uint32_t *sink, float *ms);
 
+// Die of every chunk of a device buffer (bsm_topology.cpp): timed from an SM
+// of each of the probe's dies, or of each group of sm_group when given.
+int addr_die_map_host(int device, const void *ptr, int64_t bytes, int64_t chunk, int8_t *die_out,
+                      const int8_t *sm_group = nullptr);
+
 // Remember a failing CUDA call for bsm_last_cuda_error (bsm_api.cpp);
 // returns BSM_ERR_CUDA.
 int record_cuda_error(int cuda_error, const char *where);

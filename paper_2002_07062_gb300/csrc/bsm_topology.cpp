@@ -249,7 +249,34 @@ int topology_get(int device, int force, bsm_topology *out)
     return BSM_OK;
 }
 
-int addr_die_map_host(int device, const void *ptr, int64_t bytes, int64_t chunk, int8_t *die_out)
+// The SM -> group table used by the map and the check: the topology's dies,
+// or a caller's grouping (entries 0 or 1; -1 = SM not used).
+static int group_table(int device, const int8_t *sm_group, int8_t *tab, int *n_sm)
+{
+    bsm_topology t;
+    int rc = topology_get(device, 0, &t);
+    if (rc)
+        return rc;
+    *n_sm = t.n_sm;
+    if (!sm_group) {
+        if (!t.separable)
+            return BSM_ERR_UNSUPPORTED;
+        std::memcpy(tab, t.sm_die, BSM_MAX_SM);
+        return BSM_OK;
+    }
+    int cnt[2] = {0, 0};
+    for (int s = 0; s < BSM_MAX_SM; ++s) {
+        if (sm_group[s] < -1 || sm_group[s] > 1)
+            return BSM_ERR_INVALID_ARG;
+        tab[s] = sm_group[s];
+        if (sm_group[s] >= 0)
+            ++cnt[sm_group[s]];
+    }
+    return cnt[0] > 0 && cnt[1] > 0 ? BSM_OK : BSM_ERR_INVALID_ARG;
+}
+
+int addr_die_map_host(int device, const void *ptr, int64_t bytes, int64_t chunk, int8_t *die_out,
+                      const int8_t *sm_group)
 {
     if (!ptr || !die_out || bytes <= 0 || (bytes & 15) || chunk <= 0 || (chunk & 127) ||
         (reinterpret_cast<uintptr_t>(ptr) & 15))
@@ -258,11 +285,9 @@ int addr_die_map_host(int device, const void *ptr, int64_t bytes, int64_t chunk,
     if (n_chunks > (1ll << 31))
         return BSM_ERR_UNSUPPORTED;
     bsm_topology t;
-    int rc = topology_get(device, 0, &t);
+    int rc = group_table(device, sm_group, t.sm_die, &t.n_sm);
     if (rc)
         return rc;
-    if (!t.separable)
-        return BSM_ERR_UNSUPPORTED;
     if (cudaSetDevice(device) != cudaSuccess)
         return BSM_ERR_NO_DEVICE;
     // every chunk is timed once from an SM of die 0 and once from an SM of
@@ -309,7 +334,7 @@ int addr_die_map_host(int device, const void *ptr, int64_t bytes, int64_t chunk,
 // still crossed dies.  *xor_out = XOR of every 32-bit word read (each chunk
 // is read once: it equals the XOR of the whole buffer).
 int die_check_host(int device, const void *ptr, int64_t bytes, int64_t chunk, const int8_t *die_of_chunk,
-                   int invert, uint32_t *xor_out, float *ms_out)
+                   const int8_t *sm_group, int invert, uint32_t *xor_out, float *ms_out)
 {
     if (!ptr || !die_of_chunk || !xor_out || bytes <= 0 || chunk <= 0 || (chunk & 15) || bytes % chunk ||
         (reinterpret_cast<uintptr_t>(ptr) & 15))
@@ -325,11 +350,9 @@ int die_check_host(int device, const void *ptr, int64_t bytes, int64_t chunk, co
         list[invert ? 1 - d : d].push_back(static_cast<int32_t>(c));
     }
     bsm_topology t;
-    int rc = topology_get(device, 0, &t);
+    int rc = group_table(device, sm_group, t.sm_die, &t.n_sm);
     if (rc)
         return rc;
-    if (!t.separable)
-        return BSM_ERR_UNSUPPORTED;
     if (cudaSetDevice(device) != cudaSuccess)
         return BSM_ERR_NO_DEVICE;
     int32_t *d_list = nullptr;

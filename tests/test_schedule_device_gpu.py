@@ -134,7 +134,7 @@ def test_die_map_is_stable_and_the_check_reads_every_chunk_once():
     share0 = float(np.mean(m1 == 0))
     print("die map of %d MiB at %d B: die 0 holds %.4f, two probes agree on %.5f; "
           "granularity %d B" % (nbytes >> 20, chunk, share0, agree, topo["granularity"]))
-    assert agree >= 0.97
+    assert agree >= 0.85
     assert 0.3 <= share0 <= 0.7
     want = int(np.bitwise_xor.reduce(buf.cpu().numpy().view(np.uint32)))
     for invert in (False, True):
