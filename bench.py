@@ -735,6 +735,12 @@ def other_workloads(bsm, workload, stream, dev):
     for k in (1, 2):
         res["bmm_E%d" % k] = time_bmm(bsm, workload, k, bsm.POLICY_DYNAMIC, stream, dev)
         torch.cuda.empty_cache()
+    # rows longer than a shared-memory stage (256 MiB of input each)
+    for C, dt, name in ((65536, workload.F32, "fp32_256KiB"), (262144, workload.F32, "fp32_1MiB"),
+                        (1048576, workload.F32, "fp32_4MiB"), (65536, workload.BF16, "bf16_128KiB"),
+                        (262144, workload.BF16, "bf16_512KiB"), (1048576, workload.BF16, "bf16_2MiB")):
+        res["long_rows_" + name] = time_long_rows(bsm, C, dt, stream, dev)
+        torch.cuda.empty_cache()
     return res
 
 
@@ -785,10 +791,19 @@ def sweep(args, bsm, workload, stream):
     bmm_sweep(bsm, workload, stream)
 
 
+def _moved_factor(st, op="forward"):
+    """Bytes a plan moves per algorithmic byte: rows split over groups of CTAs
+    and rows staged whole read x once; rows streamed twice read it again
+    (forward: 1.5, backward: 5/3 of the algorithmic bytes at most)."""
+    if st["group_rows"] and st["group_rows"] == st["long_items"]:
+        return 1.0
+    return 1.5 if op == "forward" else 5 / 3
+
+
 def long_row_sweep(bsm, workload, stream):
-    """Rows longer than a shared-memory stage (streamed twice in chunks):
-    GB/s of algorithmic traffic and of the bytes actually moved (the row is
-    read twice: 1.5x the algorithmic bytes forward, 5/3x backward)."""
+    """Rows longer than a shared-memory stage: GB/s of algorithmic traffic,
+    forward (rows split over groups of CTAs, or streamed twice) and backward
+    (streamed twice)."""
     import torch
     for dtype, name in ((workload.F32, "fp32"), (workload.BF16, "bf16")):
         tdt = torch.float32 if dtype == workload.F32 else torch.bfloat16
@@ -797,6 +812,9 @@ def long_row_sweep(bsm, workload, stream):
             R = max(1, (256 << 20) // (C * es))        # 256 MiB of input
             x = torch.randn(R * C, device="cuda").to(tdt)
             y = torch.empty_like(x)
+            plan = bsm.bsm_plan_create(x, y, [R], [C], dtype, bsm.POLICY_DYNAMIC)
+            st = plan.stats()
+            plan.close()
 
             def step():
                 bsm.bsm_softmax(x, y, 1, R, C, dtype, bsm.POLICY_DYNAMIC, stream)
@@ -809,7 +827,9 @@ def long_row_sweep(bsm, workload, stream):
                               "%s %d rows x %d (%d KiB rows)" % (name, R, C, C * es >> 10),
                               "policy": "dynamic", "ms": round(med, 4),
                               "GBps": round(alg / (med * 1e-3) / 1e9, 2),
-                              "moved_GBps": round(1.5 * alg / (med * 1e-3) / 1e9, 2)}), flush=True)
+                              "group_k": st["group_k"], "launches": st["launches"],
+                              "moved_GBps": round(_moved_factor(st) * alg / (med * 1e-3) / 1e9, 2)}),
+                  flush=True)
             dy = torch.randn(R * C, device="cuda").to(tdt)
 
             def bstep():
@@ -826,6 +846,51 @@ def long_row_sweep(bsm, workload, stream):
                               "moved_GBps": round(5 / 3 * alg / (med * 1e-3) / 1e9, 2)}), flush=True)
             del x, y, dy
             torch.cuda.empty_cache()
+
+
+def time_long_rows(bsm, C, dtype, stream, dev, target_s=0.5):
+    """Softmax of rows of C elements longer than a shared-memory stage, 256
+    MiB of input, the default policy: one entry of the JSON line."""
+    import torch
+    from paper_2002_07062_gb300 import workload
+    es = 4 if dtype == workload.F32 else 2
+    R = max(1, (256 << 20) // (C * es))
+    g = torch.Generator(device="cuda").manual_seed(0x2002070600 + C + dtype)
+    x = torch.randn(R * C, device="cuda", generator=g)
+    if dtype == workload.BF16:
+        x = x.to(torch.bfloat16)
+    y = torch.empty_like(x)
+    plan = bsm.bsm_plan_create(x, y, [R], [C], dtype, bsm.POLICY_DYNAMIC)
+    st = plan.stats()
+
+    def step():
+        plan.execute(stream)
+    for _ in range(5):
+        step()
+    stream.synchronize()
+    steps = _steps_for(step, stream, target_s)
+    with ClockSampler(dev) as clk:
+        total_ms, _ = time_steps(step, steps, stream)
+    ms = total_ms / steps
+    alg = 2 * R * C * es
+    peak, peak_src = measured_peak()
+    gbs = alg / (ms * 1e-3) / 1e9
+    plan.close()
+    kernel = "softmax_group" if st["group_rows"] else "softmax_persistent (long rows)"
+    return {"value": round(gbs, 2), "unit": "GB/s", "ms_per_step": round(ms, 5), "steps": steps,
+            "dtype": "f32" if dtype == workload.F32 else "bf16",
+            "config": {"workload": "%s %d rows x %d (%d KiB rows), 256 MiB, random normal"
+                                   % ("fp32" if dtype == workload.F32 else "bf16", R, C, C * es >> 10),
+                       "policy": "dynamic", "bytes_per_step": alg,
+                       "l2": "inputs larger than L2 (256 MiB vs 129 MB), no flush"},
+            "plan": {"group_k": st["group_k"], "n_groups": st["n_groups"], "launches": st["launches"],
+                     "stage_bytes": st["stage_bytes"]},
+            "gpu_launches": int(st["launches"]) * steps,
+            "roofline": {"bound": "hbm", "achieved": round(gbs, 2), "peak": peak, "unit": "GB/s",
+                         "frac": round(gbs / peak, 4), "traffic": None, "peak_source": peak_src,
+                         "kernel": kernel, "launch_ms": round(ms / max(1, st["launches"]), 5),
+                         "moved_bytes_per_step": int(_moved_factor(st) * alg)},
+            "clocks": clk.summary(), "device_status": bsm.bsm_device_status()}
 
 
 def run_bmm(args, bsm, workload, ws, rank, dev):
@@ -917,9 +982,10 @@ def run_long_rows(args, bsm, ws, rank, dev):
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
            "data": "synthetic", "config": {"workload": "fp32 %d rows x %d" % (R, C),
                                            "policy": "dynamic", "bytes_per_step": alg},
-           "moved_GBps": round(1.5 * alg / (ms * 1e-3) / 1e9, 2),
+           "moved_GBps": round(_moved_factor(st) * alg / (ms * 1e-3) / 1e9, 2),
            "gpu_launches": int(st["launches"]) * args.steps,
-           "plan": {k: st[k] for k in ("n_items", "long_items", "launches", "stage_bytes", "n_stages")},
+           "plan": {k: st[k] for k in ("n_items", "long_items", "launches", "stage_bytes", "n_stages",
+                                       "group_rows", "group_k", "n_groups")},
            "clocks": clk.summary(), "device_status": bsm.bsm_device_status()}
     plan.close()
     if rank == 0:

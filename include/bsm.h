@@ -331,7 +331,10 @@ typedef struct {
     int32_t steal;              /* 1 if CTAs steal from other dies' queues */
     int64_t map_chunk_bytes;    /* granularity of the address->die map used */
     double plan_ms;             /* host time spent in bsm_plan_create */
-    int64_t long_items;         /* rows longer than a stage (two passes over chunks) */
+    int64_t long_items;         /* rows longer than a stage (group rows included) */
+    int64_t group_rows;         /* rows split over groups of CTAs (one cooperative launch) */
+    int32_t group_k;            /* CTAs per group */
+    int32_t n_groups;           /* groups of that launch */
 } bsm_plan_stats;
 
 int bsm_plan_get_stats(const bsm_plan *plan, bsm_plan_stats *out);
@@ -406,8 +409,8 @@ typedef struct {
 typedef struct {
     int64_t stage_bytes;        /* bytes per shared-memory stage */
     int32_t n_stages;           /* stages per CTA */
-    int32_t pad;
-    int64_t n_patches;          /* phase 0 (the first or only launch) */
+    int32_t group_k;            /* CTAs per group of the rows split over groups (0: none) */
+    int64_t n_patches;          /* phase 0 (the first or only launch), group rows included */
     int64_t n_patches_phase1;   /* segments of rows cut into several (the second launch) */
     int64_t long_rows;          /* rows longer than a stage */
 } bsm_layout;

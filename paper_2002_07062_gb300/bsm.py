@@ -64,7 +64,7 @@ class Patch(ctypes.Structure):
 
 
 class Layout(ctypes.Structure):
-    _fields_ = [("stage_bytes", ctypes.c_int64), ("n_stages", ctypes.c_int32), ("pad", ctypes.c_int32),
+    _fields_ = [("stage_bytes", ctypes.c_int64), ("n_stages", ctypes.c_int32), ("group_k", ctypes.c_int32),
                 ("n_patches", ctypes.c_int64), ("n_patches_phase1", ctypes.c_int64),
                 ("long_rows", ctypes.c_int64)]
 
@@ -80,7 +80,8 @@ class PlanStats(ctypes.Structure):
                 ("stage_bytes", ctypes.c_int32), ("n_stages", ctypes.c_int32),
                 ("grid", ctypes.c_int32), ("launches", ctypes.c_int32), ("steal", ctypes.c_int32),
                 ("map_chunk_bytes", ctypes.c_int64), ("plan_ms", ctypes.c_double),
-                ("long_items", ctypes.c_int64)]
+                ("long_items", ctypes.c_int64), ("group_rows", ctypes.c_int64),
+                ("group_k", ctypes.c_int32), ("n_groups", ctypes.c_int32)]
 
 
 class PlanSchedule(ctypes.Structure):
@@ -568,7 +569,7 @@ def bsm_plan_layout_host(rows, cols, dtype: int, policy: int, n_sm: int, smem_op
     a0 = np.frombuffer(bytes(p0), dtype=dt, count=n0) if n0 else np.zeros(0, dt)
     a1 = np.frombuffer(bytes(p1), dtype=dt, count=n1) if n1 else np.zeros(0, dt)
     return {"stage_bytes": out.stage_bytes, "n_stages": out.n_stages, "long_rows": out.long_rows,
-            "phase0": a0, "phase1": a1}
+            "group_k": out.group_k, "phase0": a0, "phase1": a1}
 
 
 def bsm_schedule_host(patches: Sequence, maps: Sequence, n_banks: int, tie_seed: int,

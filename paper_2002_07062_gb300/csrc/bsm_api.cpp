@@ -141,6 +141,9 @@ struct bsm_plan {
     };
     bsm::KernelArgs args1{};         // phase 1 of plans with rows longer than a stage
     int64_t n_phase1 = 0;
+    bsm::KernelArgs argsg{};         // rows over groups of CTAs (one cooperative launch)
+    int64_t n_group = 0;
+    int grid_g = 0;
     std::vector<Launch> whole_gpu;   // WHOLE_GPU: one launch per slice
     cudaGraphExec_t whole_graph = nullptr;   // ... captured once as a CUDA graph (or null)
     void *blob = nullptr;            // device tables (patches, slice index, sm_die, heads)
@@ -149,6 +152,8 @@ struct bsm_plan {
     // (slice order) of every queue slot, the address -> die maps and the
     // planner's inputs
     std::vector<int32_t> queue;
+    int32_t q_begin[BSM_MAX_DIES] = {0, 0, 0, 0}, q_len[BSM_MAX_DIES] = {0, 0, 0, 0};
+    int32_t q_count = 0;
     std::vector<int8_t> xmap, ymap;
     std::vector<int32_t> moved;
     int64_t map_chunk = 0;
@@ -271,12 +276,81 @@ struct PatchLayout {
     std::vector<int32_t> slice_first, slice_first1;
     int64_t n_parts = 0;                // segments of rows cut into several
     int64_t long_rows = 0;              // rows longer than a stage
+    // rows split over groups of CTAs (forward): one record per row, slice
+    // order; the group launch's own stage figures
+    std::vector<Item> items_g;
+    std::vector<int32_t> slice_first_g;
+    int32_t group_k = 0, n_groups = 0;
+    int64_t stage_g = 0;
+    int n_stages_g = 0;
 };
+
+// Rows over groups of CTAs (forward pass).  A row longer than one stage is
+// cut into K parts, each staged whole by one CTA of a group of K (one read of
+// every element, one launch).  K: the fewest CTAs whose parts fit a third of
+// the shared memory (three stages: one row being written, the next one
+// reduced, a third being loaded), raised up to twice that where more SMs then
+// work (groups of n_sm / K CTAs leave n_sm mod K idle: 152 SMs take K = 4, 8,
+// 19, 38 or 76 whole).  Used when the batch's long rows fill the groups'
+// waves at least two thirds (so the one launch beats the two-launch cut of
+// few long rows into segments, which reads each row twice); K depends on
+// the longest such row and the device only, never on the policy.
+int choose_groups(const std::vector<SliceView> &slices, int es, int n_sm, int64_t smem_optin, PatchLayout &L)
+{
+    const int64_t avail = smem_optin - kSmemHeader;
+    const int64_t long_cap = max_row_bytes_for(smem_optin);
+    const int64_t vec = 16 / es;                 // elements per 16-byte vector
+    int64_t n_cand = 0, lmax = 0;
+    for (const SliceView &v : slices)
+        if (v.R > 0 && int64_t(v.C) * es > long_cap) {
+            n_cand += v.R;
+            lmax = std::max<int64_t>(lmax, v.C);
+        }
+    if (n_cand == 0)
+        return 0;
+    auto stage_for = [&](int64_t k) {
+        const int64_t part = ((lmax + k - 1) / k + vec - 1) / vec * vec;
+        return (part * es + 127) & ~int64_t(127);
+    };
+    const int64_t part_cap = (avail / 3) & ~int64_t(127);
+    const int64_t kmin = std::max<int64_t>(2, (lmax * es + part_cap - 1) / part_cap);
+    int64_t best_k = 0, best_used = 0;
+    for (int64_t k = kmin; k <= std::min<int64_t>({int64_t(kMaxGroup), 2 * kmin, int64_t(n_sm)}); ++k) {
+        if (avail / stage_for(k) < 3)
+            continue;
+        const int64_t used = (n_sm / k) * k;
+        if (used > best_used) {
+            best_used = used;
+            best_k = k;
+        }
+    }
+    if (best_k == 0)
+        return 0;
+    const int64_t G = n_sm / best_k;
+    const int64_t waves = (n_cand + G - 1) / G;
+    if (3 * n_cand < 2 * waves * G)
+        return 0;
+    L.group_k = static_cast<int32_t>(best_k);
+    L.n_groups = static_cast<int32_t>(G);
+    L.stage_g = stage_for(best_k);
+    L.n_stages_g = static_cast<int>(std::min<int64_t>(kMaxStages, avail / L.stage_g));
+    return 1;
+}
 
 int cut_patches(const bsm_plan_desc *d, const std::vector<SliceView> &slices, int64_t max_row, int n_sm,
                 int64_t smem_optin, PatchLayout &L)
 {
     const int es = esize(d->dtype);
+    // ---- rows over groups of CTAs first; the other rows set the stages
+    const bool groups = d->op == BSM_OP_FORWARD && choose_groups(slices, es, n_sm, smem_optin, L);
+    const int64_t long_cap = max_row_bytes_for(smem_optin);
+    auto is_group_row = [&](const SliceView &v) { return groups && v.R > 0 && int64_t(v.C) * es > long_cap; };
+    if (groups) {
+        max_row = 0;
+        for (const SliceView &v : slices)
+            if (v.R > 0 && !is_group_row(v))
+                max_row = std::max<int64_t>(max_row, int64_t(v.C) * es);
+    }
     // ---- stages: one CTA per SM, as many stages as fit the shared memory
     const int64_t avail = smem_optin - kSmemHeader;
     const int in_arrays = d->op == BSM_OP_BACKWARD ? 2 : 1;   // inputs sharing a stage
@@ -326,6 +400,8 @@ int cut_patches(const bsm_plan_desc *d, const std::vector<SliceView> &slices, in
     // (its second read mostly hits L2)
     int64_t n_long_rows = 0, n_short_rows = 0;
     for (const SliceView &v : slices) {
+        if (is_group_row(v))
+            continue;
         if (v.R > 0 && int64_t(v.C) * es > stage / in_arrays)
             n_long_rows += v.R;
         else
@@ -350,17 +426,30 @@ int cut_patches(const bsm_plan_desc *d, const std::vector<SliceView> &slices, in
     slice_first1.assign(slices.size() + 1, 0);
     int64_t &n_parts = L.n_parts;
     int64_t &long_rows = L.long_rows;
+    L.slice_first_g.assign(slices.size() + 1, 0);
     size_t s = 0;
     while (s < slices.size()) {
         slice_first[s] = static_cast<int32_t>(items.size());
         slice_first1[s] = static_cast<int32_t>(items1.size());
+        L.slice_first_g[s] = static_cast<int32_t>(L.items_g.size());
         const SliceView &v = slices[s];
+        if (is_group_row(v)) {
+            // one record per row, for the group launch
+            if (L.items_g.size() + size_t(v.R) >= static_cast<size_t>(INT32_MAX))
+                return BSM_ERR_UNSUPPORTED;
+            long_rows += v.R;
+            for (int32_t r = 0; r < v.R; ++r)
+                L.items_g.push_back({v.off + int64_t(r) * v.C, v.C, 1, r, v.R});
+            ++s;
+            continue;
+        }
         size_t e = s + 1;
         if (spanning && v.R > 0) {
             while (e < slices.size() && slices[e].R == v.R && slices[e].C == v.C &&
                    slices[e].off == slices[e - 1].off + int64_t(v.R) * v.C) {
                 slice_first[e] = static_cast<int32_t>(items.size());
                 slice_first1[e] = static_cast<int32_t>(items1.size());
+                L.slice_first_g[e] = static_cast<int32_t>(L.items_g.size());
                 ++e;
             }
         }
@@ -418,6 +507,7 @@ int cut_patches(const bsm_plan_desc *d, const std::vector<SliceView> &slices, in
     }
     slice_first[slices.size()] = static_cast<int32_t>(items.size());
     slice_first1[slices.size()] = static_cast<int32_t>(items1.size());
+    L.slice_first_g[slices.size()] = static_cast<int32_t>(L.items_g.size());
     if (!segs.empty())
         segs.resize(items.size(), LongSeg{0, 0, 0, 0});
     if (spanning && !items1.empty()) {
@@ -447,12 +537,12 @@ cudaGraphExec_t capture_whole_gpu(const bsm_plan *p)
     cudaGraphExec_t e = nullptr;
     bool ok = cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal) == cudaSuccess;
     if (ok) {
-        KernelArgs a = p->args, a1 = p->args1;
+        KernelArgs a = p->args, a1 = p->args1, ag = p->argsg;
         for (const auto &l : p->whole_gpu) {
-            KernelArgs &al = l.phase ? a1 : a;
+            KernelArgs &al = l.phase == 2 ? ag : (l.phase ? a1 : a);
             al.item_begin = l.begin;
             al.item_end = l.end;
-            if (launch_softmax(al, p->dtype, p->kernel_op, l.grid, st, false)) {
+            if (launch_softmax(al, p->dtype, l.phase == 2 ? OP_FORWARD_GROUP : p->kernel_op, l.grid, st, false)) {
                 ok = false;
                 break;
             }
@@ -519,7 +609,14 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     const std::vector<int32_t> &slice_first1 = lay.slice_first1;
     const int64_t n_parts = lay.n_parts;
     const int64_t long_rows = lay.long_rows;
-    const int64_t n_items = static_cast<int64_t>(items.size());
+    // the schedule covers every patch: the regular ones, then the rows split
+    // over groups of CTAs (bsm_plan_layout_host's phase-0 order)
+    std::vector<Item> &items_g = lay.items_g;
+    const int64_t n_reg = static_cast<int64_t>(items.size());
+    const int64_t n_grp = static_cast<int64_t>(items_g.size());
+    const int64_t n_items = n_reg + n_grp;
+    std::vector<Item> all(items);
+    all.insert(all.end(), items_g.begin(), items_g.end());
 
     bsm_plan *p = new bsm_plan();
     p->device = device;
@@ -537,8 +634,12 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     st.stage_bytes = static_cast<int32_t>(stage);
     st.n_stages = n_stages;
     st.long_items = long_rows;
-    p->kernel_op = d->op == BSM_OP_BACKWARD ? (long_rows > 0 ? OP_BACKWARD_LONG : OP_BACKWARD)
-                                            : (long_rows > 0 ? OP_FORWARD_LONG : OP_FORWARD);
+    st.group_rows = n_grp;
+    st.group_k = lay.group_k;
+    st.n_groups = n_grp ? lay.n_groups : 0;
+    const bool reg_long = long_rows > n_grp;   // long rows outside the groups
+    p->kernel_op = d->op == BSM_OP_BACKWARD ? (reg_long ? OP_BACKWARD_LONG : OP_BACKWARD)
+                                            : (reg_long ? OP_FORWARD_LONG : OP_FORWARD);
 
     // ---- the schedule
     std::vector<int32_t> queue;      // schedule order of the patches (queue policies)
@@ -599,8 +700,8 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
             std::vector<int64_t> pb(static_cast<size_t>(n_items)), pe(static_cast<size_t>(n_items)),
                 cost(static_cast<size_t>(n_items));
             for (int64_t i = 0; i < n_items; ++i) {
-                pb[i] = items[i].off * es;
-                pe[i] = (items[i].off + int64_t(items[i].nrows) * items[i].C) * es;
+                pb[i] = all[i].off * es;
+                pe[i] = (all[i].off + int64_t(all[i].nrows) * all[i].C) * es;
                 cost[i] = 2 * (pe[i] - pb[i]);
             }
             int32_t units[BSM_MAX_DIES] = {std::max(1, topo.sm_per_die[0]), std::max(1, topo.sm_per_die[1])};
@@ -691,19 +792,42 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     }
 
     p->queue = queue;
+    p->q_count = queue.empty() ? 0 : n_queues;
+    for (int b = 0; b < BSM_MAX_DIES; ++b) {
+        p->q_begin[b] = qbeg[b];
+        p->q_len[b] = qlen[b];
+    }
     // ---- queue policies store the patches in queue order (die 0's queue,
-    // then die 1's, ...), so a claimed queue slot is the patch record itself
+    // then die 1's, ...), so a claimed queue slot is the patch record itself;
+    // the regular patches and the group rows go to tables of their own, each
+    // in that order
+    int32_t qbeg_g[BSM_MAX_DIES] = {0}, qlen_g[BSM_MAX_DIES] = {0};
     if (!queue.empty()) {
-        std::vector<Item> ordered(items.size());
-        for (size_t k = 0; k < queue.size(); ++k)
-            ordered[k] = items[static_cast<size_t>(queue[k])];
-        items.swap(ordered);
-        if (!segs.empty()) {
-            std::vector<LongSeg> osegs(segs.size());
-            for (size_t k = 0; k < queue.size(); ++k)
-                osegs[k] = segs[static_cast<size_t>(queue[k])];
-            segs.swap(osegs);
+        std::vector<Item> ordered, ordered_g;
+        std::vector<LongSeg> osegs;
+        ordered.reserve(items.size());
+        ordered_g.reserve(items_g.size());
+        for (int b = 0; b < n_queues; ++b) {
+            const int32_t r0 = static_cast<int32_t>(ordered.size()), g0 = static_cast<int32_t>(ordered_g.size());
+            for (int32_t k = qbeg[b]; k < qbeg[b] + qlen[b]; ++k) {
+                const int64_t i = queue[static_cast<size_t>(k)];
+                if (i < n_reg) {
+                    ordered.push_back(items[static_cast<size_t>(i)]);
+                    if (!segs.empty())
+                        osegs.push_back(segs[static_cast<size_t>(i)]);
+                } else {
+                    ordered_g.push_back(items_g[static_cast<size_t>(i - n_reg)]);
+                }
+            }
+            qbeg[b] = r0;
+            qlen[b] = static_cast<int32_t>(ordered.size()) - r0;
+            qbeg_g[b] = g0;
+            qlen_g[b] = static_cast<int32_t>(ordered_g.size()) - g0;
         }
+        items.swap(ordered);
+        items_g.swap(ordered_g);
+        if (!segs.empty())
+            segs.swap(osegs);
     }
 
     // ---- upload the tables in one allocation
@@ -713,12 +837,22 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     const size_t segs_b = sizeof(LongSeg) * segs.size(), items1_b = sizeof(Item) * items1.size(),
                  segs1_b = sizeof(LongSeg) * segs1.size(), parts_b = 2 * sizeof(float) * size_t(n_parts);
     auto up = [](size_t v) { return (v + 255) & ~size_t(255); };
+    const int64_t gk = lay.group_k, gn = n_grp ? lay.n_groups : 0;
+    const size_t itemsg_b = sizeof(Item) * items_g.size(), ring_b = sizeof(uint64_t) * kGroupRing * size_t(gn),
+                 xch_b = sizeof(uint64_t) * kGroupSlots * size_t(gn * gk),
+                 xcnt_b = sizeof(uint32_t) * kGroupSlots * size_t(gn);
     const size_t o_items = 0, o_slices = up(items_b), o_smdie = o_slices + up(slices_b),
                  o_heads = o_smdie + 256, o_segs = o_heads + 256, o_items1 = o_segs + up(segs_b),
                  o_segs1 = o_items1 + up(items1_b), o_slices1 = o_segs1 + up(segs1_b),
                  o_heads1 = o_slices1 + (n1 ? up(slices_b) : 0), o_parts = o_heads1 + 256,
-                 blob_b = o_parts + up(parts_b);
+                 o_itemsg = o_parts + up(parts_b), o_slicesg = o_itemsg + up(itemsg_b),
+                 o_headsg = o_slicesg + (n_grp ? up(slices_b) : 0), o_ring = o_headsg + 256,
+                 o_xch = o_ring + up(ring_b), o_xcnt = o_xch + up(xch_b), blob_b = o_xcnt + up(xcnt_b);
     std::vector<unsigned char> host(blob_b, 0);
+    if (n_grp) {
+        std::memcpy(&host[o_itemsg], items_g.data(), itemsg_b);
+        std::memcpy(&host[o_slicesg], lay.slice_first_g.data(), slices_b);
+    }
     if (items_b)
         std::memcpy(&host[o_items], items.data(), items_b);
     std::memcpy(&host[o_slices], slice_first.data(), slices_b);
@@ -751,12 +885,12 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     unsigned char *b = static_cast<unsigned char *>(p->blob);
 
     KernelArgs &a = p->args;
+    a.n_items = static_cast<int32_t>(n_reg);
     a.x = d->x;
     a.x2 = d->op == BSM_OP_BACKWARD ? d->x2 : nullptr;
     a.y = d->y;
     a.total_elems = total;
     a.items = reinterpret_cast<const Item *>(b + o_items);
-    a.n_items = static_cast<int32_t>(n_items);
     a.slice_first_item = reinterpret_cast<const int32_t *>(b + o_slices);
     a.n_slices = static_cast<int32_t>(std::min<size_t>(slices.size(), INT32_MAX));
     a.n_queues = n_queues;
@@ -792,7 +926,33 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
         a1.heads = reinterpret_cast<uint32_t *>(b + o_heads1);
         a1.phase = 1;
     }
+    // rows over groups of CTAs: their table, queues and exchange buffers
+    p->n_group = n_grp;
+    if (n_grp) {
+        KernelArgs &ag = p->argsg;
+        ag = a;
+        ag.items = reinterpret_cast<const Item *>(b + o_itemsg);
+        ag.n_items = static_cast<int32_t>(n_grp);
+        ag.slice_first_item = reinterpret_cast<const int32_t *>(b + o_slicesg);
+        for (int q = 0; q < BSM_MAX_DIES; ++q) {
+            ag.queue_begin[q] = queue.empty() ? 0 : qbeg_g[q];
+            ag.queue_len[q] = queue.empty() ? 0 : qlen_g[q];
+        }
+        ag.heads = reinterpret_cast<uint32_t *>(b + o_headsg);
+        ag.stage_bytes = static_cast<int32_t>(lay.stage_g);
+        ag.n_stages = lay.n_stages_g;
+        ag.segs = nullptr;
+        ag.partials = nullptr;
+        ag.phase = 0;
+        ag.group_k = lay.group_k;
+        ag.n_groups = lay.n_groups;
+        ag.ring = reinterpret_cast<unsigned long long *>(b + o_ring);
+        ag.xch = reinterpret_cast<unsigned long long *>(b + o_xch);
+        ag.xcnt = reinterpret_cast<uint32_t *>(b + o_xcnt);
+        p->grid_g = lay.group_k * lay.n_groups;
+    }
 
+    const int32_t other_launches = (n_reg > 0 ? (n1 ? 2 : 1) : 0) + (n_grp > 0 ? 1 : 0);
     switch (d->policy) {
     case BSM_POLICY_WHOLE_GPU:
         a.mode = PULL_STATIC;
@@ -803,6 +963,11 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
             const int32_t n1s = slice_first1[k + 1] - slice_first1[k];
             if (n1s > 0)
                 p->whole_gpu.push_back({slice_first1[k], slice_first1[k + 1], std::min(n1s, c->n_sm), 1});
+            if (n_grp) {
+                const int32_t ng = lay.slice_first_g[k + 1] - lay.slice_first_g[k];
+                if (ng > 0)
+                    p->whole_gpu.push_back({lay.slice_first_g[k], lay.slice_first_g[k + 1], p->grid_g, 2});
+            }
         }
         p->grid = c->n_sm;
         st.launches = static_cast<int32_t>(p->whole_gpu.size());
@@ -810,15 +975,16 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     case BSM_POLICY_RR:
         a.mode = PULL_RR_SLICE;
         p->grid = static_cast<int>(std::min<int64_t>(c->n_sm, std::max<int64_t>(1, int64_t(slices.size()))));
-        st.launches = n_items > 0 ? (n1 ? 2 : 1) : 0;
+        st.launches = other_launches;
         break;
     default:
         a.mode = PULL_QUEUE;
         p->grid = c->n_sm;
-        st.launches = n_items > 0 ? (n1 ? 2 : 1) : 0;
+        st.launches = other_launches;
         break;
     }
     p->args1.mode = a.mode;
+    p->argsg.mode = a.mode;
     if (d->policy == BSM_POLICY_WHOLE_GPU && !p->whole_gpu.empty() && p->whole_gpu.size() <= kMaxGraphLaunches) {
         int prev_dev = -1;
         cudaGetDevice(&prev_dev);
@@ -852,7 +1018,8 @@ int plan_layout_host_impl(const bsm_plan_desc *d, int32_t n_sm, int64_t smem_opt
         return rc;
     out->stage_bytes = lay.stage;
     out->n_stages = lay.n_stages;
-    out->n_patches = static_cast<int64_t>(lay.items.size());
+    out->group_k = lay.items_g.empty() ? 0 : lay.group_k;
+    out->n_patches = static_cast<int64_t>(lay.items.size() + lay.items_g.size());
     out->n_patches_phase1 = static_cast<int64_t>(lay.items1.size());
     out->long_rows = lay.long_rows;
     auto put = [](const Item &it, const LongSeg *sg, bsm_patch &o) {
@@ -866,6 +1033,12 @@ int plan_layout_host_impl(const bsm_plan_desc *d, int32_t n_sm, int64_t smem_opt
     };
     for (size_t i = 0; i < lay.items.size() && static_cast<int64_t>(i) < cap0; ++i)
         put(lay.items[i], lay.segs.empty() ? nullptr : &lay.segs[i], phase0[i]);
+    // rows over groups of CTAs come last, marked part_count = -K
+    for (size_t j = 0; j < lay.items_g.size() && static_cast<int64_t>(lay.items.size() + j) < cap0; ++j) {
+        bsm_patch &o = phase0[lay.items.size() + j];
+        put(lay.items_g[j], nullptr, o);
+        o.part_count = -lay.group_k;
+    }
     for (size_t i = 0; i < lay.items1.size() && static_cast<int64_t>(i) < cap1; ++i)
         put(lay.items1[i], &lay.segs1[i], phase1[i]);
     return BSM_OK;
@@ -876,7 +1049,7 @@ int plan_execute_impl(const bsm_plan *p, bsm_stream_t stream)
     TraceRange trace("bsm_plan_execute");
     if (!p)
         return BSM_ERR_INVALID_ARG;
-    if (p->args.n_items == 0)
+    if (p->args.n_items == 0 && p->n_group == 0)
         return BSM_OK;
     int prev = -1;
     cudaGetDevice(&prev);
@@ -888,18 +1061,22 @@ int plan_execute_impl(const bsm_plan *p, bsm_stream_t stream)
         p->args.wait_limit_ns == 0) {
         err = static_cast<int>(cudaGraphLaunch(p->whole_graph, static_cast<cudaStream_t>(stream)));
     } else if (p->policy == BSM_POLICY_WHOLE_GPU) {
-        KernelArgs a = p->args, a1 = p->args1;
+        KernelArgs a = p->args, a1 = p->args1, ag = p->argsg;
         for (const auto &l : p->whole_gpu) {
-            KernelArgs &al = l.phase ? a1 : a;
+            KernelArgs &al = l.phase == 2 ? ag : (l.phase ? a1 : a);
             al.item_begin = l.begin;
             al.item_end = l.end;
-            if ((err = launch_softmax(al, p->dtype, p->kernel_op, l.grid, stream, checked)))
+            if ((err = launch_softmax(al, p->dtype, l.phase == 2 ? OP_FORWARD_GROUP : p->kernel_op, l.grid, stream,
+                                      checked)))
                 break;
         }
     } else {
-        err = launch_softmax(p->args, p->dtype, p->kernel_op, p->grid, stream, checked);
+        if (p->args.n_items > 0)
+            err = launch_softmax(p->args, p->dtype, p->kernel_op, p->grid, stream, checked);
         if (!err && p->n_phase1)
             err = launch_softmax(p->args1, p->dtype, p->kernel_op, p->grid, stream, checked);
+        if (!err && p->n_group)
+            err = launch_softmax(p->argsg, p->dtype, OP_FORWARD_GROUP, p->grid_g, stream, checked);
     }
     if (prev >= 0 && prev != p->device)
         cudaSetDevice(prev);
@@ -1042,12 +1219,12 @@ int bsm_plan_get_schedule(const bsm_plan *plan, bsm_plan_schedule *out)
     if (!plan || !out)
         return BSM_ERR_INVALID_ARG;
     const bsm_plan &p = *plan;
-    const bool queued = p.args.mode == PULL_QUEUE;
-    out->n_queues = queued ? p.args.n_queues : 0;
+    const bool queued = p.q_count > 0;
+    out->n_queues = p.q_count;
     out->count_output_bytes = p.count_y;
     for (int b = 0; b < BSM_MAX_DIES; ++b) {
-        out->queue_begin[b] = queued ? p.args.queue_begin[b] : 0;
-        out->queue_len[b] = queued ? p.args.queue_len[b] : 0;
+        out->queue_begin[b] = queued ? p.q_begin[b] : 0;
+        out->queue_len[b] = queued ? p.q_len[b] : 0;
         out->units[b] = p.units[b];
     }
     out->l_near = p.w_near;
@@ -1070,10 +1247,10 @@ int bsm_plan_get_schedule(const bsm_plan *plan, bsm_plan_schedule *out)
 
 int bsm_plan_device_table(const bsm_plan *plan, int phase, bsm_patch *out, int64_t cap, int64_t *n_out)
 {
-    if (!plan || !n_out || (phase != 0 && phase != 1) || cap < 0 || (cap > 0 && !out))
+    if (!plan || !n_out || phase < 0 || phase > 2 || cap < 0 || (cap > 0 && !out))
         return BSM_ERR_INVALID_ARG;
-    const KernelArgs &a = phase ? plan->args1 : plan->args;
-    const int64_t n = phase && !plan->n_phase1 ? 0 : a.n_items;
+    const KernelArgs &a = phase == 2 ? plan->argsg : (phase ? plan->args1 : plan->args);
+    const int64_t n = (phase == 1 && !plan->n_phase1) || (phase == 2 && !plan->n_group) ? 0 : a.n_items;
     *n_out = n;
     const int64_t m = std::min(n, cap);
     if (m <= 0)
@@ -1099,7 +1276,7 @@ int bsm_plan_device_table(const bsm_plan *plan, int phase, bsm_patch *out, int64
         out[i].row0 = items[i].row0;
         out[i].slice_rows = items[i].R;
         out[i].col0 = segs.empty() ? 0 : segs[i].col0;
-        out[i].part_count = segs.empty() ? 0 : segs[i].part_count;
+        out[i].part_count = phase == 2 ? -a.group_k : (segs.empty() ? 0 : segs[i].part_count);
     }
     return BSM_OK;
 }
@@ -1132,12 +1309,16 @@ int bsm_plan_debug(bsm_plan *plan, int what, int64_t arg)
         plan->args.wait_limit_ns = 0;
         plan->args1.debug = 0;
         plan->args1.wait_limit_ns = 0;
+        plan->argsg.debug = 0;
+        plan->argsg.wait_limit_ns = 0;
         return BSM_OK;
     case BSM_DEBUG_WITHHOLD_STAGE:
         if (arg <= 0)
             return BSM_ERR_INVALID_ARG;
         plan->args.debug |= KDEBUG_WITHHOLD_STAGE0;
         plan->args.wait_limit_ns = static_cast<uint64_t>(arg);
+        plan->argsg.debug |= KDEBUG_WITHHOLD_STAGE0;
+        plan->argsg.wait_limit_ns = static_cast<uint64_t>(arg);
         return BSM_OK;
     case BSM_DEBUG_CORRUPT_PATCH: {
         if (arg < 0 || arg >= plan->args.n_items)

@@ -50,8 +50,20 @@ enum Op : int32_t {
     OP_FORWARD = 0,     // y = softmax(x [+ causal mask])
     OP_BACKWARD = 1,    // y = x * (x2 - rowsum(x * x2)): x = softmax output, x2 = its gradient
     OP_FORWARD_LONG = 2, // OP_FORWARD for plans with rows longer than a stage (two passes)
-    OP_BACKWARD_LONG = 3 // OP_BACKWARD for plans with rows longer than half a stage (two passes)
+    OP_BACKWARD_LONG = 3, // OP_BACKWARD for plans with rows longer than half a stage (two passes)
+    OP_FORWARD_GROUP = 4 // OP_FORWARD of rows split over groups of CTAs (one read; see KernelArgs)
 };
+
+// Rows split over groups of CTAs (OP_FORWARD_GROUP): group g is CTAs
+// [g*K, g*K + K); its rank-0 CTA claims rows and announces them in the
+// group's ring of kGroupRing claim words (row sequence number + 1 in the high
+// half, the row's position in the table in the low half); each member stages
+// its part of the row, publishes its (max, sum) in one of kGroupSlots
+// exchange slots and counts it in that slot's counter.  Rings and counters
+// are reset by the last CTA of every launch.
+constexpr int kGroupRing = 16;
+constexpr int kGroupSlots = 4;
+constexpr int kMaxGroup = 128;
 
 // A row longer than one stage is cut into segments of whole stage-sized
 // chunks, each its own patch (nrows = 1, off/C = the segment).  An execute
@@ -95,6 +107,12 @@ struct KernelArgs {
     const LongSeg *segs;        // per patch, in the order of `items`; NULL: no long rows
     float *partials;            // 2 floats per segment
     int32_t phase;              // 0: segments leave their partials; 1: combine and write
+    // rows split over groups of CTAs (OP_FORWARD_GROUP): items are whole rows
+    int32_t group_k;            // CTAs per group (2..kMaxGroup); the grid is n_groups * group_k
+    int32_t n_groups;
+    unsigned long long *ring;   // n_groups x kGroupRing claim words
+    unsigned long long *xch;    // n_groups x kGroupSlots x group_k partials: (max, sum) as two floats
+    uint32_t *xcnt;             // n_groups x kGroupSlots arrival counters
 };
 
 // Test-only fault injection (bsm_plan_debug).

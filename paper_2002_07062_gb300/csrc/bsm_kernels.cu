@@ -38,9 +38,10 @@ namespace bsm {
 namespace {
 
 constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s
+constexpr uint32_t kClaimAhead = 2;                 // rows a group's rank 0 announces ahead
 constexpr float kLog2e = 1.4426950408889634f;
 
-enum : int32_t { KIND_DATA = 0, KIND_SKIP = 1, KIND_DONE = 2, KIND_LONG = 3 };
+enum : int32_t { KIND_DATA = 0, KIND_SKIP = 1, KIND_DONE = 2, KIND_LONG = 3, KIND_GROUP = 4 };
 
 struct alignas(16) StageMeta {
     int64_t off;
@@ -1023,8 +1024,12 @@ __device__ __forceinline__ int consume_stage(const unsigned char *sbuf, const St
 
 // -------------------------------------------------------------- the schedule
 
+// The pulling unit is a CTA, or for rows split over groups of CTAs a whole
+// group (unit = group index, n_units = groups): the static and round-robin
+// deals and the tail rule count units, not CTAs.
 struct Puller {
     const KernelArgs &a;
+    int32_t unit, n_units;
     int32_t k = 0;           // PULL_STATIC: patches taken so far
     int32_t slice = -1;      // PULL_RR_SLICE
     int32_t cur = 0, end = 0;
@@ -1032,14 +1037,20 @@ struct Puller {
     int32_t die = 0;
     uint32_t fetch = kFetch; // PULL_QUEUE: patches per claim (1 near the end of a queue)
 
-    __device__ explicit Puller(const KernelArgs &args) : a(args)
+    __device__ explicit Puller(const KernelArgs &args)
+        : Puller(args, static_cast<int32_t>(blockIdx.x), static_cast<int32_t>(gridDim.x))
+    {
+    }
+
+    __device__ Puller(const KernelArgs &args, int32_t unit_, int32_t n_units_)
+        : a(args), unit(unit_), n_units(n_units_)
     {
         if (a.mode == PULL_QUEUE && a.sm_die) {
             int d = a.sm_die[sm_id() & (BSM_MAX_SM - 1)];
             die = (d >= 0 && d < a.n_queues) ? d : 0;
         }
         if (a.mode == PULL_RR_SLICE)
-            slice = static_cast<int32_t>(blockIdx.x) - static_cast<int32_t>(gridDim.x);
+            slice = unit - n_units;
     }
 
     // Positions in a.items of this CTA's next patches (up to `most`, at most
@@ -1050,7 +1061,7 @@ struct Puller {
         if (a.mode == PULL_STATIC) {
 #pragma unroll
             for (int j = 0; j < kFetch; ++j) {
-                const int64_t idx = (int64_t)a.item_begin + blockIdx.x + (int64_t)(k + j) * gridDim.x;
+                const int64_t idx = (int64_t)a.item_begin + unit + (int64_t)(k + j) * n_units;
                 if (j < most && idx < a.item_end)
                     pos[n++] = static_cast<int32_t>(idx);
             }
@@ -1059,7 +1070,7 @@ struct Puller {
         }
         if (a.mode == PULL_RR_SLICE) {
             while (cur >= end) {
-                slice += gridDim.x;
+                slice += n_units;
                 if (slice >= a.n_slices)
                     return 0;
                 cur = a.slice_first_item[slice];
@@ -1086,7 +1097,7 @@ struct Puller {
                         pos[n++] = a.queue_begin[qq] + static_cast<int32_t>(t + j);
                 // near the end of the queue, claim one patch at a time so the
                 // last patches spread over the SMs instead of queueing in fours
-                if (len - t < 2u * kFetch * gridDim.x)
+                if (len - t < 2u * kFetch * static_cast<uint32_t>(n_units))
                     fetch = 1;
                 return n;
             }
@@ -1534,6 +1545,381 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
     }
 }
 
+
+// ------------------------------------------------ rows over groups of CTAs
+// A row too long for one SM's shared memory is cut into K parts of equal
+// length (whole 16-byte vectors; the last may be shorter or empty), and the K
+// CTAs of a group each stage one part in one stage: every element is read
+// from memory once.  Each CTA takes its part's running (max, rescaled sum)
+// -- lanes, then warps in a fixed order, as for the long rows above --,
+// publishes it in global memory and counts it in its slot's counter
+// (release); every member then waits for the K partials of the row
+// (acquire), combines them in the same fixed order (a per-lane sum over
+// ranks l, l + 32, ..., then the xor tree), and writes its part of y from
+// its stage.  The consumers are one row ahead: they take the next row's
+// partial before waiting for the previous row's group, so the exchange
+// overlaps work.  The group's rank-0 CTA claims the rows (any policy's puller,
+// with the group as the unit) and announces them to its members through a
+// ring of claim words.  The launch is cooperative, so every member of a group
+// is resident and each wait ends; every wait is bounded all the same.
+
+__device__ __forceinline__ void st_release_u64(unsigned long long *p, unsigned long long v)
+{
+    asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+
+__device__ __forceinline__ void st_relaxed_u64(unsigned long long *p, unsigned long long v)
+{
+    asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+
+__device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long long *p)
+{
+    unsigned long long v;
+    asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ unsigned long long ld_relaxed_u64(const unsigned long long *p)
+{
+    unsigned long long v;
+    asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t *p)
+{
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void red_release_add(uint32_t *p, uint32_t v)
+{
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// Wait until the claim word at p carries sequence number seq (bounded).
+__device__ __noinline__ bool wait_claim(const unsigned long long *p, uint32_t seq, const volatile int32_t *abort,
+                                        uint64_t limit_ns, unsigned long long &word)
+{
+    word = ld_acquire_u64(p);
+    if (static_cast<uint32_t>(word >> 32) == seq)
+        return true;
+    const uint64_t t0 = global_timer_ns();
+    for (uint32_t it = 0; it < (1u << 26); ++it) {
+        __nanosleep(32);
+        word = ld_acquire_u64(p);
+        if (static_cast<uint32_t>(word >> 32) == seq)
+            return true;
+        if ((abort && *abort) || global_timer_ns() - t0 > limit_ns)
+            return false;
+    }
+    return false;
+}
+
+// Wait until the counter at p reaches target (it only grows within a launch).
+__device__ __noinline__ bool wait_count(const uint32_t *p, uint32_t target, const volatile int32_t *abort,
+                                        uint64_t limit_ns)
+{
+    if (ld_acquire_u32(p) >= target)
+        return true;
+    const uint64_t t0 = global_timer_ns();
+    for (uint32_t it = 0; it < (1u << 26); ++it) {
+        __nanosleep(32);
+        if (ld_acquire_u32(p) >= target)
+            return true;
+        if ((abort && *abort) || global_timer_ns() - t0 > limit_ns)
+            return false;
+    }
+    return false;
+}
+
+__device__ __forceinline__ unsigned long long pack_ms(float m, float sum)
+{
+    return (static_cast<unsigned long long>(__float_as_uint(sum)) << 32) | __float_as_uint(m);
+}
+
+template <typename Tag, bool Checked>
+__global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
+{
+    using E = Elem<Tag>;
+    constexpr int EPV = E::kPerVec;
+    extern __shared__ __align__(1024) unsigned char smem[];
+    SmemHeader &h = *reinterpret_cast<SmemHeader *>(smem);
+    unsigned char *stages = smem + kSmemHeader;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int S = a.n_stages;
+    const int K = a.group_k;
+    const int grp = static_cast<int>(blockIdx.x) / K, rank = static_cast<int>(blockIdx.x) % K;
+    const uint64_t wait_limit = a.wait_limit_ns ? a.wait_limit_ns : kWaitLimitNs;
+    unsigned long long *ring = a.ring + static_cast<size_t>(grp) * kGroupRing;
+    unsigned long long *xch = a.xch + static_cast<size_t>(grp) * kGroupSlots * K;
+    uint32_t *xcnt = a.xcnt + static_cast<size_t>(grp) * kGroupSlots;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(&h.full[s], 1);
+            mbar_init(&h.empty[s], kConsumerWarps);
+        }
+        mbar_init(&h.xwarp, kConsumerWarps);
+        h.abort_flag = 0;
+        mbar_init_fence();
+    }
+    __syncthreads();
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+
+    if (warp == kConsumerWarps) {
+        // ------------------------------------------------------- producer
+        if (lane == 0) {
+            Puller pull(a, grp, a.n_groups);
+            uint32_t issued_phase[kMaxStages];
+            bool issued[kMaxStages];
+            for (int s = 0; s < kMaxStages; ++s)
+                issued[s] = false;
+            bool aborted = false;
+            uint32_t it = 0, posted = 0;
+            bool post_done = false;
+            for (uint32_t t = 0; !aborted; ++t) {
+                if (rank == 0) {
+                    // announce rows up to kClaimAhead beyond this one
+                    while (!post_done && posted <= t + kClaimAhead) {
+                        int32_t p1[kFetch];
+                        const int n = pull.next_batch(p1, 1);
+                        const uint32_t pos = n > 0 ? static_cast<uint32_t>(p1[0]) : 0xFFFFFFFFu;
+                        st_release_u64(&ring[posted % kGroupRing],
+                                       (static_cast<unsigned long long>(posted + 1) << 32) | pos);
+                        ++posted;
+                        post_done = n == 0;
+                    }
+                }
+                unsigned long long word = 0;
+                if (!wait_claim(&ring[t % kGroupRing], t + 1, &h.abort_flag, wait_limit, word)) {
+                    aborted = true;
+                    break;
+                }
+                const uint32_t pos = static_cast<uint32_t>(word);
+                const int s = static_cast<int>(it % S);
+                const uint32_t ph = (it / S) & 1u;
+                if (!mbar_wait_bounded(&h.empty[s], ph ^ 1u, &h.abort_flag, wait_limit)) {
+                    aborted = true;
+                    break;
+                }
+                issued[s] = false;
+                ++it;
+                StageMeta &mt = h.meta[s];
+                if (pos == 0xFFFFFFFFu) {
+                    mt.kind = KIND_DONE;
+                    mbar_arrive(&h.full[s]);
+                    break;
+                }
+                if ((a.debug & KDEBUG_WITHHOLD_STAGE0) && it == 1)
+                    continue;                      // test hook: stage 0 is never filled
+                const bool in = pos < static_cast<uint32_t>(a.n_items);
+                const Item item = in ? a.items[pos] : Item{-1, 0, 0, 0, 0};
+                // this member's part (the same cut in every member)
+                const int64_t part = ((int64_t(item.C) + K - 1) / K + EPV - 1) / EPV * EPV;
+                const int64_t c0 = part * rank;
+                const int64_t cn = item.C - c0 < 0 ? 0 : (item.C - c0 < part ? item.C - c0 : part);
+                const bool ok = in && item.off >= 0 && item.C > 0 && item.nrows == 1 && item.R > 0 &&
+                                item.row0 >= 0 && item.row0 < item.R && item.off + item.C <= a.total_elems &&
+                                ((item.off * E::kSize) & 15) == 0 && ((int64_t(item.C) * E::kSize) & 15) == 0 &&
+                                part * E::kSize <= a.stage_bytes;
+                if (!ok) {
+                    // every member sees the same record and skips the row alike
+                    atomicOr(a.status, BSM_DEV_BOUNDS);
+                    mt.kind = KIND_SKIP;
+                    mbar_arrive(&h.full[s]);
+                    continue;
+                }
+                mt.off = item.off + c0;
+                mt.C = static_cast<int32_t>(cn);
+                mt.nrows = 1;
+                mt.row0 = item.row0;
+                mt.R = item.R;
+                mt.col0 = static_cast<int32_t>(c0);
+                mt.pass = 0;
+                mt.kind = KIND_GROUP;
+                if (cn == 0) {
+                    mbar_arrive(&h.full[s]);
+                    continue;
+                }
+                const uint32_t bytes = static_cast<uint32_t>(cn * E::kSize);
+                unsigned char *dst = stages + static_cast<size_t>(s) * a.stage_bytes;
+                const unsigned char *src = static_cast<const unsigned char *>(a.x) + (item.off + c0) * E::kSize;
+                if (Checked) {
+                    const unsigned char *x0 = static_cast<const unsigned char *>(a.x);
+                    if (src < x0 || src + bytes > x0 + a.total_elems * E::kSize ||
+                        (reinterpret_cast<uintptr_t>(src) & 15) || (smem_addr(dst) & 15) ||
+                        bytes > static_cast<uint32_t>(a.stage_bytes) ||
+                        dst + bytes > smem + kSmemHeader + static_cast<size_t>(S) * a.stage_bytes) {
+                        check_fail(a.status, 3, pos, bytes);
+                        mt.kind = KIND_SKIP;       // the group's other members time out
+                        mbar_arrive(&h.full[s]);
+                        continue;
+                    }
+                }
+                mbar_arrive_expect_tx(&h.full[s], bytes);
+                bulk_load(dst, src, bytes, &h.full[s]);
+                issued[s] = true;
+                issued_phase[s] = ph;
+            }
+            if (aborted) {
+                atomicOr(a.status, BSM_DEV_TIMEOUT);
+                h.abort_flag = 1;
+            }
+            for (int s = 0; s < S; ++s)
+                if (issued[s])
+                    mbar_wait_bounded(&h.full[s], issued_phase[s], nullptr, wait_limit);
+        }
+        __syncwarp();
+    } else {
+        // ----------------------------------------------------------- consumers
+        const bool causal = (a.flags & BSM_FLAG_CAUSAL) != 0;
+        unsigned char *y = static_cast<unsigned char *>(a.y);
+        const Bounds bd0{nullptr, nullptr, y, y + a.total_elems * E::kSize, a.status};
+        uint32_t xt = 0;            // group rows this CTA took part in (the exchange sequence)
+        int pend = -1;              // stage of the row whose group exchange is outstanding
+        StageMeta pmt{};
+        uint32_t pxt = 0;
+        // the row of stage ps (exchange number x1): wait for its K partials,
+        // combine them, write this member's part, release the stage
+        auto finish = [&](int ps, const StageMeta &m1, uint32_t x1) -> bool {
+            const uint32_t slot = x1 & (kGroupSlots - 1);
+            const uint32_t target = static_cast<uint32_t>(K) * ((x1 / kGroupSlots) + 1);
+            int okw = 1;
+            if (lane == 0)
+                okw = wait_count(&xcnt[slot], target, &h.abort_flag, wait_limit) ? 1 : 0;
+            okw = __shfl_sync(0xFFFFFFFFu, okw, 0);
+            if (!okw) {
+                if (lane == 0) {
+                    atomicOr(a.status, BSM_DEV_TIMEOUT);
+                    h.abort_flag = 1;
+                }
+                return false;
+            }
+            (void)ld_acquire_u32(&xcnt[slot]);   // this lane's reads below come after the count
+            float mv[kMaxGroup / 32], sv[kMaxGroup / 32];
+            float M = -INFINITY;
+#pragma unroll
+            for (int j = 0; j < kMaxGroup / 32; ++j) {
+                const int r = lane + 32 * j;
+                mv[j] = -INFINITY;
+                sv[j] = 0.0f;
+                if (r < K) {
+                    const unsigned long long w = ld_relaxed_u64(&xch[slot * K + r]);
+                    mv[j] = __uint_as_float(static_cast<uint32_t>(w));
+                    sv[j] = __uint_as_float(static_cast<uint32_t>(w >> 32));
+                    M = fmaxf(M, mv[j]);
+                }
+            }
+            M = group_max<32>(M);
+            float sum = 0.0f;
+#pragma unroll
+            for (int j = 0; j < kMaxGroup / 32; ++j)
+                if (lane + 32 * j < K)
+                    sum += mv[j] == M ? sv[j] : sv[j] * ex2((mv[j] - M) * kLog2e);
+            sum = group_sum<32>(sum);
+            if (m1.C > 0) {
+                StageMeta mw = m1;
+                mw.pass = 1;
+                float dm = -INFINITY, ds = 0.0f;
+                long_chunk<Tag, Checked>(stages + static_cast<size_t>(ps) * a.stage_bytes, mw, y, causal, warp,
+                                         lane, bd0, dm, ds, M * kLog2e, __frcp_rn(sum));
+            }
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(&h.empty[ps]);
+            return true;
+        };
+        bool failed = false;
+        for (uint32_t it = 0;; ++it) {
+            const int s = static_cast<int>(it % S);
+            const uint32_t ph = (it / S) & 1u;
+            // the whole warp gives up together (a shuffle below needs all lanes)
+            if (!__all_sync(0xFFFFFFFFu, mbar_wait_bounded(&h.full[s], ph, &h.abort_flag, wait_limit))) {
+                if (lane == 0) {
+                    atomicOr(a.status, BSM_DEV_TIMEOUT);
+                    h.abort_flag = 1;
+                }
+                failed = true;
+                break;
+            }
+            const StageMeta mt = h.meta[s];
+            if (mt.kind == KIND_DONE)
+                break;
+            if (mt.kind != KIND_GROUP) {
+                __syncwarp();
+                if (lane == 0)
+                    mbar_arrive(&h.empty[s]);
+                continue;
+            }
+            // pass 0: this member's (max, sum) of its part
+            float m_l = -INFINITY, s_l = 0.0f;
+            if (mt.C > 0)
+                long_chunk<Tag, Checked>(stages + static_cast<size_t>(s) * a.stage_bytes, mt, y, causal, warp, lane,
+                                         bd0, m_l, s_l, 0.0f, 0.0f);
+#pragma unroll
+            for (int o = 16; o >= 1; o >>= 1) {
+                const float mo = __shfl_xor_sync(0xFFFFFFFFu, m_l, o);
+                const float so = __shfl_xor_sync(0xFFFFFFFFu, s_l, o);
+                combine_ms(m_l, s_l, mo, so);
+            }
+            const int par = xt & 1;
+            if (lane == 0) {
+                h.partial[par][warp] = make_float2(m_l, s_l);
+                mbar_arrive(&h.xwarp);
+            }
+            if (!__all_sync(0xFFFFFFFFu, mbar_wait_bounded(&h.xwarp, xt & 1u, &h.abort_flag, wait_limit))) {
+                if (lane == 0) {
+                    atomicOr(a.status, BSM_DEV_TIMEOUT);
+                    h.abort_flag = 1;
+                }
+                failed = true;
+                break;
+            }
+            if (warp == 0 && lane == 0) {
+                float m = -INFINITY, sum = 0.0f;
+                for (int w = 0; w < kConsumerWarps; ++w)
+                    combine_ms(m, sum, h.partial[par][w].x, h.partial[par][w].y);
+                const uint32_t slot = xt & (kGroupSlots - 1);
+                st_relaxed_u64(&xch[slot * K + rank], pack_ms(m, sum));
+                red_release_add(&xcnt[slot], 1u);
+            }
+            // the previous row's partials are (nearly) in by now: finish it
+            if (pend >= 0 && !finish(pend, pmt, pxt)) {
+                failed = true;
+                break;
+            }
+            pend = s;
+            pmt = mt;
+            pxt = xt;
+            ++xt;
+        }
+        if (pend >= 0 && !failed)
+            finish(pend, pmt, pxt);
+        __syncwarp();
+    }
+    // the last CTA out resets the queue heads, the claim rings and the
+    // exchange counters for the next launch
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        const uint32_t prev = atomicAdd(&a.heads[BSM_MAX_DIES], 1u);
+        if (prev == gridDim.x - 1) {
+            __threadfence();
+            for (int d = 0; d < BSM_MAX_DIES; ++d)
+                atomicExch(&a.heads[d], 0u);
+            for (int i = 0; i < a.n_groups * kGroupRing; ++i)
+                a.ring[i] = 0ull;
+            for (int i = 0; i < a.n_groups * kGroupSlots; ++i)
+                a.xcnt[i] = 0u;
+            __threadfence();
+            atomicExch(&a.heads[BSM_MAX_DIES], 0u);
+        }
+    }
+}
+
 }  // namespace
 
 int kernel_set_smem_limit(int bytes)
@@ -1554,7 +1940,11 @@ int kernel_set_smem_limit(int bytes)
         reinterpret_cast<const void *>(softmax_persistent<F32, OP_BACKWARD_LONG, false>),
         reinterpret_cast<const void *>(softmax_persistent<BF16, OP_BACKWARD_LONG, false>),
         reinterpret_cast<const void *>(softmax_persistent<F32, OP_BACKWARD_LONG, true>),
-        reinterpret_cast<const void *>(softmax_persistent<BF16, OP_BACKWARD_LONG, true>)};
+        reinterpret_cast<const void *>(softmax_persistent<BF16, OP_BACKWARD_LONG, true>),
+        reinterpret_cast<const void *>(softmax_group<F32, false>),
+        reinterpret_cast<const void *>(softmax_group<BF16, false>),
+        reinterpret_cast<const void *>(softmax_group<F32, true>),
+        reinterpret_cast<const void *>(softmax_group<BF16, true>)};
     for (const void *f : fns) {
         cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
         if (e != cudaSuccess)
@@ -1587,13 +1977,40 @@ void launch_one(const KernelArgs &a, int grid, size_t smem, cudaStream_t st, boo
     else
         cudaLaunchKernelEx(&cfg, softmax_persistent<Tag, Op, false>, a);
 }
+
+// Rows over groups of CTAs: a cooperative launch (every CTA resident at once,
+// so the members of a group can wait on one another), without the
+// programmatic overlap with the previous kernel.
+template <typename Tag>
+void launch_group(const KernelArgs &a, int grid, size_t smem, cudaStream_t st, bool checked)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(grid));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (checked)
+        cudaLaunchKernelEx(&cfg, softmax_group<Tag, true>, a);
+    else
+        cudaLaunchKernelEx(&cfg, softmax_group<Tag, false>, a);
+}
 }  // namespace
 
 int launch_softmax(const KernelArgs &a, int dtype, int op, int grid, void *stream, bool checked)
 {
     const size_t smem = kSmemHeader + (size_t)a.n_stages * a.stage_bytes;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    if (op == OP_BACKWARD) {
+    if (op == OP_FORWARD_GROUP) {
+        if (dtype == BSM_F32)
+            launch_group<F32>(a, grid, smem, st, checked);
+        else
+            launch_group<BF16>(a, grid, smem, st, checked);
+    } else if (op == OP_BACKWARD) {
         if (dtype == BSM_F32)
             launch_one<F32, OP_BACKWARD>(a, grid, smem, st, checked);
         else

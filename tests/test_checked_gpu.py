@@ -53,9 +53,9 @@ def test_checked_forward_every_routine(dtype, flags, col_steps):
 
 @pytest.mark.parametrize("R,caps", [(3, 1), (400, 1), (400, 2)])
 def test_checked_long_rows(R, caps):
-    """3 rows: segments over two launches; 400 rows: one launch per row, of
-    two chunks (staged whole between the passes) or three (the last chunk
-    kept, the others copied again)."""
+    """3 rows: segments over two launches; 400 rows: split over groups of
+    two or four CTAs (one cooperative launch; the self-checking group kernel
+    checks its bulk copies, stage reads and stores too)."""
     import torch
     es = 4
     C = caps * (bsm.bsm_max_row_bytes() // es) + 64

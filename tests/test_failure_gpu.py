@@ -172,3 +172,31 @@ def test_whole_gpu_graph_and_debug_launches():
     assert bsm.bsm_device_status() == 0
     check_all_against_oracle(w, to_host(y))
     p.close()
+
+
+def test_withheld_stage_in_a_group_launch_times_out_and_context_survives():
+    """Rows split over groups of CTAs: the members of a group wait on one
+    another too; with a stage withheld every wait still ends (timeout
+    status), and the next execute is right."""
+    import time
+    import torch
+    w = workload.uniform("fail group", workload.F32, 1, 40, 65536, 2.0, 0xFA12).materialize()
+    x = to_device(w.x)
+    y = torch.zeros_like(x)
+    bsm.bsm_device_status_clear()
+    p = bsm.bsm_plan_create(x, y, w.rows, w.cols, w.dtype, bsm.POLICY_DYNAMIC)
+    assert p.stats()["group_rows"] == 40
+    bsm.bsm_plan_debug(p, bsm.DEBUG_WITHHOLD_STAGE, 100_000_000)      # 0.1 s waits
+    t0 = time.time()
+    p.execute()
+    torch.cuda.synchronize()
+    assert time.time() - t0 < 5.0
+    assert bsm.bsm_device_status() & bsm.DEV_TIMEOUT
+    bsm.bsm_plan_debug(p, bsm.DEBUG_NONE)
+    bsm.bsm_device_status_clear()
+    y.fill_(float("nan"))
+    p.execute()
+    torch.cuda.synchronize()
+    assert bsm.bsm_device_status() == 0
+    check_all_against_oracle(w, to_host(y))
+    p.close()

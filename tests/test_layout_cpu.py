@@ -4,9 +4,11 @@ checked here from the batch itself.  Sec. 4 cuts a batch into patches (blocks
 of consecutive rows); every row must then run exactly once, each patch must
 fit a shared-memory stage, a row longer than a stage must be covered by its
 segments exactly once, and the two launches of segmented rows must hold the
-same segments.  Worked figures: workload 2 (384 x 512 x 512 fp32) is 6144
-patches of 32 rows in three 64 KiB stages; 64 rows of 4 MiB fp32 are 1216
-segments over two launches."""
+same segments; a row split over a group of CTAs must be one record whose
+parts fit a stage of the group launch.  Worked figures: workload 2
+(384 x 512 x 512 fp32) is 6144 patches of 32 rows in three 64 KiB stages; 64
+rows of 4 MiB fp32 go to two groups of 76 CTAs; one such row is 37 segments
+over two launches."""
 import random
 from collections import Counter
 
@@ -38,6 +40,7 @@ def _slices(rows, cols, offsets):
 
 def check_layout(rows, cols, dtype, policy, n_sm=152, smem=SMEM, offsets=None, rows_per_item=0, op=0):
     es = 4 if dtype == bsm.F32 else 2
+    vec = 16 // es
     ins = 2 if op == bsm.OP_BACKWARD else 1
     L = bsm.bsm_plan_layout_host(rows, cols, dtype, policy, n_sm, smem, offsets=offsets,
                                  rows_per_item=rows_per_item, op=op)
@@ -48,22 +51,53 @@ def check_layout(rows, cols, dtype, policy, n_sm=152, smem=SMEM, offsets=None, r
 
     sl = _slices(rows, cols, offsets)
     row_owner = {}                                 # element offset of a row -> (slice, row)
-    long_rows = set()
     for s, (off, R, C) in enumerate(sl):
         for r in range(R):
             row_owner[off + r * C] = (s, r)
-            if C * es * ins > stage:
-                long_rows.add(off + r * C)
     # a row that fits half the shared memory (with its partner row, for the
     # backward pass) is staged whole: never long
     whole_cap = (((avail // 2) & ~127) // ins) & ~127
+
+    # rows split over groups of K CTAs (forward only): one record each, last
+    # in phase 0, part_count = -K; they are all the rows longer than a stage
+    # of their own, each part fits a third of the shared memory (three
+    # stages), and the groups' waves are at least two thirds full
+    K = L["group_k"]
+    grp = [p for p in L["phase0"] if int(p["part_count"]) < 0]
+    group_rows = set()
+    if grp:
+        assert op == 0 and 2 <= K <= min(n_sm, 128)
+        assert all(int(p["part_count"]) < 0 for p in L["phase0"][len(L["phase0"]) - len(grp):])
+        for p in grp:
+            off, C, n, r0, R = (int(p[k]) for k in ("elem_offset", "cols", "nrows", "row0", "slice_rows"))
+            assert int(p["part_count"]) == -K and n == 1 and int(p["col0"]) == 0
+            assert off in row_owner and off not in group_rows
+            s, r = row_owner[off]
+            assert (r, R, C) == (r0, sl[s][1], sl[s][2])
+            part = -(-(-(-C // K)) // vec) * vec      # ceil(C / K), whole vectors
+            assert part * es <= (avail // 3) & ~127
+            group_rows.add(off)
+        assert group_rows == {o for o, (s, _) in row_owner.items() if sl[s][2] * es > whole_cap}
+        G = n_sm // K
+        waves = -(-len(grp) // G)
+        assert 3 * len(grp) >= 2 * waves * G
+    else:
+        assert K == 0
+
+    long_rows = set()
+    for s, (off, R, C) in enumerate(sl):
+        for r in range(R):
+            if C * es * ins > stage and off + r * C not in group_rows:
+                long_rows.add(off + r * C)
     assert all(C * es > whole_cap for (_, R, C) in sl if R > 0 and C * es * ins > stage)
-    assert L["long_rows"] == len(long_rows)
-    n_short = len(row_owner) - len(long_rows)
+    assert L["long_rows"] == len(long_rows) + len(group_rows)
+    n_short = len(row_owner) - len(long_rows) - len(group_rows)
 
     seen = Counter()
     segs = {}                                      # long row -> [(col0, cols, part_count)]
     for p in L["phase0"]:
+        if int(p["part_count"]) < 0:
+            continue                               # a group row, checked above
         off, C, n, r0, R = (int(p[k]) for k in ("elem_offset", "cols", "nrows", "row0", "slice_rows"))
         assert n >= 1 and 0 <= r0 < R
         first = off - int(p["col0"])
@@ -87,10 +121,10 @@ def check_layout(rows, cols, dtype, policy, n_sm=152, smem=SMEM, offsets=None, r
             assert r0 + n <= R                     # RR / WHOLE_GPU: inside its slice
         for k in range(n):
             row = off + k * C
-            assert row in row_owner and row not in long_rows, (off, k)
+            assert row in row_owner and row not in long_rows and row not in group_rows, (off, k)
             assert sl[row_owner[row][0]][2] == C   # rows of one patch share a length
             seen[row] += 1
-    short_rows = [o for o in row_owner if o not in long_rows]
+    short_rows = [o for o in row_owner if o not in long_rows and o not in group_rows]
     assert set(seen) == set(short_rows) and all(v == 1 for v in seen.values())
 
     # long rows: segments cover [0, C) once; every segment carries its row's count
@@ -123,20 +157,41 @@ def test_workload2_six_thousand_patches_of_32_rows():
     assert len(L["phase1"]) == 0
 
 
-def test_four_mib_rows_are_1216_segments_over_two_launches():
+def test_four_mib_rows_go_to_two_groups_of_76():
+    """64 fp32 rows of 4 MiB: parts of at most a third of the shared memory
+    (75.25 KiB) need 55 CTAs a row; 76 (half the SMs) is the group size that
+    leaves none idle: two groups, 32 rows each, one launch, no segments."""
     L = check_layout([64], [1 << 20], bsm.F32, bsm.POLICY_DYNAMIC)
-    assert (L["stage_bytes"], L["n_stages"]) == (115712, 2)       # the 113 KiB cap
-    assert len(L["phase0"]) == 1216 and len(L["phase1"]) == 1216   # 19 per row
+    assert L["group_k"] == 76 and len(L["phase0"]) == 64 and len(L["phase1"]) == 0
     assert L["long_rows"] == 64
 
 
-def test_rows_of_two_chunks_stay_staged():
-    """bf16 rows of 128 KiB: three stages of half a row (two chunks per row),
-    each row one patch, whole in one launch."""
-    L = check_layout([2048], [65536], bsm.BF16, bsm.POLICY_DYNAMIC)
-    assert (L["stage_bytes"], L["n_stages"]) == (65536, 3)
-    assert len(L["phase0"]) == 2048 and len(L["phase1"]) == 0
-    assert set(L["phase0"]["part_count"]) == {1} and set(L["phase0"]["cols"]) == {65536}
+def test_one_four_mib_row_is_cut_into_segments_over_two_launches():
+    """A single 4 MiB row would keep one of the two groups idle: it is cut
+    into 37 segments of whole 113 KiB chunks instead (two launches)."""
+    L = check_layout([1], [1 << 20], bsm.F32, bsm.POLICY_DYNAMIC)
+    assert L["group_k"] == 0
+    assert (L["stage_bytes"], L["n_stages"]) == (115712, 2)       # the 113 KiB cap
+    assert len(L["phase0"]) == 37 and len(L["phase1"]) == 37
+
+
+@pytest.mark.parametrize("C,dtype,k", [(65536, bsm.F32, 4), (262144, bsm.F32, 19),
+                                       (65536, bsm.BF16, 2), (262144, bsm.BF16, 8),
+                                       (1048576, bsm.BF16, 38)])
+def test_long_rows_group_sizes(C, dtype, k):
+    """256 MiB of long rows (the bench's long-row cases): fp32 256 KiB and
+    1 MiB rows, bf16 128 KiB, 512 KiB and 2 MiB rows go to groups of 4, 19,
+    2, 8 and 38 CTAs -- divisors of 152 -- and each CTA stages one part."""
+    es = 4 if dtype == bsm.F32 else 2
+    R = (256 << 20) // (C * es)
+    L = check_layout([R], [C], dtype, bsm.POLICY_DYNAMIC)
+    assert L["group_k"] == k and len(L["phase0"]) == R and len(L["phase1"]) == 0
+
+
+def test_backward_long_rows_keep_one_cta_per_row():
+    """The backward pass keeps its long-row paths (no groups)."""
+    L = check_layout([2048], [65536], bsm.BF16, bsm.POLICY_DYNAMIC, op=bsm.OP_BACKWARD)
+    assert L["group_k"] == 0 and L["long_rows"] == 2048
 
 
 @pytest.mark.parametrize("policy", [bsm.POLICY_WHOLE_GPU, bsm.POLICY_RR] + list(QUEUE_POLICIES))

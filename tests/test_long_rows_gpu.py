@@ -1,6 +1,9 @@
-"""Rows longer than one shared-memory stage (streamed twice in chunks: a
-running max and rescaled sum, then the output) against the oracle, under
-every policy, bit-identical across policies."""
+"""Rows longer than one shared-memory stage against the oracle, under every
+policy, bit-identical across policies: forward rows split over groups of CTAs
+(each CTA stages one part; the group exchanges (max, sum) partials), and the
+paths that stream a row twice in chunks (a running max and rescaled sum,
+then the output): few long rows cut into segments over two launches, and
+the backward pass."""
 import numpy as np
 import pytest
 
@@ -85,12 +88,9 @@ def test_non_finite_long_rows():
 
 
 @pytest.mark.parametrize("dtype", [workload.F32, workload.BF16])
-def test_many_long_rows_stream_whole_rows_in_one_launch(dtype):
-    """With at least two waves of long rows each row is one segment that one
-    CTA streams in a single launch (fewer rows are cut into segments over two
-    launches).  Rows just over the cap get three stages of half a row: a row
-    (two chunks) stays staged for its second pass.  Against the oracle, all
-    policies bit-identical."""
+def test_many_rows_just_over_a_stage_go_to_groups_of_two(dtype):
+    """Two waves of rows just over the single-stage limit: each row is split
+    over a group of two CTAs (one launch, each CTA stages half a row)."""
     import torch
     es = 4 if dtype == workload.F32 else 2
     limit = bsm.bsm_max_row_bytes() // es
@@ -101,7 +101,7 @@ def test_many_long_rows_stream_whole_rows_in_one_launch(dtype):
     p = bsm.bsm_plan_create(x, x, w.rows, w.cols, dtype, bsm.POLICY_DYNAMIC)
     st = p.stats()
     assert st["long_items"] == R and st["launches"] == 1 and st["n_items"] == R
-    assert st["n_stages"] == 3 and 2 * st["stage_bytes"] >= C * es
+    assert st["group_rows"] == R and st["group_k"] == 2
     p.close()
     y = _all(w, x)
     check_all_against_oracle(w, to_host(y))
@@ -124,11 +124,11 @@ def test_few_long_rows_are_segmented_over_two_launches():
 
 @pytest.mark.parametrize("dtype", [workload.F32, workload.BF16])
 @pytest.mark.parametrize("chunks,flags", [(3, workload.CAUSAL), (4, 0)])
-def test_many_long_rows_of_several_chunks(dtype, chunks, flags):
-    """Whole rows of three and four chunks in the one-launch path: the
-    second pass starts on the chunk still staged and runs backwards; under
-    the causal mask most of every row is masked (the row index is below the
-    column count), so the kept last chunk is a masked one."""
+def test_many_rows_of_several_stages(dtype, chunks, flags):
+    """Rows of three and four stages' length, two waves of them: groups of
+    four and eight CTAs; under the causal mask most of every row is masked
+    (the row index is below the column count), so most members hold a wholly
+    masked part."""
     import torch
     es = 4 if dtype == workload.F32 else 2
     limit = bsm.bsm_max_row_bytes() // es
@@ -140,7 +140,83 @@ def test_many_long_rows_of_several_chunks(dtype, chunks, flags):
     p = bsm.bsm_plan_create(x, x, w.rows, w.cols, dtype, bsm.POLICY_DYNAMIC, flags=flags)
     st = p.stats()
     assert st["long_items"] == R and st["launches"] == 1
+    assert st["group_rows"] == R and st["group_k"] == (4 if chunks == 3 else 8)
     p.close()
     y = _all(w, x)
     check_all_against_oracle(w, to_host(y))
     assert bsm.bsm_device_status() == 0
+
+
+# rows over groups: (rows, row length, dtype, group size) -- each fills the
+# groups' waves; every group size the long-row bench uses on 152 SMs
+GROUP_CASES = [(40, 65536, workload.F32, 4), (8, 262144, workload.F32, 19),
+               (2, 1048576, workload.F32, 76), (80, 65536, workload.BF16, 2),
+               (20, 262144, workload.BF16, 8), (4, 1048576, workload.BF16, 38)]
+
+
+@pytest.mark.parametrize("case", range(len(GROUP_CASES)))
+@pytest.mark.parametrize("flags", [0, workload.CAUSAL])
+def test_group_rows_every_group_size(case, flags):
+    import torch
+    R, C, dtype, k = GROUP_CASES[case]
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    w = workload.uniform("group rows", dtype, 1, R, C, 3.0, 0x6A0 + case + flags, flags).materialize()
+    x = to_device(w.x)
+    p = bsm.bsm_plan_create(x, torch.empty_like(x), w.rows, w.cols, dtype, bsm.POLICY_DYNAMIC,
+                            flags=flags)
+    st = p.stats()
+    p.close()
+    if n_sm == 152:
+        assert st["group_k"] == k
+    assert st["group_rows"] == R and st["launches"] == 1
+    y = _all(w, x)
+    check_all_against_oracle(w, to_host(y))
+    assert bsm.bsm_device_status() == 0
+
+
+def test_group_rows_beside_short_rows_two_launches():
+    """A ragged batch: short rows (one launch of the regular kernel) and a
+    wave of rows split over groups (a second, cooperative launch), slices
+    interleaved and not contiguous."""
+    rows = np.array([3, 20, 5, 19, 1, 0, 7], np.int32)
+    cols = np.array([512, 200000, 64, 180000, 4096, 64, 2048], np.int32)
+    sizes = rows.astype(np.int64) * cols
+    off = np.concatenate([[0], np.cumsum(sizes + 64)[:-1]]).astype(np.int64)
+    w = workload.Workload("group mix", workload.F32, rows, cols, off, 0, 0x6B0, 3.0)
+    w.materialize()
+    import torch
+    x = to_device(w.x)
+    p = bsm.bsm_plan_create(x, torch.empty_like(x), w.rows, w.cols, workload.F32,
+                            bsm.POLICY_DYNAMIC, offsets=w.offsets)
+    st = p.stats()
+    p.close()
+    assert st["group_rows"] == 39 and st["launches"] == 2
+    y = _all(w, x)
+    check_all_against_oracle(w, to_host(y))
+    assert bsm.bsm_device_status() == 0
+
+
+def test_non_finite_group_rows():
+    """NaN, +inf, a row all -inf but one element and a row all -inf, inside
+    a wave of rows split over groups: the same results as the definition."""
+    C, R = 100000, 19
+    rng = np.random.default_rng(5)
+    x = rng.normal(0, 3, (R, C)).astype(np.float32)
+    x[1, 77777] = np.nan
+    x[2, 5] = np.inf
+    x[3, :] = -np.inf
+    x[3, 99999] = 1.0
+    x[4, :] = -np.inf
+    w = workload.uniform("group nonfinite", workload.F32, 1, R, C, 1.0, 0)
+    w.x = x.reshape(-1)
+    import torch
+    xd = to_device(w.x)
+    p = bsm.bsm_plan_create(xd, torch.empty_like(xd), w.rows, w.cols, workload.F32,
+                            bsm.POLICY_DYNAMIC)
+    assert p.stats()["group_rows"] == R
+    p.close()
+    y = _all(w, xd)
+    yh = to_host(y).reshape(R, C)
+    assert np.isnan(yh[1]).all() and np.isnan(yh[2]).all() and np.isnan(yh[4]).all()
+    assert yh[3, 99999] == 1.0 and np.count_nonzero(yh[3]) == 1
+    check_all_against_oracle(w, to_host(y))
