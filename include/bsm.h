@@ -276,8 +276,8 @@ typedef struct {
     int32_t policy;             /* bsm_policy */
     uint32_t flags;             /* BSM_FLAG_* */
     int32_t rows_per_item;      /* rows per patch at most; 0 = as many as fill one stage
-                                   (the queue policies cut a batch of fewer than four such
-                                   patches per SM into ceil(rows / (4 * SMs))-row patches) */
+                                   (the queue policies cut a batch of fewer such patches
+                                   than SMs into ceil(rows / SMs)-row patches: one per SM) */
     uint64_t tie_seed;          /* seed of the CBMF equal-share coin */
     int32_t lb_weighted;        /* CBMF_LB: 1 = weights from measured latency, 0 = equal */
     int32_t count_output_bytes; /* CBMF: 1 = a patch's bytes on a die count x and y */

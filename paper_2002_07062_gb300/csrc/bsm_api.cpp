@@ -407,14 +407,14 @@ int cut_patches(const bsm_plan_desc *d, const std::vector<SliceView> &slices, in
         else
             n_short_rows += v.R;
     }
-    // Under the queue policies a CTA's first claim takes kFetch patches.  A
-    // batch of fewer than kFetch stage-filling patches per SM (up to a few
-    // tens of MB) is therefore cut into patches of at most
-    // ceil(rows / (kFetch * SMs)) rows, so that the first claims reach every
-    // SM instead of a few (8 x 64 x 64 fp32 ran on 2 SMs).  RR and WHOLE_GPU
-    // keep their own units.
-    const int64_t spread_rows =
-        std::max<int64_t>(1, (n_short_rows + int64_t(kFetch) * n_sm - 1) / (int64_t(kFetch) * n_sm));
+    // Under the queue policies a CTA claims kFetch patches at a time, one at
+    // a time on a short queue (fewer than 2 * kFetch patches per SM).  A
+    // batch of fewer stage-filling patches than SMs (up to about 10 MB) is
+    // therefore cut into about one patch per SM -- at most
+    // ceil(rows / SMs) rows each -- so that every SM takes one patch with one
+    // claim and one copy (8 x 64 x 64 fp32 ran on 2 SMs with whole-stage
+    // patches).  RR and WHOLE_GPU keep their own units.
+    const int64_t spread_rows = std::max<int64_t>(1, (n_short_rows + n_sm - 1) / n_sm);
     const int64_t chunk_elems = stage / in_arrays / es;
     const int64_t want_segs = n_long_rows > 0 && n_long_rows < 2 * n_sm
                                   ? std::max<int64_t>(1, (8 * n_sm + n_long_rows - 1) / n_long_rows)
@@ -831,7 +831,7 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     }
 
     // ---- upload the tables in one allocation
-    const size_t items_b = sizeof(Item) * static_cast<size_t>(n_items);
+    const size_t items_b = sizeof(Item) * items.size();          // the regular patches only
     const size_t slices_b = sizeof(int32_t) * slice_first.size();
     const int64_t n1 = static_cast<int64_t>(items1.size());
     const size_t segs_b = sizeof(LongSeg) * segs.size(), items1_b = sizeof(Item) * items1.size(),

@@ -1049,6 +1049,10 @@ struct Puller {
             int d = a.sm_die[sm_id() & (BSM_MAX_SM - 1)];
             die = (d >= 0 && d < a.n_queues) ? d : 0;
         }
+        // a short queue (small batch: about a patch per SM) is claimed one
+        // patch at a time from the first claim on, so every SM gets one
+        if (a.mode == PULL_QUEUE && static_cast<uint32_t>(a.queue_len[die]) < 2u * kFetch * static_cast<uint32_t>(n_units))
+            fetch = 1;
         if (a.mode == PULL_RR_SLICE)
             slice = unit - n_units;
     }

@@ -141,10 +141,10 @@ int softmax_noalloc(const void *x, void *y, int64_t B, int64_t R, int64_t C, int
     if (row_bytes > ((avail / 2) & ~int64_t(127)))
         return BSM_ERR_UNSUPPORTED;
     const int n_stages = static_cast<int>(avail / stage < kMaxStages ? avail / stage : kMaxStages);
-    // a small batch (fewer than kFetch stage-filling patches per SM) is cut
-    // into patches of at most ceil(rows / (kFetch * SMs)) rows, as the planned
-    // dynamic schedule cuts it, so that the CTAs' first claims reach every SM
-    const int64_t spread = (rows + int64_t(kFetch) * nd->n_sm - 1) / (int64_t(kFetch) * nd->n_sm);
+    // a small batch (fewer stage-filling patches than SMs) is cut into
+    // patches of at most ceil(rows / SMs) rows, as the planned dynamic
+    // schedule cuts it, so that every SM takes one
+    const int64_t spread = (rows + nd->n_sm - 1) / nd->n_sm;
     const int64_t rpi = spread < rpi_stage ? (spread > 0 ? spread : 1) : rpi_stage;
     const int64_t n_items = (rows + rpi - 1) / rpi;
     if (n_items > kNoAllocMaxPatches)

@@ -116,7 +116,7 @@ def check_layout(rows, cols, dtype, policy, n_sm=152, smem=SMEM, offsets=None, r
         if policy == bsm.POLICY_WHOLE_GPU:
             assert n <= -(-R // n_sm)
         if policy in QUEUE_POLICIES:
-            assert n <= max(1, -(-n_short // (4 * n_sm)))
+            assert n <= max(1, -(-n_short // n_sm))
         if policy not in QUEUE_POLICIES:
             assert r0 + n <= R                     # RR / WHOLE_GPU: inside its slice
         for k in range(n):
@@ -196,8 +196,8 @@ def test_backward_long_rows_keep_one_cta_per_row():
 
 @pytest.mark.parametrize("policy", [bsm.POLICY_WHOLE_GPU, bsm.POLICY_RR] + list(QUEUE_POLICIES))
 def test_patches_never_cross_slices_under_rr_and_whole_gpu(policy):
-    # 9010 rows: the queue policies' patches are 15 rows (ceil(9010 / 608)),
-    # which do not divide 3001
+    # patches of at most 16 rows, which do not divide 3001: the queue
+    # policies' patches run on into the next slice of the same shape
     rows, cols = [3001, 3001, 3001, 7], [256, 256, 256, 256]
     L = check_layout(rows, cols, bsm.F32, policy, rows_per_item=16)
     spans = any(int(p["row0"]) + int(p["nrows"]) > int(p["slice_rows"]) for p in L["phase0"])
@@ -205,17 +205,17 @@ def test_patches_never_cross_slices_under_rr_and_whole_gpu(policy):
 
 
 def test_small_batches_spread_over_every_sm():
-    """A CTA's first claim takes four patches: a batch of fewer than four
-    stage-filling patches per SM is cut into patches of ceil(rows / (4 x SMs))
-    rows under the queue policies, so that the first claims reach every SM."""
+    """A batch of fewer stage-filling patches than SMs is cut into patches of
+    ceil(rows / SMs) rows under the queue policies (whose short queues are
+    claimed one patch at a time), so that every SM takes one patch."""
     L = check_layout([64] * 8, [64] * 8, bsm.F32, bsm.POLICY_DYNAMIC)     # 8 x 64 x 64
-    assert len(L["phase0"]) == 512 and set(L["phase0"]["nrows"]) == {1}
+    assert len(L["phase0"]) == 128 and set(L["phase0"]["nrows"]) == {4}
     L = check_layout([64] * 8, [64] * 8, bsm.F32, bsm.POLICY_RR)          # one patch per slice
     assert len(L["phase0"]) == 8
-    L = check_layout([512] * 30, [512] * 30, bsm.F32, bsm.POLICY_CBMF_LB)  # 15360 rows
-    assert len(L["phase0"]) == 591 and max(L["phase0"]["nrows"]) == 26
-    # past four stage-filling patches per SM nothing changes
-    L = check_layout([512] * 40, [512] * 40, bsm.F32, bsm.POLICY_DYNAMIC)
+    L = check_layout([512] * 8, [512] * 8, bsm.F32, bsm.POLICY_CBMF_LB)   # 4096 rows
+    assert len(L["phase0"]) == 152 and max(L["phase0"]["nrows"]) == 27
+    # from one stage-filling patch per SM on, nothing changes
+    L = check_layout([512] * 10, [512] * 10, bsm.F32, bsm.POLICY_DYNAMIC)
     assert set(L["phase0"]["nrows"]) == {32}
 
 
