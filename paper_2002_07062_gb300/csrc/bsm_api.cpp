@@ -985,7 +985,10 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     }
     p->args1.mode = a.mode;
     p->argsg.mode = a.mode;
-    if (d->policy == BSM_POLICY_WHOLE_GPU && !p->whole_gpu.empty() && p->whole_gpu.size() <= kMaxGraphLaunches) {
+    // (rows over groups of CTAs use cooperative launches, which stay out of
+    // the graph: such plans launch kernel by kernel)
+    if (d->policy == BSM_POLICY_WHOLE_GPU && !p->whole_gpu.empty() && p->whole_gpu.size() <= kMaxGraphLaunches &&
+        n_grp == 0) {
         int prev_dev = -1;
         cudaGetDevice(&prev_dev);
         cudaSetDevice(device);
