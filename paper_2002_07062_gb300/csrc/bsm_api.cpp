@@ -939,6 +939,12 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
             ag.queue_len[q] = queue.empty() ? 0 : qlen_g[q];
         }
         ag.heads = reinterpret_cast<uint32_t *>(b + o_headsg);
+        // a group pulls from the die queue of its rank-0 CTA's SM, and from
+        // the other die's once that is empty -- also under CBMF: the groups
+        // (a group may span both dies) need not cover both dies, and every
+        // queue must be drained
+        if (ag.n_queues > 1)
+            ag.steal = 1;
         ag.stage_bytes = static_cast<int32_t>(lay.stage_g);
         ag.n_stages = lay.n_stages_g;
         ag.segs = nullptr;
