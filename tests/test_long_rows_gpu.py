@@ -149,9 +149,10 @@ def test_many_rows_of_several_stages(dtype, chunks, flags):
 
 # rows over groups: (rows, row length, dtype, group size) -- each fills the
 # groups' waves; every group size the long-row bench uses on 152 SMs
-GROUP_CASES = [(40, 65536, workload.F32, 4), (8, 262144, workload.F32, 19),
-               (2, 1048576, workload.F32, 76), (80, 65536, workload.BF16, 2),
-               (20, 262144, workload.BF16, 8), (4, 1048576, workload.BF16, 38)]
+# (one full wave: as many rows as groups, n_sm / K)
+GROUP_CASES = [(38, 65536, workload.F32, 4), (8, 262144, workload.F32, 19),
+               (2, 1048576, workload.F32, 76), (76, 65536, workload.BF16, 2),
+               (19, 262144, workload.BF16, 8), (4, 1048576, workload.BF16, 38)]
 
 
 @pytest.mark.parametrize("case", range(len(GROUP_CASES)))
