@@ -439,7 +439,10 @@ int bsm_plan_device_table(const bsm_plan *plan, int phase, bsm_patch *out, int64
  *   BSM_DEBUG_CORRUPT_PATCH   the device patch table entry at position arg is
  *                             rewritten to start past the end of the buffers; the
  *                             kernel's bounds check skips it and sets
- *                             BSM_DEV_BOUNDS (its rows are not written).
+ *                             BSM_DEV_BOUNDS (its rows are not written).  Positions
+ *                             past the regular table's address the table of rows
+ *                             split over groups of CTAs (every member of the
+ *                             group skips such a row alike).
  *   BSM_DEBUG_NONE            restore the normal wait limit and switch the
  *                             withheld stage off (a corrupted entry stays).
  * Synchronous.  Returns BSM_ERR_INVALID_ARG for an unknown `what` or arg. */

@@ -1330,10 +1330,15 @@ int bsm_plan_debug(bsm_plan *plan, int what, int64_t arg)
         plan->argsg.wait_limit_ns = static_cast<uint64_t>(arg);
         return BSM_OK;
     case BSM_DEBUG_CORRUPT_PATCH: {
-        if (arg < 0 || arg >= plan->args.n_items)
+        // slots of the regular table first, then those of the group rows
+        if (arg < 0 || arg >= int64_t(plan->args.n_items) + plan->n_group)
             return BSM_ERR_INVALID_ARG;
         const int64_t past_end = plan->args.total_elems;
-        unsigned char *entry = static_cast<unsigned char *>(plan->blob) + sizeof(Item) * static_cast<size_t>(arg);
+        unsigned char *entry =
+            arg < plan->args.n_items
+                ? static_cast<unsigned char *>(plan->blob) + sizeof(Item) * static_cast<size_t>(arg)
+                : reinterpret_cast<unsigned char *>(const_cast<Item *>(plan->argsg.items)) +
+                      sizeof(Item) * static_cast<size_t>(arg - plan->args.n_items);
         int prev = -1;
         cudaGetDevice(&prev);
         cudaSetDevice(plan->device);

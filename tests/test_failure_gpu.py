@@ -85,8 +85,9 @@ def test_corrupted_patch_is_skipped_with_bounds_status():
 
 
 def _w_long():
-    """Two waves of rows just over a stage: the one-launch long-row path
-    (rows staged whole between their passes)."""
+    """Two waves of rows just over a stage: rows split over groups of two
+    CTAs (one cooperative launch; the members of a group wait on each
+    other's partials)."""
     import torch
     n_sm = torch.cuda.get_device_properties(0).multi_processor_count
     C = bsm.bsm_max_row_bytes() // 4 + 64
