@@ -312,11 +312,14 @@ int choose_groups(const std::vector<SliceView> &slices, int es, int n_sm, int64_
         const int64_t part = ((lmax + k - 1) / k + vec - 1) / vec * vec;
         return (part * es + 127) & ~int64_t(127);
     };
-    const int64_t part_cap = (avail / 3) & ~int64_t(127);
+    // a part fits a third of the shared memory (three stages) and the
+    // registers of the consumer threads (kGroupVecs vectors each)
+    const int64_t part_cap = std::min<int64_t>((avail / 3) & ~int64_t(127),
+                                               int64_t(kGroupVecs) * 16 * kConsumerWarps * 32);
     const int64_t kmin = std::max<int64_t>(2, (lmax * es + part_cap - 1) / part_cap);
     int64_t best_k = 0, best_used = 0;
     for (int64_t k = kmin; k <= std::min<int64_t>({int64_t(kMaxGroup), 2 * kmin, int64_t(n_sm)}); ++k) {
-        if (avail / stage_for(k) < 3)
+        if (avail / stage_for(k) < 3 || stage_for(k) > part_cap)
             continue;
         const int64_t used = (n_sm / k) * k;
         if (used > best_used) {

@@ -64,6 +64,10 @@ enum Op : int32_t {
 constexpr int kGroupRing = 16;
 constexpr int kGroupSlots = 4;
 constexpr int kMaxGroup = 128;
+// A member's part is held in registers while its group exchanges partials:
+// at most kGroupVecs 16-byte vectors per consumer thread, i.e. parts of at
+// most kGroupVecs * 16 * 512 bytes = 64 KiB.
+constexpr int kGroupVecs = 8;
 
 // A row longer than one stage is cut into segments of whole stage-sized
 // chunks, each its own patch (nrows = 1, off/C = the segment).  An execute

@@ -1644,6 +1644,95 @@ __device__ __forceinline__ unsigned long long pack_ms(float m, float sum)
     return (static_cast<unsigned long long>(__float_as_uint(sum)) << 32) | __float_as_uint(m);
 }
 
+// A member's part of a group row held in registers: consumer thread t (of
+// the kConsumerWarps * 32) holds the part's 16-byte vectors t, t + 512, ...
+constexpr int kConsumerThreads = kConsumerWarps * 32;
+
+template <typename Tag, bool Checked>
+__device__ __forceinline__ void group_load(uint4 (&r)[kGroupVecs], const unsigned char *sbuf, int nvec, int tid,
+                                           const Bounds &bd)
+{
+    using E = Elem<Tag>;
+#pragma unroll
+    for (int j = 0; j < kGroupVecs; ++j) {
+        const int vi = tid + j * kConsumerThreads;
+        r[j] = E::neg_inf_vec();
+        if (vi < nvec) {
+            uint4 t;
+            if (load_vec<Checked>(sbuf + 16 * vi, bd, t))
+                r[j] = t;
+        }
+    }
+}
+
+// This thread's (max, sum of exp(v - max)) over its vectors of the part in
+// the stage: the maximum first (exact), then the sum in vector order; a part
+// whose values are all -inf (masked) adds 0, a NaN or +inf makes the sum NaN.
+template <typename Tag, bool Checked>
+__device__ __forceinline__ void group_partial(const unsigned char *sbuf, int nvec, int tid, int col0, int row,
+                                              bool causal, const Bounds &bd, float &m, float &s)
+{
+    using E = Elem<Tag>;
+    constexpr int EPV = E::kPerVec;
+    m = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < kGroupVecs; ++j) {
+        const int vi = tid + j * kConsumerThreads;
+        const int col = col0 + vi * EPV;
+        uint4 raw;
+        if (vi < nvec && !(causal && col > row) && load_vec<Checked>(sbuf + 16 * vi, bd, raw)) {
+            float v[EPV];
+            E::unpack(raw, v);
+            if (causal && col + EPV - 1 > row)
+                apply_causal<EPV>(v, col, row);
+            m = fmaxf(m, tree_max<EPV>(v));
+        }
+    }
+    const float mL = m * kLog2e;
+    s = 0.0f;
+#pragma unroll
+    for (int j = 0; j < kGroupVecs; ++j) {
+        const int vi = tid + j * kConsumerThreads;
+        uint4 raw;
+        if (vi < nvec && load_vec<Checked>(sbuf + 16 * vi, bd, raw)) {
+            const int col = col0 + vi * EPV;
+            const bool masked = causal && col > row;
+            float v[EPV];
+            E::unpack(raw, v);
+            if (causal && !masked && col + EPV - 1 > row)
+                apply_causal<EPV>(v, col, row);
+            vec_exp<EPV>(v, mL, masked || m == -INFINITY);
+            s += tree_sum<EPV>(v);
+        }
+    }
+}
+
+// y = exp(v - M) / S for this thread's vectors of the part (mL = M log2 e).
+template <typename Tag, bool Checked>
+__device__ __forceinline__ void group_write(const uint4 (&r)[kGroupVecs], int nvec, int tid, int col0, int row,
+                                            bool causal, float mL, float inv, unsigned char *ypart, const Bounds &bd)
+{
+    using E = Elem<Tag>;
+    constexpr int EPV = E::kPerVec;
+#pragma unroll
+    for (int j = 0; j < kGroupVecs; ++j) {
+        const int vi = tid + j * kConsumerThreads;
+        if (vi < nvec) {
+            const int col = col0 + vi * EPV;
+            const bool masked = causal && col > row;
+            float v[EPV];
+            E::unpack(r[j], v);
+            if (causal && !masked && col + EPV - 1 > row)
+                apply_causal<EPV>(v, col, row);
+            vec_exp<EPV>(v, mL, masked);
+#pragma unroll
+            for (int e = 0; e < EPV; ++e)
+                v[e] *= inv;
+            store_vec<Checked>(ypart + 16 * vi, bd, E::pack(v));
+        }
+    }
+}
+
 template <typename Tag, bool Checked>
 __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
 {
@@ -1728,7 +1817,8 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
                 const bool ok = in && item.off >= 0 && item.C > 0 && item.nrows == 1 && item.R > 0 &&
                                 item.row0 >= 0 && item.row0 < item.R && item.off + item.C <= a.total_elems &&
                                 ((item.off * E::kSize) & 15) == 0 && ((int64_t(item.C) * E::kSize) & 15) == 0 &&
-                                part * E::kSize <= a.stage_bytes;
+                                part * E::kSize <= a.stage_bytes &&
+                                part * E::kSize <= int64_t(kGroupVecs) * 16 * kConsumerThreads;
                 if (!ok) {
                     // every member sees the same record and skips the row alike
                     atomicOr(a.status, BSM_DEV_BOUNDS);
@@ -1779,18 +1869,26 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
         __syncwarp();
     } else {
         // ----------------------------------------------------------- consumers
+        // A member takes a row's partial straight from its stage, then writes
+        // the previous row -- held in registers (thread t of the 512 consumer
+        // threads holds its vectors t, t + 512, ...: at most kGroupVecs), whose
+        // group exchange has had a whole row's time to complete -- and then
+        // moves this row from the stage into the registers and releases the
+        // stage.  So one stage is held at a time, the others are in flight.
         const bool causal = (a.flags & BSM_FLAG_CAUSAL) != 0;
         unsigned char *y = static_cast<unsigned char *>(a.y);
-        const Bounds bd0{nullptr, nullptr, y, y + a.total_elems * E::kSize, a.status};
+        const Bounds bdy{nullptr, nullptr, y, y + a.total_elems * E::kSize, a.status};
+        const int tid = warp * 32 + lane;
         uint32_t xt = 0;            // group rows this CTA took part in (the exchange sequence)
-        int pend = -1;              // stage of the row whose group exchange is outstanding
-        StageMeta pmt{};
-        uint32_t pxt = 0;
-        // the row of stage ps (exchange number x1): wait for its K partials,
-        // combine them, write this member's part, release the stage
-        auto finish = [&](int ps, const StageMeta &m1, uint32_t x1) -> bool {
-            const uint32_t slot = x1 & (kGroupSlots - 1);
-            const uint32_t target = static_cast<uint32_t>(K) * ((x1 / kGroupSlots) + 1);
+        uint4 rr[kGroupVecs];       // the row one behind: published, not yet written
+        StageMeta rm{};
+        uint32_t rx = 0;
+        bool rh = false;
+        // the row held in rr: wait for its K partials, combine them in rank
+        // order, write this member's part
+        auto finish = [&]() -> bool {
+            const uint32_t slot = rx & (kGroupSlots - 1);
+            const uint32_t target = static_cast<uint32_t>(K) * ((rx / kGroupSlots) + 1);
             int okw = 1;
             if (lane == 0)
                 okw = wait_count(&xcnt[slot], target, &h.abort_flag, wait_limit) ? 1 : 0;
@@ -1807,11 +1905,11 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
             float M = -INFINITY;
 #pragma unroll
             for (int j = 0; j < kMaxGroup / 32; ++j) {
-                const int r = lane + 32 * j;
+                const int r2 = lane + 32 * j;
                 mv[j] = -INFINITY;
                 sv[j] = 0.0f;
-                if (r < K) {
-                    const unsigned long long w = ld_relaxed_u64(&xch[slot * K + r]);
+                if (r2 < K) {
+                    const unsigned long long w = ld_relaxed_u64(&xch[slot * K + r2]);
                     mv[j] = __uint_as_float(static_cast<uint32_t>(w));
                     sv[j] = __uint_as_float(static_cast<uint32_t>(w >> 32));
                     M = fmaxf(M, mv[j]);
@@ -1824,23 +1922,16 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
                 if (lane + 32 * j < K)
                     sum += mv[j] == M ? sv[j] : sv[j] * ex2((mv[j] - M) * kLog2e);
             sum = group_sum<32>(sum);
-            if (m1.C > 0) {
-                StageMeta mw = m1;
-                mw.pass = 1;
-                float dm = -INFINITY, ds = 0.0f;
-                long_chunk<Tag, Checked>(stages + static_cast<size_t>(ps) * a.stage_bytes, mw, y, causal, warp,
-                                         lane, bd0, dm, ds, M * kLog2e, __frcp_rn(sum));
-            }
-            __syncwarp();
-            if (lane == 0)
-                mbar_arrive(&h.empty[ps]);
+            group_write<Tag, Checked>(rr, (rm.C * E::kSize) >> 4, tid, rm.col0, rm.row0, causal, M * kLog2e,
+                                      __frcp_rn(sum), y + rm.off * E::kSize, bdy);
+            rh = false;
             return true;
         };
         bool failed = false;
         for (uint32_t it = 0;; ++it) {
             const int s = static_cast<int>(it % S);
             const uint32_t ph = (it / S) & 1u;
-            // the whole warp gives up together (a shuffle below needs all lanes)
+            // the whole warp gives up together (the shuffles need all lanes)
             if (!__all_sync(0xFFFFFFFFu, mbar_wait_bounded(&h.full[s], ph, &h.abort_flag, wait_limit))) {
                 if (lane == 0) {
                     atomicOr(a.status, BSM_DEV_TIMEOUT);
@@ -1858,16 +1949,19 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
                     mbar_arrive(&h.empty[s]);
                 continue;
             }
-            // pass 0: this member's (max, sum) of its part
-            float m_l = -INFINITY, s_l = 0.0f;
-            if (mt.C > 0)
-                long_chunk<Tag, Checked>(stages + static_cast<size_t>(s) * a.stage_bytes, mt, y, causal, warp, lane,
-                                         bd0, m_l, s_l, 0.0f, 0.0f);
+            const int nvec = (mt.C * E::kSize) >> 4;
+            const unsigned char *sbuf = stages + static_cast<size_t>(s) * a.stage_bytes;
+            Bounds bs = bdy;
+            bs.s_lo = sbuf;
+            bs.s_hi = sbuf + static_cast<size_t>(mt.C) * E::kSize;
+            // this member's (max, sum) of its part, from the stage
+            float m_l, s_l;
+            group_partial<Tag, Checked>(sbuf, nvec, tid, mt.col0, mt.row0, causal, bs, m_l, s_l);
 #pragma unroll
-            for (int o = 16; o >= 1; o >>= 1) {
-                const float mo = __shfl_xor_sync(0xFFFFFFFFu, m_l, o);
-                const float so = __shfl_xor_sync(0xFFFFFFFFu, s_l, o);
-                combine_ms(m_l, s_l, mo, so);
+            for (int o2 = 16; o2 >= 1; o2 >>= 1) {
+                const float mo2 = __shfl_xor_sync(0xFFFFFFFFu, m_l, o2);
+                const float so2 = __shfl_xor_sync(0xFFFFFFFFu, s_l, o2);
+                combine_ms(m_l, s_l, mo2, so2);
             }
             const int par = xt & 1;
             if (lane == 0) {
@@ -1890,18 +1984,23 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
                 st_relaxed_u64(&xch[slot * K + rank], pack_ms(m, sum));
                 red_release_add(&xcnt[slot], 1u);
             }
-            // the previous row's partials are (nearly) in by now: finish it
-            if (pend >= 0 && !finish(pend, pmt, pxt)) {
+            // the previous row: its partials are (nearly) in by now
+            if (rh && !finish()) {
                 failed = true;
                 break;
             }
-            pend = s;
-            pmt = mt;
-            pxt = xt;
+            // this row into the registers; the stage is free
+            group_load<Tag, Checked>(rr, sbuf, nvec, tid, bs);
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(&h.empty[s]);
+            rm = mt;
+            rx = xt;
+            rh = true;
             ++xt;
         }
-        if (pend >= 0 && !failed)
-            finish(pend, pmt, pxt);
+        if (!failed && rh)
+            finish();
         __syncwarp();
     }
     // the last CTA out resets the queue heads, the claim rings and the
