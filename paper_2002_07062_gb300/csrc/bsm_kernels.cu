@@ -1665,12 +1665,13 @@ __device__ __forceinline__ void group_load(uint4 (&r)[kGroupVecs], const unsigne
     }
 }
 
-// This thread's (max, sum of exp(v - max)) over its vectors of the part in
-// the stage: the maximum first (exact), then the sum in vector order; a part
-// whose values are all -inf (masked) adds 0, a NaN or +inf makes the sum NaN.
-template <typename Tag, bool Checked>
-__device__ __forceinline__ void group_partial(const unsigned char *sbuf, int nvec, int tid, int col0, int row,
-                                              bool causal, const Bounds &bd, float &m, float &s)
+// This thread's (max, sum of exp(v - max)) over its vectors of the part,
+// from the registers: the maximum first (exact), then the sum in vector
+// order; a part whose values are all -inf (masked) adds 0, a NaN or +inf
+// makes the sum NaN.
+template <typename Tag>
+__device__ __forceinline__ void group_partial(const uint4 (&r)[kGroupVecs], int nvec, int tid, int col0, int row,
+                                              bool causal, float &m, float &s)
 {
     using E = Elem<Tag>;
     constexpr int EPV = E::kPerVec;
@@ -1679,10 +1680,9 @@ __device__ __forceinline__ void group_partial(const unsigned char *sbuf, int nve
     for (int j = 0; j < kGroupVecs; ++j) {
         const int vi = tid + j * kConsumerThreads;
         const int col = col0 + vi * EPV;
-        uint4 raw;
-        if (vi < nvec && !(causal && col > row) && load_vec<Checked>(sbuf + 16 * vi, bd, raw)) {
+        if (vi < nvec && !(causal && col > row)) {
             float v[EPV];
-            E::unpack(raw, v);
+            E::unpack(r[j], v);
             if (causal && col + EPV - 1 > row)
                 apply_causal<EPV>(v, col, row);
             m = fmaxf(m, tree_max<EPV>(v));
@@ -1693,12 +1693,11 @@ __device__ __forceinline__ void group_partial(const unsigned char *sbuf, int nve
 #pragma unroll
     for (int j = 0; j < kGroupVecs; ++j) {
         const int vi = tid + j * kConsumerThreads;
-        uint4 raw;
-        if (vi < nvec && load_vec<Checked>(sbuf + 16 * vi, bd, raw)) {
+        if (vi < nvec) {
             const int col = col0 + vi * EPV;
             const bool masked = causal && col > row;
             float v[EPV];
-            E::unpack(raw, v);
+            E::unpack(r[j], v);
             if (causal && !masked && col + EPV - 1 > row)
                 apply_causal<EPV>(v, col, row);
             vec_exp<EPV>(v, mL, masked || m == -INFINITY);
@@ -1869,65 +1868,18 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
         __syncwarp();
     } else {
         // ----------------------------------------------------------- consumers
-        // A member takes a row's partial straight from its stage, then writes
-        // the previous row -- held in registers (thread t of the 512 consumer
-        // threads holds its vectors t, t + 512, ...: at most kGroupVecs), whose
-        // group exchange has had a whole row's time to complete -- and then
-        // moves this row from the stage into the registers and releases the
-        // stage.  So one stage is held at a time, the others are in flight.
+        // A member moves its part from the stage into registers (thread t of
+        // the 512 consumer threads holds its vectors t, t + 512, ...: at most
+        // kGroupVecs, eight independent loads) and releases the stage at once,
+        // so that every stage is in flight while the group exchanges; then it
+        // takes its partial, publishes it, waits for the group's and writes
+        // its part, all from the registers.
         const bool causal = (a.flags & BSM_FLAG_CAUSAL) != 0;
         unsigned char *y = static_cast<unsigned char *>(a.y);
         const Bounds bdy{nullptr, nullptr, y, y + a.total_elems * E::kSize, a.status};
         const int tid = warp * 32 + lane;
         uint32_t xt = 0;            // group rows this CTA took part in (the exchange sequence)
-        uint4 rr[kGroupVecs];       // the row one behind: published, not yet written
-        StageMeta rm{};
-        uint32_t rx = 0;
-        bool rh = false;
-        // the row held in rr: wait for its K partials, combine them in rank
-        // order, write this member's part
-        auto finish = [&]() -> bool {
-            const uint32_t slot = rx & (kGroupSlots - 1);
-            const uint32_t target = static_cast<uint32_t>(K) * ((rx / kGroupSlots) + 1);
-            int okw = 1;
-            if (lane == 0)
-                okw = wait_count(&xcnt[slot], target, &h.abort_flag, wait_limit) ? 1 : 0;
-            okw = __shfl_sync(0xFFFFFFFFu, okw, 0);
-            if (!okw) {
-                if (lane == 0) {
-                    atomicOr(a.status, BSM_DEV_TIMEOUT);
-                    h.abort_flag = 1;
-                }
-                return false;
-            }
-            (void)ld_acquire_u32(&xcnt[slot]);   // this lane's reads below come after the count
-            float mv[kMaxGroup / 32], sv[kMaxGroup / 32];
-            float M = -INFINITY;
-#pragma unroll
-            for (int j = 0; j < kMaxGroup / 32; ++j) {
-                const int r2 = lane + 32 * j;
-                mv[j] = -INFINITY;
-                sv[j] = 0.0f;
-                if (r2 < K) {
-                    const unsigned long long w = ld_relaxed_u64(&xch[slot * K + r2]);
-                    mv[j] = __uint_as_float(static_cast<uint32_t>(w));
-                    sv[j] = __uint_as_float(static_cast<uint32_t>(w >> 32));
-                    M = fmaxf(M, mv[j]);
-                }
-            }
-            M = group_max<32>(M);
-            float sum = 0.0f;
-#pragma unroll
-            for (int j = 0; j < kMaxGroup / 32; ++j)
-                if (lane + 32 * j < K)
-                    sum += mv[j] == M ? sv[j] : sv[j] * ex2((mv[j] - M) * kLog2e);
-            sum = group_sum<32>(sum);
-            group_write<Tag, Checked>(rr, (rm.C * E::kSize) >> 4, tid, rm.col0, rm.row0, causal, M * kLog2e,
-                                      __frcp_rn(sum), y + rm.off * E::kSize, bdy);
-            rh = false;
-            return true;
-        };
-        bool failed = false;
+        uint4 rr[kGroupVecs];
         for (uint32_t it = 0;; ++it) {
             const int s = static_cast<int>(it % S);
             const uint32_t ph = (it / S) & 1u;
@@ -1937,7 +1889,6 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
                     atomicOr(a.status, BSM_DEV_TIMEOUT);
                     h.abort_flag = 1;
                 }
-                failed = true;
                 break;
             }
             const StageMeta mt = h.meta[s];
@@ -1954,9 +1905,13 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
             Bounds bs = bdy;
             bs.s_lo = sbuf;
             bs.s_hi = sbuf + static_cast<size_t>(mt.C) * E::kSize;
-            // this member's (max, sum) of its part, from the stage
+            group_load<Tag, Checked>(rr, sbuf, nvec, tid, bs);
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(&h.empty[s]);          // the part is in registers: the stage is free
+            // this member's (max, sum): lanes, then warps in order
             float m_l, s_l;
-            group_partial<Tag, Checked>(sbuf, nvec, tid, mt.col0, mt.row0, causal, bs, m_l, s_l);
+            group_partial<Tag>(rr, nvec, tid, mt.col0, mt.row0, causal, m_l, s_l);
 #pragma unroll
             for (int o2 = 16; o2 >= 1; o2 >>= 1) {
                 const float mo2 = __shfl_xor_sync(0xFFFFFFFFu, m_l, o2);
@@ -1973,34 +1928,46 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
                     atomicOr(a.status, BSM_DEV_TIMEOUT);
                     h.abort_flag = 1;
                 }
-                failed = true;
                 break;
             }
+            const uint32_t slot = xt & (kGroupSlots - 1);
             if (warp == 0 && lane == 0) {
                 float m = -INFINITY, sum = 0.0f;
                 for (int w = 0; w < kConsumerWarps; ++w)
                     combine_ms(m, sum, h.partial[par][w].x, h.partial[par][w].y);
-                const uint32_t slot = xt & (kGroupSlots - 1);
                 st_relaxed_u64(&xch[slot * K + rank], pack_ms(m, sum));
                 red_release_add(&xcnt[slot], 1u);
             }
-            // the previous row: its partials are (nearly) in by now
-            if (rh && !finish()) {
-                failed = true;
+            // the group's K partials of this row, combined in rank order
+            const uint32_t target = static_cast<uint32_t>(K) * ((xt / kGroupSlots) + 1);
+            int okw = 1;
+            if (lane == 0)
+                okw = wait_count(&xcnt[slot], target, &h.abort_flag, wait_limit) ? 1 : 0;
+            okw = __shfl_sync(0xFFFFFFFFu, okw, 0);
+            if (!okw) {
+                if (lane == 0) {
+                    atomicOr(a.status, BSM_DEV_TIMEOUT);
+                    h.abort_flag = 1;
+                }
                 break;
             }
-            // this row into the registers; the stage is free
-            group_load<Tag, Checked>(rr, sbuf, nvec, tid, bs);
-            __syncwarp();
-            if (lane == 0)
-                mbar_arrive(&h.empty[s]);
-            rm = mt;
-            rx = xt;
-            rh = true;
+            (void)ld_acquire_u32(&xcnt[slot]);   // this lane's reads below come after the count
+            float M = -INFINITY;
+            for (int r2 = lane; r2 < K; r2 += 32)
+                M = fmaxf(M, __uint_as_float(static_cast<uint32_t>(ld_relaxed_u64(&xch[slot * K + r2]))));
+            M = group_max<32>(M);
+            float sum = 0.0f;
+            for (int r2 = lane; r2 < K; r2 += 32) {
+                const unsigned long long w = ld_relaxed_u64(&xch[slot * K + r2]);
+                const float mr = __uint_as_float(static_cast<uint32_t>(w));
+                const float sr = __uint_as_float(static_cast<uint32_t>(w >> 32));
+                sum += mr == M ? sr : sr * ex2((mr - M) * kLog2e);
+            }
+            sum = group_sum<32>(sum);
+            group_write<Tag, Checked>(rr, nvec, tid, mt.col0, mt.row0, causal, M * kLog2e, __frcp_rn(sum),
+                                      y + mt.off * E::kSize, bdy);
             ++xt;
         }
-        if (!failed && rh)
-            finish();
         __syncwarp();
     }
     // the last CTA out resets the queue heads, the claim rings and the
