@@ -1665,43 +1665,58 @@ __device__ __forceinline__ void group_load(uint4 (&r)[kGroupVecs], const unsigne
     }
 }
 
-// This thread's (max, sum of exp(v - max)) over its vectors of the part,
-// from the registers: the maximum first (exact), then the sum in vector
-// order; a part whose values are all -inf (masked) adds 0, a NaN or +inf
-// makes the sum NaN.
-template <typename Tag>
-__device__ __forceinline__ void group_partial(const uint4 (&r)[kGroupVecs], int nvec, int tid, int col0, int row,
-                                              bool causal, float &m, float &s)
+// This thread's running (max, sum of exp(v - max)) over its vectors of the
+// part in the stage, in chunks of 16 elements (4 fp32 or 2 bf16 vectors, so
+// the chunk's unpacked values and the held row fit the registers): a chunk's vectors are
+// loaded first (independent loads), then its maximum taken and, when it
+// grows the running one, the sum rescaled; then the chunk's exponentials
+// added in vector order.  While the running maximum is -inf every value seen
+// is -inf (masked) or NaN: it adds 0 (NaN).
+template <typename Tag, bool Checked>
+__device__ __forceinline__ void group_partial(const unsigned char *sbuf, int nvec, int tid, int col0, int row,
+                                              bool causal, const Bounds &bd, float &m, float &s)
 {
     using E = Elem<Tag>;
     constexpr int EPV = E::kPerVec;
+    constexpr int kGroupChunk = 16 / EPV;
     m = -INFINITY;
-#pragma unroll
-    for (int j = 0; j < kGroupVecs; ++j) {
-        const int vi = tid + j * kConsumerThreads;
-        const int col = col0 + vi * EPV;
-        if (vi < nvec && !(causal && col > row)) {
-            float v[EPV];
-            E::unpack(r[j], v);
-            if (causal && col + EPV - 1 > row)
-                apply_causal<EPV>(v, col, row);
-            m = fmaxf(m, tree_max<EPV>(v));
-        }
-    }
-    const float mL = m * kLog2e;
     s = 0.0f;
 #pragma unroll
-    for (int j = 0; j < kGroupVecs; ++j) {
-        const int vi = tid + j * kConsumerThreads;
-        if (vi < nvec) {
+    for (int c = 0; c < kGroupVecs; c += kGroupChunk) {
+        uint4 raw[kGroupChunk];
+#pragma unroll
+        for (int j = 0; j < kGroupChunk; ++j) {
+            const int vi = tid + (c + j) * kConsumerThreads;
+            raw[j] = E::neg_inf_vec();
+            if (vi < nvec) {
+                uint4 t;
+                if (load_vec<Checked>(sbuf + 16 * vi, bd, t))
+                    raw[j] = t;
+            }
+        }
+        float cm = -INFINITY;
+        float v[kGroupChunk][EPV];
+#pragma unroll
+        for (int j = 0; j < kGroupChunk; ++j) {
+            const int col = col0 + (tid + (c + j) * kConsumerThreads) * EPV;
+            E::unpack(raw[j], v[j]);
+            if (causal && col + EPV - 1 > row)
+                apply_causal<EPV>(v[j], col, row);
+            cm = fmaxf(cm, tree_max<EPV>(v[j]));
+        }
+        if (cm > m) {
+            s *= ex2((m - cm) * kLog2e);
+            m = cm;
+        }
+        const float mL = m * kLog2e;
+#pragma unroll
+        for (int j = 0; j < kGroupChunk; ++j) {
+            const int vi = tid + (c + j) * kConsumerThreads;
             const int col = col0 + vi * EPV;
-            const bool masked = causal && col > row;
-            float v[EPV];
-            E::unpack(r[j], v);
-            if (causal && !masked && col + EPV - 1 > row)
-                apply_causal<EPV>(v, col, row);
-            vec_exp<EPV>(v, mL, masked || m == -INFINITY);
-            s += tree_sum<EPV>(v);
+            if (vi < nvec) {
+                vec_exp<EPV>(v[j], mL, (causal && col > row) || m == -INFINITY);
+                s += tree_sum<EPV>(v[j]);
+            }
         }
     }
 }
@@ -1868,18 +1883,58 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
         __syncwarp();
     } else {
         // ----------------------------------------------------------- consumers
-        // A member moves its part from the stage into registers (thread t of
-        // the 512 consumer threads holds its vectors t, t + 512, ...: at most
-        // kGroupVecs, eight independent loads) and releases the stage at once,
-        // so that every stage is in flight while the group exchanges; then it
-        // takes its partial, publishes it, waits for the group's and writes
-        // its part, all from the registers.
+        // A member takes a row's partial straight from its stage, then writes
+        // the previous row -- held in registers (thread t of the 512 consumer
+        // threads holds its vectors t, t + 512, ...: at most kGroupVecs), whose
+        // group exchange has had this row's partial to complete -- and then
+        // moves this row from the stage into the registers and releases the
+        // stage.  One stage is held at a time; the others are in flight.
         const bool causal = (a.flags & BSM_FLAG_CAUSAL) != 0;
         unsigned char *y = static_cast<unsigned char *>(a.y);
         const Bounds bdy{nullptr, nullptr, y, y + a.total_elems * E::kSize, a.status};
         const int tid = warp * 32 + lane;
         uint32_t xt = 0;            // group rows this CTA took part in (the exchange sequence)
-        uint4 rr[kGroupVecs];
+        uint4 rr[kGroupVecs];       // the row one behind: published, not yet written
+        StageMeta rm{};
+        uint32_t rx = 0;
+        bool rh = false;
+        // the row held in rr: wait for its K partials, combine them in rank
+        // order, write this member's part
+        auto finish = [&]() -> bool {
+            const uint32_t slot = rx & (kGroupSlots - 1);
+            const uint32_t target = static_cast<uint32_t>(K) * ((rx / kGroupSlots) + 1);
+            int okw = 1;
+            if (lane == 0)
+                okw = wait_count(&xcnt[slot], target, &h.abort_flag, wait_limit) ? 1 : 0;
+            // lane 0's acquire, then the warp barrier: the other lanes' reads
+            // below come after the count
+            __syncwarp();
+            okw = __shfl_sync(0xFFFFFFFFu, okw, 0);
+            if (!okw) {
+                if (lane == 0) {
+                    atomicOr(a.status, BSM_DEV_TIMEOUT);
+                    h.abort_flag = 1;
+                }
+                return false;
+            }
+            float M = -INFINITY;
+            for (int r2 = lane; r2 < K; r2 += 32)
+                M = fmaxf(M, __uint_as_float(static_cast<uint32_t>(ld_relaxed_u64(&xch[slot * K + r2]))));
+            M = group_max<32>(M);
+            float sum = 0.0f;
+            for (int r2 = lane; r2 < K; r2 += 32) {
+                const unsigned long long w = ld_relaxed_u64(&xch[slot * K + r2]);
+                const float mr = __uint_as_float(static_cast<uint32_t>(w));
+                const float sr = __uint_as_float(static_cast<uint32_t>(w >> 32));
+                sum += mr == M ? sr : sr * ex2((mr - M) * kLog2e);
+            }
+            sum = group_sum<32>(sum);
+            group_write<Tag, Checked>(rr, (rm.C * E::kSize) >> 4, tid, rm.col0, rm.row0, causal, M * kLog2e,
+                                      __frcp_rn(sum), y + rm.off * E::kSize, bdy);
+            rh = false;
+            return true;
+        };
+        bool failed = false;
         for (uint32_t it = 0;; ++it) {
             const int s = static_cast<int>(it % S);
             const uint32_t ph = (it / S) & 1u;
@@ -1889,6 +1944,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
                     atomicOr(a.status, BSM_DEV_TIMEOUT);
                     h.abort_flag = 1;
                 }
+                failed = true;
                 break;
             }
             const StageMeta mt = h.meta[s];
@@ -1905,13 +1961,9 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
             Bounds bs = bdy;
             bs.s_lo = sbuf;
             bs.s_hi = sbuf + static_cast<size_t>(mt.C) * E::kSize;
-            group_load<Tag, Checked>(rr, sbuf, nvec, tid, bs);
-            __syncwarp();
-            if (lane == 0)
-                mbar_arrive(&h.empty[s]);          // the part is in registers: the stage is free
-            // this member's (max, sum): lanes, then warps in order
+            // this member's (max, sum) of its part, from the stage
             float m_l, s_l;
-            group_partial<Tag>(rr, nvec, tid, mt.col0, mt.row0, causal, m_l, s_l);
+            group_partial<Tag, Checked>(sbuf, nvec, tid, mt.col0, mt.row0, causal, bs, m_l, s_l);
 #pragma unroll
             for (int o2 = 16; o2 >= 1; o2 >>= 1) {
                 const float mo2 = __shfl_xor_sync(0xFFFFFFFFu, m_l, o2);
@@ -1928,46 +1980,34 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
                     atomicOr(a.status, BSM_DEV_TIMEOUT);
                     h.abort_flag = 1;
                 }
+                failed = true;
                 break;
             }
-            const uint32_t slot = xt & (kGroupSlots - 1);
             if (warp == 0 && lane == 0) {
                 float m = -INFINITY, sum = 0.0f;
                 for (int w = 0; w < kConsumerWarps; ++w)
                     combine_ms(m, sum, h.partial[par][w].x, h.partial[par][w].y);
+                const uint32_t slot = xt & (kGroupSlots - 1);
                 st_relaxed_u64(&xch[slot * K + rank], pack_ms(m, sum));
                 red_release_add(&xcnt[slot], 1u);
             }
-            // the group's K partials of this row, combined in rank order
-            const uint32_t target = static_cast<uint32_t>(K) * ((xt / kGroupSlots) + 1);
-            int okw = 1;
-            if (lane == 0)
-                okw = wait_count(&xcnt[slot], target, &h.abort_flag, wait_limit) ? 1 : 0;
-            okw = __shfl_sync(0xFFFFFFFFu, okw, 0);
-            if (!okw) {
-                if (lane == 0) {
-                    atomicOr(a.status, BSM_DEV_TIMEOUT);
-                    h.abort_flag = 1;
-                }
+            // the previous row: its partials are (nearly) in by now
+            if (rh && !finish()) {
+                failed = true;
                 break;
             }
-            (void)ld_acquire_u32(&xcnt[slot]);   // this lane's reads below come after the count
-            float M = -INFINITY;
-            for (int r2 = lane; r2 < K; r2 += 32)
-                M = fmaxf(M, __uint_as_float(static_cast<uint32_t>(ld_relaxed_u64(&xch[slot * K + r2]))));
-            M = group_max<32>(M);
-            float sum = 0.0f;
-            for (int r2 = lane; r2 < K; r2 += 32) {
-                const unsigned long long w = ld_relaxed_u64(&xch[slot * K + r2]);
-                const float mr = __uint_as_float(static_cast<uint32_t>(w));
-                const float sr = __uint_as_float(static_cast<uint32_t>(w >> 32));
-                sum += mr == M ? sr : sr * ex2((mr - M) * kLog2e);
-            }
-            sum = group_sum<32>(sum);
-            group_write<Tag, Checked>(rr, nvec, tid, mt.col0, mt.row0, causal, M * kLog2e, __frcp_rn(sum),
-                                      y + mt.off * E::kSize, bdy);
+            // this row into the registers; the stage is free
+            group_load<Tag, Checked>(rr, sbuf, nvec, tid, bs);
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(&h.empty[s]);
+            rm = mt;
+            rx = xt;
+            rh = true;
             ++xt;
         }
+        if (!failed && rh)
+            finish();
         __syncwarp();
     }
     // the last CTA out resets the queue heads, the claim rings and the
