@@ -66,6 +66,7 @@ struct SmemHeader {
     uint64_t full[kMaxStages];
     uint64_t empty[kMaxStages];
     uint64_t xwarp;                 // long rows: the consumer warps' partials are in
+    uint64_t xwarp2[2];             // rows over groups: the same, by row parity (warp 0 alone waits)
     StageMeta meta[kMaxStages];
     float2 partial[2][kConsumerWarps];   // long rows: (max, sum) per warp, two rows deep
     int32_t abort_flag;
@@ -1598,6 +1599,15 @@ __device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t *p)
     return v;
 }
 
+__device__ __forceinline__ uint32_t ld_relaxed_u32(const uint32_t *p)
+{
+    uint32_t v;
+    asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
+
 __device__ __forceinline__ void red_release_add(uint32_t *p, uint32_t v)
 {
     asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
@@ -1769,7 +1779,8 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
             mbar_init(&h.full[s], 1);
             mbar_init(&h.empty[s], kConsumerWarps);
         }
-        mbar_init(&h.xwarp, kConsumerWarps);
+        mbar_init(&h.xwarp2[0], kConsumerWarps);
+        mbar_init(&h.xwarp2[1], kConsumerWarps);
         h.abort_flag = 0;
         mbar_init_fence();
     }
@@ -1898,16 +1909,18 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
         StageMeta rm{};
         uint32_t rx = 0;
         bool rh = false;
-        // the row held in rr: wait for its K partials, combine them in rank
-        // order, write this member's part
-        auto finish = [&]() -> bool {
+        // the row held in rr: wait for its K partials (pre: the counter read
+        // early, relaxed), combine them in rank order, write this member's part
+        auto finish = [&](uint32_t pre) -> bool {
             const uint32_t slot = rx & (kGroupSlots - 1);
             const uint32_t target = static_cast<uint32_t>(K) * ((rx / kGroupSlots) + 1);
             int okw = 1;
-            if (lane == 0)
-                okw = wait_count(&xcnt[slot], target, &h.abort_flag, wait_limit) ? 1 : 0;
-            // lane 0's acquire, then the warp barrier: the other lanes' reads
-            // below come after the count
+            if (lane == 0) {
+                if (pre < target)
+                    okw = wait_count(&xcnt[slot], target, &h.abort_flag, wait_limit) ? 1 : 0;
+                fence_acq_rel_gpu();        // the count seen: the partials it counts are visible
+            }
+            // then the warp barrier: the other lanes' reads below come after it
             __syncwarp();
             okw = __shfl_sync(0xFFFFFFFFu, okw, 0);
             if (!okw) {
@@ -1917,17 +1930,27 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
                 }
                 return false;
             }
-            float M = -INFINITY;
-            for (int r2 = lane; r2 < K; r2 += 32)
-                M = fmaxf(M, __uint_as_float(static_cast<uint32_t>(ld_relaxed_u64(&xch[slot * K + r2]))));
+            // the K partials in one round of loads: lane l holds ranks l, l + 32, ...
+            float mv[kMaxGroup / 32], sv[kMaxGroup / 32];
+#pragma unroll
+            for (int j = 0; j < kMaxGroup / 32; ++j) {
+                const int r2 = lane + 32 * j;
+                unsigned long long w = 0xFF800000ull;        // (-inf, 0)
+                if (r2 < K)
+                    w = ld_relaxed_u64(&xch[slot * K + r2]);
+                mv[j] = __uint_as_float(static_cast<uint32_t>(w));
+                sv[j] = __uint_as_float(static_cast<uint32_t>(w >> 32));
+            }
+            float M = mv[0];
+#pragma unroll
+            for (int j = 1; j < kMaxGroup / 32; ++j)
+                M = fmaxf(M, mv[j]);
             M = group_max<32>(M);
             float sum = 0.0f;
-            for (int r2 = lane; r2 < K; r2 += 32) {
-                const unsigned long long w = ld_relaxed_u64(&xch[slot * K + r2]);
-                const float mr = __uint_as_float(static_cast<uint32_t>(w));
-                const float sr = __uint_as_float(static_cast<uint32_t>(w >> 32));
-                sum += mr == M ? sr : sr * ex2((mr - M) * kLog2e);
-            }
+#pragma unroll
+            for (int j = 0; j < kMaxGroup / 32; ++j)
+                if (lane + 32 * j < K)
+                    sum += mv[j] == M ? sv[j] : sv[j] * ex2((mv[j] - M) * kLog2e);
             sum = group_sum<32>(sum);
             group_write<Tag, Checked>(rr, (rm.C * E::kSize) >> 4, tid, rm.col0, rm.row0, causal, M * kLog2e,
                                       __frcp_rn(sum), y + rm.off * E::kSize, bdy);
@@ -1956,6 +1979,11 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
                     mbar_arrive(&h.empty[s]);
                 continue;
             }
+            // the held row's exchange counter, read now and used after this
+            // row's partial (its latency overlaps the partial)
+            uint32_t pre = 0;
+            if (rh && lane == 0)
+                pre = ld_relaxed_u32(&xcnt[rx & (kGroupSlots - 1)]);
             const int nvec = (mt.C * E::kSize) >> 4;
             const unsigned char *sbuf = stages + static_cast<size_t>(s) * a.stage_bytes;
             Bounds bs = bdy;
@@ -1970,29 +1998,39 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
                 const float so2 = __shfl_xor_sync(0xFFFFFFFFu, s_l, o2);
                 combine_ms(m_l, s_l, mo2, so2);
             }
+            // the warps' partials (two barriers by row parity: a warp may run a
+            // row ahead of warp 0, never two); warp 0 alone waits, combines
+            // them (a fixed tree over 16 lanes) and publishes the CTA's
             const int par = xt & 1;
             if (lane == 0) {
                 h.partial[par][warp] = make_float2(m_l, s_l);
-                mbar_arrive(&h.xwarp);
+                mbar_arrive(&h.xwarp2[par]);
             }
-            if (!__all_sync(0xFFFFFFFFu, mbar_wait_bounded(&h.xwarp, xt & 1u, &h.abort_flag, wait_limit))) {
-                if (lane == 0) {
-                    atomicOr(a.status, BSM_DEV_TIMEOUT);
-                    h.abort_flag = 1;
+            if (warp == 0) {
+                if (!__all_sync(0xFFFFFFFFu,
+                                mbar_wait_bounded(&h.xwarp2[par], (xt >> 1) & 1u, &h.abort_flag, wait_limit))) {
+                    if (lane == 0) {
+                        atomicOr(a.status, BSM_DEV_TIMEOUT);
+                        h.abort_flag = 1;
+                    }
+                    failed = true;
+                    break;
                 }
-                failed = true;
-                break;
-            }
-            if (warp == 0 && lane == 0) {
-                float m = -INFINITY, sum = 0.0f;
-                for (int w = 0; w < kConsumerWarps; ++w)
-                    combine_ms(m, sum, h.partial[par][w].x, h.partial[par][w].y);
-                const uint32_t slot = xt & (kGroupSlots - 1);
-                st_relaxed_u64(&xch[slot * K + rank], pack_ms(m, sum));
-                red_release_add(&xcnt[slot], 1u);
+                float2 pw = lane < kConsumerWarps ? h.partial[par][lane] : make_float2(-INFINITY, 0.0f);
+#pragma unroll
+                for (int o2 = kConsumerWarps / 2; o2 >= 1; o2 >>= 1) {
+                    const float mo2 = __shfl_xor_sync(0xFFFFFFFFu, pw.x, o2);
+                    const float so2 = __shfl_xor_sync(0xFFFFFFFFu, pw.y, o2);
+                    combine_ms(pw.x, pw.y, mo2, so2);
+                }
+                if (lane == 0) {
+                    const uint32_t slot = xt & (kGroupSlots - 1);
+                    st_relaxed_u64(&xch[slot * K + rank], pack_ms(pw.x, pw.y));
+                    red_release_add(&xcnt[slot], 1u);
+                }
             }
             // the previous row: its partials are (nearly) in by now
-            if (rh && !finish()) {
+            if (rh && !finish(pre)) {
                 failed = true;
                 break;
             }
@@ -2007,7 +2045,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
             ++xt;
         }
         if (!failed && rh)
-            finish();
+            finish(0u);
         __syncwarp();
     }
     // the last CTA out resets the queue heads, the claim rings and the
