@@ -842,15 +842,14 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     auto up = [](size_t v) { return (v + 255) & ~size_t(255); };
     const int64_t gk = lay.group_k, gn = n_grp ? lay.n_groups : 0;
     const size_t itemsg_b = sizeof(Item) * items_g.size(), ring_b = sizeof(uint64_t) * kGroupRing * size_t(gn),
-                 xch_b = sizeof(uint64_t) * kGroupSlots * size_t(gn * gk),
-                 xcnt_b = sizeof(uint32_t) * kGroupSlots * size_t(gn);
+                 xch_b = 2 * sizeof(uint64_t) * kGroupSlots * size_t(gn * gk);
     const size_t o_items = 0, o_slices = up(items_b), o_smdie = o_slices + up(slices_b),
                  o_heads = o_smdie + 256, o_segs = o_heads + 256, o_items1 = o_segs + up(segs_b),
                  o_segs1 = o_items1 + up(items1_b), o_slices1 = o_segs1 + up(segs1_b),
                  o_heads1 = o_slices1 + (n1 ? up(slices_b) : 0), o_parts = o_heads1 + 256,
                  o_itemsg = o_parts + up(parts_b), o_slicesg = o_itemsg + up(itemsg_b),
                  o_headsg = o_slicesg + (n_grp ? up(slices_b) : 0), o_ring = o_headsg + 256,
-                 o_xch = o_ring + up(ring_b), o_xcnt = o_xch + up(xch_b), blob_b = o_xcnt + up(xcnt_b);
+                 o_xch = o_ring + up(ring_b), blob_b = o_xch + up(xch_b);
     std::vector<unsigned char> host(blob_b, 0);
     if (n_grp) {
         std::memcpy(&host[o_itemsg], items_g.data(), itemsg_b);
@@ -957,7 +956,6 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
         ag.n_groups = lay.n_groups;
         ag.ring = reinterpret_cast<unsigned long long *>(b + o_ring);
         ag.xch = reinterpret_cast<unsigned long long *>(b + o_xch);
-        ag.xcnt = reinterpret_cast<uint32_t *>(b + o_xcnt);
         p->grid_g = lay.group_k * lay.n_groups;
     }
 

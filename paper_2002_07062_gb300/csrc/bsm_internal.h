@@ -58,9 +58,10 @@ enum Op : int32_t {
 // [g*K, g*K + K); its rank-0 CTA claims rows and announces them in the
 // group's ring of kGroupRing claim words (row sequence number + 1 in the high
 // half, the row's position in the table in the low half); each member stages
-// its part of the row, publishes its (max, sum) in one of kGroupSlots
-// exchange slots and counts it in that slot's counter.  Rings and counters
-// are reset by the last CTA of every launch.
+// its part of the row and publishes its (max, sum) in one of kGroupSlots
+// exchange slots as two words (the row sequence number + 1 in the high half
+// of each, max or sum in the low half).  Rings and exchange words are reset
+// by the last CTA of every launch.
 constexpr int kGroupRing = 16;
 constexpr int kGroupSlots = 4;
 constexpr int kMaxGroup = 128;
@@ -115,8 +116,7 @@ struct KernelArgs {
     int32_t group_k;            // CTAs per group (2..kMaxGroup); the grid is n_groups * group_k
     int32_t n_groups;
     unsigned long long *ring;   // n_groups x kGroupRing claim words
-    unsigned long long *xch;    // n_groups x kGroupSlots x group_k partials: (max, sum) as two floats
-    uint32_t *xcnt;             // n_groups x kGroupSlots arrival counters
+    unsigned long long *xch;    // n_groups x kGroupSlots x group_k x 2 tagged words: max, sum
 };
 
 // Test-only fault injection (bsm_plan_debug).

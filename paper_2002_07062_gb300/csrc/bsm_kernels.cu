@@ -1556,17 +1556,17 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
 // length (whole 16-byte vectors; the last may be shorter or empty), and the K
 // CTAs of a group each stage one part in one stage: every element is read
 // from memory once.  Each CTA takes its part's running (max, rescaled sum)
-// -- lanes, then warps in a fixed order, as for the long rows above --,
-// publishes it in global memory and counts it in its slot's counter
-// (release); every member then waits for the K partials of the row
-// (acquire), combines them in the same fixed order (a per-lane sum over
-// ranks l, l + 32, ..., then the xor tree), and writes its part of y from
-// its stage.  The consumers are one row ahead: they take the next row's
-// partial before waiting for the previous row's group, so the exchange
-// overlaps work.  The group's rank-0 CTA claims the rows (any policy's puller,
-// with the group as the unit) and announces them to its members through a
-// ring of claim words.  The launch is cooperative, so every member of a group
-// is resident and each wait ends; every wait is bounded all the same.
+// -- threads, then warps in a fixed order -- and publishes it in global
+// memory as two words tagged with the row's sequence number; every member
+// then reads the K partials until all carry the tag, combines them in the
+// same fixed order (a per-lane sum over ranks l, l + 32, ..., then the xor
+// tree), and writes its part of y.  The consumers work one row ahead: they
+// take the next row's partial (from its stage) before finishing the previous
+// row (held in registers), so the exchange overlaps work.  The group's
+// rank-0 CTA claims the rows (any policy's puller, with the group as the
+// unit) and announces them to its members through a ring of claim words.
+// The launch is cooperative, so every member of a group is resident and each
+// wait ends; every wait is bounded all the same.
 
 __device__ __forceinline__ void st_release_u64(unsigned long long *p, unsigned long long v)
 {
@@ -1592,27 +1592,6 @@ __device__ __forceinline__ unsigned long long ld_relaxed_u64(const unsigned long
     return v;
 }
 
-__device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t *p)
-{
-    uint32_t v;
-    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-    return v;
-}
-
-__device__ __forceinline__ uint32_t ld_relaxed_u32(const uint32_t *p)
-{
-    uint32_t v;
-    asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-    return v;
-}
-
-__device__ __forceinline__ void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
-
-__device__ __forceinline__ void red_release_add(uint32_t *p, uint32_t v)
-{
-    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
-}
-
 // Wait until the claim word at p carries sequence number seq (bounded).
 __device__ __noinline__ bool wait_claim(const unsigned long long *p, uint32_t seq, const volatile int32_t *abort,
                                         uint64_t limit_ns, unsigned long long &word)
@@ -1625,23 +1604,6 @@ __device__ __noinline__ bool wait_claim(const unsigned long long *p, uint32_t se
         __nanosleep(32);
         word = ld_acquire_u64(p);
         if (static_cast<uint32_t>(word >> 32) == seq)
-            return true;
-        if ((abort && *abort) || global_timer_ns() - t0 > limit_ns)
-            return false;
-    }
-    return false;
-}
-
-// Wait until the counter at p reaches target (it only grows within a launch).
-__device__ __noinline__ bool wait_count(const uint32_t *p, uint32_t target, const volatile int32_t *abort,
-                                        uint64_t limit_ns)
-{
-    if (ld_acquire_u32(p) >= target)
-        return true;
-    const uint64_t t0 = global_timer_ns();
-    for (uint32_t it = 0; it < (1u << 26); ++it) {
-        __nanosleep(32);
-        if (ld_acquire_u32(p) >= target)
             return true;
         if ((abort && *abort) || global_timer_ns() - t0 > limit_ns)
             return false;
@@ -1771,8 +1733,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
     const int grp = static_cast<int>(blockIdx.x) / K, rank = static_cast<int>(blockIdx.x) % K;
     const uint64_t wait_limit = a.wait_limit_ns ? a.wait_limit_ns : kWaitLimitNs;
     unsigned long long *ring = a.ring + static_cast<size_t>(grp) * kGroupRing;
-    unsigned long long *xch = a.xch + static_cast<size_t>(grp) * kGroupSlots * K;
-    uint32_t *xcnt = a.xcnt + static_cast<size_t>(grp) * kGroupSlots;
+    unsigned long long *xch = a.xch + 2 * static_cast<size_t>(grp) * kGroupSlots * K;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
@@ -1909,37 +1870,46 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
         StageMeta rm{};
         uint32_t rx = 0;
         bool rh = false;
-        // the row held in rr: wait for its K partials (pre: the counter read
-        // early, relaxed), combine them in rank order, write this member's part
-        auto finish = [&](uint32_t pre) -> bool {
+        // the row held in rr: poll its K partials (each two words carrying the
+        // row's tag) until all are in, combine them in rank order, write this
+        // member's part
+        auto finish = [&]() -> bool {
             const uint32_t slot = rx & (kGroupSlots - 1);
-            const uint32_t target = static_cast<uint32_t>(K) * ((rx / kGroupSlots) + 1);
-            int okw = 1;
-            if (lane == 0) {
-                if (pre < target)
-                    okw = wait_count(&xcnt[slot], target, &h.abort_flag, wait_limit) ? 1 : 0;
-                fence_acq_rel_gpu();        // the count seen: the partials it counts are visible
+            const uint32_t tag = rx + 1;
+            const unsigned long long *xs = &xch[2 * static_cast<size_t>(slot) * K];
+            float mv[kMaxGroup / 32], sv[kMaxGroup / 32];
+            bool in = false;
+            const uint64_t t0 = global_timer_ns();
+            for (uint32_t tries = 0; tries < (1u << 24); ++tries) {
+                bool all = true;
+#pragma unroll
+                for (int j = 0; j < kMaxGroup / 32; ++j) {
+                    const int r2 = lane + 32 * j;
+                    mv[j] = -INFINITY;
+                    sv[j] = 0.0f;
+                    if (r2 < K) {
+                        const unsigned long long w0 = ld_relaxed_u64(&xs[2 * r2]);
+                        const unsigned long long w1 = ld_relaxed_u64(&xs[2 * r2 + 1]);
+                        all = all && static_cast<uint32_t>(w0 >> 32) == tag && static_cast<uint32_t>(w1 >> 32) == tag;
+                        mv[j] = __uint_as_float(static_cast<uint32_t>(w0));
+                        sv[j] = __uint_as_float(static_cast<uint32_t>(w1));
+                    }
+                }
+                if (__all_sync(0xFFFFFFFFu, all)) {
+                    in = true;
+                    break;
+                }
+                const int give_up = (h.abort_flag || global_timer_ns() - t0 > wait_limit) ? 1 : 0;
+                if (__any_sync(0xFFFFFFFFu, give_up))
+                    break;
+                __nanosleep(32);
             }
-            // then the warp barrier: the other lanes' reads below come after it
-            __syncwarp();
-            okw = __shfl_sync(0xFFFFFFFFu, okw, 0);
-            if (!okw) {
+            if (!in) {
                 if (lane == 0) {
                     atomicOr(a.status, BSM_DEV_TIMEOUT);
                     h.abort_flag = 1;
                 }
                 return false;
-            }
-            // the K partials in one round of loads: lane l holds ranks l, l + 32, ...
-            float mv[kMaxGroup / 32], sv[kMaxGroup / 32];
-#pragma unroll
-            for (int j = 0; j < kMaxGroup / 32; ++j) {
-                const int r2 = lane + 32 * j;
-                unsigned long long w = 0xFF800000ull;        // (-inf, 0)
-                if (r2 < K)
-                    w = ld_relaxed_u64(&xch[slot * K + r2]);
-                mv[j] = __uint_as_float(static_cast<uint32_t>(w));
-                sv[j] = __uint_as_float(static_cast<uint32_t>(w >> 32));
             }
             float M = mv[0];
 #pragma unroll
@@ -1979,11 +1949,6 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
                     mbar_arrive(&h.empty[s]);
                 continue;
             }
-            // the held row's exchange counter, read now and used after this
-            // row's partial (its latency overlaps the partial)
-            uint32_t pre = 0;
-            if (rh && lane == 0)
-                pre = ld_relaxed_u32(&xcnt[rx & (kGroupSlots - 1)]);
             const int nvec = (mt.C * E::kSize) >> 4;
             const unsigned char *sbuf = stages + static_cast<size_t>(s) * a.stage_bytes;
             Bounds bs = bdy;
@@ -2024,13 +1989,18 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
                     combine_ms(pw.x, pw.y, mo2, so2);
                 }
                 if (lane == 0) {
+                    // two self-validating words (value, row tag): 8-byte stores
+                    // are single-copy atomic, so a reader that sees the tag
+                    // sees the value written with it
                     const uint32_t slot = xt & (kGroupSlots - 1);
-                    st_relaxed_u64(&xch[slot * K + rank], pack_ms(pw.x, pw.y));
-                    red_release_add(&xcnt[slot], 1u);
+                    const unsigned long long tag = static_cast<unsigned long long>(xt + 1) << 32;
+                    unsigned long long *w = &xch[2 * (static_cast<size_t>(slot) * K + rank)];
+                    st_relaxed_u64(w, tag | __float_as_uint(pw.x));
+                    st_relaxed_u64(w + 1, tag | __float_as_uint(pw.y));
                 }
             }
             // the previous row: its partials are (nearly) in by now
-            if (rh && !finish(pre)) {
+            if (rh && !finish()) {
                 failed = true;
                 break;
             }
@@ -2045,7 +2015,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
             ++xt;
         }
         if (!failed && rh)
-            finish(0u);
+            finish();
         __syncwarp();
     }
     // the last CTA out resets the queue heads, the claim rings and the
@@ -2060,8 +2030,8 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
                 atomicExch(&a.heads[d], 0u);
             for (int i = 0; i < a.n_groups * kGroupRing; ++i)
                 a.ring[i] = 0ull;
-            for (int i = 0; i < a.n_groups * kGroupSlots; ++i)
-                a.xcnt[i] = 0u;
+            for (int i = 0; i < 2 * a.n_groups * kGroupSlots * a.group_k; ++i)
+                a.xch[i] = 0ull;
             __threadfence();
             atomicExch(&a.heads[BSM_MAX_DIES], 0u);
         }
