@@ -66,7 +66,7 @@ struct SmemHeader {
     uint64_t full[kMaxStages];
     uint64_t empty[kMaxStages];
     uint64_t xwarp;                 // long rows: the consumer warps' partials are in
-    uint64_t xwarp2[2];             // rows over groups: the same, by row parity (warp 0 alone waits)
+    uint32_t xarrive[2];            // rows over groups: warps whose partial is in, by row parity
     StageMeta meta[kMaxStages];
     float2 partial[2][kConsumerWarps];   // long rows: (max, sum) per warp, two rows deep
     int32_t abort_flag;
@@ -1740,8 +1740,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
             mbar_init(&h.full[s], 1);
             mbar_init(&h.empty[s], kConsumerWarps);
         }
-        mbar_init(&h.xwarp2[0], kConsumerWarps);
-        mbar_init(&h.xwarp2[1], kConsumerWarps);
+        h.xarrive[0] = h.xarrive[1] = 0u;
         h.abort_flag = 0;
         mbar_init_fence();
     }
@@ -1873,7 +1872,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
         // the row held in rr: poll its K partials (each two words carrying the
         // row's tag) until all are in, combine them in rank order, write this
         // member's part
-        auto finish = [&]() -> bool {
+        auto finish = [&](unsigned long long pre0, unsigned long long pre1) -> bool {
             const uint32_t slot = rx & (kGroupSlots - 1);
             const uint32_t tag = rx + 1;
             const unsigned long long *xs = &xch[2 * static_cast<size_t>(slot) * K];
@@ -1888,8 +1887,10 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
                     mv[j] = -INFINITY;
                     sv[j] = 0.0f;
                     if (r2 < K) {
-                        const unsigned long long w0 = ld_relaxed_u64(&xs[2 * r2]);
-                        const unsigned long long w1 = ld_relaxed_u64(&xs[2 * r2 + 1]);
+                        // the first round of rank `lane` was loaded early
+                        const bool early = tries == 0 && j == 0;
+                        const unsigned long long w0 = early ? pre0 : ld_relaxed_u64(&xs[2 * r2]);
+                        const unsigned long long w1 = early ? pre1 : ld_relaxed_u64(&xs[2 * r2 + 1]);
                         all = all && static_cast<uint32_t>(w0 >> 32) == tag && static_cast<uint32_t>(w1 >> 32) == tag;
                         mv[j] = __uint_as_float(static_cast<uint32_t>(w0));
                         sv[j] = __uint_as_float(static_cast<uint32_t>(w1));
@@ -1954,6 +1955,14 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
             Bounds bs = bdy;
             bs.s_lo = sbuf;
             bs.s_hi = sbuf + static_cast<size_t>(mt.C) * E::kSize;
+            // the held row's exchange words of rank `lane`, loaded now and
+            // used after this row's partial (their latency overlaps it)
+            unsigned long long pre0 = 0, pre1 = 0;
+            if (rh && lane < K) {
+                const unsigned long long *xs = &xch[2 * static_cast<size_t>(rx & (kGroupSlots - 1)) * K];
+                pre0 = ld_relaxed_u64(&xs[2 * lane]);
+                pre1 = ld_relaxed_u64(&xs[2 * lane + 1]);
+            }
             // this member's (max, sum) of its part, from the stage
             float m_l, s_l;
             group_partial<Tag, Checked>(sbuf, nvec, tid, mt.col0, mt.row0, causal, bs, m_l, s_l);
@@ -1963,24 +1972,24 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
                 const float so2 = __shfl_xor_sync(0xFFFFFFFFu, s_l, o2);
                 combine_ms(m_l, s_l, mo2, so2);
             }
-            // the warps' partials (two barriers by row parity: a warp may run a
-            // row ahead of warp 0, never two); warp 0 alone waits, combines
-            // them (a fixed tree over 16 lanes) and publishes the CTA's
+            // the warps' partials: the last warp to bring its own combines them
+            // (a fixed tree over 16 lanes) and publishes the CTA's; nobody
+            // waits.  (A warp's partial of row t + 2 comes after its finish of
+            // row t, i.e. after row t's publication: two slots by row parity.)
             const int par = xt & 1;
+            int last = 0;
             if (lane == 0) {
                 h.partial[par][warp] = make_float2(m_l, s_l);
-                mbar_arrive(&h.xwarp2[par]);
-            }
-            if (warp == 0) {
-                if (!__all_sync(0xFFFFFFFFu,
-                                mbar_wait_bounded(&h.xwarp2[par], (xt >> 1) & 1u, &h.abort_flag, wait_limit))) {
-                    if (lane == 0) {
-                        atomicOr(a.status, BSM_DEV_TIMEOUT);
-                        h.abort_flag = 1;
-                    }
-                    failed = true;
-                    break;
+                __threadfence_block();
+                last = atomicAdd(&h.xarrive[par], 1u) == static_cast<uint32_t>(kConsumerWarps - 1) ? 1 : 0;
+                if (last) {
+                    __threadfence_block();
+                    h.xarrive[par] = 0u;
                 }
+            }
+            last = __shfl_sync(0xFFFFFFFFu, last, 0);
+            if (last) {
+                __syncwarp();
                 float2 pw = lane < kConsumerWarps ? h.partial[par][lane] : make_float2(-INFINITY, 0.0f);
 #pragma unroll
                 for (int o2 = kConsumerWarps / 2; o2 >= 1; o2 >>= 1) {
@@ -2000,7 +2009,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
                 }
             }
             // the previous row: its partials are (nearly) in by now
-            if (rh && !finish()) {
+            if (rh && !finish(pre0, pre1)) {
                 failed = true;
                 break;
             }
@@ -2015,7 +2024,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
             ++xt;
         }
         if (!failed && rh)
-            finish();
+            finish(0ull, 0ull);
         __syncwarp();
     }
     // the last CTA out resets the queue heads, the claim rings and the
