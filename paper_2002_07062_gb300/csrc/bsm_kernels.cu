@@ -1645,76 +1645,12 @@ __device__ __forceinline__ void group_load(uint4 (&r)[kGroupVecs], const unsigne
 // added in vector order.  While the running maximum is -inf every value seen
 // is -inf (masked) or NaN: it adds 0 (NaN).
 template <typename Tag, bool Checked>
-__device__ __forceinline__ void group_partial(unsigned char *sbuf, int nvec, int tid, int col0, int row,
+__device__ __forceinline__ void group_partial(const unsigned char *sbuf, int nvec, int tid, int col0, int row,
                                               bool causal, const Bounds &bd, float &m, float &s)
 {
     using E = Elem<Tag>;
     constexpr int EPV = E::kPerVec;
     constexpr int kGroupChunk = 16 / EPV;
-    if constexpr (E::kSize == 4) {
-        // fp32: the maximum first, then p = exp(v - m) written back over the
-        // part in the stage and summed, so the write needs no exponential
-        // (y = p * exp(m - M) / S); the proxy fence orders these writes before
-        // the bulk copy that later refills the stage
-        m = -INFINITY;
-        s = 0.0f;
-#pragma unroll
-        for (int c = 0; c < kGroupVecs; c += kGroupChunk) {
-            uint4 raw[kGroupChunk];
-#pragma unroll
-            for (int j = 0; j < kGroupChunk; ++j) {
-                const int vi = tid + (c + j) * kConsumerThreads;
-                raw[j] = E::neg_inf_vec();
-                if (vi < nvec) {
-                    uint4 t;
-                    if (load_vec<Checked>(sbuf + 16 * vi, bd, t))
-                        raw[j] = t;
-                }
-            }
-#pragma unroll
-            for (int j = 0; j < kGroupChunk; ++j) {
-                const int col = col0 + (tid + (c + j) * kConsumerThreads) * EPV;
-                float v[EPV];
-                E::unpack(raw[j], v);
-                if (causal && col + EPV - 1 > row)
-                    apply_causal<EPV>(v, col, row);
-                m = fmaxf(m, tree_max<EPV>(v));
-            }
-        }
-        const float mL = m * kLog2e;
-#pragma unroll
-        for (int c = 0; c < kGroupVecs; c += kGroupChunk) {
-            uint4 raw[kGroupChunk];
-#pragma unroll
-            for (int j = 0; j < kGroupChunk; ++j) {
-                const int vi = tid + (c + j) * kConsumerThreads;
-                raw[j] = E::neg_inf_vec();
-                if (vi < nvec) {
-                    uint4 t;
-                    if (load_vec<Checked>(sbuf + 16 * vi, bd, t))
-                        raw[j] = t;
-                }
-            }
-#pragma unroll
-            for (int j = 0; j < kGroupChunk; ++j) {
-                const int vi = tid + (c + j) * kConsumerThreads;
-                const int col = col0 + vi * EPV;
-                if (vi < nvec) {
-                    float v[EPV];
-                    E::unpack(raw[j], v);
-                    const bool masked = causal && col > row;
-                    if (causal && !masked && col + EPV - 1 > row)
-                        apply_causal<EPV>(v, col, row);
-                    vec_exp<EPV>(v, mL, masked || m == -INFINITY);
-                    s += tree_sum<EPV>(v);
-                    if (!Checked || (sbuf + 16 * vi >= bd.s_lo && sbuf + 16 * vi + 16 <= bd.s_hi))
-                        sts128(sbuf + 16 * vi, E::pack(v));
-                }
-            }
-        }
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        return;
-    }
     m = -INFINITY;
     s = 0.0f;
 #pragma unroll
@@ -1760,28 +1696,10 @@ __device__ __forceinline__ void group_partial(unsigned char *sbuf, int nvec, int
 // y = exp(v - M) / S for this thread's vectors of the part (mL = M log2 e).
 template <typename Tag, bool Checked>
 __device__ __forceinline__ void group_write(const uint4 (&r)[kGroupVecs], int nvec, int tid, int col0, int row,
-                                            bool causal, float mL, float inv, float mt, unsigned char *ypart,
-                                            const Bounds &bd)
+                                            bool causal, float mL, float inv, unsigned char *ypart, const Bounds &bd)
 {
     using E = Elem<Tag>;
     constexpr int EPV = E::kPerVec;
-    if constexpr (E::kSize == 4) {
-        // fp32: the registers hold p = exp(v - mt) (mt: this thread's maximum)
-        const float f = (mt == -INFINITY && mL != -INFINITY ? 0.0f : ex2(fmaf(mt, kLog2e, -mL))) * inv;
-#pragma unroll
-        for (int j = 0; j < kGroupVecs; ++j) {
-            const int vi = tid + j * kConsumerThreads;
-            if (vi < nvec) {
-                float v[EPV];
-                E::unpack(r[j], v);
-#pragma unroll
-                for (int e = 0; e < EPV; ++e)
-                    v[e] *= f;
-                store_vec<Checked>(ypart + 16 * vi, bd, E::pack(v));
-            }
-        }
-        return;
-    }
 #pragma unroll
     for (int j = 0; j < kGroupVecs; ++j) {
         const int vi = tid + j * kConsumerThreads;
@@ -1948,7 +1866,6 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
         const int tid = warp * 32 + lane;
         uint32_t xt = 0;            // group rows this CTA took part in (the exchange sequence)
         uint4 rr[kGroupVecs];       // the row one behind: published, not yet written
-        float rmt = -INFINITY;      // fp32: this thread's maximum of that row (rr holds exp(v - rmt))
         StageMeta rm{};
         uint32_t rx = 0;
         bool rh = false;
@@ -2007,7 +1924,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
                     sum += mv[j] == M ? sv[j] : sv[j] * ex2((mv[j] - M) * kLog2e);
             sum = group_sum<32>(sum);
             group_write<Tag, Checked>(rr, (rm.C * E::kSize) >> 4, tid, rm.col0, rm.row0, causal, M * kLog2e,
-                                      __frcp_rn(sum), rmt, y + rm.off * E::kSize, bdy);
+                                      __frcp_rn(sum), y + rm.off * E::kSize, bdy);
             rh = false;
             return true;
         };
@@ -2034,7 +1951,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
                 continue;
             }
             const int nvec = (mt.C * E::kSize) >> 4;
-            unsigned char *sbuf = stages + static_cast<size_t>(s) * a.stage_bytes;
+            const unsigned char *sbuf = stages + static_cast<size_t>(s) * a.stage_bytes;
             Bounds bs = bdy;
             bs.s_lo = sbuf;
             bs.s_hi = sbuf + static_cast<size_t>(mt.C) * E::kSize;
@@ -2049,7 +1966,6 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
             // this member's (max, sum) of its part, from the stage
             float m_l, s_l;
             group_partial<Tag, Checked>(sbuf, nvec, tid, mt.col0, mt.row0, causal, bs, m_l, s_l);
-            const float m_self = m_l;
 #pragma unroll
             for (int o2 = 16; o2 >= 1; o2 >>= 1) {
                 const float mo2 = __shfl_xor_sync(0xFFFFFFFFu, m_l, o2);
@@ -2103,7 +2019,6 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
             if (lane == 0)
                 mbar_arrive(&h.empty[s]);
             rm = mt;
-            rmt = m_self;
             rx = xt;
             rh = true;
             ++xt;
