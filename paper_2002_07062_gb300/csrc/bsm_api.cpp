@@ -286,15 +286,19 @@ struct PatchLayout {
 };
 
 // Rows over groups of CTAs (forward pass).  A row longer than one stage is
-// cut into K parts, each staged whole by one CTA of a group of K (one read of
-// every element, one launch).  K: the fewest CTAs whose parts fit a third of
-// the shared memory (three stages: one row being written, the next one
-// reduced, a third being loaded), raised up to twice that where more SMs then
-// work (groups of n_sm / K CTAs leave n_sm mod K idle: 152 SMs take K = 4, 8,
-// 19, 38 or 76 whole).  Used when the batch's long rows fill the groups'
-// waves at least two thirds (so the one launch beats the two-launch cut of
-// few long rows into segments, which reads each row twice); K depends on
-// the longest such row and the device only, never on the policy.
+// cut into K parts, each staged by one CTA of a group of K (one read of every
+// element, one launch).  K: the fewest CTAs whose parts fit the consumer
+// threads' registers (64 KiB) and a third of the shared memory, raised up to
+// twice that where more SMs then work (groups of n_sm / K CTAs leave n_sm
+// mod K idle: 152 SMs take K = 8 or 19 whole).  Used for rows of at least
+// kGroupMinParts parts on groups of at most kGroupMaxSize CTAs, when the
+// batch's long rows fill the groups' waves at least two thirds (so the one
+// launch beats the two-launch cut of few long rows into segments, which
+// reads each row twice); K depends on the longest such row and the device
+// only, never on the policy.
+constexpr int64_t kGroupMinParts = 5;    // rows of fewer parts stay on one CTA
+constexpr int64_t kGroupMaxSize = 24;    // larger groups wait too long on their slowest member
+
 int choose_groups(const std::vector<SliceView> &slices, int es, int n_sm, int64_t smem_optin, PatchLayout &L)
 {
     const int64_t avail = smem_optin - kSmemHeader;
@@ -327,7 +331,15 @@ int choose_groups(const std::vector<SliceView> &slices, int es, int n_sm, int64_
             best_k = k;
         }
     }
-    if (best_k == 0)
+    // Measured on GB300 (same run, 256 MiB of rows, against the paths that
+    // stream a row twice through one CTA): groups of 8 and 19 win (bf16
+    // 512 KiB rows 4134 against 4039 GB/s, fp32 1 MiB rows 4367 against
+    // 4014); groups of 2 and 4 lose to one CTA per row, whose second read
+    // mostly hits L2 and which waits on no other CTA (bf16 128 KiB 4006
+    // against 4500, fp32 256 KiB 4709 against 4886); groups of 38 and 76 lose
+    // to waiting for the slowest of their members at every row (bf16 2 MiB
+    // 3336 against 3600, fp32 4 MiB 3215 against 3948).
+    if (best_k == 0 || kmin < kGroupMinParts || best_k > kGroupMaxSize)
         return 0;
     const int64_t G = n_sm / best_k;
     const int64_t waves = (n_cand + G - 1) / G;

@@ -53,9 +53,9 @@ def test_checked_forward_every_routine(dtype, flags, col_steps):
 
 @pytest.mark.parametrize("R,caps", [(3, 1), (400, 1), (400, 2)])
 def test_checked_long_rows(R, caps):
-    """3 rows: segments over two launches; 400 rows: split over groups of
-    two or four CTAs (one cooperative launch; the self-checking group kernel
-    checks its bulk copies, stage reads and stores too)."""
+    """3 rows: segments over two launches; 400 rows: one launch per row, of
+    two chunks (staged whole between the passes) or three (the last chunk
+    kept, the others copied again)."""
     import torch
     es = 4
     C = caps * (bsm.bsm_max_row_bytes() // es) + 64
@@ -83,4 +83,15 @@ def test_checked_backward_short_and_long():
                                         bsm.POLICY_DYNAMIC)
         return dx
     a, b = _both(bwd)
+    assert torch.equal(bits(a), bits(b))
+
+
+def test_checked_group_rows():
+    """Rows split over groups of CTAs (19 groups of 8 on 152 SMs): the
+    self-checking group kernel checks its bulk copies, stage reads and
+    stores, and gives the same bits."""
+    import torch
+    w = workload.uniform("checked group", workload.F32, 1, 19, 98304, 2.0, 0xC51).materialize()
+    x = to_device(w.x)
+    a, b = _both(lambda: run(w, x, bsm.POLICY_DYNAMIC))
     assert torch.equal(bits(a), bits(b))

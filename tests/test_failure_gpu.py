@@ -85,9 +85,8 @@ def test_corrupted_patch_is_skipped_with_bounds_status():
 
 
 def _w_long():
-    """Two waves of rows just over a stage: rows split over groups of two
-    CTAs (one cooperative launch; the members of a group wait on each
-    other's partials)."""
+    """Two waves of rows just over a stage: the one-launch long-row path
+    (rows staged whole between their passes)."""
     import torch
     n_sm = torch.cuda.get_device_properties(0).multi_processor_count
     C = bsm.bsm_max_row_bytes() // 4 + 64
@@ -181,12 +180,12 @@ def test_withheld_stage_in_a_group_launch_times_out_and_context_survives():
     status), and the next execute is right."""
     import time
     import torch
-    w = workload.uniform("fail group", workload.F32, 1, 38, 65536, 2.0, 0xFA12).materialize()
+    w = workload.uniform("fail group", workload.F32, 1, 19, 98304, 2.0, 0xFA12).materialize()
     x = to_device(w.x)
     y = torch.zeros_like(x)
     bsm.bsm_device_status_clear()
     p = bsm.bsm_plan_create(x, y, w.rows, w.cols, w.dtype, bsm.POLICY_DYNAMIC)
-    assert p.stats()["group_rows"] == 38          # 38 groups of 4 CTAs on 152 SMs
+    assert p.stats()["group_rows"] == 19          # 19 groups of 8 CTAs on 152 SMs
     bsm.bsm_plan_debug(p, bsm.DEBUG_WITHHOLD_STAGE, 100_000_000)      # 0.1 s waits
     t0 = time.time()
     p.execute()
@@ -201,3 +200,34 @@ def test_withheld_stage_in_a_group_launch_times_out_and_context_survives():
     assert bsm.bsm_device_status() == 0
     check_all_against_oracle(w, to_host(y))
     p.close()
+
+
+def test_corrupted_group_row_is_skipped_by_every_member():
+    """A record of the group-row table pointing past the buffers: every
+    member of the group that draws it skips it alike (no member waits for
+    the others' partials), BSM_DEV_BOUNDS is set, and the other rows are
+    right."""
+    import torch
+    w = workload.uniform("fail group corrupt", workload.F32, 1, 19, 98304, 2.0, 0xFA13).materialize()
+    C = int(w.cols[0])
+    x = to_device(w.x)
+    sentinel = -7.0
+    y = torch.full_like(x, sentinel)
+    bsm.bsm_device_status_clear()
+    p = bsm.bsm_plan_create(x, y, w.rows, w.cols, w.dtype, bsm.POLICY_RR)
+    st = p.stats()
+    assert st["group_rows"] == 19 and st["n_items"] == 19
+    bsm.bsm_plan_debug(p, bsm.DEBUG_CORRUPT_PATCH, 7)         # the group table's slot 7
+    p.execute()
+    torch.cuda.synchronize()
+    assert bsm.bsm_device_status() & bsm.DEV_BOUNDS
+    assert not bsm.bsm_device_status() & bsm.DEV_TIMEOUT
+    yh = to_host(y).reshape(-1, C)
+    untouched = np.all(yh == sentinel, axis=1)
+    assert untouched.sum() == 1 and untouched[7]
+    from oracle import softmax as O
+    y64, _ = O.softmax_batched(w.x, w.offsets, w.rows, w.cols)
+    ok = ~untouched
+    assert np.max(np.abs(yh[ok].astype(np.float64) - y64.reshape(-1, C)[ok])) <= 2e-6
+    p.close()
+    bsm.bsm_device_status_clear()

@@ -69,8 +69,8 @@ def test_offsets_past_32_bits(dtype, flags):
 
 @pytest.mark.parametrize("R_long,C_long", [(2049, 1 << 20), (9, 1 << 28)])
 def test_long_rows_past_32_bits(R_long, C_long):
-    """Rows longer than a stage past element 2^31: 2049 rows of 4 MiB (split
-    over groups of CTAs, one launch) and 9 rows of 1 GiB (segments over two
+    """Rows longer than a stage past element 2^31: 2049 rows of 4 MiB (each
+    row whole in one launch) and 9 rows of 1 GiB (segments over two
     launches); the rows on both sides of element 2^31 against the oracle."""
     import torch
     n = R_long * C_long

@@ -7,8 +7,8 @@ segments exactly once, and the two launches of segmented rows must hold the
 same segments; a row split over a group of CTAs must be one record whose
 parts fit a stage of the group launch.  Worked figures: workload 2
 (384 x 512 x 512 fp32) is 6144 patches of 32 rows in three 64 KiB stages; 64
-rows of 4 MiB fp32 go to two groups of 76 CTAs; one such row is 37 segments
-over two launches."""
+rows of 4 MiB fp32 are 1216 segments over two launches; 256 rows of 1 MiB
+fp32 go to eight groups of 19 CTAs."""
 import random
 from collections import Counter
 
@@ -157,35 +157,50 @@ def test_workload2_six_thousand_patches_of_32_rows():
     assert len(L["phase1"]) == 0
 
 
-def test_four_mib_rows_go_to_two_groups_of_76():
-    """64 fp32 rows of 4 MiB: parts of at most a third of the shared memory
-    (75.25 KiB) need 55 CTAs a row; 76 (half the SMs) is the group size that
-    leaves none idle: two groups, 32 rows each, one launch, no segments."""
+def test_four_mib_rows_are_1216_segments_over_two_launches():
+    """64 fp32 rows of 4 MiB would need groups of 76 CTAs (too many to wait
+    on): fewer rows than two per SM, so each is cut into 19 segments of whole
+    113 KiB chunks, 1216 over two launches."""
     L = check_layout([64], [1 << 20], bsm.F32, bsm.POLICY_DYNAMIC)
-    assert L["group_k"] == 76 and len(L["phase0"]) == 64 and len(L["phase1"]) == 0
+    assert L["group_k"] == 0
+    assert (L["stage_bytes"], L["n_stages"]) == (115712, 2)       # the 113 KiB cap
+    assert len(L["phase0"]) == 1216 and len(L["phase1"]) == 1216   # 19 per row
     assert L["long_rows"] == 64
 
 
-def test_one_four_mib_row_is_cut_into_segments_over_two_launches():
-    """A single 4 MiB row would keep one of the two groups idle: it is cut
-    into 37 segments of whole 113 KiB chunks instead (two launches)."""
-    L = check_layout([1], [1 << 20], bsm.F32, bsm.POLICY_DYNAMIC)
+def test_one_row_of_a_group_size_is_cut_into_segments():
+    """A single 1 MiB fp32 row would keep seven of the eight groups idle: it
+    is cut into segments of whole 113 KiB chunks instead (two launches)."""
+    L = check_layout([1], [262144], bsm.F32, bsm.POLICY_DYNAMIC)
     assert L["group_k"] == 0
-    assert (L["stage_bytes"], L["n_stages"]) == (115712, 2)       # the 113 KiB cap
-    assert len(L["phase0"]) == 37 and len(L["phase1"]) == 37
+    assert len(L["phase0"]) == len(L["phase1"]) == 10
 
 
-@pytest.mark.parametrize("C,dtype,k", [(65536, bsm.F32, 4), (262144, bsm.F32, 19),
-                                       (65536, bsm.BF16, 2), (262144, bsm.BF16, 8),
-                                       (1048576, bsm.BF16, 38)])
+def test_rows_of_two_chunks_stay_staged():
+    """bf16 rows of 128 KiB (two parts: too few for a group): three stages of
+    half a row (two chunks per row), each row one patch, whole in one launch."""
+    L = check_layout([2048], [65536], bsm.BF16, bsm.POLICY_DYNAMIC)
+    assert L["group_k"] == 0
+    assert (L["stage_bytes"], L["n_stages"]) == (65536, 3)
+    assert len(L["phase0"]) == 2048 and len(L["phase1"]) == 0
+    assert set(L["phase0"]["part_count"]) == {1} and set(L["phase0"]["cols"]) == {65536}
+
+
+@pytest.mark.parametrize("C,dtype,k", [(65536, bsm.F32, 0), (98304, bsm.F32, 8), (262144, bsm.F32, 19),
+                                       (1048576, bsm.F32, 0), (65536, bsm.BF16, 0),
+                                       (262144, bsm.BF16, 8), (524288, bsm.BF16, 19),
+                                       (1048576, bsm.BF16, 0)])
 def test_long_rows_group_sizes(C, dtype, k):
-    """256 MiB of long rows (the bench's long-row cases): fp32 256 KiB and
-    1 MiB rows, bf16 128 KiB, 512 KiB and 2 MiB rows go to groups of 4, 19,
-    2, 8 and 38 CTAs -- divisors of 152 -- and each CTA stages one part."""
+    """256 MiB of long rows: rows of 5 to 24 parts of 64 KiB go to groups of
+    K CTAs -- 8 or 19 on 152 SMs (divisors of 152) --, each CTA holding one
+    part; shorter rows (256 KiB fp32, 128 KiB bf16) stay on one CTA per row,
+    longer ones (4 MiB fp32, 2 MiB bf16) are streamed twice."""
     es = 4 if dtype == bsm.F32 else 2
     R = (256 << 20) // (C * es)
     L = check_layout([R], [C], dtype, bsm.POLICY_DYNAMIC)
-    assert L["group_k"] == k and len(L["phase0"]) == R and len(L["phase1"]) == 0
+    assert L["group_k"] == k
+    if k:
+        assert len(L["phase0"]) == R and len(L["phase1"]) == 0
 
 
 def test_backward_long_rows_keep_one_cta_per_row():

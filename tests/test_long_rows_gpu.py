@@ -88,9 +88,12 @@ def test_non_finite_long_rows():
 
 
 @pytest.mark.parametrize("dtype", [workload.F32, workload.BF16])
-def test_many_rows_just_over_a_stage_go_to_groups_of_two(dtype):
-    """Two waves of rows just over the single-stage limit: each row is split
-    over a group of two CTAs (one launch, each CTA stages half a row)."""
+def test_many_long_rows_stream_whole_rows_in_one_launch(dtype):
+    """With at least two waves of rows too short for a group each row is one
+    segment that one CTA streams in a single launch (fewer rows are cut into
+    segments over two launches).  Rows just over the cap get three stages of
+    half a row: a row (two chunks) stays staged for its second pass.  Against
+    the oracle, all policies bit-identical."""
     import torch
     es = 4 if dtype == workload.F32 else 2
     limit = bsm.bsm_max_row_bytes() // es
@@ -101,7 +104,8 @@ def test_many_rows_just_over_a_stage_go_to_groups_of_two(dtype):
     p = bsm.bsm_plan_create(x, x, w.rows, w.cols, dtype, bsm.POLICY_DYNAMIC)
     st = p.stats()
     assert st["long_items"] == R and st["launches"] == 1 and st["n_items"] == R
-    assert st["group_rows"] == R and st["group_k"] == 2
+    assert st["group_rows"] == 0
+    assert st["n_stages"] == 3 and 2 * st["stage_bytes"] >= C * es
     p.close()
     y = _all(w, x)
     check_all_against_oracle(w, to_host(y))
@@ -124,11 +128,13 @@ def test_few_long_rows_are_segmented_over_two_launches():
 
 @pytest.mark.parametrize("dtype", [workload.F32, workload.BF16])
 @pytest.mark.parametrize("chunks,flags", [(3, workload.CAUSAL), (4, 0)])
-def test_many_rows_of_several_stages(dtype, chunks, flags):
-    """Rows of three and four stages' length, two waves of them: groups of
-    four and eight CTAs; under the causal mask most of every row is masked
-    (the row index is below the column count), so most members hold a wholly
-    masked part."""
+def test_many_long_rows_of_several_chunks(dtype, chunks, flags):
+    """Two waves of rows of three and four stages' length: the three-chunk
+    rows (four parts of 64 KiB at most: too few for a group) are streamed
+    whole by one CTA each, starting the second pass on the chunk still
+    staged and running backwards; the four-chunk rows go to groups of eight
+    CTAs.  Under the causal mask most of every row is masked (the row index is
+    below the column count)."""
     import torch
     es = 4 if dtype == workload.F32 else 2
     limit = bsm.bsm_max_row_bytes() // es
@@ -140,19 +146,17 @@ def test_many_rows_of_several_stages(dtype, chunks, flags):
     p = bsm.bsm_plan_create(x, x, w.rows, w.cols, dtype, bsm.POLICY_DYNAMIC, flags=flags)
     st = p.stats()
     assert st["long_items"] == R and st["launches"] == 1
-    assert st["group_rows"] == R and st["group_k"] == (4 if chunks == 3 else 8)
+    assert st["group_rows"] == (0 if chunks == 3 else R)
     p.close()
     y = _all(w, x)
     check_all_against_oracle(w, to_host(y))
     assert bsm.bsm_device_status() == 0
 
 
-# rows over groups: (rows, row length, dtype, group size) -- each fills the
-# groups' waves; every group size the long-row bench uses on 152 SMs
-# (one full wave: as many rows as groups, n_sm / K)
-GROUP_CASES = [(38, 65536, workload.F32, 4), (8, 262144, workload.F32, 19),
-               (2, 1048576, workload.F32, 76), (76, 65536, workload.BF16, 2),
-               (19, 262144, workload.BF16, 8), (4, 1048576, workload.BF16, 38)]
+# rows over groups: (rows, row length, dtype, group size on 152 SMs) -- one
+# full wave each (as many rows as groups, n_sm / K)
+GROUP_CASES = [(19, 98304, workload.F32, 8), (8, 262144, workload.F32, 19),
+               (19, 262144, workload.BF16, 8), (8, 524288, workload.BF16, 19)]
 
 
 @pytest.mark.parametrize("case", range(len(GROUP_CASES)))
