@@ -440,13 +440,15 @@ def main():
             return time_steps_flushed(fn, n, stream, flush_buf)
         return time_steps(fn, n, stream)
 
-    for _ in range(args.warmup):
-        step()
-    stream.synchronize()
-    if ws > 1:
-        dist.barrier()
-    torch.cuda.synchronize()
+    # the clock sampler starts first (it needs a moment), then the warm-up
+    # steps, so that the timed steps follow busy ones instead of an idle gap
     with ClockSampler(dev) as clk:
+        for _ in range(args.warmup):
+            step()
+        stream.synchronize()
+        if ws > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
         total_ms, _ = timed(step, args.steps)
     torch.cuda.synchronize()
     if ws > 1:
@@ -609,6 +611,9 @@ def time_softmax(bsm, w, x, y, pol, stream, dev, target_s=1.0, clocks=True):
     torch.cuda.synchronize()
     if clocks:
         with ClockSampler(dev) as clk:
+            for _ in range(3):
+                step()
+            torch.cuda.synchronize()
             total_ms, _ = (time_steps_flushed(step, steps, stream, flush_buf) if small
                            else time_steps(step, steps, stream))
     else:
@@ -683,6 +688,9 @@ def time_bmm(bsm, workload, k, pol, stream, dev, target_s=1.0, clocks=True):
     clk = None
     if clocks:
         with ClockSampler(dev) as clk:
+            for _ in range(3):
+                step()
+            stream.synchronize()
             total_ms, _ = time_steps(step, steps, stream)
     else:
         total_ms, _ = time_steps(step, steps, stream)
@@ -870,6 +878,9 @@ def time_long_rows(bsm, C, dtype, stream, dev, target_s=0.5):
     stream.synchronize()
     steps = _steps_for(step, stream, target_s)
     with ClockSampler(dev) as clk:
+        for _ in range(3):
+            step()
+        stream.synchronize()
         total_ms, _ = time_steps(step, steps, stream)
     ms = total_ms / steps
     alg = 2 * R * C * es
@@ -916,6 +927,9 @@ def run_bmm(args, bsm, workload, ws, rank, dev):
         import torch.distributed as dist
         dist.barrier()
     with ClockSampler(dev) as clk:
+        for _ in range(3):
+            step()
+        stream.synchronize()
         total_ms, _ = time_steps(step, args.steps, stream)
     torch.cuda.synchronize()
     if ws > 1:
@@ -969,6 +983,9 @@ def run_long_rows(args, bsm, ws, rank, dev):
         import torch.distributed as dist
         dist.barrier()
     with ClockSampler(dev) as clk:
+        for _ in range(3):
+            step()
+        stream.synchronize()
         total_ms, _ = time_steps(step, args.steps, stream)
     torch.cuda.synchronize()
     if ws > 1:
