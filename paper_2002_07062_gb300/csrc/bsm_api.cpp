@@ -921,33 +921,12 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     a.segs = segs.empty() ? nullptr : reinterpret_cast<const LongSeg *>(b + o_segs);
     a.partials = n_parts ? reinterpret_cast<float *>(b + o_parts) : nullptr;
     a.phase = 0;
-    // the natural cut of a uniform batch packed from element 0 (in table
-    // order): the kernel computes the records instead of reading them
-    a.nat_rpi = 0;
-    if (!items.empty() && segs.empty() && items[0].off == 0 && items[0].row0 == 0) {
-        const Item &f = items[0];
-        int64_t rows = 0;
-        bool nat = true;
-        for (size_t i = 0; i < items.size() && nat; ++i) {
-            const Item &it = items[i];
-            nat = it.C == f.C && it.R == f.R && it.off == rows * f.C && it.row0 == rows % f.R &&
-                  (it.nrows == f.nrows || i + 1 == items.size()) && it.nrows <= f.nrows;
-            rows += it.nrows;
-        }
-        if (nat) {
-            a.nat_rpi = f.nrows;
-            a.nat_R = f.R;
-            a.nat_C = f.C;
-            a.nat_rows = rows;
-        }
-    }
     // phase 1 (rows longer than a stage): their segments again, one queue
     // (or the same static / round-robin split as phase 0)
     p->n_phase1 = n1;
     if (n1) {
         KernelArgs &a1 = p->args1;
         a1 = a;
-        a1.nat_rpi = 0;
         a1.items = reinterpret_cast<const Item *>(b + o_items1);
         a1.segs = reinterpret_cast<const LongSeg *>(b + o_segs1);
         a1.n_items = static_cast<int32_t>(n1);
@@ -966,7 +945,6 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     if (n_grp) {
         KernelArgs &ag = p->argsg;
         ag = a;
-        ag.nat_rpi = 0;
         ag.items = reinterpret_cast<const Item *>(b + o_itemsg);
         ag.n_items = static_cast<int32_t>(n_grp);
         ag.slice_first_item = reinterpret_cast<const int32_t *>(b + o_slicesg);
@@ -1026,6 +1004,15 @@ int plan_create_impl(bsm_plan **out, const bsm_plan_desc *d)
     }
     p->args1.mode = a.mode;
     p->argsg.mode = a.mode;
+    // one queue no longer than the grid (a small batch: a patch per SM at
+    // most): CTA u takes queue slot u and nothing else, with no claim before
+    // its copy and no queue head to rewind after it -- the static deal over
+    // the queue's slots
+    if (a.mode == PULL_QUEUE && a.n_queues == 1 && a.queue_len[0] <= p->grid) {
+        a.mode = PULL_STATIC;
+        a.item_begin = a.queue_begin[0];
+        a.item_end = a.queue_begin[0] + a.queue_len[0];
+    }
     // (rows over groups of CTAs use cooperative launches, which stay out of
     // the graph: such plans launch kernel by kernel)
     if (d->policy == BSM_POLICY_WHOLE_GPU && !p->whole_gpu.empty() && p->whole_gpu.size() <= kMaxGraphLaunches &&
@@ -1348,12 +1335,12 @@ int bsm_plan_debug(bsm_plan *plan, int what, int64_t arg)
     if (!plan)
         return noalloc_debug(what, arg);
     switch (what) {
-    case BSM_DEBUG_NONE:       // (a rewritten table stays rewritten)
-        plan->args.debug &= KDEBUG_TABLE_WRITTEN;
+    case BSM_DEBUG_NONE:
+        plan->args.debug = 0;
         plan->args.wait_limit_ns = 0;
-        plan->args1.debug &= KDEBUG_TABLE_WRITTEN;
+        plan->args1.debug = 0;
         plan->args1.wait_limit_ns = 0;
-        plan->argsg.debug &= KDEBUG_TABLE_WRITTEN;
+        plan->argsg.debug = 0;
         plan->argsg.wait_limit_ns = 0;
         return BSM_OK;
     case BSM_DEBUG_WITHHOLD_STAGE:
@@ -1369,10 +1356,6 @@ int bsm_plan_debug(bsm_plan *plan, int what, int64_t arg)
         if (arg < 0 || arg >= int64_t(plan->args.n_items) + plan->n_group)
             return BSM_ERR_INVALID_ARG;
         const int64_t past_end = plan->args.total_elems;
-        // the kernel reads the (rewritten) table from now on, launch by launch
-        plan->args.nat_rpi = 0;
-        plan->args.debug |= KDEBUG_TABLE_WRITTEN;
-        plan->argsg.debug |= KDEBUG_TABLE_WRITTEN;
         unsigned char *entry =
             arg < plan->args.n_items
                 ? static_cast<unsigned char *>(plan->blob) + sizeof(Item) * static_cast<size_t>(arg)

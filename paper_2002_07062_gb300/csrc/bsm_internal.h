@@ -112,12 +112,6 @@ struct KernelArgs {
     const LongSeg *segs;        // per patch, in the order of `items`; NULL: no long rows
     float *partials;            // 2 floats per segment
     int32_t phase;              // 0: segments leave their partials; 1: combine and write
-    // a uniform batch packed from element 0 whose patch table is the natural
-    // cut (patch i = rows [i * nat_rpi, + nat_rpi) of the (B*R) x C matrix, in
-    // that order): the records are computed from the index, not read
-    int32_t nat_rpi;            // 0: read the records
-    int32_t nat_R, nat_C;
-    int64_t nat_rows;
     // rows split over groups of CTAs (OP_FORWARD_GROUP): items are whole rows
     int32_t group_k;            // CTAs per group (2..kMaxGroup); the grid is n_groups * group_k
     int32_t n_groups;
@@ -127,8 +121,6 @@ struct KernelArgs {
 
 // Test-only fault injection (bsm_plan_debug).
 constexpr uint32_t KDEBUG_WITHHOLD_STAGE0 = 1u;   // producer never fills stage 0 of its first round
-constexpr uint32_t KDEBUG_TABLE_WRITTEN = 2u;     // the device table was rewritten: no effect in the
-                                                  // kernel, keeps the plan off its captured graph
 
 // One output tile of the batched matrix product: rows [m0, m0 + 128) and
 // columns [n0, n0 + BN) of slice `slice`.

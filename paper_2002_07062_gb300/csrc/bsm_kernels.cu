@@ -1028,14 +1028,6 @@ __device__ __forceinline__ int consume_stage(const unsigned char *sbuf, const St
 // The pulling unit is a CTA, or for rows split over groups of CTAs a whole
 // group (unit = group index, n_units = groups): the static and round-robin
 // deals and the tail rule count units, not CTAs.
-// Patch i of a uniform batch packed from element 0, cut naturally.
-__device__ __forceinline__ Item natural_item(const KernelArgs &a, int32_t i)
-{
-    const int64_t g0 = static_cast<int64_t>(i) * a.nat_rpi;
-    const int64_t nr = a.nat_rows - g0 < a.nat_rpi ? a.nat_rows - g0 : a.nat_rpi;
-    return Item{g0 * a.nat_C, a.nat_C, static_cast<int32_t>(nr), static_cast<int32_t>(g0 % a.nat_R), a.nat_R};
-}
-
 struct Puller {
     const KernelArgs &a;
     int32_t unit, n_units;
@@ -1045,9 +1037,6 @@ struct Puller {
     int32_t q = 0;           // PULL_QUEUE: index into the try order
     int32_t die = 0;
     uint32_t fetch = kFetch; // PULL_QUEUE: patches per claim (1 near the end of a queue)
-    // PULL_QUEUE, one short queue: unit u takes slot u first without a claim
-    // (no round trip before its first copy); later claims are counter + units
-    bool static_first = false;
 
     __device__ explicit Puller(const KernelArgs &args)
         : Puller(args, static_cast<int32_t>(blockIdx.x), static_cast<int32_t>(gridDim.x))
@@ -1063,10 +1052,8 @@ struct Puller {
         }
         // a short queue (small batch: about a patch per SM) is claimed one
         // patch at a time from the first claim on, so every SM gets one
-        if (a.mode == PULL_QUEUE && static_cast<uint32_t>(a.queue_len[die]) < 2u * kFetch * static_cast<uint32_t>(n_units)) {
+        if (a.mode == PULL_QUEUE && static_cast<uint32_t>(a.queue_len[die]) < 2u * kFetch * static_cast<uint32_t>(n_units))
             fetch = 1;
-            static_first = a.n_queues == 1;
-        }
         if (a.mode == PULL_RR_SLICE)
             slice = unit - n_units;
     }
@@ -1102,23 +1089,6 @@ struct Puller {
         }
         // PULL_QUEUE: claim kFetch consecutive slots of the own die's queue,
         // then (steal) of the other dies' queues in order.
-        if (static_first) {
-            const uint32_t len = static_cast<uint32_t>(a.queue_len[0]);
-            if (k == 0) {
-                k = 1;
-                if (static_cast<uint32_t>(unit) < len) {
-                    pos[0] = a.queue_begin[0] + unit;
-                    return 1;
-                }
-                return 0;
-            }
-            const uint32_t t = atomicAdd(&a.heads[0], 1u) + static_cast<uint32_t>(n_units);
-            if (t < len) {
-                pos[0] = a.queue_begin[0] + static_cast<int32_t>(t);
-                return 1;
-            }
-            return 0;
-        }
         const int tries = a.steal ? a.n_queues : 1;
         while (q < tries) {
             const int qq = (die + q) % a.n_queues;
@@ -1230,7 +1200,7 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
 #pragma unroll
                     for (int j = 0; j < kFetch; ++j)
                         if (j < n && pos[j] >= 0 && pos[j] < a.n_items) {
-                            batch[j] = a.nat_rpi > 0 ? natural_item(a, pos[j]) : a.items[pos[j]];
+                            batch[j] = a.items[pos[j]];
                             if (kLong && a.segs)
                                 lseg[j] = a.segs[pos[j]];
                         }

@@ -168,7 +168,11 @@ int softmax_noalloc(const void *x, void *y, int64_t B, int64_t R, int64_t C, int
     a.total_elems = rows * C;
     a.items = items;
     a.n_items = static_cast<int32_t>(n_items);
-    a.mode = PULL_QUEUE;
+    // at most a patch per SM: CTA u takes patch u with no claim (the static
+    // deal); otherwise the device-wide queue
+    a.mode = n_items <= nd->n_sm ? PULL_STATIC : PULL_QUEUE;
+    a.item_begin = 0;
+    a.item_end = static_cast<int32_t>(n_items);
     a.n_queues = 1;
     a.queue_begin[0] = 0;
     a.queue_len[0] = static_cast<int32_t>(n_items);
