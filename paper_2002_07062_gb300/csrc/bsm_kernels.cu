@@ -1112,6 +1112,60 @@ struct Puller {
     }
 };
 
+// Warm L2 with the patches this CTA most likely copies first, before the
+// wait on the previous kernel: the slots of its first batch (the static
+// deal's and round robin's exactly; under a queue, slots r*kFetch .. of queue
+// u mod n_queues for CTA u = r*n_queues + (u mod n_queues), so that the CTAs
+// together cover the first claims).  A prefetch into L2 carries no data to
+// the SM and has no effect on what any load returns (L2 is the point of
+// coherence), so it may run while the previous kernel still writes; what it
+// buys is that DRAM serves these lines during that kernel's last wave
+// instead of after it.  Records are checked like the producer checks them;
+// one that fails is skipped.
+__device__ __forceinline__ void prefetch_l2(const void *p, uint32_t bytes)
+{
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+
+template <int ES>
+__device__ __forceinline__ void prefetch_first_batch(const KernelArgs &a, bool two_inputs)
+{
+    int64_t first = 0, end = 0, step = 1;
+    const int64_t u = blockIdx.x;
+    if (a.mode == PULL_STATIC) {
+        first = a.item_begin + u;
+        end = a.item_end;
+        step = gridDim.x;
+    } else if (a.mode == PULL_RR_SLICE) {
+        if (u >= a.n_slices)
+            return;
+        first = a.slice_first_item[u];
+        end = a.slice_first_item[u + 1];
+    } else {
+        const int nq = a.n_queues > 0 ? a.n_queues : 1;
+        const int q = static_cast<int>(u % nq);
+        first = a.queue_begin[q] + (u / nq) * kFetch;
+        end = (int64_t)a.queue_begin[q] + a.queue_len[q];
+    }
+    if (end > a.n_items)
+        end = a.n_items;
+    const int64_t cap = two_inputs ? a.stage_bytes / 2 : a.stage_bytes;
+    for (int j = 0; j < kFetch; ++j) {
+        const int64_t idx = first + j * step;
+        if (idx < 0 || idx >= end)
+            break;
+        const Item it = a.items[idx];
+        const int64_t ne = (int64_t)it.nrows * it.C;
+        const int64_t nbytes = ne * ES;
+        if (it.off < 0 || it.C <= 0 || it.nrows <= 0 || it.off + ne > a.total_elems || nbytes > cap ||
+            (nbytes & 15) != 0 || ((it.off * ES) & 15) != 0)
+            continue;
+        prefetch_l2(static_cast<const unsigned char *>(a.x) + it.off * ES, static_cast<uint32_t>(nbytes));
+        if (two_inputs)
+            prefetch_l2(static_cast<const unsigned char *>(a.x2) + it.off * ES, static_cast<uint32_t>(nbytes));
+    }
+}
+
 template <typename Tag, int Op, bool Checked>
 __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelArgs a)
 {
@@ -1137,10 +1191,15 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_persistent(const KernelAr
         mbar_init_fence();
     }
     __syncthreads();
+    // rows that fit a stage: the first batch's bytes are prefetched into L2
+    // (a hint: it reads nothing into this CTA and writes nothing)
+    if (!kLong && warp == kConsumerWarps && lane == 0)
+        prefetch_first_batch<E::kSize>(a, kBwd);
     // Programmatic dependent launch: this kernel may have started while the
-    // previous kernel of the stream was finishing.  No role touches memory or
-    // starts a bounded wait before that kernel is done (a no-op without such
-    // a predecessor); then the next kernel may begin its own launch.
+    // previous kernel of the stream was finishing.  No role loads data,
+    // stores or starts a bounded wait before that kernel is done (a no-op
+    // without such a predecessor); then the next kernel may begin its own
+    // launch.
     asm volatile("griddepcontrol.wait;" ::: "memory");
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
