@@ -144,16 +144,6 @@ __device__ __forceinline__ void tma_load_3d(void *dst, const CUtensorMap *map, i
         : "memory");
 }
 
-// Prefetch into L2 of the same 3-D box (no data reaches the SM, and no
-// load returns anything different for it: L2 is the point of coherence).
-__device__ __forceinline__ void tma_prefetch_3d(const CUtensorMap *map, int32_t c0, int32_t c1, int32_t c2)
-{
-    asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];" ::"l"(
-                     reinterpret_cast<uint64_t>(map)),
-                 "r"(c0), "r"(c1), "r"(c2)
-                 : "memory");
-}
-
 // Tile record of queue entry idx: read from the plan, or computed when the
 // plan keeps tiles in their natural order (slice, row block, column block).
 template <int BN> __device__ __forceinline__ GemmItem tile_at(const GemmArgs &a, int32_t idx)
@@ -353,20 +343,6 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             bar_init(&h.drain, 1);
             h.abort_flag = 0;
             asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-            // the first tile's operands are prefetched into L2 while the
-            // previous kernel of the stream may still be finishing (a hint:
-            // no operand byte reaches this CTA, nothing is written; the tile
-            // record comes from the plan's constant table), so that DRAM
-            // serves them during that kernel's last wave
-            if (idx >= 0) {
-                const GemmItem f = tile_at<BN>(a, idx);
-                if (f.slice >= 0 && f.slice < a.B && f.m0 >= 0 && f.m0 + kBM <= a.M && f.n0 >= 0 &&
-                    f.n0 + BN <= a.N)
-                    for (int kb = 0; kb < NS; ++kb) {
-                        tma_prefetch_3d(&tmA, 0, f.slice * a.M + f.m0, kb * G);
-                        tma_prefetch_3d(&tmB, 0, f.slice * a.N + f.n0, kb * G);
-                    }
-            }
             // launched early behind the previous kernel of the stream: from
             // here on memory is touched, so wait until that kernel is done
             grid_dependency_wait();

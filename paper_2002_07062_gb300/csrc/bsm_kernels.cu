@@ -1113,15 +1113,20 @@ struct Puller {
 };
 
 // Warm L2 with the patches this CTA most likely copies first, before the
-// wait on the previous kernel: the slots of its first batch (the static
-// deal's and round robin's exactly; under a queue, slots r*kFetch .. of queue
-// u mod n_queues for CTA u = r*n_queues + (u mod n_queues), so that the CTAs
-// together cover the first claims).  A prefetch into L2 carries no data to
+// wait on the previous kernel: the first kPrefetch slots of its first batch
+// (the static deal's and round robin's exactly; under a queue, slots
+// r*kFetch .. of queue u mod n_queues for CTA u = r*n_queues + (u mod
+// n_queues), so that the CTAs together cover the first claims).  Two patches
+// (19.5 MB over 152 SMs at 64 KiB) measured best: 1, 3 and 4 gave 0.4-0.7 %
+// less on 384 x 512 x 512 rows, a second batch 2-5 % less (the prefetches
+// then slow the previous kernel's last wave).  A prefetch into L2 carries no data to
 // the SM and has no effect on what any load returns (L2 is the point of
 // coherence), so it may run while the previous kernel still writes; what it
 // buys is that DRAM serves these lines during that kernel's last wave
 // instead of after it.  Records are checked like the producer checks them;
 // one that fails is skipped.
+constexpr int kPrefetch = 2;
+
 __device__ __forceinline__ void prefetch_l2(const void *p, uint32_t bytes)
 {
     asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
@@ -1150,7 +1155,7 @@ __device__ __forceinline__ void prefetch_first_batch(const KernelArgs &a, bool t
     if (end > a.n_items)
         end = a.n_items;
     const int64_t cap = two_inputs ? a.stage_bytes / 2 : a.stage_bytes;
-    for (int j = 0; j < kFetch; ++j) {
+    for (int j = 0; j < kPrefetch; ++j) {
         const int64_t idx = first + j * step;
         if (idx < 0 || idx >= end)
             break;
