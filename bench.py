@@ -62,15 +62,17 @@ def kernel_hash() -> str:
     return hashlib.sha256(open(KERNEL_SRC, "rb").read()).hexdigest()[:16]
 
 
-def profiled_traffic(workload_k: int):
-    """DRAM bytes per launch of the softmax kernel on workload k (steady
-    state: consecutive launches, caches not flushed) from a committed ncu
-    summary taken on the current kernel source, else None."""
+def profiled_traffic(workload_k):
+    """DRAM bytes per launch of the softmax kernel on workload k (an int), or
+    on the case a key names (e.g. "long_fp32_1024KiB"), in steady state
+    (consecutive launches, caches not flushed) from a committed ncu summary
+    taken on the current kernel source, else None."""
     import glob
-    for path in sorted(glob.glob(os.path.join(PROFILE_DIR, "softmax_persistent*.md"))):
+    key = "workload%d" % workload_k if isinstance(workload_k, int) else str(workload_k)
+    for path in sorted(glob.glob(os.path.join(PROFILE_DIR, "softmax_*.md"))):
         text = open(path).read()
         m_hash = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]{16})", text)
-        m_traf = re.search(r"dram_bytes_per_launch_workload%d:\s*([0-9]+)" % workload_k, text)
+        m_traf = re.search(r"dram_bytes_per_launch_%s:\s*([0-9]+)" % re.escape(key), text)
         if m_hash and m_traf and m_hash.group(1) == kernel_hash():
             return int(m_traf.group(1))
     return None
@@ -898,7 +900,11 @@ def time_long_rows(bsm, C, dtype, stream, dev, target_s=0.5):
                      "stage_bytes": st["stage_bytes"]},
             "gpu_launches": int(st["launches"]) * steps,
             "roofline": {"bound": "hbm", "achieved": round(gbs, 2), "peak": peak, "unit": "GB/s",
-                         "frac": round(gbs / peak, 4), "traffic": None, "peak_source": peak_src,
+                         "frac": round(gbs / peak, 4),
+                         "traffic": profiled_traffic("long_%s_%dKiB" % ("fp32" if dtype == workload.F32
+                                                                        else "bf16", C * es >> 10))
+                         if st["launches"] == 1 else None,
+                         "peak_source": peak_src,
                          "kernel": kernel, "launch_ms": round(ms / max(1, st["launches"]), 5),
                          "moved_bytes_per_step": int(_moved_factor(st) * alg)},
             "clocks": clk.summary(), "device_status": bsm.bsm_device_status()}
