@@ -540,6 +540,27 @@ def main():
         out["e2e"] = {"value": round(ws * bytes_step / (e_ms * 1e-3) / 1e9, 2), "unit": "GB/s",
                       "h2d_bytes_per_step": nb, "d2h_bytes_per_step": nb,
                       "ms_per_step": round(e_ms, 4), "api": "bsm_softmax_host, pinned host buffers read and written by the kernel over the host link"}
+        if ws == 1:
+            # beside it, not the e2e figure: the same call on pageable host
+            # buffers, which the library stages through its device buffers in
+            # chunks (a device-to-host copy into pageable memory blocks the
+            # host, so the host times these steps)
+            import numpy as np
+            xh = xp.view(torch.int32 if x.element_size() == 4 else torch.int16).numpy().copy()
+            yh = np.empty_like(xh)
+            bsm.bsm_softmax_host(xh, yh, B, R, C, w.dtype, pol, w.flags, stream)
+            stream.synchronize()
+            n_pg = 3
+            t0 = time.perf_counter()
+            for _ in range(n_pg):
+                bsm.bsm_softmax_host(xh, yh, B, R, C, w.dtype, pol, w.flags, stream)
+            stream.synchronize()
+            pg_ms = (time.perf_counter() - t0) * 1e3 / n_pg
+            out["e2e"]["pageable"] = {
+                "value": round(bytes_step / (pg_ms * 1e-3) / 1e9, 2), "unit": "GB/s",
+                "ms_per_step": round(pg_ms, 3), "steps": n_pg,
+                "api": "bsm_softmax_host, pageable host buffers staged through device buffers in "
+                       "48 MiB chunks (host clock)"}
     if not args.no_cpu_baseline and rank == 0 and ws == 1:
         out["cpu_baseline"] = cpu_baseline(w)
 

@@ -6,13 +6,17 @@
 // straight to y_host -- no staging memory, both link directions busy at once.
 //
 // Pageable buffers go through a staged pipeline: the batch is cut into
-// chunks of whole slices; every chunk goes through
-// three stages on three streams of the library -- copy in (host to device),
-// the softmax kernel (the plan-cached bsm_softmax_ex path on a device staging
-// buffer), copy out (device to host) -- with two staging buffers, so chunk i
-// is copied in while chunk i-1 is computed and chunk i-2 is copied out.  The
-// two copy directions use the link at the same time; the end-to-end time
-// approaches the slower direction instead of the sum of both.
+// chunks of whole slices; every chunk goes through three stages on three
+// streams of the library -- copy in (host to device), the softmax kernel (the
+// plan-cached bsm_softmax_ex path on a device staging buffer), copy out
+// (device to host) -- with two staging buffers.  A device-to-host copy into
+// pageable memory returns to the host only once it has finished, so the
+// host thread issues chunk i's copy-in and kernel before chunk i-1's
+// copy-out: while the host waits on that copy-out, chunk i moves in and is
+// computed.  Both link directions are then busy at once, but only in pairs
+// of chunks (the copy-in of chunk i+1 is issued after chunk i-1's copy-out
+// has finished), and the driver stages pageable copies through its own
+// buffers; pinned buffers are the fast path.
 
 #include <cuda_runtime.h>
 
@@ -135,6 +139,20 @@ int softmax_host(const void *x_host, void *y_host, int64_t B, int64_t R, int64_t
         return record_cuda_error(static_cast<int>(e), "host pipeline start");
     const unsigned char *xs = static_cast<const unsigned char *>(x_host);
     unsigned char *ys = static_cast<unsigned char *>(y_host);
+    // copy-out of a computed chunk (staging buffer b, its place in y); it
+    // waits for that chunk's kernel only (ev_k[b], recorded after it)
+    auto copy_out = [&](int b, int64_t off, int64_t bytes) -> int {
+        cudaError_t ee;
+        if ((ee = cudaStreamWaitEvent(p.s_out, p.ev_k[b], 0)) ||
+            (ee = cudaMemcpyAsync(ys + off, p.dy[b], static_cast<size_t>(bytes), cudaMemcpyDeviceToHost,
+                                  p.s_out)) ||
+            (ee = cudaEventRecord(p.ev_out[b], p.s_out)))
+            return record_cuda_error(static_cast<int>(ee), "host pipeline copy out");
+        p.out_recorded[b] = true;
+        return BSM_OK;
+    };
+    int pend_b = -1;                 // the chunk computed but not yet copied out
+    int64_t pend_off = 0, pend_bytes = 0;
     for (int64_t first = 0, i = 0; first < B; first += per_chunk, ++i) {
         const int b = static_cast<int>(i & 1);
         const int64_t n = std::min<int64_t>(per_chunk, B - first);
@@ -150,13 +168,20 @@ int softmax_host(const void *x_host, void *y_host, int64_t B, int64_t R, int64_t
         if (int rc = bsm_softmax_ex(p.dx[b], p.dy[b], n, R, C, dtype, policy, flags,
                                     reinterpret_cast<bsm_stream_t>(p.s_k)))
             return rc;
-        if ((e = cudaEventRecord(p.ev_k[b], p.s_k)) || (e = cudaStreamWaitEvent(p.s_out, p.ev_k[b], 0)) ||
-            (e = cudaMemcpyAsync(ys + off, p.dy[b], static_cast<size_t>(bytes), cudaMemcpyDeviceToHost,
-                                 p.s_out)) ||
-            (e = cudaEventRecord(p.ev_out[b], p.s_out)))
-            return record_cuda_error(static_cast<int>(e), "host pipeline copy out");
-        p.out_recorded[b] = true;
+        if ((e = cudaEventRecord(p.ev_k[b], p.s_k)))
+            return record_cuda_error(static_cast<int>(e), "host pipeline kernel");
+        // the previous chunk's copy-out after this chunk's copy-in and kernel
+        // are queued (it may block the host until it has finished)
+        if (pend_b >= 0)
+            if (int rc = copy_out(pend_b, pend_off, pend_bytes))
+                return rc;
+        pend_b = b;
+        pend_off = off;
+        pend_bytes = bytes;
     }
+    if (pend_b >= 0)
+        if (int rc = copy_out(pend_b, pend_off, pend_bytes))
+            return rc;
     if ((e = cudaEventRecord(p.ev_end, p.s_out)) || (e = cudaStreamWaitEvent(caller, p.ev_end, 0)))
         return record_cuda_error(static_cast<int>(e), "host pipeline end");
     return BSM_OK;

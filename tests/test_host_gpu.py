@@ -35,8 +35,10 @@ def test_host_pipeline_matches_device_path(k):
 
 def test_host_pipeline_ragged_tail_in_place_and_pageable():
     import torch
-    # 211 slices of 96 x 1024 fp32 (384 KiB each): chunks of 128 slices + a tail of 83
-    w = workload.uniform("host tail", workload.F32, 211, 96, 1024, 2.0, 0x4057).materialize()
+    # 339 slices of 96 x 1024 fp32 (384 KiB each): two chunks of 128 slices
+    # and a tail of 83, so both staging buffers are reused and a copy-out
+    # is always issued after the next chunk's copy-in and kernel
+    w = workload.uniform("host tail", workload.F32, 339, 96, 1024, 2.0, 0x4057).materialize()
     x = to_device(w.x)
     y_dev = torch.empty_like(x)
     bsm.bsm_softmax(x, y_dev, w.nslices, 96, 1024, w.dtype, bsm.POLICY_RR)
