@@ -160,20 +160,23 @@ def test_workload2_six_thousand_patches_of_32_rows():
 def test_four_mib_rows_are_1216_segments_over_two_launches():
     """64 fp32 rows of 4 MiB would need groups of 76 CTAs (too many to wait
     on): fewer rows than two per SM, so each is cut into 19 segments of whole
-    113 KiB chunks, 1216 over two launches."""
+    chunks, 1216 over two launches.  fp32 rows streamed in chunks get three
+    stages of a third of the shared memory: (232448 - 1024) / 3 rounded down
+    to 128 bytes = 77056."""
     L = check_layout([64], [1 << 20], bsm.F32, bsm.POLICY_DYNAMIC)
     assert L["group_k"] == 0
-    assert (L["stage_bytes"], L["n_stages"]) == (115712, 2)       # the 113 KiB cap
+    assert (L["stage_bytes"], L["n_stages"]) == (77056, 3)
     assert len(L["phase0"]) == 1216 and len(L["phase1"]) == 1216   # 19 per row
     assert L["long_rows"] == 64
 
 
 def test_one_row_of_a_group_size_is_cut_into_segments():
     """A single 1 MiB fp32 row would keep seven of the eight groups idle: it
-    is cut into segments of whole 113 KiB chunks instead (two launches)."""
+    is cut into segments of whole chunks instead (two launches): 1 MiB in
+    chunks of at most 77056 bytes is 14 chunks, one segment each."""
     L = check_layout([1], [262144], bsm.F32, bsm.POLICY_DYNAMIC)
     assert L["group_k"] == 0
-    assert len(L["phase0"]) == len(L["phase1"]) == 10
+    assert len(L["phase0"]) == len(L["phase1"]) == 14
 
 
 def test_rows_of_two_chunks_stay_staged():
