@@ -398,6 +398,19 @@ int cut_patches(const bsm_plan_desc *d, const std::vector<SliceView> &slices, in
             // bf16 2 MiB rows lose, 3609 -> 3533, and keep two stages; four
             // stages gain nothing)
             stage = std::min<int64_t>(stage, std::max<int64_t>(min_stage, (avail / 3) & ~int64_t(127)));
+        else if (d->op == BSM_OP_BACKWARD) {
+            // the backward pass's rows streamed by one CTA each (at least two
+            // waves of them): three stages as well (same box: fp32 256 KiB
+            // rows 5240 -> 5382 GB/s, bf16 128 KiB 5519 -> 5952, bf16 512 KiB
+            // 4411 -> 4468); rows cut into segments over two launches keep
+            // two (they lose 0.2-0.5 %)
+            int64_t n_over = 0;
+            for (const SliceView &v : slices)
+                if (v.R > 0 && int64_t(v.C) * es > max_row_bytes_for(smem_optin) / in_arrays)
+                    n_over += v.R;
+            if (n_over >= 2 * int64_t(n_sm))
+                stage = std::min<int64_t>(stage, std::max<int64_t>(min_stage, (avail / 3) & ~int64_t(255)));
+        }
     }
     const int n_stages = static_cast<int>(std::min<int64_t>(kMaxStages, avail / stage));
     if (n_stages < 2)
