@@ -288,16 +288,16 @@ struct PatchLayout {
 // Rows over groups of CTAs (forward pass).  A row longer than one stage is
 // cut into K parts, each staged by one CTA of a group of K (one read of every
 // element, one launch).  K: the fewest CTAs whose parts fit the consumer
-// threads' registers (64 KiB) and a third of the shared memory, raised up to
-// twice that where more SMs then work (groups of n_sm / K CTAs leave n_sm
-// mod K idle: 152 SMs take K = 8 or 19 whole).  Used for rows of at least
+// threads' registers (64 KiB) and a third of the shared memory (groups of
+// n_sm / K CTAs; n_sm mod K SMs stay idle).  Used for rows of at least
 // kGroupMinParts parts on groups of at most kGroupMaxSize CTAs, when the
 // batch's long rows fill the groups' waves at least two thirds (so the one
 // launch beats the two-launch cut of few long rows into segments, which
 // reads each row twice); K depends on the longest such row and the device
 // only, never on the policy.
 constexpr int64_t kGroupMinParts = 5;    // rows of fewer parts stay on one CTA
-constexpr int64_t kGroupMaxSize = 24;    // larger groups wait too long on their slowest member
+constexpr int64_t kGroupMaxSize = 32;    // larger groups wait too long on their slowest member
+constexpr int64_t kGroupMaxSizeBf16 = 24; // (bf16: 32 already loses to the two-launch segments)
 
 int choose_groups(const std::vector<SliceView> &slices, int es, int n_sm, int64_t smem_optin, PatchLayout &L)
 {
@@ -321,25 +321,27 @@ int choose_groups(const std::vector<SliceView> &slices, int es, int n_sm, int64_
     const int64_t part_cap = std::min<int64_t>((avail / 3) & ~int64_t(127),
                                                int64_t(kGroupVecs) * 16 * kConsumerWarps * 32);
     const int64_t kmin = std::max<int64_t>(2, (lmax * es + part_cap - 1) / part_cap);
-    int64_t best_k = 0, best_used = 0;
-    for (int64_t k = kmin; k <= std::min<int64_t>({int64_t(kMaxGroup), 2 * kmin, int64_t(n_sm)}); ++k) {
-        if (avail / stage_for(k) < 3 || stage_for(k) > part_cap)
-            continue;
-        const int64_t used = (n_sm / k) * k;
-        if (used > best_used) {
-            best_used = used;
+    // The smallest group whose parts fit: a member's time per row goes by
+    // the vectors each of its threads holds (kGroupVecs at the cap), so the
+    // fewest members with full parts move the most bytes per exchange, even
+    // when n_sm / K groups leave SMs idle.  Measured on GB300 (256 MiB of
+    // rows, GB/s): fp32 1 MiB rows K = 16 (9 groups) 4746 against K = 19 (8
+    // groups) 4347, 17 and 18 lower still; bf16 1 MiB the same (3952 against
+    // 3635); bf16 512 KiB K = 8 4139 against K = 16 2612 and K = 19 2316;
+    // fp32 2 MiB K = 32 4336 against K = 38 3748.  Against the paths that
+    // stream a row twice through one CTA: groups of 2 and 4 lose (bf16
+    // 128 KiB 4006 against 4500, fp32 256 KiB 4709 against 4886), whose
+    // second read mostly hits L2 and which wait on no other CTA; groups of
+    // 64 lose to the two-launch segments (fp32 4 MiB rows 3612 against
+    // 3983), while fp32 2 MiB rows gain at K = 32 (4318 against 3978) and
+    // bf16 2 MiB rows lose a little there (3570 against 3602).
+    int64_t best_k = 0;
+    for (int64_t k = kmin; k <= std::min<int64_t>(int64_t(kMaxGroup), int64_t(n_sm)); ++k)
+        if (avail / stage_for(k) >= 3 && stage_for(k) <= part_cap) {
             best_k = k;
+            break;
         }
-    }
-    // Measured on GB300 (same run, 256 MiB of rows, against the paths that
-    // stream a row twice through one CTA): groups of 8 and 19 win (bf16
-    // 512 KiB rows 4134 against 4039 GB/s, fp32 1 MiB rows 4367 against
-    // 4014); groups of 2 and 4 lose to one CTA per row, whose second read
-    // mostly hits L2 and which waits on no other CTA (bf16 128 KiB 4006
-    // against 4500, fp32 256 KiB 4709 against 4886); groups of 38 and 76 lose
-    // to waiting for the slowest of their members at every row (bf16 2 MiB
-    // 3336 against 3600, fp32 4 MiB 3215 against 3948).
-    if (best_k == 0 || kmin < kGroupMinParts || best_k > kGroupMaxSize)
+    if (best_k == 0 || kmin < kGroupMinParts || best_k > (es == 2 ? kGroupMaxSizeBf16 : kGroupMaxSize))
         return 0;
     const int64_t G = n_sm / best_k;
     const int64_t waves = (n_cand + G - 1) / G;

@@ -87,7 +87,7 @@ def test_checked_backward_short_and_long():
 
 
 def test_checked_group_rows():
-    """Rows split over groups of CTAs (19 groups of 8 on 152 SMs): the
+    """Rows split over groups of CTAs (19 of the 25 groups of 6 on 152 SMs): the
     self-checking group kernel checks its bulk copies, stage reads and
     stores, and gives the same bits."""
     import torch

@@ -185,7 +185,7 @@ def test_withheld_stage_in_a_group_launch_times_out_and_context_survives():
     y = torch.zeros_like(x)
     bsm.bsm_device_status_clear()
     p = bsm.bsm_plan_create(x, y, w.rows, w.cols, w.dtype, bsm.POLICY_DYNAMIC)
-    assert p.stats()["group_rows"] == 19          # 19 groups of 8 CTAs on 152 SMs
+    assert p.stats()["group_rows"] == 19          # 19 of the 25 groups of 6 CTAs on 152 SMs
     bsm.bsm_plan_debug(p, bsm.DEBUG_WITHHOLD_STAGE, 100_000_000)      # 0.1 s waits
     t0 = time.time()
     p.execute()

@@ -189,15 +189,16 @@ def test_rows_of_two_chunks_stay_staged():
     assert set(L["phase0"]["part_count"]) == {1} and set(L["phase0"]["cols"]) == {65536}
 
 
-@pytest.mark.parametrize("C,dtype,k", [(65536, bsm.F32, 0), (98304, bsm.F32, 8), (262144, bsm.F32, 19),
-                                       (1048576, bsm.F32, 0), (65536, bsm.BF16, 0),
-                                       (262144, bsm.BF16, 8), (524288, bsm.BF16, 19),
-                                       (1048576, bsm.BF16, 0)])
+@pytest.mark.parametrize("C,dtype,k", [(65536, bsm.F32, 0), (98304, bsm.F32, 6), (262144, bsm.F32, 16),
+                                       (524288, bsm.F32, 32), (1048576, bsm.F32, 0),
+                                       (65536, bsm.BF16, 0), (262144, bsm.BF16, 8),
+                                       (524288, bsm.BF16, 16), (1048576, bsm.BF16, 0)])
 def test_long_rows_group_sizes(C, dtype, k):
-    """256 MiB of long rows: rows of 5 to 24 parts of 64 KiB go to groups of
-    K CTAs -- 8 or 19 on 152 SMs (divisors of 152) --, each CTA holding one
-    part; shorter rows (256 KiB fp32, 128 KiB bf16) stay on one CTA per row,
-    longer ones (4 MiB fp32, 2 MiB bf16) are streamed twice."""
+    """256 MiB of long rows: rows of 5 to 32 parts of at most 64 KiB (24 for
+    bf16) go to groups of K CTAs, the fewest whose parts fit (K = ceil(row /
+    64 KiB)), each CTA holding one part; shorter rows (256 KiB fp32, 128 KiB
+    bf16) stay on one CTA per row, longer ones (4 MiB fp32, 2 MiB bf16) are
+    streamed twice."""
     es = 4 if dtype == bsm.F32 else 2
     R = (256 << 20) // (C * es)
     L = check_layout([R], [C], dtype, bsm.POLICY_DYNAMIC)

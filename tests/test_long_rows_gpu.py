@@ -154,9 +154,10 @@ def test_many_long_rows_of_several_chunks(dtype, chunks, flags):
 
 
 # rows over groups: (rows, row length, dtype, group size on 152 SMs) -- one
-# full wave each (as many rows as groups, n_sm / K)
-GROUP_CASES = [(19, 98304, workload.F32, 8), (8, 262144, workload.F32, 19),
-               (19, 262144, workload.BF16, 8), (8, 524288, workload.BF16, 19)]
+# full wave each (as many rows as groups, n_sm // K)
+GROUP_CASES = [(25, 98304, workload.F32, 6), (9, 262144, workload.F32, 16),
+               (4, 524288, workload.F32, 32), (19, 262144, workload.BF16, 8),
+               (9, 524288, workload.BF16, 16)]
 
 
 @pytest.mark.parametrize("case", range(len(GROUP_CASES)))
