@@ -392,13 +392,15 @@ int cut_patches(const bsm_plan_desc *d, const std::vector<SliceView> &slices, in
         const int64_t two_chunk = std::max<int64_t>(min_stage, in_arrays * half);
         if (3 * two_chunk <= avail)
             stage = two_chunk;
-        else if (d->op == BSM_OP_FORWARD && es == 4)
-            // fp32 rows streamed in chunks: three stages of a third of the
-            // shared memory rather than two of the cap, so that a chunk is on
-            // its way while one is written and one computed (measured, same
-            // box: 256 KiB rows 4890 -> 5061 GB/s, 4 MiB rows 3950 -> 3977;
-            // bf16 2 MiB rows lose, 3609 -> 3533, and keep two stages; four
-            // stages gain nothing)
+        else if (d->op == BSM_OP_FORWARD && es == 4 && max_row > 2 * row_cap)
+            // fp32 rows streamed in more than two chunks of the cap: three
+            // stages of a third of the shared memory rather than two of the
+            // cap, so that a chunk is on its way while one is written and one
+            // computed (measured, same box: 256 KiB rows 4890 -> 5061 GB/s,
+            // 4 MiB rows 3950 -> 3977; bf16 2 MiB rows lose, 3609 -> 3533, and
+            // keep two stages; four stages gain nothing).  Rows of two chunks
+            // of the cap keep them: the smaller stages would cut them into
+            // three and re-read more (160 KiB rows 5235 against 4878)
             stage = std::min<int64_t>(stage, std::max<int64_t>(min_stage, (avail / 3) & ~int64_t(127)));
         else if (d->op == BSM_OP_BACKWARD) {
             // the backward pass's rows streamed by one CTA each (at least two
