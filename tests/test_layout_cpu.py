@@ -315,3 +315,23 @@ def test_edge_cases():
     L = check_layout([3], [1 << 22], bsm.BF16, bsm.POLICY_DYNAMIC, op=bsm.OP_BACKWARD)
     assert len(L["phase0"]) == len(L["phase1"]) == 3 * 145
     assert set(L["phase1"]["part_count"]) == {145}
+
+
+@pytest.mark.parametrize("rows,cols,dtype,op,stage,n_stages", [
+    # fp32 rows of two chunks of the 113 KiB cap keep two stages of the cap
+    (1638, 40960, bsm.F32, bsm.OP_FORWARD, 115712, 2),
+    # longer fp32 rows: three stages of a third of the shared memory
+    (1024, 65536, bsm.F32, bsm.OP_FORWARD, 77056, 3),
+    # bf16 rows streamed in chunks keep two stages of the cap
+    (1024, 131072, bsm.BF16, bsm.OP_FORWARD, 115712, 2),
+    # backward rows streamed by one CTA each (two waves or more): three stages
+    (1024, 65536, bsm.F32, bsm.OP_BACKWARD, 77056, 3),
+    # backward rows cut into segments (fewer than two per SM): two of the cap
+    (256, 262144, bsm.F32, bsm.OP_BACKWARD, 115712, 2),
+])
+def test_stage_size_of_streamed_rows(rows, cols, dtype, op, stage, n_stages):
+    """The stages that rows longer than one stage are streamed through, by
+    row length, dtype and pass (232448 bytes of shared memory, 152 SMs)."""
+    L = check_layout([rows], [cols], dtype, bsm.POLICY_DYNAMIC, op=op)
+    assert L["group_k"] == 0
+    assert (L["stage_bytes"], L["n_stages"]) == (stage, n_stages)
