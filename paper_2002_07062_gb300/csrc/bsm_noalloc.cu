@@ -8,7 +8,8 @@
 // whole device up front, a framework allocator that must see every byte), or
 // code that must not add cudaMalloc/cudaFree calls, which synchronise the
 // device, to a latency-critical path.  This entry point runs the same
-// persistent kernel under the one-queue dynamic schedule, with its scratch
+// persistent kernel under the one-queue dynamic schedule (a batch of at most
+// one patch per SM dealt statically, as the planned path deals it), with its scratch
 // (patch table, queue counters, status words) in one file-scope __device__
 // array of fixed size instead of allocated memory.  The caller still passes
 // x and y.  Rows must fit one shared-memory stage (BSM_NOALLOC_MAX_ROW_BYTES,
