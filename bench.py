@@ -1109,24 +1109,19 @@ def run_die_check(bsm, dev, dump=None):
     return 0
 
 def _sweep_cell(bsm, w, x, y, pol, rpi, reps, stream):
-    """Median ms of one policy on one workload; rpi > 0 caps the rows per
-    patch (a plan of its own), 0 lets patches fill a stage."""
-    plan = None
-    if rpi:
-        plan = bsm.bsm_plan_create(x, y, w.rows, w.cols, w.dtype, pol, offsets=w.offsets,
-                                   flags=w.flags, rows_per_item=rpi)
+    """Median ms of one policy on one workload, timed on a plan (one C call
+    per execute, so that the host never paces the kernels); rpi > 0 caps the
+    rows per patch, 0 lets patches fill a stage."""
+    plan = bsm.bsm_plan_create(x, y, w.rows, w.cols, w.dtype, pol, offsets=w.offsets,
+                               flags=w.flags, rows_per_item=rpi)
 
     def step():
-        if plan is not None:
-            plan.execute(stream)
-        else:
-            bsm.bsm_softmax_ragged(x, y, w.offsets, w.rows, w.cols, w.dtype, pol, w.flags, stream)
+        plan.execute(stream)
     for _ in range(3):
         step()
     stream.synchronize()
     med = _median_ms(step, reps, stream)
-    if plan is not None:
-        plan.close()
+    plan.close()
     return med
 
 

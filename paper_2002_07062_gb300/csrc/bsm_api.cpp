@@ -1611,6 +1611,21 @@ void bsm_set_device_checks(int on) { g_checked.store(on ? 1 : 0); }
 
 const char *bsm_last_cuda_error(void) { return t_last_error.c_str(); }
 
+int64_t bsm_ragged_extent(int64_t n, const int64_t *offsets, const int32_t *rows, const int32_t *cols)
+{
+    if (n < 0 || (n > 0 && (!offsets || !rows || !cols)))
+        return -1;
+    int64_t end = 0;
+    for (int64_t s = 0; s < n; ++s) {
+        if (rows[s] <= 0)
+            continue;
+        if (offsets[s] < 0 || cols[s] < 0)
+            return -1;
+        end = std::max<int64_t>(end, offsets[s] + int64_t(rows[s]) * cols[s]);
+    }
+    return end;
+}
+
 int64_t bsm_max_row_bytes(int device)
 {
     DeviceCtx *c = nullptr;

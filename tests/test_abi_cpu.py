@@ -224,3 +224,25 @@ def test_binding_rejects_host_strided_and_short_tensors():
     assert e.value.status == bsm.ERR_NO_DEVICE
     # empty batches need no buffer at all
     bsm.bsm_softmax(None, None, 0, 4, 64, bsm.F32, bsm.POLICY_RR)
+
+
+def test_ragged_extent_host_helper():
+    """bsm_ragged_extent: the end of the furthest non-empty slice, 0 for none,
+    -1 for a negative offset or column count (host only, no device)."""
+    import numpy as np
+    from paper_2002_07062_gb300 import bsm
+
+    def ext(off, rows, cols):
+        o = np.asarray(off, np.int64)
+        r = np.asarray(rows, np.int32)
+        c = np.asarray(cols, np.int32)
+        return int(bsm.lib().bsm_ragged_extent(len(o), o.ctypes.data_as(bsm.c_i64p),
+                                               r.ctypes.data_as(bsm.c_i32p),
+                                               c.ctypes.data_as(bsm.c_i32p)))
+    assert ext([0, 10], [0, 2], [5, 3]) == 16            # the empty slice is ignored
+    assert ext([100, 0], [1, 4], [8, 16]) == 108         # furthest end, not the last slice
+    assert ext([], [], []) == 0
+    assert ext([0], [0], [7]) == 0
+    assert ext([1 << 40], [3], [1 << 20]) == (1 << 40) + 3 * (1 << 20)
+    assert ext([-8], [1], [4]) == -1
+    assert ext([0], [1], [-4]) == -1
