@@ -324,6 +324,16 @@ int build_plan(GemmPlan *p, const GemmDev &dev)
         if (fit >= 2 || bufs <= 2 || p->want_bufs)
             break;
     }
+    // an output-heavy tile left with two stages: a third stage beats the
+    // extra store buffers (E1, 384 x (512x64)(64x512): 3 stages x 2 buffers
+    // 41.60 us against 2 x 4 41.85 us, same box)
+    if (!p->want_bufs && !p->want_stages && fit == 2 && bufs > 2) {
+        const int fit2 = (dev.smem_optin - gemm_fixed_smem(bn, p->out_bf16, 2)) / (kbs * gemm_stage_bytes(bn));
+        if (fit2 >= 3) {
+            bufs = 2;
+            fit = fit2;
+        }
+    }
     a.epi_bufs = bufs;
     a.kbs = kbs;
     a.identity = use_die ? 0 : 1;
