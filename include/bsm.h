@@ -595,7 +595,8 @@ int64_t bsm_max_row_bytes(int device);
  * offsets[s] + rows[s] * cols[s] (0 for none), for a caller that checks its
  * buffers before bsm_softmax_ragged (the Python binding does).  Host only;
  * offsets/rows/cols: host arrays of n entries (NULL allowed when n == 0).
- * Returns -1 for n < 0, a NULL array or a negative offset or column count. */
+ * Returns -1 for n < 0, a NULL array, a negative offset or column count, or
+ * an end past INT64_MAX. */
 int64_t bsm_ragged_extent(int64_t n, const int64_t *offsets, const int32_t *rows, const int32_t *cols);
 
 /* Static description of a status code. */

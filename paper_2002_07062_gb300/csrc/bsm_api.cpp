@@ -1621,7 +1621,10 @@ int64_t bsm_ragged_extent(int64_t n, const int64_t *offsets, const int32_t *rows
             continue;
         if (offsets[s] < 0 || cols[s] < 0)
             return -1;
-        end = std::max<int64_t>(end, offsets[s] + int64_t(rows[s]) * cols[s]);
+        const int64_t span = int64_t(rows[s]) * cols[s];     // < 2^62
+        if (offsets[s] > INT64_MAX - span)
+            return -1;
+        end = std::max<int64_t>(end, offsets[s] + span);
     }
     return end;
 }

@@ -246,3 +246,4 @@ def test_ragged_extent_host_helper():
     assert ext([1 << 40], [3], [1 << 20]) == (1 << 40) + 3 * (1 << 20)
     assert ext([-8], [1], [4]) == -1
     assert ext([0], [1], [-4]) == -1
+    assert ext([(1 << 63) - 8], [1], [16]) == -1               # past INT64_MAX
