@@ -1707,10 +1707,11 @@ __device__ __forceinline__ void group_load(uint4 (&r)[kGroupVecs], const unsigne
 // loaded first (independent loads), then its maximum taken and, when it
 // grows the running one, the sum rescaled; then the chunk's exponentials
 // added in vector order.  While the running maximum is -inf every value seen
-// is -inf (masked) or NaN: it adds 0 (NaN).
-template <typename Tag, bool Checked>
+// is -inf (masked) or NaN: it adds 0 (NaN).  `mid` runs halfway through (the
+// caller issues its exchange loads there).
+template <typename Tag, bool Checked, typename Mid>
 __device__ __forceinline__ void group_partial(const unsigned char *sbuf, int nvec, int tid, int col0, int row,
-                                              bool causal, const Bounds &bd, float &m, float &s)
+                                              bool causal, const Bounds &bd, float &m, float &s, Mid &&mid)
 {
     using E = Elem<Tag>;
     constexpr int EPV = E::kPerVec;
@@ -1719,6 +1720,8 @@ __device__ __forceinline__ void group_partial(const unsigned char *sbuf, int nve
     s = 0.0f;
 #pragma unroll
     for (int c = 0; c < kGroupVecs; c += kGroupChunk) {
+        if (c == kGroupVecs / 2)
+            mid();
         uint4 raw[kGroupChunk];
 #pragma unroll
         for (int j = 0; j < kGroupChunk; ++j) {
@@ -2019,17 +2022,21 @@ __global__ void __launch_bounds__(kThreads, 1) softmax_group(const KernelArgs a)
             Bounds bs = bdy;
             bs.s_lo = sbuf;
             bs.s_hi = sbuf + static_cast<size_t>(mt.C) * E::kSize;
-            // the held row's exchange words of rank `lane`, loaded now and
-            // used after this row's partial (their latency overlaps it)
+            // the held row's exchange words of rank `lane`, loaded halfway
+            // through this row's partial and used after it: late enough that
+            // most members have published, early enough that the second half
+            // covers the loads' latency
             unsigned long long pre0 = 0, pre1 = 0;
-            if (rh && lane < K) {
-                const unsigned long long *xs = &xch[2 * static_cast<size_t>(rx & (kGroupSlots - 1)) * K];
-                pre0 = ld_relaxed_u64(&xs[2 * lane]);
-                pre1 = ld_relaxed_u64(&xs[2 * lane + 1]);
-            }
+            auto poll = [&]() {
+                if (rh && lane < K) {
+                    const unsigned long long *xs = &xch[2 * static_cast<size_t>(rx & (kGroupSlots - 1)) * K];
+                    pre0 = ld_relaxed_u64(&xs[2 * lane]);
+                    pre1 = ld_relaxed_u64(&xs[2 * lane + 1]);
+                }
+            };
             // this member's (max, sum) of its part, from the stage
             float m_l, s_l;
-            group_partial<Tag, Checked>(sbuf, nvec, tid, mt.col0, mt.row0, causal, bs, m_l, s_l);
+            group_partial<Tag, Checked>(sbuf, nvec, tid, mt.col0, mt.row0, causal, bs, m_l, s_l, poll);
 #pragma unroll
             for (int o2 = 16; o2 >= 1; o2 >>= 1) {
                 const float mo2 = __shfl_xor_sync(0xFFFFFFFFu, m_l, o2);
