@@ -365,6 +365,9 @@ def main():
                          "(nested under 'workloads' in the JSON line)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=20)
+    ap.add_argument("--slices", type=int, default=0,
+                    help="run only the first N slices of the workload (same shapes and values): a "
+                         "smaller case of the same kernel, e.g. for a profiler capture of workload 4")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -404,7 +407,10 @@ def main():
     if args.long_rows:
         return run_long_rows(args, bsm, ws, rank, dev)
 
-    w = workload.config(args.workload).materialize()
+    w = workload.config(args.workload)
+    if 0 < args.slices < w.nslices:
+        w = workload.slice_sample(w, list(range(args.slices)))
+    w = w.materialize()
     pol = policy_code(args.policy)
     xh = w.x
     x = torch.from_numpy(xh.view(np.int16) if w.dtype == workload.BF16 else xh).cuda()
@@ -477,7 +483,8 @@ def main():
     # step is nothing but its launches)
     launch_ms = total_ms / (args.steps * launches_per_step)
     achieved = bytes_step / launches_per_step / (launch_ms * 1e-3) / 1e9
-    traffic = profiled_traffic(args.workload)
+    # (a sample of the workload's slices has no profiled figure of its own)
+    traffic = profiled_traffic(args.workload) if not args.slices else None
 
     out = {
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": ws,
