@@ -495,6 +495,50 @@ template <> __device__ __forceinline__ bool vec_poisons<BF16>(uint4 r)
     return !(lo < INFINITY) || !(hi < INFINITY);
 }
 
+// p = 2^(v*log2e - mL) for one vector in fp32 pairs (each pair two IEEE
+// fmas: the bits of vec_exp), and the vector's sum in tree_sum's order
+// ((p0 + p1) + (p2 + p3), and so on).
+template <int EPV>
+__device__ __forceinline__ float vec_exp_sum_pairs(float (&v)[EPV], float mL)
+{
+    const float2 l2 = make_float2(kLog2e, kLog2e), nm = make_float2(-mL, -mL);
+#pragma unroll
+    for (int e = 0; e < EPV; e += 2) {
+        const float2 t = fma2(make_float2(v[e], v[e + 1]), l2, nm);
+        v[e] = ex2(t.x);
+        v[e + 1] = ex2(t.y);
+    }
+    if constexpr (EPV == 4) {
+        const float2 a = add2(make_float2(v[0], v[2]), make_float2(v[1], v[3]));
+        return a.x + a.y;
+    } else {
+        const float2 a = add2(make_float2(v[0], v[4]), make_float2(v[1], v[5]));
+        const float2 b = add2(make_float2(v[2], v[6]), make_float2(v[3], v[7]));
+        const float2 c = add2(a, b);
+        return c.x + c.y;
+    }
+}
+
+// The maximum of a chunk's vectors as loaded: bf16 on the packed words
+// (exact; a NaN operand loses, as with fmaxf), fp32 through tree_max.
+template <typename Tag, int N>
+__device__ __forceinline__ float raw_max(const uint4 (&raw)[N], const float (&v)[N][Elem<Tag>::kPerVec])
+{
+    if constexpr (Elem<Tag>::kSize == 2) {
+        uint32_t mw = 0xFF80FF80u;
+#pragma unroll
+        for (int j = 0; j < N; ++j)
+            mw = bmax2(mw, bmax2(bmax2(raw[j].x, raw[j].y), bmax2(raw[j].z, raw[j].w)));
+        return fmaxf(__uint_as_float(mw << 16), __uint_as_float(mw & 0xFFFF0000u));
+    } else {
+        float m = -INFINITY;
+#pragma unroll
+        for (int j = 0; j < N; ++j)
+            m = fmaxf(m, tree_max<Elem<Tag>::kPerVec>(v[j]));
+        return m;
+    }
+}
+
 // Register-resident bf16 row (bf16 rows move 4 bytes per element, so
 // instruction issue matters): T lanes, V vectors per lane (vector j of lane l
 // is vector j*T + l of the row).  Arithmetic, the same in both variants and
@@ -1704,10 +1748,13 @@ __device__ __forceinline__ void group_load(uint4 (&r)[kGroupVecs], const unsigne
 // This thread's running (max, sum of exp(v - max)) over its vectors of the
 // part in the stage, in chunks of 16 elements (4 fp32 or 2 bf16 vectors, so
 // the chunk's unpacked values and the held row fit the registers): a chunk's vectors are
-// loaded first (independent loads), then its maximum taken and, when it
-// grows the running one, the sum rescaled; then the chunk's exponentials
-// added in vector order.  While the running maximum is -inf every value seen
-// is -inf (masked) or NaN: it adds 0 (NaN).  `mid` runs halfway through (the
+// loaded first (independent loads), then its maximum taken (bf16 without
+// the causal mask: on the packed words) and, when it grows the running one,
+// the sum rescaled; then the chunk's exponentials added in vector order,
+// computed in fp32 pairs (the same bits as one at a time: each pair is two
+// IEEE operations, each vector's sum in tree_sum's order).  While the
+// running maximum is -inf every value seen is -inf (masked) or NaN: it adds
+// 0 (NaN).  `mid` runs halfway through (the
 // caller issues its exchange loads there).
 template <typename Tag, bool Checked, typename Mid>
 __device__ __forceinline__ void group_partial(const unsigned char *sbuf, int nvec, int tid, int col0, int row,
@@ -1735,13 +1782,20 @@ __device__ __forceinline__ void group_partial(const unsigned char *sbuf, int nve
         }
         float cm = -INFINITY;
         float v[kGroupChunk][EPV];
+        if (causal) {
 #pragma unroll
-        for (int j = 0; j < kGroupChunk; ++j) {
-            const int col = col0 + (tid + (c + j) * kConsumerThreads) * EPV;
-            E::unpack(raw[j], v[j]);
-            if (causal && col + EPV - 1 > row)
-                apply_causal<EPV>(v[j], col, row);
-            cm = fmaxf(cm, tree_max<EPV>(v[j]));
+            for (int j = 0; j < kGroupChunk; ++j) {
+                const int col = col0 + (tid + (c + j) * kConsumerThreads) * EPV;
+                E::unpack(raw[j], v[j]);
+                if (col + EPV - 1 > row)
+                    apply_causal<EPV>(v[j], col, row);
+                cm = fmaxf(cm, tree_max<EPV>(v[j]));
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < kGroupChunk; ++j)
+                E::unpack(raw[j], v[j]);
+            cm = raw_max<Tag, kGroupChunk>(raw, v);
         }
         if (cm > m) {
             s *= ex2((m - cm) * kLog2e);
@@ -1753,14 +1807,19 @@ __device__ __forceinline__ void group_partial(const unsigned char *sbuf, int nve
             const int vi = tid + (c + j) * kConsumerThreads;
             const int col = col0 + vi * EPV;
             if (vi < nvec) {
-                vec_exp<EPV>(v[j], mL, (causal && col > row) || m == -INFINITY);
-                s += tree_sum<EPV>(v[j]);
+                if ((causal && col > row) || m == -INFINITY) {
+                    vec_exp<EPV>(v[j], mL, true);
+                    s += tree_sum<EPV>(v[j]);
+                } else {
+                    s += vec_exp_sum_pairs<EPV>(v[j], mL);
+                }
             }
         }
     }
 }
 
-// y = exp(v - M) / S for this thread's vectors of the part (mL = M log2 e).
+// y = exp(v - M) / S for this thread's vectors of the part (mL = M log2 e),
+// in fp32 pairs where no element is masked.
 template <typename Tag, bool Checked>
 __device__ __forceinline__ void group_write(const uint4 (&r)[kGroupVecs], int nvec, int tid, int col0, int row,
                                             bool causal, float mL, float inv, unsigned char *ypart, const Bounds &bd)
@@ -1777,10 +1836,22 @@ __device__ __forceinline__ void group_write(const uint4 (&r)[kGroupVecs], int nv
             E::unpack(r[j], v);
             if (causal && !masked && col + EPV - 1 > row)
                 apply_causal<EPV>(v, col, row);
-            vec_exp<EPV>(v, mL, masked);
+            if (masked) {
+                vec_exp<EPV>(v, mL, true);
 #pragma unroll
-            for (int e = 0; e < EPV; ++e)
-                v[e] *= inv;
+                for (int e = 0; e < EPV; ++e)
+                    v[e] *= inv;
+            } else {
+                const float2 l2 = make_float2(kLog2e, kLog2e), nm = make_float2(-mL, -mL);
+                const float2 i2 = make_float2(inv, inv);
+#pragma unroll
+                for (int e = 0; e < EPV; e += 2) {
+                    const float2 t = fma2(make_float2(v[e], v[e + 1]), l2, nm);
+                    const float2 y2 = mul2(make_float2(ex2(t.x), ex2(t.y)), i2);
+                    v[e] = y2.x;
+                    v[e + 1] = y2.y;
+                }
+            }
             store_vec<Checked>(ypart + 16 * vi, bd, E::pack(v));
         }
     }
