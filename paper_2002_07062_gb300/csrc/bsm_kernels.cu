@@ -922,9 +922,14 @@ __device__ __forceinline__ void long_chunk(const unsigned char *sbuf, const Stag
                 }
             }
             // while the running max is still -inf every value seen is -inf (or
-            // NaN): it adds 0 (NaN), as a masked vector does
-            vec_exp<EPV>(v, m_l * kLog2e, masked || m_l == -INFINITY);
-            s_l += tree_sum<EPV>(v);
+            // NaN): it adds 0 (NaN), as a masked vector does; otherwise the
+            // exponentials in fp32 pairs (the same bits as one at a time)
+            if (masked || m_l == -INFINITY) {
+                vec_exp<EPV>(v, m_l * kLog2e, true);
+                s_l += tree_sum<EPV>(v);
+            } else {
+                s_l += vec_exp_sum_pairs<EPV>(v, m_l * kLog2e);
+            }
         } else {
             vec_exp<EPV>(v, mL, masked);
 #pragma unroll
