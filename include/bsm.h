@@ -61,7 +61,7 @@
  *     into segments spread over the SMs and the execute takes two launches
  *     (segment partials, then combine and write); otherwise each row stays
  *     on one SM within one launch.  Forward rows of 5 to 32 parts of at most
- *     64 KiB (24 for bf16), enough of them to fill two thirds of the groups'
+ *     64 KiB, enough of them to fill two thirds of the groups'
  *     waves, are instead split over groups of K CTAs (K = ceil(row / 64
  *     KiB); n_sm / K groups) in one cooperative launch: each CTA stages one
  *     part, the group exchanges (max, sum) partials through global memory

@@ -297,7 +297,6 @@ struct PatchLayout {
 // only, never on the policy.
 constexpr int64_t kGroupMinParts = 5;    // rows of fewer parts stay on one CTA
 constexpr int64_t kGroupMaxSize = 32;    // larger groups wait too long on their slowest member
-constexpr int64_t kGroupMaxSizeBf16 = 24; // (bf16: 32 already loses to the two-launch segments)
 
 int choose_groups(const std::vector<SliceView> &slices, int es, int n_sm, int64_t smem_optin, PatchLayout &L)
 {
@@ -333,15 +332,17 @@ int choose_groups(const std::vector<SliceView> &slices, int es, int n_sm, int64_
     // 128 KiB 4006 against 4500, fp32 256 KiB 4709 against 4886), whose
     // second read mostly hits L2 and which wait on no other CTA; groups of
     // 64 lose to the two-launch segments (fp32 4 MiB rows 3612 against
-    // 3983), while fp32 2 MiB rows gain at K = 32 (4318 against 3978) and
-    // bf16 2 MiB rows lose a little there (3570 against 3602).
+    // 3983), while fp32 2 MiB rows gain at K = 32 (4318 against 3978).  bf16
+    // rows of 1.75 and 2 MiB (K = 28, 32) lost a little to the segments with
+    // scalar arithmetic in the group routines (3570 against 3602) and gain
+    // with pair arithmetic (4042 against 3700, 3756 against 3650).
     int64_t best_k = 0;
     for (int64_t k = kmin; k <= std::min<int64_t>(int64_t(kMaxGroup), int64_t(n_sm)); ++k)
         if (avail / stage_for(k) >= 3 && stage_for(k) <= part_cap) {
             best_k = k;
             break;
         }
-    if (best_k == 0 || kmin < kGroupMinParts || best_k > (es == 2 ? kGroupMaxSizeBf16 : kGroupMaxSize))
+    if (best_k == 0 || kmin < kGroupMinParts || best_k > kGroupMaxSize)
         return 0;
     const int64_t G = n_sm / best_k;
     const int64_t waves = (n_cand + G - 1) / G;

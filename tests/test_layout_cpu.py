@@ -192,13 +192,14 @@ def test_rows_of_two_chunks_stay_staged():
 @pytest.mark.parametrize("C,dtype,k", [(65536, bsm.F32, 0), (98304, bsm.F32, 6), (262144, bsm.F32, 16),
                                        (524288, bsm.F32, 32), (1048576, bsm.F32, 0),
                                        (65536, bsm.BF16, 0), (262144, bsm.BF16, 8),
-                                       (524288, bsm.BF16, 16), (1048576, bsm.BF16, 0)])
+                                       (524288, bsm.BF16, 16), (1048576, bsm.BF16, 32),
+                                       (2097152, bsm.BF16, 0)])
 def test_long_rows_group_sizes(C, dtype, k):
-    """256 MiB of long rows: rows of 5 to 32 parts of at most 64 KiB (24 for
-    bf16) go to groups of K CTAs, the fewest whose parts fit (K = ceil(row /
-    64 KiB)), each CTA holding one part; shorter rows (256 KiB fp32, 128 KiB
-    bf16) stay on one CTA per row, longer ones (4 MiB fp32, 2 MiB bf16) are
-    streamed twice."""
+    """256 MiB of long rows: rows of 5 to 32 parts of at most 64 KiB go to
+    groups of K CTAs, the fewest whose parts fit (K = ceil(row / 64 KiB)),
+    each CTA holding one part; shorter rows (256 KiB fp32, 128 KiB bf16) stay
+    on one CTA per row, longer ones (4 MiB of either type) are streamed
+    twice."""
     es = 4 if dtype == bsm.F32 else 2
     R = (256 << 20) // (C * es)
     L = check_layout([R], [C], dtype, bsm.POLICY_DYNAMIC)

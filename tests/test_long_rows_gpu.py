@@ -157,7 +157,7 @@ def test_many_long_rows_of_several_chunks(dtype, chunks, flags):
 # full wave each (as many rows as groups, n_sm // K)
 GROUP_CASES = [(25, 98304, workload.F32, 6), (9, 262144, workload.F32, 16),
                (4, 524288, workload.F32, 32), (19, 262144, workload.BF16, 8),
-               (9, 524288, workload.BF16, 16)]
+               (9, 524288, workload.BF16, 16), (4, 1048576, workload.BF16, 32)]
 
 
 @pytest.mark.parametrize("case", range(len(GROUP_CASES)))
