@@ -192,8 +192,8 @@ def test_rows_of_two_chunks_stay_staged():
 @pytest.mark.parametrize("C,dtype,k", [(65536, bsm.F32, 0), (98304, bsm.F32, 6), (262144, bsm.F32, 16),
                                        (524288, bsm.F32, 32), (1048576, bsm.F32, 0),
                                        (65536, bsm.BF16, 0), (262144, bsm.BF16, 8),
-                                       (524288, bsm.BF16, 16), (1048576, bsm.BF16, 32),
-                                       (2097152, bsm.BF16, 0)])
+                                       (524288, bsm.BF16, 16), (917504, bsm.BF16, 28),
+                                       (1048576, bsm.BF16, 32), (2097152, bsm.BF16, 0)])
 def test_long_rows_group_sizes(C, dtype, k):
     """256 MiB of long rows: rows of 5 to 32 parts of at most 64 KiB go to
     groups of K CTAs, the fewest whose parts fit (K = ceil(row / 64 KiB)),
